@@ -1,0 +1,199 @@
+"""fp64 CPU oracle of the PIC decode synthesis (Sec. 3.1 Eq. 1, Sec. 4.1, App. A).
+
+TEST INFRASTRUCTURE ONLY: the parity oracle for the CUDA decoder.  Only the
+tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py``
+import this module.  It shares no code with the CUDA path and never imports
+the ``paper_2609_09020_gb300`` package.
+
+The arithmetic lives in ``pic_oracle.c`` (plain C, double precision, compiled
+with ``-O2 -ffp-contract=off``); this module compiles it with gcc and marshals
+numpy arrays through ctypes.
+
+Parity status of each function (what pins it is in tests/test_oracle.py):
+  dequant             pinned (exact integer x power-of-two products)
+  bilinear/upsample   pinned (constants, affine grids, brute-force
+                      half-pixel interpolation, hand-computed grids)
+  mlp                 pinned (zero/identity weights, hand-computed layers,
+                      GELU closed forms)
+  decode              pinned (hand-computed 4x4 image, reductions to the
+                      pieces above, planted-mistake runs)
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "pic_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libpic_oracle.so")
+
+ACT_RELU = 0
+ACT_GELU = 1
+ACTS = {"relu": ACT_RELU, "gelu": ACT_GELU}
+
+_lock = threading.Lock()
+_lib = None
+
+
+def compile_oracle(src: str = _SRC, out: str = _LIB_PATH, extra_flags=()) -> str:
+    """Compiles the oracle C file into a shared library with gcc; returns its path."""
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    cmd = ["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fopenmp", "-shared",
+           "-fPIC", "-std=c11", *extra_flags, "-o", out + ".tmp", src, "-lm"]
+    subprocess.run(cmd, check=True, capture_output=True, text=True)
+    os.replace(out + ".tmp", out)
+    return out
+
+
+def _needs_build() -> bool:
+    return (not os.path.exists(_LIB_PATH)) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC)
+
+
+def _declare(lib):
+    c_int, c_i64, c_dbl = ctypes.c_int, ctypes.c_int64, ctypes.c_double
+    p = ctypes.c_void_p
+    lib.pic_oracle_level_size.argtypes = [c_int, c_int]
+    lib.pic_oracle_level_size.restype = c_int
+    lib.pic_oracle_latent_count.argtypes = [c_int, c_int, c_int, c_int]
+    lib.pic_oracle_latent_count.restype = c_i64
+    lib.pic_oracle_param_count.argtypes = [c_int, p]
+    lib.pic_oracle_param_count.restype = c_i64
+    lib.pic_oracle_dequant.argtypes = [p, c_i64, c_dbl, p]
+    lib.pic_oracle_dequant.restype = None
+    lib.pic_oracle_bilinear_at.argtypes = [p, c_int, c_int, c_int, c_int, c_int, c_int]
+    lib.pic_oracle_bilinear_at.restype = c_dbl
+    lib.pic_oracle_upsample.argtypes = [p, c_int, c_int, c_int, c_int, p]
+    lib.pic_oracle_upsample.restype = None
+    lib.pic_oracle_act.argtypes = [c_dbl, c_int]
+    lib.pic_oracle_act.restype = c_dbl
+    lib.pic_oracle_mlp.argtypes = [p, p, c_int, p, c_int, p]
+    lib.pic_oracle_mlp.restype = c_int
+    lib.pic_oracle_clamp01.argtypes = [c_dbl]
+    lib.pic_oracle_clamp01.restype = c_dbl
+    lib.pic_oracle_decode.argtypes = [p, p, p, c_int, c_int, c_int, p, c_int, c_int,
+                                      c_int, c_int, p, p, c_int]
+    lib.pic_oracle_decode.restype = c_int
+    lib.pic_oracle_decode_pixels.argtypes = [p, p, p, c_int, c_int, c_int, p, c_int, c_int,
+                                             c_int, c_int, p, c_i64, p, p]
+    lib.pic_oracle_decode_pixels.restype = c_int
+    return lib
+
+
+def load(path: str | None = None):
+    """Returns the ctypes handle of the oracle library, compiling it if needed.
+
+    With ``path`` given, loads that (already compiled) library instead; the
+    planted-mistake tests use this for mutated copies of the oracle."""
+    global _lib
+    if path is not None:
+        return Oracle(_declare(ctypes.CDLL(path)))
+    with _lock:
+        if _lib is None:
+            if _needs_build():
+                compile_oracle()
+            _lib = Oracle(_declare(ctypes.CDLL(_LIB_PATH)))
+    return _lib
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+class Oracle:
+    """numpy front end of one compiled copy of the oracle library."""
+
+    def __init__(self, lib):
+        self.lib = lib
+
+    # ---- shapes -------------------------------------------------------
+    def level_size(self, n: int, l: int) -> int:
+        return int(self.lib.pic_oracle_level_size(n, l))
+
+    def latent_count(self, H: int, W: int, L: int, C: int) -> int:
+        return int(self.lib.pic_oracle_latent_count(H, W, L, C))
+
+    def param_count(self, dims) -> int:
+        d = np.ascontiguousarray(dims, dtype=np.int32)
+        return int(self.lib.pic_oracle_param_count(len(d) - 1, _ptr(d)))
+
+    # ---- pieces ------------------------------------------------------
+    def dequant(self, q: np.ndarray, step: float) -> np.ndarray:
+        q = np.ascontiguousarray(q, dtype=np.int32)
+        y = np.empty(q.shape, dtype=np.float64)
+        self.lib.pic_oracle_dequant(_ptr(q), q.size, float(step), _ptr(y))
+        return y
+
+    def bilinear_at(self, g: np.ndarray, H: int, W: int, x: int, y: int) -> float:
+        g = np.ascontiguousarray(g, dtype=np.float64)
+        return float(self.lib.pic_oracle_bilinear_at(_ptr(g), g.shape[0], g.shape[1], H, W, x, y))
+
+    def upsample(self, g: np.ndarray, H: int, W: int) -> np.ndarray:
+        g = np.ascontiguousarray(g, dtype=np.float64)
+        out = np.empty((H, W), dtype=np.float64)
+        self.lib.pic_oracle_upsample(_ptr(g), g.shape[0], g.shape[1], H, W, _ptr(out))
+        return out
+
+    def act(self, z: float, act: str) -> float:
+        return float(self.lib.pic_oracle_act(float(z), ACTS[act]))
+
+    def mlp(self, feat: np.ndarray, weights: np.ndarray, dims, act: str) -> np.ndarray:
+        feat = np.ascontiguousarray(feat, dtype=np.float64)
+        w = np.ascontiguousarray(weights, dtype=np.float64)
+        d = np.ascontiguousarray(dims, dtype=np.int32)
+        out = np.empty(int(d[-1]), dtype=np.float64)
+        rc = self.lib.pic_oracle_mlp(_ptr(feat), _ptr(w), len(d) - 1, _ptr(d), ACTS[act], _ptr(out))
+        if rc != 0:
+            raise ValueError("oracle mlp rejected the dims")
+        return out
+
+    def clamp01(self, v: float) -> float:
+        return float(self.lib.pic_oracle_clamp01(float(v)))
+
+    # ---- whole decode --------------------------------------------------
+    def decode(self, latents, steps, weights, H, W, L, C, dims, act, clamp=True,
+               nthreads: int = 1) -> np.ndarray:
+        """Decodes one image; returns planar fp64 [3][H][W]."""
+        q = np.ascontiguousarray(latents, dtype=np.int32).ravel()
+        s = np.ascontiguousarray(steps, dtype=np.float64).ravel()
+        w = np.ascontiguousarray(weights, dtype=np.float64).ravel()
+        d = np.ascontiguousarray(dims, dtype=np.int32)
+        if q.size != self.latent_count(H, W, L, C) or s.size != L or w.size != self.param_count(d):
+            raise ValueError("oracle decode: buffer sizes do not match the shapes")
+        out = np.empty((3, H, W), dtype=np.float64)
+        work = np.empty(max(q.size, 1), dtype=np.float64)
+        rc = self.lib.pic_oracle_decode(_ptr(q), _ptr(s), _ptr(w), L, C, len(d) - 1, _ptr(d),
+                                        ACTS[act], int(bool(clamp)), H, W, _ptr(out), _ptr(work),
+                                        int(nthreads))
+        if rc != 0:
+            raise ValueError("oracle decode rejected the arguments")
+        return out
+
+    def decode_pixels(self, latents, steps, weights, H, W, L, C, dims, act, pix,
+                      clamp=True) -> np.ndarray:
+        """Decodes the pixels with flat indices ``pix`` (y * W + x); returns [n][3]."""
+        q = np.ascontiguousarray(latents, dtype=np.int32).ravel()
+        s = np.ascontiguousarray(steps, dtype=np.float64).ravel()
+        w = np.ascontiguousarray(weights, dtype=np.float64).ravel()
+        d = np.ascontiguousarray(dims, dtype=np.int32)
+        p = np.ascontiguousarray(pix, dtype=np.int64).ravel()
+        if q.size != self.latent_count(H, W, L, C) or s.size != L or w.size != self.param_count(d):
+            raise ValueError("oracle decode_pixels: buffer sizes do not match the shapes")
+        out = np.empty((p.size, 3), dtype=np.float64)
+        work = np.empty(max(q.size, 1), dtype=np.float64)
+        rc = self.lib.pic_oracle_decode_pixels(_ptr(q), _ptr(s), _ptr(w), L, C, len(d) - 1,
+                                               _ptr(d), ACTS[act], int(bool(clamp)), H, W,
+                                               _ptr(p), p.size, _ptr(out), _ptr(work))
+        if rc != 0:
+            raise ValueError("oracle decode_pixels rejected the arguments")
+        return out
+
+
+def build() -> str:
+    """Compiles the oracle library (used by the build step); returns its path."""
+    with _lock:
+        return compile_oracle()

@@ -1,0 +1,261 @@
+/*
+ * pic_oracle.c -- plain, slow, fp64 CPU decoder for the PIC synthesis g_r
+ * (Sec. 3.1, Eq. 1; Sec. 3.3; Sec. 4.1 "Implementation Details"; App. A).
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the parity oracle for the CUDA
+ * decoder.  Only the test suite, the smoke check and the CPU-baseline leg of
+ * the benchmark load it.  It shares no code, header, table or constant with
+ * the CUDA path, and the CUDA path never calls it.
+ *
+ * What it computes, per output pixel (x, y) of an H x W image:
+ *   1. dequantisation of the integer latent symbols of every pyramid level
+ *      (Fig. 1: the decoder reconstructs real latents from quantised symbols):
+ *          y_l[c][v][u] = q_l[c][v][u] * step_l
+ *   2. upsampling of every level to H x W (Sec. 3.1, after Eq. 1: "y_hat is
+ *      upsampled to y_u in R^{C x H x W}").  The paper does not name the
+ *      kernel; this oracle uses bilinear interpolation with half-pixel
+ *      centres and edge clamping, the size-based scale W_l / W and H_l / H.
+ *   3. per-pixel concatenation of all levels into the feature vector that
+ *      feeds g_s (Sec. 3.1: y_u has C channels at every pixel).  Order:
+ *      level-major, finest level first, channel-minor.
+ *   4. the synthesis MLP g_s (Sec. 4.1: an MLP with ReLU activations; the
+ *      decoder only needs the fused weights w', b', App. A):
+ *          h_{k+1} = act(W_k h_k + b_k) for hidden layers, linear last layer.
+ *      act is ReLU, or GELU in its exact erf form.
+ *   5. clamp of the RGB output to [0, 1].
+ *
+ * Notation: the paper numbers levels i = 1..L with i = L the finest
+ * (H_i = H / 2^(L-i), Eq. 1).  Here l = L - i, so l = 0 is the full-resolution
+ * level and H_l = ceil(H / 2^l), W_l = ceil(W / 2^l) (Eq. 1 assumes exact
+ * division; the ceiling covers sizes that are not multiples of 2^l).
+ *
+ * Memory layouts (all row-major, contiguous):
+ *   latents : levels l = 0..L-1 concatenated, each level planar [C][H_l][W_l]
+ *   steps   : [L]
+ *   weights : for k = 0..n-1: W_k [dims[k+1]][dims[k]] then b_k [dims[k+1]]
+ *   out_rgb : planar [3][H][W]
+ *
+ * Arithmetic is double throughout, every sum in index order; build with
+ * -O2 -ffp-contract=off so that no fused multiply-add changes the rounding.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stddef.h>
+
+#define PIC_ORACLE_ACT_RELU 0
+#define PIC_ORACLE_ACT_GELU 1
+
+#define PIC_ORACLE_MAX_LEVELS 16
+#define PIC_ORACLE_MAX_WIDTH 512
+
+/* Size of pyramid level l: ceil(n / 2^l) (Eq. 1, ceiling reading). */
+static int level_size(int n, int l)
+{
+    int64_t p = (int64_t)1 << l;
+    return (int)(((int64_t)n + p - 1) / p);
+}
+
+int pic_oracle_level_size(int n, int l)
+{
+    if (n <= 0 || l < 0 || l > 30) return -1;
+    return level_size(n, l);
+}
+
+/* Number of int32 symbols of one image's pyramid: sum_l C * H_l * W_l. */
+int64_t pic_oracle_latent_count(int H, int W, int L, int C)
+{
+    int64_t n = 0;
+    for (int l = 0; l < L; ++l)
+        n += (int64_t)C * level_size(H, l) * level_size(W, l);
+    return n;
+}
+
+/* Number of weight + bias values of the MLP: sum_k d_{k+1} (d_k + 1). */
+int64_t pic_oracle_param_count(int n_layers, const int *dims)
+{
+    int64_t n = 0;
+    for (int k = 0; k < n_layers; ++k)
+        n += (int64_t)dims[k + 1] * dims[k] + dims[k + 1];
+    return n;
+}
+
+/* Step 1: dequantisation y = q * step, element by element. */
+void pic_oracle_dequant(const int32_t *q, int64_t n, double step, double *y)
+{
+    for (int64_t i = 0; i < n; ++i)
+        y[i] = (double)q[i] * step;
+}
+
+/*
+ * Step 2 at one output pixel: bilinear sample of a Hl x Wl grid g, seen as an
+ * image stretched over H x W output pixels.  The source coordinate of output
+ * pixel centre x + 1/2 is (x + 1/2) * Wl / W - 1/2, clamped below at 0; the
+ * right/bottom neighbour index is clamped at the last row/column.
+ */
+double pic_oracle_bilinear_at(const double *g, int Hl, int Wl, int H, int W,
+                              int x, int y)
+{
+    double sx = ((double)x + 0.5) * ((double)Wl / (double)W) - 0.5;
+    double sy = ((double)y + 0.5) * ((double)Hl / (double)H) - 0.5;
+    if (sx < 0.0) sx = 0.0;
+    if (sy < 0.0) sy = 0.0;
+    int u0 = (int)floor(sx);
+    int v0 = (int)floor(sy);
+    int u1 = (u0 + 1 < Wl) ? u0 + 1 : Wl - 1;
+    int v1 = (v0 + 1 < Hl) ? v0 + 1 : Hl - 1;
+    double a = sx - (double)u0; /* weight of column u1 */
+    double b = sy - (double)v0; /* weight of row v1 */
+    double top = (1.0 - a) * g[(int64_t)v0 * Wl + u0] + a * g[(int64_t)v0 * Wl + u1];
+    double bot = (1.0 - a) * g[(int64_t)v1 * Wl + u0] + a * g[(int64_t)v1 * Wl + u1];
+    return (1.0 - b) * top + b * bot;
+}
+
+/* Step 2 over a whole image: out[y][x] = bilinear sample at (x, y). */
+void pic_oracle_upsample(const double *g, int Hl, int Wl, int H, int W, double *out)
+{
+    for (int y = 0; y < H; ++y)
+        for (int x = 0; x < W; ++x)
+            out[(int64_t)y * W + x] = pic_oracle_bilinear_at(g, Hl, Wl, H, W, x, y);
+}
+
+/* Hidden activation.  GELU(z) = z * Phi(z) = 0.5 z (1 + erf(z / sqrt 2)). */
+double pic_oracle_act(double z, int act)
+{
+    if (act == PIC_ORACLE_ACT_GELU)
+        return 0.5 * z * (1.0 + erf(z / sqrt(2.0)));
+    return z > 0.0 ? z : 0.0;
+}
+
+/*
+ * Step 4: g_s on one feature vector.  W_k is [dims[k+1]][dims[k]] row-major
+ * followed by b_k; z_i = sum_j W_k[i][j] h_j + b_k[i], summed in j order.
+ * Returns 0, or -1 for unsupported dims.
+ */
+int pic_oracle_mlp(const double *in, const double *weights, int n_layers,
+                   const int *dims, int act, double *out)
+{
+    double h[PIC_ORACLE_MAX_WIDTH], z[PIC_ORACLE_MAX_WIDTH];
+    if (n_layers < 1) return -1;
+    for (int k = 0; k <= n_layers; ++k)
+        if (dims[k] < 1 || dims[k] > PIC_ORACLE_MAX_WIDTH) return -1;
+    for (int j = 0; j < dims[0]; ++j) h[j] = in[j];
+    const double *p = weights;
+    for (int k = 0; k < n_layers; ++k) {
+        int din = dims[k], dout = dims[k + 1];
+        const double *Wk = p;
+        const double *bk = p + (int64_t)dout * din;
+        for (int i = 0; i < dout; ++i) {
+            double s = 0.0;
+            for (int j = 0; j < din; ++j) s += Wk[(int64_t)i * din + j] * h[j];
+            z[i] = s + bk[i];
+        }
+        int last = (k == n_layers - 1);
+        for (int i = 0; i < dout; ++i) h[i] = last ? z[i] : pic_oracle_act(z[i], act);
+        p = bk + dout;
+    }
+    for (int i = 0; i < dims[n_layers]; ++i) out[i] = h[i];
+    return 0;
+}
+
+/* Step 5: clamp to [0, 1]. */
+double pic_oracle_clamp01(double v)
+{
+    if (v < 0.0) return 0.0;
+    if (v > 1.0) return 1.0;
+    return v;
+}
+
+/* Checks shared by the two decode entry points. */
+static int check_args(int H, int W, int L, int C, int n_layers, const int *dims)
+{
+    if (H < 1 || W < 1 || L < 1 || L > PIC_ORACLE_MAX_LEVELS || C < 1) return -1;
+    if (n_layers < 1 || dims[0] != L * C || dims[n_layers] != 3) return -1;
+    for (int k = 0; k <= n_layers; ++k)
+        if (dims[k] < 1 || dims[k] > PIC_ORACLE_MAX_WIDTH) return -1;
+    return 0;
+}
+
+/*
+ * Steps 1-5 at one pixel, given the dequantised levels y[l] (planar [C][H_l][W_l]).
+ */
+static int decode_pixel(double *const *y, int L, int C, const double *weights,
+                        int n_layers, const int *dims, int act, int clamp,
+                        int H, int W, int x, int yy, double *rgb)
+{
+    double f[PIC_ORACLE_MAX_WIDTH];
+    int d = 0;
+    for (int l = 0; l < L; ++l) {
+        int Hl = level_size(H, l), Wl = level_size(W, l);
+        for (int c = 0; c < C; ++c)
+            f[d++] = pic_oracle_bilinear_at(y[l] + (int64_t)c * Hl * Wl, Hl, Wl, H, W, x, yy);
+    }
+    if (pic_oracle_mlp(f, weights, n_layers, dims, act, rgb) != 0) return -1;
+    if (clamp)
+        for (int c = 0; c < 3; ++c) rgb[c] = pic_oracle_clamp01(rgb[c]);
+    return 0;
+}
+
+/* Dequantises every level of one pyramid into `work`; fills y[l]. */
+static void dequant_pyramid(const int32_t *latents, const double *steps, int L, int C,
+                            int H, int W, double *work, double **y)
+{
+    int64_t off = 0;
+    for (int l = 0; l < L; ++l) {
+        int64_t n = (int64_t)C * level_size(H, l) * level_size(W, l);
+        y[l] = work + off;
+        pic_oracle_dequant(latents + off, n, steps[l], y[l]);
+        off += n;
+    }
+}
+
+/*
+ * Full decode of one image.  `work` must hold pic_oracle_latent_count(H, W, L, C)
+ * doubles.  nthreads > 1 splits the output rows over OpenMP threads (the
+ * arithmetic of each pixel does not change).  Returns 0 or -1.
+ */
+int pic_oracle_decode(const int32_t *latents, const double *steps, const double *weights,
+                      int L, int C, int n_layers, const int *dims, int act, int clamp,
+                      int H, int W, double *out_rgb, double *work, int nthreads)
+{
+    double *y[PIC_ORACLE_MAX_LEVELS];
+    if (check_args(H, W, L, C, n_layers, dims) != 0) return -1;
+    dequant_pyramid(latents, steps, L, C, H, W, work, y);
+    int64_t plane = (int64_t)H * W;
+    int bad = 0;
+#ifdef _OPENMP
+#pragma omp parallel for num_threads(nthreads > 0 ? nthreads : 1) schedule(static) reduction(| : bad)
+#endif
+    for (int yy = 0; yy < H; ++yy) {
+        for (int x = 0; x < W; ++x) {
+            double rgb[3];
+            if (decode_pixel(y, L, C, weights, n_layers, dims, act, clamp, H, W, x, yy, rgb) != 0) {
+                bad = 1;
+                continue;
+            }
+            for (int c = 0; c < 3; ++c) out_rgb[c * plane + (int64_t)yy * W + x] = rgb[c];
+        }
+    }
+    (void)nthreads;
+    return bad ? -1 : 0;
+}
+
+/*
+ * Decode only the listed pixels (index y * W + x) of one image; out is
+ * [npix][3].  Used to check full-size outputs at sampled positions.
+ */
+int pic_oracle_decode_pixels(const int32_t *latents, const double *steps, const double *weights,
+                             int L, int C, int n_layers, const int *dims, int act, int clamp,
+                             int H, int W, const int64_t *pix, int64_t npix, double *out,
+                             double *work)
+{
+    double *y[PIC_ORACLE_MAX_LEVELS];
+    if (check_args(H, W, L, C, n_layers, dims) != 0) return -1;
+    dequant_pyramid(latents, steps, L, C, H, W, work, y);
+    for (int64_t i = 0; i < npix; ++i) {
+        if (pix[i] < 0 || pix[i] >= (int64_t)H * W) return -1;
+        int yy = (int)(pix[i] / W), x = (int)(pix[i] % W);
+        if (decode_pixel(y, L, C, weights, n_layers, dims, act, clamp, H, W, x, yy, out + 3 * i) != 0)
+            return -1;
+    }
+    return 0;
+}

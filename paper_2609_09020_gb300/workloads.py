@@ -1,0 +1,206 @@
+"""Seeded synthetic inputs shaped like PIC's decode workloads.
+
+This module only draws random inputs and describes their shapes.  It holds
+none of the decoder's arithmetic (no dequantisation, interpolation or MLP), so
+both the fp64 oracle side and the CUDA side of the tests may use it.
+
+Shapes follow the decoder's statement of the problem (Sec. 3.1, Eq. 1): an
+H x W image is represented by L latent grids, level l (0 = full resolution)
+of size ceil(H / 2^l) x ceil(W / 2^l) with C channels, and by the weights of
+the synthesis MLP g_s (Sec. 4.1).  The paper evaluates on Kodak (24 images of
+768 x 512) and on CLIC high-resolution images (Sec. 4.1 "Dataset"); neither
+dataset is available, so seeded stand-ins are drawn instead:
+
+* latent symbols: a discretised Laplacian, round(Laplace(0, scale)) clipped to
+  +-clip, int32 -- the heavy-tailed, zero-peaked statistics of quantised
+  transform-coded symbols (Sec. 3.2 quantises DCT coefficients of the latents);
+* per-level quantisation step 2^-l;
+* MLP weights W_k ~ N(0, 1/fan_in) in the nn.Linear layout [out][in], biases
+  0.01 * N(0, 1); fp32, or fp16 (round-to-nearest-even of the draw) where the
+  workload fixes fp16 weights.
+
+Draw order for one image with generator PCG64(seed): for l = 0..L-1, for
+c = 0..C-1 the level's symbols; then for k = 0..n-1 the weight matrix W_k
+followed by the bias b_k.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+
+ACTS = ("relu", "gelu")
+PRECISIONS = ("fp32", "fp16_tc")
+
+
+def level_size(n: int, l: int) -> int:
+    """ceil(n / 2^l): the side of pyramid level l for an image side n (Eq. 1)."""
+    p = 1 << l
+    return (n + p - 1) // p
+
+
+def level_shapes(H: int, W: int, L: int):
+    return [(level_size(H, l), level_size(W, l)) for l in range(L)]
+
+
+def latent_count(H: int, W: int, L: int, C: int) -> int:
+    return sum(C * h * w for h, w in level_shapes(H, W, L))
+
+
+def param_count(dims) -> int:
+    return sum(dims[k + 1] * dims[k] + dims[k + 1] for k in range(len(dims) - 1))
+
+
+@dataclass(frozen=True)
+class Workload:
+    """One decode workload: image size, pyramid, MLP and input statistics."""
+
+    name: str
+    H: int
+    W: int
+    L: int
+    C: int
+    dims: tuple
+    act: str
+    weight_dtype: str          # "fp32" or "fp16": the dtype the weights are defined in
+    lap_scale: float
+    clip: int
+    seeds: tuple               # one seed per image; len(seeds) = batch size
+    precisions: tuple = ("fp32",)   # decoder paths that run this workload
+    note: str = field(default="", compare=False)
+
+    @property
+    def B(self) -> int:
+        return len(self.seeds)
+
+    @property
+    def pixels(self) -> int:
+        return self.B * self.H * self.W
+
+    @property
+    def n_latents(self) -> int:
+        return latent_count(self.H, self.W, self.L, self.C)
+
+    @property
+    def n_params(self) -> int:
+        return param_count(self.dims)
+
+    @property
+    def macs_per_pixel(self) -> int:
+        return sum(self.dims[k] * self.dims[k + 1] for k in range(len(self.dims) - 1))
+
+    @property
+    def hidden_per_pixel(self) -> int:
+        return sum(self.dims[1:-1])
+
+    def replace(self, **kw) -> "Workload":
+        d = dict(self.__dict__)
+        d.update(kw)
+        return Workload(**d)
+
+
+# The five decode workloads.  Kodak-sized images stand in for the Kodak set,
+# 1080p and 2160p images for the CLIC high-resolution set.
+WORKLOADS = {
+    "c1": Workload("c1", H=256, W=256, L=4, C=1, dims=(4, 16, 16, 3), act="relu",
+                   weight_dtype="fp32", lap_scale=2.0, clip=15, seeds=(0,),
+                   note="256x256, 4 levels x 1 ch, 4-16-16-3 ReLU, fp32"),
+    "c2": Workload("c2", H=512, W=768, L=7, C=1, dims=(7, 40, 40, 3), act="gelu",
+                   weight_dtype="fp32", lap_scale=3.0, clip=31, seeds=(1,),
+                   note="768x512 (Kodak size), 7 levels x 1 ch, 7-40-40-3 GELU, fp32"),
+    "c3": Workload("c3", H=1080, W=1920, L=7, C=2, dims=(14, 64, 64, 3), act="relu",
+                   weight_dtype="fp32", lap_scale=3.0, clip=31, seeds=(2,),
+                   note="1920x1080, 7 levels x 2 ch, 14-64-64-3 ReLU, fp32"),
+    "c4": Workload("c4", H=2160, W=3840, L=8, C=2, dims=(16, 64, 64, 64, 3), act="gelu",
+                   weight_dtype="fp32", lap_scale=4.0, clip=63, seeds=(3,),
+                   precisions=("fp32", "fp16_tc"),
+                   note="3840x2160, 8 levels x 2 ch, 16-64-64-64-3 GELU, fp32 + fp16 copy"),
+    "c5": Workload("c5", H=512, W=768, L=7, C=1, dims=(7, 64, 64, 3), act="relu",
+                   weight_dtype="fp16", lap_scale=3.0, clip=31, seeds=tuple(range(100, 164)),
+                   precisions=("fp16_tc",),
+                   note="batch of 64 Kodak-sized images, 7-64-64-3 ReLU, fp16 weights"),
+}
+
+
+@dataclass
+class Inputs:
+    """Host arrays for a batch of B images of one workload."""
+
+    wl: Workload
+    latents: np.ndarray      # int32 [B, n_latents]: levels concatenated, each [C][H_l][W_l]
+    steps: np.ndarray        # float32 [B, L]
+    weights: np.ndarray      # float32 or float16 [B, n_params]: the defined weights
+    weights_fp16: np.ndarray | None = None   # fp16 copy (RNE) of fp32 weights, for the TC path
+
+    def weights_for(self, precision: str) -> np.ndarray:
+        """The weight blob a decoder path consumes: fp32 for the CUDA-core path,
+        fp16 for the tensor-core path."""
+        if precision == "fp32":
+            return self.weights.astype(np.float32)
+        if self.weights.dtype == np.float16:
+            return self.weights
+        if self.weights_fp16 is None:
+            self.weights_fp16 = self.weights.astype(np.float16)
+        return self.weights_fp16
+
+    def oracle_weights(self, precision: str) -> np.ndarray:
+        """The weights the oracle uses as the definition: the defined weights
+        (fp32 draw, or fp16 where the workload defines fp16 weights), exactly
+        widened to fp64."""
+        return self.weights.astype(np.float64)
+
+
+def _draw_image(rng: np.random.Generator, H, W, L, C, dims, lap_scale, clip, weight_dtype):
+    levels = []
+    for l in range(L):
+        h, w = level_size(H, l), level_size(W, l)
+        for _c in range(C):
+            q = np.clip(np.rint(rng.laplace(0.0, lap_scale, (h, w))), -clip, clip).astype(np.int32)
+            levels.append(q.ravel())
+    params = []
+    for k in range(len(dims) - 1):
+        din, dout = dims[k], dims[k + 1]
+        Wk = rng.standard_normal((dout, din)) / np.sqrt(din)
+        bk = 0.01 * rng.standard_normal(dout)
+        params.append(Wk.ravel())
+        params.append(bk)
+    p64 = np.concatenate(params)
+    weights = p64.astype(np.float16) if weight_dtype == "fp16" else p64.astype(np.float32)
+    return np.concatenate(levels), weights
+
+
+def make_inputs(wl: Workload | str, batch: int | None = None) -> Inputs:
+    """Draws the inputs of a workload (all its images, or the first `batch`)."""
+    if isinstance(wl, str):
+        wl = WORKLOADS[wl]
+    seeds = wl.seeds if batch is None else wl.seeds[:batch]
+    lat, wts = [], []
+    for s in seeds:
+        rng = np.random.Generator(np.random.PCG64(s))
+        q, w = _draw_image(rng, wl.H, wl.W, wl.L, wl.C, wl.dims, wl.lap_scale, wl.clip,
+                           wl.weight_dtype)
+        lat.append(q)
+        wts.append(w)
+    steps = np.array([[2.0 ** -l for l in range(wl.L)]] * len(seeds), dtype=np.float32)
+    return Inputs(wl=wl, latents=np.stack(lat), steps=steps, weights=np.stack(wts))
+
+
+def custom(name: str, H: int, W: int, L: int, C: int, dims, act: str = "relu",
+           weight_dtype: str = "fp32", lap_scale: float = 3.0, clip: int = 31,
+           seed: int = 0, batch: int = 1, precisions=("fp32",)) -> Workload:
+    """A workload with arbitrary shapes (odd sizes, edge cases) for tests."""
+    return Workload(name, H=H, W=W, L=L, C=C, dims=tuple(dims), act=act,
+                    weight_dtype=weight_dtype, lap_scale=lap_scale, clip=clip,
+                    seeds=tuple(seed + i for i in range(batch)), precisions=tuple(precisions))
+
+
+def sample_pixels(H: int, W: int, n: int, seed: int) -> np.ndarray:
+    """Flat pixel indices (y * W + x) to check at full size: the four corners,
+    the middle of every border, and n seeded random positions."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    fixed = [(0, 0), (0, W - 1), (H - 1, 0), (H - 1, W - 1),
+             (0, W // 2), (H - 1, W // 2), (H // 2, 0), (H // 2, W - 1)]
+    ys = rng.integers(0, H, n)
+    xs = rng.integers(0, W, n)
+    idx = [y * W + x for y, x in fixed] + list(ys * W + xs)
+    return np.unique(np.array(idx, dtype=np.int64))

@@ -1,0 +1,298 @@
+"""Pins of the fp64 oracle: facts fixed by the paper's definitions and by
+mathematics, independent of the oracle's own code.
+
+Each pin takes an ``oracle.Oracle`` and raises AssertionError when the oracle
+disagrees.  ``test_oracle.py`` runs every pin on the real oracle;
+``test_oracle_mutations.py`` runs them on copies of the oracle with a planted
+mistake and requires every planted mistake to fail at least one pin.
+"""
+from __future__ import annotations
+
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _frac(tok: str) -> float:
+    return float(Fraction(tok))
+
+
+def load_golden(name: str) -> dict:
+    out = {}
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            key, *vals = line.split()
+            out[key] = vals
+    return out
+
+
+# ---------------------------------------------------------------- shapes
+def pin_level_sizes(o):
+    """Eq. 1 with the ceiling reading: H_l = ceil(H / 2^l)."""
+    assert [o.level_size(1080, l) for l in range(7)] == [1080, 540, 270, 135, 68, 34, 17]
+    assert [o.level_size(1920, l) for l in range(7)] == [1920, 960, 480, 240, 120, 60, 30]
+    assert [o.level_size(768, l) for l in range(7)] == [768, 384, 192, 96, 48, 24, 12]
+    assert [o.level_size(5, l) for l in range(4)] == [5, 3, 2, 1]
+    assert o.latent_count(256, 256, 4, 1) == 256 ** 2 + 128 ** 2 + 64 ** 2 + 32 ** 2
+    assert o.latent_count(5, 3, 3, 2) == 2 * (15 + 6 + 2)
+    assert o.param_count([4, 16, 16, 3]) == 16 * 5 + 16 * 17 + 3 * 17
+
+
+# ---------------------------------------------------------------- dequant
+def pin_dequant_exact(o):
+    """y = q * step; with step = 2^-l every product is an exact dyadic."""
+    q = np.arange(-63, 64, dtype=np.int32)
+    for l in range(8):
+        y = o.dequant(q, 2.0 ** -l)
+        assert np.array_equal(y, q.astype(np.float64) / (1 << l))
+    y = o.dequant(np.array([3, -5], dtype=np.int32), 0.3)
+    assert y[0] == 3 * 0.3 and y[1] == -5 * 0.3
+
+
+# ---------------------------------------------------------------- upsampling
+def _src_coord(x: int, n_in: int, n_out: int) -> Fraction:
+    """Half-pixel-centre source coordinate, exact, clamped to [0, n_in - 1]."""
+    s = (Fraction(2 * x + 1) * n_in) / (2 * n_out) - Fraction(1, 2)
+    return min(max(s, Fraction(0)), Fraction(n_in - 1))
+
+
+def pin_upsample_constant(o):
+    """A constant grid upsamples to the same constant everywhere."""
+    for (hl, wl, H, W) in [(1, 1, 7, 5), (2, 3, 4, 6), (17, 30, 135, 240), (3, 2, 5, 3)]:
+        g = np.full((hl, wl), -2.75)
+        out = o.upsample(g, H, W)
+        assert np.array_equal(out, np.full((H, W), -2.75))
+
+
+def pin_upsample_affine(o):
+    """Bilinear interpolation reproduces an affine grid a + b u + c v exactly,
+    at the (clamped) source coordinate of every output pixel.  Dyadic values
+    and power-of-two scales keep every fp64 operation exact."""
+    a, b, c = 1.5, 0.25, -2.0
+    for (hl, wl, H, W) in [(8, 4, 32, 16), (2, 2, 4, 4), (4, 8, 32, 64), (1, 4, 8, 16)]:
+        v, u = np.mgrid[0:hl, 0:wl]
+        g = a + b * u + c * v
+        out = o.upsample(g, H, W)
+        for y in range(H):
+            sy = float(_src_coord(y, hl, H))
+            for x in range(W):
+                sx = float(_src_coord(x, wl, W))
+                assert out[y, x] == a + b * sx + c * sy, (hl, wl, H, W, x, y)
+
+
+def pin_upsample_separable_bruteforce(o):
+    """Bilinear upsampling of an outer product is the outer product of the two
+    1-D linear interpolations; each 1-D weight is the tent (1 - |s - u|)^+ at
+    the exact rational source coordinate, written out here by brute force.
+    Covers ceil-sized (non power-of-two) ratios."""
+    rng = np.random.Generator(np.random.PCG64(7))
+    for (hl, wl, H, W) in [(3, 5, 5, 9), (17, 30, 135, 240), (2, 1, 3, 1), (34, 60, 270, 480),
+                           (1, 2, 1, 3), (68, 120, 1080, 1920)]:
+        r = rng.integers(-31, 32, hl).astype(np.float64)
+        cvec = rng.integers(-31, 32, wl).astype(np.float64)
+        g = np.outer(r, cvec)
+
+        def interp_1d(vals, n_in, n_out, x):
+            s = _src_coord(x, n_in, n_out)
+            return sum(float(max(Fraction(0), 1 - abs(s - u))) * vals[u] for u in range(n_in))
+
+        ys = np.unique(np.linspace(0, H - 1, min(H, 24)).astype(int))
+        xs = np.unique(np.linspace(0, W - 1, min(W, 24)).astype(int))
+        ry = {int(y): interp_1d(r, hl, H, int(y)) for y in ys}
+        cx = {int(x): interp_1d(cvec, wl, W, int(x)) for x in xs}
+        for y in ys:
+            for x in xs:
+                got = o.bilinear_at(g, H, W, int(x), int(y))
+                want = ry[int(y)] * cx[int(x)]
+                assert abs(got - want) <= 1e-12 * (1 + abs(want)), (hl, wl, H, W, x, y, got, want)
+        full = o.upsample(g, H, W)
+        assert np.array_equal(full[ys][:, xs], np.array([[o.bilinear_at(g, H, W, int(x), int(y))
+                                                          for x in xs] for y in ys]))
+
+
+def pin_upsample_identity_scale(o):
+    """Level 0 (scale 1) is the identity."""
+    rng = np.random.Generator(np.random.PCG64(3))
+    g = rng.standard_normal((7, 11))
+    assert np.array_equal(o.upsample(g, 7, 11), g)
+
+
+def pin_upsample_factor2_weights(o):
+    """2x upsampling with half-pixel centres uses the weights 3/4, 1/4: output
+    column 2u+1 = 3/4 g[u] + 1/4 g[u+1], column 2u+2 = 1/4 g[u] + 3/4 g[u+1]."""
+    g = np.array([[1.0, 5.0, -3.0, 8.0]])
+    out = o.upsample(g, 1, 8)[0]
+    want = [1.0, 0.75 * 1 + 0.25 * 5, 0.25 * 1 + 0.75 * 5, 0.75 * 5 + 0.25 * -3,
+            0.25 * 5 + 0.75 * -3, 0.75 * -3 + 0.25 * 8, 0.25 * -3 + 0.75 * 8, 8.0]
+    assert np.array_equal(out, np.array(want))
+    col = o.upsample(g.T.copy(), 8, 1)[:, 0]
+    assert np.array_equal(col, np.array(want))
+
+
+# ---------------------------------------------------------------- MLP
+def pin_act_closed_forms(o):
+    """ReLU(z) = max(z, 0).  GELU(z) = z Phi(z): GELU(0) = 0, GELU(1) = Phi(1),
+    GELU(z) - GELU(-z) = z (since Phi(z) + Phi(-z) = 1), GELU(z) -> z, 0 at
+    +-infinity, and the textbook value Phi(1) = 0.8413447460685429..."""
+    assert o.act(0.0, "relu") == 0.0 and o.act(-3.5, "relu") == 0.0 and o.act(2.25, "relu") == 2.25
+    assert o.act(0.0, "gelu") == 0.0
+    assert abs(o.act(1.0, "gelu") - 0.8413447460685429) < 1e-15
+    assert abs(o.act(-1.0, "gelu") - (0.8413447460685429 - 1.0)) < 1e-15
+    for z in [0.1, 0.5, 1.7, 3.0, 6.0]:
+        assert abs(o.act(z, "gelu") - o.act(-z, "gelu") - z) < 1e-14
+    assert abs(o.act(12.0, "gelu") - 12.0) < 1e-20
+    assert abs(o.act(-12.0, "gelu")) < 1e-20
+    # Phi(2) = 0.9772498680518208 (standard normal table value)
+    assert abs(o.act(2.0, "gelu") - 2 * 0.9772498680518208) < 1e-14
+
+
+def pin_mlp_zero_weights(o):
+    """All weights zero: the output is the last bias, whatever the input."""
+    dims = [5, 8, 3]
+    w = np.zeros(8 * 5 + 8 + 3 * 8 + 3)
+    w[-3:] = [0.25, -1.5, 7.0]
+    for act in ("relu", "gelu"):
+        out = o.mlp(np.array([1.0, -2, 3, -4, 5]), w, dims, act)
+        assert np.array_equal(out, np.array([0.25, -1.5, 7.0]))
+
+
+def _blob(layers):
+    return np.concatenate([np.concatenate([np.asarray(Wm, float).ravel(), np.asarray(b, float)])
+                           for Wm, b in layers])
+
+
+def pin_mlp_hand(o):
+    """A two-layer MLP worked by hand; exposes transposed weights, dropped or
+    misplaced biases, and an activation on the output layer."""
+    W0 = [[1.0, 2.0, 0.0], [0.0, -1.0, 1.0]]          # 3 -> 2
+    b0 = [0.5, -4.0]
+    W1 = [[2.0, 0.0], [1.0, 1.0], [0.0, -3.0]]         # 2 -> 3
+    b1 = [0.0, -10.0, 1.0]
+    x = np.array([1.0, 2.0, 3.0])
+    # z0 = (1 + 4 + 0 + 0.5, 0 - 2 + 3 - 4) = (5.5, -3); relu -> (5.5, 0)
+    # out = (11, 5.5 - 10, 0 + 1) = (11, -4.5, 1)
+    out = o.mlp(x, _blob([(W0, b0), (W1, b1)]), [3, 2, 3], "relu")
+    assert np.array_equal(out, np.array([11.0, -4.5, 1.0]))
+    # GELU hidden: h = (5.5 Phi(5.5), -3 Phi(-3))
+    phi = lambda z: 0.5 * (1 + math.erf(z / math.sqrt(2)))
+    h = [5.5 * phi(5.5), -3 * phi(-3)]
+    want = [2 * h[0], h[0] + h[1] - 10, -3 * h[1] + 1]
+    out = o.mlp(x, _blob([(W0, b0), (W1, b1)]), [3, 2, 3], "gelu")
+    assert np.allclose(out, want, rtol=0, atol=1e-13)
+
+
+def pin_mlp_identity(o):
+    """Identity hidden layers with ReLU pass the positive part through."""
+    n = 6
+    eye = np.eye(n)
+    Wout = np.zeros((3, n))
+    Wout[0, 0], Wout[1, 3], Wout[2, 5] = 1.0, 2.0, -1.0
+    w = _blob([(eye, np.zeros(n)), (eye, np.zeros(n)), (Wout, [0.0, 0.0, 0.5])])
+    x = np.array([1.5, -2.0, 3.0, 0.25, -1.0, -4.0])
+    out = o.mlp(x, w, [n, n, n, 3], "relu")
+    assert np.array_equal(out, np.array([1.5, 0.5, 0.5]))
+
+
+def pin_mlp_random_matmul(o):
+    """Against independent fp64 matrix products (numpy) on random weights."""
+    rng = np.random.Generator(np.random.PCG64(11))
+    dims = [7, 40, 40, 3]
+    layers = [(rng.standard_normal((dims[k + 1], dims[k])), rng.standard_normal(dims[k + 1]))
+              for k in range(3)]
+    x = rng.standard_normal(7) * 3
+    h = x
+    for k, (Wm, b) in enumerate(layers):
+        z = Wm @ h + b
+        h = z if k == 2 else np.maximum(z, 0)
+    out = o.mlp(x, _blob(layers), dims, "relu")
+    assert np.allclose(out, h, rtol=1e-13, atol=1e-13)
+
+
+def pin_clamp(o):
+    assert o.clamp01(-0.5) == 0.0 and o.clamp01(1.5) == 1.0 and o.clamp01(0.375) == 0.375
+
+
+# ---------------------------------------------------------------- decode
+def pin_decode_hand_4x4(o):
+    """The hand-computed 4x4 image (tests/golden/hand_4x4.txt)."""
+    g = load_golden("hand_4x4.txt")
+    H, W, L, C = int(g["H"][0]), int(g["W"][0]), int(g["L"][0]), int(g["C"][0])
+    dims = [int(v) for v in g["dims"]]
+    lat = np.array([int(v) for v in g["latents_l0"] + g["latents_l1"]], dtype=np.int32)
+    steps = np.array([_frac(v) for v in g["steps"]])
+    w = np.array([_frac(v) for v in g["weights"]])
+    out = o.decode(lat, steps, w, H, W, L, C, dims, g["act"][0], clamp=True)
+    for c, key in enumerate("RGB"):
+        want = np.array([_frac(v) for v in g[key]]).reshape(H, W)
+        assert np.allclose(out[c], want, rtol=0, atol=1e-15), (key, out[c], want)
+    # the upsampled level-1 plane, through the upsampler alone
+    y1 = o.dequant(np.array([int(v) for v in g["latents_l1"]], dtype=np.int32), steps[1])
+    u1 = o.upsample(y1.reshape(2, 2), H, W)
+    assert np.array_equal(u1, np.array([_frac(v) for v in g["U1"]]).reshape(H, W))
+    # unclamped: B at (3, 3) is 1 - 6/4 = -1/2
+    raw = o.decode(lat, steps, w, H, W, L, C, dims, "relu", clamp=False)
+    assert raw[2, 3, 3] == -0.5 and raw[1, 3, 3] == 1.0
+
+
+def pin_decode_feature_order(o):
+    """The feature is level-major (finest first), channel-minor: a first layer
+    that selects feature index j reproduces exactly level l = j // C, channel
+    c = j % C, upsampled."""
+    rng = np.random.Generator(np.random.PCG64(5))
+    H, W, L, C = 9, 7, 3, 2
+    shapes = [((H + (1 << l) - 1) >> l, (W + (1 << l) - 1) >> l) for l in range(L)]
+    planes = [rng.integers(-9, 10, (h, w)).astype(np.int32) for (h, w) in shapes for _ in range(C)]
+    lat = np.concatenate([p.ravel() for p in planes])
+    steps = np.array([1.0, 0.5, 0.25])
+    D = L * C
+    for j in range(D):
+        W0 = np.zeros((3, D))
+        W0[0, j] = 1.0
+        W0[1, j] = -1.0
+        W0[2, (j + 1) % D] = 0.5
+        w = np.concatenate([W0.ravel(), np.zeros(3)])
+        out = o.decode(lat, steps, w, H, W, L, C, [D, 3], "relu", clamp=False)
+        l, c = divmod(j, C)
+        want = o.upsample(planes[j].astype(np.float64) * steps[l], H, W)
+        assert np.array_equal(out[0], want) and np.array_equal(out[1], -want)
+        l2, _ = divmod((j + 1) % D, C)
+        want2 = o.upsample(planes[(j + 1) % D].astype(np.float64) * steps[l2], H, W) * 0.5
+        assert np.array_equal(out[2], want2)
+
+
+def pin_decode_single_level(o):
+    """L = 1: no interpolation; out = clamp(W1 relu(W0 q s + b0) + b1) per pixel,
+    against numpy matrix products."""
+    rng = np.random.Generator(np.random.PCG64(9))
+    H, W = 6, 5
+    q = rng.integers(-15, 16, (1, H, W)).astype(np.int32)
+    W0, b0 = rng.standard_normal((4, 1)), rng.standard_normal(4)
+    W1, b1 = rng.standard_normal((3, 4)) * 0.3, rng.standard_normal(3) * 0.3 + 0.5
+    out = o.decode(q.ravel(), [0.125], _blob([(W0, b0), (W1, b1)]), H, W, 1, 1, [1, 4, 3], "relu")
+    f = q.reshape(1, -1).astype(np.float64) * 0.125
+    want = np.clip(W1 @ np.maximum(W0 @ f + b0[:, None], 0) + b1[:, None], 0, 1).reshape(3, H, W)
+    assert np.allclose(out, want, rtol=0, atol=1e-14)
+
+
+def pin_decode_pixels_match(o):
+    """decode_pixels returns the same values as the full decode at those pixels."""
+    rng = np.random.Generator(np.random.PCG64(21))
+    H, W, L, C = 13, 10, 3, 1
+    n = sum(((H + (1 << l) - 1) >> l) * ((W + (1 << l) - 1) >> l) for l in range(L))
+    lat = rng.integers(-31, 32, n).astype(np.int32)
+    dims = [3, 8, 3]
+    w = rng.standard_normal(8 * 3 + 8 + 3 * 8 + 3) * 0.4
+    full = o.decode(lat, [1, .5, .25], w, H, W, L, C, dims, "gelu")
+    pix = np.array([0, 9, 55, 129, 64], dtype=np.int64)
+    part = o.decode_pixels(lat, [1, .5, .25], w, H, W, L, C, dims, "gelu", pix)
+    assert np.array_equal(part, full.reshape(3, -1)[:, pix].T)
+
+
+PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

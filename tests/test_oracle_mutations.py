@@ -1,0 +1,112 @@
+"""Planted mistakes in the oracle must be caught by its pins.
+
+Each case copies oracle/pic_oracle.c to a temporary directory, replaces one
+expression with a plausible wrong one (a dropped term, a wrong sign or index,
+a transposed operand, a swapped weight), compiles the copy and runs every pin
+of tests/oracle_pins.py against it.  The case passes when at least one pin
+fails, i.e. the pins would have exposed that mistake.  Every mutation keeps
+all memory accesses in bounds.
+"""
+import os
+import tempfile
+
+import pytest
+
+import oracle
+import oracle_pins
+
+SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "oracle",
+                   "pic_oracle.c")
+
+MUTATIONS = {
+    "no_half_pixel_offset": (
+        "double sx = ((double)x + 0.5) * ((double)Wl / (double)W) - 0.5;",
+        "double sx = ((double)x) * ((double)Wl / (double)W);"),
+    "x_uses_row_scale": (
+        "double sx = ((double)x + 0.5) * ((double)Wl / (double)W) - 0.5;",
+        "double sx = ((double)x + 0.5) * ((double)Hl / (double)H) - 0.5;"),
+    "y_uses_x_coordinate": (
+        "double sy = ((double)y + 0.5)",
+        "double sy = ((double)x + 0.5)"),
+    "align_corners_scale": (
+        "double sx = ((double)x + 0.5) * ((double)Wl / (double)W) - 0.5;",
+        "double sx = (W > 1) ? (double)x * ((double)(Wl - 1) / (double)(W - 1)) : 0.0;"),
+    "no_lower_clamp": (
+        "if (sx < 0.0) sx = 0.0;",
+        "if (sx < -1.0) sx = 0.0;"),
+    "swapped_column_weights": (
+        "double top = (1.0 - a) * g[(int64_t)v0 * Wl + u0] + a * g[(int64_t)v0 * Wl + u1];",
+        "double top = a * g[(int64_t)v0 * Wl + u0] + (1.0 - a) * g[(int64_t)v0 * Wl + u1];"),
+    "swapped_row_weights": (
+        "return (1.0 - b) * top + b * bot;",
+        "return b * top + (1.0 - b) * bot;"),
+    "wrapping_right_neighbour": (
+        "int u1 = (u0 + 1 < Wl) ? u0 + 1 : Wl - 1;",
+        "int u1 = (u0 + 1 < Wl) ? u0 + 1 : 0;"),
+    "bottom_row_uses_top_row": (
+        "double bot = (1.0 - a) * g[(int64_t)v1 * Wl + u0] + a * g[(int64_t)v1 * Wl + u1];",
+        "double bot = (1.0 - a) * g[(int64_t)v0 * Wl + u0] + a * g[(int64_t)v0 * Wl + u1];"),
+    "floor_level_size": (
+        "return (int)(((int64_t)n + p - 1) / p);",
+        "return (int)((int64_t)n / p > 0 ? (int64_t)n / p : 1);"),
+    "step_ignored": (
+        "y[i] = (double)q[i] * step;",
+        "y[i] = (double)q[i];"),
+    "transposed_weights": (
+        "s += Wk[(int64_t)i * din + j] * h[j];",
+        "s += Wk[(int64_t)(j % dout) * din + (i % din)] * h[j];"),
+    "dropped_bias": (
+        "z[i] = s + bk[i];",
+        "z[i] = s;"),
+    "activation_on_output_layer": (
+        "h[i] = last ? z[i] : pic_oracle_act(z[i], act);",
+        "h[i] = pic_oracle_act(z[i], act);"),
+    "no_hidden_activation": (
+        "h[i] = last ? z[i] : pic_oracle_act(z[i], act);",
+        "h[i] = z[i];"),
+    "gelu_wrong_scale": (
+        "return 0.5 * z * (1.0 + erf(z / sqrt(2.0)));",
+        "return 0.5 * z * (1.0 + erf(z / 2.0));"),
+    "gelu_tanh_form": (
+        "return 0.5 * z * (1.0 + erf(z / sqrt(2.0)));",
+        "return 0.5 * z * (1.0 + tanh(0.7978845608028654 * (z + 0.044715 * z * z * z)));"),
+    "leaky_relu": (
+        "return z > 0.0 ? z : 0.0;",
+        "return z > 0.0 ? z : 0.01 * z;"),
+    "no_upper_clamp": (
+        "if (v > 1.0) return 1.0;",
+        "if (v > 1.0) return v;"),
+    "levels_coarsest_first": (
+        "f[d++] = pic_oracle_bilinear_at(y[l] + (int64_t)c * Hl * Wl, Hl, Wl, H, W, x, yy);",
+        "f[(L - 1 - l) * C + c] = pic_oracle_bilinear_at(y[l] + (int64_t)c * Hl * Wl, Hl, Wl, H, W, x, yy); d++;"),
+    "channel_major_features": (
+        "f[d++] = pic_oracle_bilinear_at(y[l] + (int64_t)c * Hl * Wl, Hl, Wl, H, W, x, yy);",
+        "f[c * L + l] = pic_oracle_bilinear_at(y[l] + (int64_t)c * Hl * Wl, Hl, Wl, H, W, x, yy); d++;"),
+    "channel_offset_dropped": (
+        "f[d++] = pic_oracle_bilinear_at(y[l] + (int64_t)c * Hl * Wl, Hl, Wl, H, W, x, yy);",
+        "f[d++] = pic_oracle_bilinear_at(y[l], Hl, Wl, H, W, x, yy);"),
+}
+
+
+def _compile_mutant(name: str, tmp: str) -> str:
+    with open(SRC) as f:
+        src = f.read()
+    old, new = MUTATIONS[name]
+    assert src.count(old) == 1, f"mutation anchor for {name!r} not found exactly once"
+    path = os.path.join(tmp, f"{name}.c")
+    with open(path, "w") as f:
+        f.write(src.replace(old, new))
+    return oracle.compile_oracle(src=path, out=os.path.join(tmp, f"lib{name}.so"))
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_planted_mistake_is_caught(name):
+    with tempfile.TemporaryDirectory() as tmp:
+        mutant = oracle.load(_compile_mutant(name, tmp))
+        failed = []
+        for pin in oracle_pins.PINS:
+            try:
+                pin(mutant)
+            except (AssertionError, ValueError):
+                failed.append(pin.__name__)
+        assert failed, f"no pin exposes the planted mistake {name!r}"

@@ -1,0 +1,55 @@
+"""Host-side checks of the seeded input generator (shapes, determinism,
+statistics); no decoder arithmetic is involved."""
+import numpy as np
+import pytest
+
+from paper_2609_09020_gb300 import workloads as wk
+
+
+def test_level_shapes_match_ceiling_rule():
+    assert wk.level_shapes(1080, 1920, 7)[-1] == (17, 30)
+    assert wk.level_shapes(2160, 3840, 8)[-1] == (17, 30)
+    assert wk.level_shapes(512, 768, 7)[-1] == (8, 12)
+
+
+@pytest.mark.parametrize("name,lat,params", [
+    ("c1", 87_040, 403), ("c2", 524_256, 2083), ("c3", 2 * 2_764_710, 5315),
+    ("c4", 2 * 11_059_110, 9603), ("c5", 524_256, 4867)])
+def test_workload_sizes(name, lat, params):
+    wl = wk.WORKLOADS[name]
+    assert wl.n_latents == lat
+    assert wl.n_params == params
+
+
+def test_generator_is_deterministic_and_bounded():
+    a = wk.make_inputs("c1")
+    b = wk.make_inputs("c1")
+    assert np.array_equal(a.latents, b.latents) and np.array_equal(a.weights, b.weights)
+    assert a.latents.dtype == np.int32 and a.latents.shape == (1, 87_040)
+    assert np.abs(a.latents).max() <= 15
+    assert a.steps.tolist() == [[1.0, 0.5, 0.25, 0.125]]
+    # discretised Laplace(0, 2): P(q = 0) = 1 - exp(-1/4) ~ 0.221
+    p0 = np.mean(a.latents == 0)
+    assert 0.20 < p0 < 0.24
+
+
+def test_batch_uses_one_seed_per_image():
+    x = wk.make_inputs("c5", batch=3)
+    assert x.latents.shape == (3, 524_256) and x.weights.dtype == np.float16
+    assert not np.array_equal(x.latents[0], x.latents[1])
+    y = wk.make_inputs(wk.WORKLOADS["c5"].replace(seeds=(101,)))
+    assert np.array_equal(y.latents[0], x.latents[1])
+
+
+def test_fp16_copy_is_round_to_nearest():
+    x = wk.make_inputs(wk.custom("t", 8, 8, 2, 1, (2, 4, 3)))
+    h = x.weights_for("fp16_tc")
+    assert h.dtype == np.float16
+    assert np.array_equal(h, x.weights.astype(np.float16))
+
+
+def test_sample_pixels_include_corners():
+    p = wk.sample_pixels(10, 7, 20, 0)
+    for idx in (0, 6, 63, 69):
+        assert idx in p
+    assert p.min() >= 0 and p.max() < 70
