@@ -1,0 +1,376 @@
+"""Throughput benchmark of the fused PIC decode synthesis on GB300.
+
+One step = one pass of the whole hot path (dequantise, upsample, concatenate,
+MLP, clamp) over one batch of synthetic input: by default the 64-image
+throughput workload (64 independent 768x512 images, 7 levels x 1 channel,
+7-64-64-3 ReLU, fp16 weights) decoded by one ``pic_decode_batch`` call.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c5]
+                    [--precision fp16_tc|fp32] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  ``value`` is decoded megapixels/s over all
+ranks (weak scaling: each rank decodes its own batch; no collective on the
+data path).  ``--impl reference`` times the fp64 CPU oracle on the host cores
+on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_09020_gb300 import workloads as wk  # noqa: E402
+
+METRIC = "decoded megapixels/s and images/s at 1 GB300; % of binding roofline"
+UNIT = "MP/s"
+SM_COUNT = 152
+SM_MAX_MHZ = 2070.0
+FP32_LANES_PER_SM = 128
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained"), "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def fp32_peak_tflops():
+    """FP32 CUDA-core peak: SMs x 128 FMA lanes x 2 FLOP x max SM clock."""
+    return SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
+
+
+def algorithmic(wl: wk.Workload, batch: int):
+    """Per-launch algorithmic work: unpadded MLP FLOPs and the bytes the decode
+    must move at least once (int32 latents, weights, steps, fp32 RGB)."""
+    px = batch * wl.H * wl.W
+    flops = 2.0 * wl.macs_per_pixel * px
+    wbytes = 2 if wl.weight_dtype == "fp16" else 4
+    nbytes = batch * (wl.n_latents * 4 + wl.n_params * wbytes + wl.L * 4 + 3 * wl.H * wl.W * 4)
+    return flops, nbytes
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_09020_gb300", "csrc")
+    for fn in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, fn), "rb") as f:
+            h.update(fn.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel_name: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    e = rec.get(f"{kernel_name}/{workload}")
+    if not e or e.get("source_hash") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        mhz, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in getattr(self, "lines", []):
+            f = [s.strip() for s in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                mhz.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not mhz:
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(mhz)}
+
+
+def cpu_baseline(wl: wk.Workload, x: wk.Inputs, precision: str, budget_s: float):
+    """The fp64 oracle, as it stands, on the host cores: full images decoded
+    one after another until about budget_s seconds have passed."""
+    import oracle
+    orc = oracle.load()
+    cores = os.cpu_count() or 1
+    w = x.weights_for(precision)
+    n, t0 = 0, time.perf_counter()
+    while True:
+        b = n % x.latents.shape[0]
+        orc.decode(x.latents[b], x.steps[b].astype(np.float64), w[b].astype(np.float64), wl.H,
+                   wl.W, wl.L, wl.C, wl.dims, wl.act, nthreads=cores)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s:
+            break
+    mp = n * wl.H * wl.W / 1e6
+    return {"value": mp / el, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{n} full {wl.W}x{wl.H} image(s) of workload {wl.name} in {el:.1f} s "
+                      f"(fp64 C oracle, OpenMP over rows, {cores} threads)",
+            "images_per_s": n / el}
+
+
+def workload_desc(wl: wk.Workload, precision: str):
+    mlp = "-".join(str(d) for d in wl.dims) + " " + wl.act
+    return {"workload": f"{wl.name}: {wl.B} x {wl.W}x{wl.H}, {wl.L} levels x {wl.C} ch, MLP {mlp}, "
+                        f"{wl.weight_dtype} weights, {precision} path",
+            "images": wl.B, "H": wl.H, "W": wl.W, "levels": wl.L, "channels": wl.C,
+            "mlp": mlp, "precision": precision}
+
+
+def run_reference(args, wl, precision, rank):
+    if rank != 0:
+        return
+    x = wk.make_inputs(wl, batch=min(wl.B, 4))
+    budget = args.ref_step_s
+    for _ in range(args.warmup):
+        cpu_baseline(wl, x, precision, 0.0)
+    vals, imgs = [], []
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        r = cpu_baseline(wl, x, precision, budget)
+        vals.append(r["value"])
+        imgs.append(r["images_per_s"])
+    el = time.perf_counter() - t0
+    v = statistics.median(vals)
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * el / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded, workload-shaped)",
+            "config": {**workload_desc(wl, precision), "parallelism": "host cores"},
+            "images_per_s": statistics.median(imgs),
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": os.cpu_count() or 1,
+                             "kind": "oracle",
+                             "sample": f"each step: full images decoded for about {budget:.0f} s"},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default="c5", choices=sorted(wk.WORKLOADS))
+    ap.add_argument("--precision", default=None, choices=["fp32", "fp16_tc"])
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-budget-s", type=float, default=12.0)
+    ap.add_argument("--ref-step-s", type=float, default=5.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+
+    wl = wk.WORKLOADS[args.workload]
+    precision = args.precision or wl.precisions[-1]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if world > 1:
+            import torch.distributed as dist
+            dist.init_process_group("gloo")
+        run_reference(args, wl, precision, rank)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+
+    import torch
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    from paper_2609_09020_gb300 import build, pic
+    if rank == 0:
+        build.build()
+    barrier()
+    build.build()  # no-op once built
+
+    # Each rank decodes its own batch: image seeds offset by rank (weak scaling).
+    wl_r = wl.replace(seeds=tuple(s + 1000 * rank for s in wl.seeds)) if rank else wl
+    x = wk.make_inputs(wl_r)
+    B = x.latents.shape[0]
+    dec = pic.Decoder.for_workload(wl, precision, max_batch=B)
+    w_host = np.ascontiguousarray(x.weights_for(precision))
+    lat = torch.from_numpy(x.latents).to(dev)
+    steps_t = torch.from_numpy(x.steps).to(dev)
+    wts = torch.from_numpy(w_host).to(dev)
+    out = torch.empty((B, 3, wl.H, wl.W), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    for _ in range(max(args.warmup, 3)):
+        dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B)
+    dec.check(stream)
+    torch.cuda.synchronize(dev)
+
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local_rank) as clk:
+        barrier()
+        torch.cuda.synchronize(dev)
+        ev0.record(stream)
+        for _ in range(args.steps):
+            dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B)
+        ev1.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier()
+    dec.check(stream)
+    ms = ev0.elapsed_time(ev1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    px_total = world * B * wl.H * wl.W
+    value = px_total / (ms * 1e-3) / 1e6
+    images_per_s = world * B / (ms * 1e-3)
+
+    # End to end through the C ABI with host buffers (pinned): H2D of the
+    # inputs, the decode, D2H of the RGB planes, every step.
+    e2e = None
+    if not args.no_e2e:
+        lat_h = torch.from_numpy(x.latents).pin_memory()
+        st_h = torch.from_numpy(x.steps).pin_memory()
+        w_h = torch.from_numpy(w_host).pin_memory()
+        out_h = torch.empty((B, 3, wl.H, wl.W), dtype=torch.float32).pin_memory()
+        sp = stream.cuda_stream
+        ptrs = (lat_h.data_ptr(), st_h.data_ptr(), w_h.data_ptr(), out_h.data_ptr())
+
+        def host_call():
+            rc = pic.pic_decode_batch_host(dec.handle, B, ptrs[0], ptrs[1], ptrs[2], wl.H, wl.W,
+                                           ptrs[3], sp)
+            if rc != pic.PIC_OK:
+                raise pic.PicError(rc, "pic_decode_batch_host")
+
+        host_call()
+        e_steps = max(3, min(args.steps, 10))
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(e_steps):
+            host_call()
+        el = time.perf_counter() - t0
+        if world > 1:
+            t = torch.tensor([el], device=dev)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            el = float(t.item())
+        h2d = lat_h.numel() * 4 + st_h.numel() * 4 + w_h.numel() * w_h.element_size()
+        e2e = {"value": px_total * e_steps / el / 1e6, "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(out_h.numel() * 4),
+               "ms_per_step": 1e3 * el / e_steps}
+
+    peaks = load_peaks()
+    flops, nbytes = algorithmic(wl, B)
+    t_s = ms * 1e-3
+    kname = dec.kernel_name
+    if precision == "fp16_tc":
+        peak_tf = peaks["bf16_tflops"]  # fp16 dense tensor rate = bf16 rate
+        t_pipe = flops / (peak_tf * 1e12)
+        roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": peak_tf,
+                "unit": "TFLOP/s", "peak_source": f"bf16 dense burst, {peaks['source']}"}
+    else:
+        peak_tf = fp32_peak_tflops()
+        t_pipe = flops / (peak_tf * 1e12)
+        roof = {"bound": "alu", "achieved": flops / t_s / 1e12, "peak": peak_tf,
+                "unit": "TFLOP/s",
+                "peak_source": "FP32 FMA: 152 SMs x 128 lanes x 2 FLOP x 2070 MHz"}
+    t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
+    if t_hbm > t_pipe:
+        roof.update({"bound": "hbm", "achieved": nbytes / t_s / 1e9, "peak": peaks["hbm_gbs"],
+                     "unit": "GB/s", "peak_source": f"copy bandwidth, {peaks['source']}"})
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = recorded_traffic(kname, wl.name)
+    roof["kernel"] = kname
+    roof["algorithmic_flops_per_launch"] = flops
+    roof["algorithmic_bytes_per_launch"] = nbytes
+    roof["binding_time_us"] = max(t_pipe, t_hbm) * 1e6
+    roof["avg_launch_us"] = ms * 1e3
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(wl, x, precision, args.cpu_budget_s)
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+                "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f16 operands (hi+lo split), f32 accumulate" if precision == "fp16_tc"
+                else "f32",
+                "data": "synthetic (seeded Laplacian int latents, N(0,1/fan_in) weights)",
+                "config": {**workload_desc(wl, precision), "parallelism": f"dp{world}",
+                           "l2": "inputs larger than L2 (no flush needed)"
+                           if nbytes > 129e6 else "inputs smaller than L2; back-to-back calls",
+                           "batch_per_gpu": B},
+                "images_per_s": images_per_s,
+                "roofline": roof, "clocks": clk.summary(), "e2e": e2e,
+                "gpu_launches": args.steps, "cpu_baseline": cpu}
+        print(json.dumps(line), flush=True)
+    dec.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,163 @@
+/*
+ * pic_decode.h -- C ABI of the GB300 decoder for the PIC synthesis g_r
+ * (arxiv 2609.09020, "PIC: Revisiting INR for Image Coding with Fast Encoding
+ * and Sub-Millisecond Decoding").
+ *
+ * The decode problem (Sec. 3.1, Eq. 1; Sec. 4.1; App. A): an H x W image is
+ * represented by L quantised latent grids y_hat = {y_l}, level l of size
+ * ceil(H / 2^l) x ceil(W / 2^l) with C channels (l = 0 is full resolution;
+ * the paper's index is i = L - l), plus the weights of the per-pixel synthesis
+ * MLP g_s (the decoder only needs the fused weights w', b' of App. A).  For
+ * every output pixel the decoder
+ *   1. dequantises the integer symbols of every level: y = q * step_l,
+ *   2. upsamples every level to H x W (bilinear, half-pixel centres, edge
+ *      clamp, source coordinate (x + 1/2) * W_l / W - 1/2),
+ *   3. concatenates the levels into a feature of L * C values (level-major,
+ *      finest level first, channel-minor),
+ *   4. runs g_s: h_{k+1} = act(W_k h_k + b_k) for hidden layers (act = ReLU,
+ *      or GELU in its erf form), a linear last layer with 3 outputs,
+ *   5. clamps the RGB result to [0, 1].
+ * Steps 1-5 run fused in one kernel launch per call: features and hidden
+ * activations never leave the chip.
+ *
+ * Conventions for every entry point below:
+ *   - Device pointers are CUDA global-memory pointers on the current device,
+ *     owned by the caller, contiguous, at least 16-byte aligned; the library
+ *     never takes ownership of, frees, or keeps them after the call.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Decode
+ *     calls are asynchronous on it: they enqueue work and return without a
+ *     host synchronisation.  Outputs are ready when the stream reaches them.
+ *   - Every function returns a pic_status.  Argument errors are detected on
+ *     the host before anything is launched.  No function calls exit(),
+ *     abort() or traps on the device.
+ *   - A handle is not thread-safe: calls on one handle must not overlap in
+ *     host threads.  Different handles are independent.
+ */
+#ifndef PIC_DECODE_H
+#define PIC_DECODE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct pic_decoder pic_decoder; /* opaque handle */
+
+typedef enum {
+    PIC_OK = 0,
+    PIC_ERR_INVALID_ARG = -1, /* NULL pointer, bad size, misaligned pointer, arch mismatch */
+    PIC_ERR_UNSUPPORTED = -2, /* arch outside the supported envelope, or no sm_103 device */
+    PIC_ERR_CUDA = -3,        /* a CUDA runtime call or kernel launch failed */
+    PIC_ERR_ALLOC = -4,       /* device or host allocation failed (create only) */
+    PIC_ERR_TIMEOUT = -5      /* a bounded device-side wait gave up (reported by pic_decode_check) */
+} pic_status;
+
+typedef enum {
+    PIC_ACT_RELU = 0, /* max(z, 0) (Sec. 4.1) */
+    PIC_ACT_GELU = 1  /* z * Phi(z) = z/2 (1 + erf(z / sqrt 2)) */
+} pic_act;
+
+typedef enum {
+    /* fp32 weights; all arithmetic in fp32 on the CUDA cores. */
+    PIC_PREC_FP32 = 0,
+    /* fp16 weights; the MLP runs on the tensor cores with fp16 operands and
+     * fp32 accumulation.  Every activation operand (features and hidden
+     * values) is split into two fp16 terms hi + lo, so the products carry
+     * about 22 significant bits; the weights are used exactly as given. */
+    PIC_PREC_FP16_TC = 1
+} pic_prec;
+
+/* Architecture of one decoder instance (fixed at create). */
+typedef struct {
+    int num_levels;         /* L, 1..12 */
+    int channels_per_level; /* C, 1..4 */
+    int num_layers;         /* n linear layers, 1..6 */
+    int dims[7];            /* dims[0] = L*C, dims[n] = 3; every dim 1..128 */
+    int hidden_act;         /* pic_act */
+    int precision;          /* pic_prec */
+    int clamp_output;       /* 1: clamp to [0, 1] (the decode); 0: raw MLP output */
+    int max_H, max_W;       /* largest image accepted by the decode calls */
+    int max_batch;          /* largest B accepted by pic_decode_batch */
+} pic_arch;
+
+/*
+ * Creates a decoder for `arch` on the current CUDA device.  Validates the
+ * arch, selects the kernel, and allocates the handle's small device state.
+ * May synchronise.  On success *out receives the handle (destroy it with
+ * pic_decode_destroy); on failure *out is set to NULL.
+ * Errors: PIC_ERR_INVALID_ARG (NULL arch/out, inconsistent dims),
+ * PIC_ERR_UNSUPPORTED (limits above, or the current device is not sm_103),
+ * PIC_ERR_ALLOC, PIC_ERR_CUDA.
+ */
+int pic_decode_create(const pic_arch *arch, pic_decoder **out);
+
+/*
+ * Decodes one image (steps 1-5 above) on `stream`.
+ *   latents : int32, device; levels l = 0..L-1 concatenated, each planar
+ *             [C][H_l][W_l] row-major, H_l = ceil(H / 2^l), W_l = ceil(W / 2^l);
+ *             pic_latent_count(H, W, L, C) values.
+ *   steps   : float, device; [L] dequantisation step of each level.
+ *   weights : device; for k = 0..n-1: W_k [dims[k+1]][dims[k]] row-major, then
+ *             b_k [dims[k+1]]; pic_param_count(arch) values; float for
+ *             PIC_PREC_FP32, IEEE half (uint16 bits) for PIC_PREC_FP16_TC.
+ *   H, W    : image size, 1..max_H, 1..max_W.
+ *   out_rgb : float, device; planar [3][H][W] (R, G, B planes).
+ * Errors: PIC_ERR_INVALID_ARG (NULL handle/pointer, misaligned pointer, H or W
+ * out of range) with nothing launched; PIC_ERR_CUDA if the launch failed.
+ */
+int pic_decode(pic_decoder *h, const int32_t *latents, const float *steps, const void *weights,
+               int H, int W, float *out_rgb, void *stream);
+
+/*
+ * Decodes B independent images of the same size in one launch.  Image b uses
+ * latents + b * pic_latent_count(H, W, L, C), steps + b * L,
+ * weights + b * pic_param_count(arch) and writes out_rgb + b * 3 * H * W
+ * (all images' buffers are contiguous, image-major).  B in 1..max_batch;
+ * other arguments and errors as pic_decode.
+ */
+int pic_decode_batch(pic_decoder *h, int B, const int32_t *latents, const float *steps,
+                     const void *weights, int H, int W, float *out_rgb, void *stream);
+
+/*
+ * End-to-end convenience for callers holding HOST buffers (same layouts as
+ * pic_decode_batch, host pointers, preferably pinned): copies the inputs to
+ * device buffers owned by the handle, decodes, copies the RGB planes back,
+ * and synchronises `stream` before returning.  The staging buffers are
+ * allocated on first use for max_batch images of max_H x max_W and kept
+ * until destroy.
+ * Errors: as pic_decode_batch, plus PIC_ERR_ALLOC.
+ */
+int pic_decode_batch_host(pic_decoder *h, int B, const int32_t *latents, const float *steps,
+                          const void *weights, int H, int W, float *out_rgb, void *stream);
+
+/*
+ * Synchronises `stream` and reports whether any kernel of this handle
+ * launched on it since the last check hit a bounded device-side wait limit
+ * (PIC_ERR_TIMEOUT; the handle's flag is then cleared), or PIC_OK.
+ * Errors: PIC_ERR_INVALID_ARG (NULL handle), PIC_ERR_CUDA.
+ */
+int pic_decode_check(pic_decoder *h, void *stream);
+
+/* Frees the handle and its device state.  NULL is a no-op.  Synchronises the
+ * device first, so that no kernel of this handle is still running. */
+void pic_decode_destroy(pic_decoder *h);
+
+/* Name of the kernel selected at create (static string), or "" for NULL. */
+const char *pic_decode_kernel_name(const pic_decoder *h);
+
+/* sum_l C * ceil(H/2^l) * ceil(W/2^l), or -1 for invalid arguments. */
+int64_t pic_latent_count(int H, int W, int L, int C);
+
+/* sum_k dims[k+1] * (dims[k] + 1), or -1 for an invalid arch. */
+int64_t pic_param_count(const pic_arch *arch);
+
+/* Static description of a status code. */
+const char *pic_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PIC_DECODE_H */

@@ -1,0 +1,110 @@
+// pic_common.cuh -- launch parameters and device helpers shared by the decode
+// kernels (the CUDA path only; the fp64 oracle shares nothing with this file).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda_fp16.h>
+
+namespace pic {
+
+constexpr int kMaxLevels = 12;
+constexpr int kMaxLayers = 6;
+constexpr int kMaxDim = 128;
+
+// Geometry of one pyramid level (Eq. 1 with the ceiling rule): size, offset
+// of the level inside one image's latent block, and the size ratios
+// W_l / W, H_l / H that map output pixel centres to source coordinates.
+struct LevelGeom {
+  int H, W;
+  long long off;   // element offset of level l within one image's latents
+  float sx, sy;    // W_l / W and H_l / H, rounded to fp32
+};
+
+// Everything a decode launch needs; passed by value (kernel parameter space).
+struct DecodeParams {
+  const int32_t* latents;
+  const float* steps;
+  const void* weights;
+  float* out;
+  int H, W, B, L, C;
+  int clamp;
+  long long lat_per_image;     // sum_l C H_l W_l
+  long long params_per_image;  // sum_k d_{k+1} (d_k + 1)
+  int tiles_per_row;
+  long long tiles_per_image;
+  long long total_tiles;
+  int* status;                 // device word: nonzero after a bounded wait gave up
+  int n_layers;
+  int dims[kMaxLayers + 1];
+  int act;
+  LevelGeom lv[kMaxLevels];
+};
+
+enum { ACT_RELU = 0, ACT_GELU = 1 };
+
+// GELU in its erf form, z * Phi(z), with CUDA's erff.
+__device__ __forceinline__ float gelu_erf(float z) {
+  return 0.5f * z * (1.0f + erff(z * 0.70710678118654752f));
+}
+
+template <int ACT>
+__device__ __forceinline__ float activate(float z) {
+  if constexpr (ACT == ACT_GELU) return gelu_erf(z);
+  else return fmaxf(z, 0.0f);
+}
+
+__device__ __forceinline__ float activate_rt(float z, int act) {
+  return act == ACT_GELU ? gelu_erf(z) : fmaxf(z, 0.0f);
+}
+
+// ---- packed fp32 pairs (sm_100+ f32x2 instructions) ----------------------
+__device__ __forceinline__ unsigned long long pack2(float lo, float hi) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ float2 unpack2(unsigned long long v) {
+  float2 r;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
+  return r;
+}
+// d = a * b + c on both halves (one instruction, two FMAs).
+__device__ __forceinline__ unsigned long long fma2(unsigned long long a, unsigned long long b,
+                                                   unsigned long long c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+
+// Bilinear source coordinate of output index x along one axis: the pixel
+// centre x + 1/2 maps to (x + 1/2) * ratio - 1/2, clamped below at 0; i0 is
+// its floor, i1 the next index clamped to n - 1, and frac the weight of i1.
+struct Tap {
+  int i0, i1;
+  float frac;
+};
+__device__ __forceinline__ Tap bilinear_tap(int x, float ratio, int n) {
+  float s = fmaxf(fmaf(static_cast<float>(x) + 0.5f, ratio, -0.5f), 0.0f);
+  int i0 = static_cast<int>(s);
+  Tap t;
+  t.i0 = min(i0, n - 1);
+  t.i1 = min(i0 + 1, n - 1);
+  t.frac = s - static_cast<float>(i0);
+  return t;
+}
+
+// One bilinear sample of integer grid `q` (row stride w), in fp32: the two
+// horizontal lerps use exact integer differences, then one vertical lerp.
+__device__ __forceinline__ float bilinear_sample(const int32_t* __restrict__ q, int w, Tap tx,
+                                                 Tap ty) {
+  const int32_t* r0 = q + static_cast<long long>(ty.i0) * w;
+  const int32_t* r1 = q + static_cast<long long>(ty.i1) * w;
+  int a = __ldg(r0 + tx.i0), b = __ldg(r0 + tx.i1);
+  int c = __ldg(r1 + tx.i0), d = __ldg(r1 + tx.i1);
+  float top = fmaf(tx.frac, static_cast<float>(b - a), static_cast<float>(a));
+  float bot = fmaf(tx.frac, static_cast<float>(d - c), static_cast<float>(c));
+  return fmaf(ty.frac, bot - top, top);
+}
+
+}  // namespace pic

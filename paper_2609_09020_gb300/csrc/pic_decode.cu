@@ -1,0 +1,332 @@
+// pic_decode.cu -- the C ABI (include/pic_decode.h): argument validation,
+// kernel selection, launch.  Host code only; the kernels live in k_*.cu.
+#include <cstdint>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+
+#include <cuda_runtime.h>
+
+#include "pic_common.cuh"
+#include "pic_kernels.h"
+#include "pic_decode.h"
+
+using pic::DecodeParams;
+using pic::KernelInfo;
+
+struct pic_decoder {
+  pic_arch arch;
+  int device;
+  int sm_count;
+  KernelInfo kern;
+  int grid_cap;          // resident CTAs over all SMs
+  int* d_status;         // bounded-wait failure flag (device word)
+  long long n_params;    // per image
+  // staging for pic_decode_batch_host (allocated on first use)
+  int32_t* s_lat;
+  float* s_steps;
+  void* s_w;
+  float* s_out;
+};
+
+namespace {
+
+int level_size(int n, int l) { return static_cast<int>((static_cast<long long>(n) + (1LL << l) - 1) >> l); }
+
+bool arch_valid(const pic_arch* a) {
+  if (a->num_levels < 1 || a->num_levels > pic::kMaxLevels) return false;
+  if (a->channels_per_level < 1 || a->channels_per_level > 4) return false;
+  if (a->num_layers < 1 || a->num_layers > pic::kMaxLayers) return false;
+  if (a->dims[0] != a->num_levels * a->channels_per_level) return false;
+  if (a->dims[a->num_layers] != 3) return false;
+  for (int k = 0; k <= a->num_layers; ++k)
+    if (a->dims[k] < 1 || a->dims[k] > pic::kMaxDim) return false;
+  if (a->hidden_act != PIC_ACT_RELU && a->hidden_act != PIC_ACT_GELU) return false;
+  if (a->precision != PIC_PREC_FP32 && a->precision != PIC_PREC_FP16_TC) return false;
+  if (a->clamp_output != 0 && a->clamp_output != 1) return false;
+  if (a->max_H < 1 || a->max_W < 1 || a->max_batch < 1) return false;
+  if (a->max_H > 65536 || a->max_W > 65536 || a->max_batch > 65536) return false;
+  return true;
+}
+
+bool kernel_matches(const KernelInfo& k, const pic_arch* a) {
+  if (k.generic || k.precision != a->precision || k.C != a->channels_per_level ||
+      k.n_layers != a->num_layers || k.act != a->hidden_act)
+    return false;
+  for (int i = 0; i <= a->num_layers; ++i)
+    if (k.dims[i] != a->dims[i]) return false;
+  return true;
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int check_decode_args(const pic_decoder* h, int B, const int32_t* latents, const float* steps,
+                      const void* weights, int H, int W, const float* out) {
+  if (!h || !latents || !steps || !weights || !out) return PIC_ERR_INVALID_ARG;
+  if (B < 1 || B > h->arch.max_batch) return PIC_ERR_INVALID_ARG;
+  if (H < 1 || W < 1 || H > h->arch.max_H || W > h->arch.max_W) return PIC_ERR_INVALID_ARG;
+  if (!aligned(latents, 16) || !aligned(weights, 16) || !aligned(out, 16) || !aligned(steps, 4))
+    return PIC_ERR_INVALID_ARG;
+  return PIC_OK;
+}
+
+void fill_params(const pic_decoder* h, DecodeParams& p, int B, const int32_t* latents,
+                 const float* steps, const void* weights, int H, int W, float* out) {
+  std::memset(&p, 0, sizeof(p));
+  const pic_arch& a = h->arch;
+  p.latents = latents;
+  p.steps = steps;
+  p.weights = weights;
+  p.out = out;
+  p.H = H;
+  p.W = W;
+  p.B = B;
+  p.L = a.num_levels;
+  p.C = a.channels_per_level;
+  p.clamp = a.clamp_output;
+  p.status = h->d_status;
+  p.n_layers = a.num_layers;
+  for (int k = 0; k <= a.num_layers; ++k) p.dims[k] = a.dims[k];
+  p.act = a.hidden_act;
+  long long off = 0;
+  for (int l = 0; l < a.num_levels; ++l) {
+    pic::LevelGeom& g = p.lv[l];
+    g.H = level_size(H, l);
+    g.W = level_size(W, l);
+    g.off = off;
+    g.sx = static_cast<float>(static_cast<double>(g.W) / W);
+    g.sy = static_cast<float>(static_cast<double>(g.H) / H);
+    off += static_cast<long long>(a.channels_per_level) * g.H * g.W;
+  }
+  p.lat_per_image = off;
+  p.params_per_image = h->n_params;
+  const int tp = h->kern.tile_px;
+  p.tiles_per_row = (W + tp - 1) / tp;
+  p.tiles_per_image = static_cast<long long>(p.tiles_per_row) * H;
+  p.total_tiles = p.tiles_per_image * B;
+}
+
+int launch(pic_decoder* h, const DecodeParams& p, cudaStream_t stream) {
+  long long grid = p.total_tiles < h->grid_cap ? p.total_tiles : h->grid_cap;
+  if (grid < 1) grid = 1;
+  void* args[] = {const_cast<DecodeParams*>(&p)};
+  cudaError_t e = cudaLaunchKernel(h->kern.fn, dim3(static_cast<unsigned>(grid)),
+                                   dim3(h->kern.threads), args, h->kern.smem_bytes, stream);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  return PIC_OK;
+}
+
+size_t weight_elem_bytes(const pic_arch& a) { return a.precision == PIC_PREC_FP16_TC ? 2 : 4; }
+
+}  // namespace
+
+extern "C" {
+
+const char* pic_status_string(int s) {
+  switch (s) {
+    case PIC_OK: return "ok";
+    case PIC_ERR_INVALID_ARG: return "invalid argument";
+    case PIC_ERR_UNSUPPORTED: return "unsupported architecture or device";
+    case PIC_ERR_CUDA: return "CUDA error";
+    case PIC_ERR_ALLOC: return "allocation failed";
+    case PIC_ERR_TIMEOUT: return "device-side wait timed out";
+    default: return "unknown status";
+  }
+}
+
+int64_t pic_latent_count(int H, int W, int L, int C) {
+  if (H < 1 || W < 1 || L < 1 || L > 30 || C < 1) return -1;
+  int64_t n = 0;
+  for (int l = 0; l < L; ++l) n += static_cast<int64_t>(C) * level_size(H, l) * level_size(W, l);
+  return n;
+}
+
+int64_t pic_param_count(const pic_arch* a) {
+  if (!a || a->num_layers < 1 || a->num_layers > pic::kMaxLayers) return -1;
+  int64_t n = 0;
+  for (int k = 0; k < a->num_layers; ++k) {
+    if (a->dims[k] < 1 || a->dims[k + 1] < 1) return -1;
+    n += static_cast<int64_t>(a->dims[k + 1]) * (a->dims[k] + 1);
+  }
+  return n;
+}
+
+int pic_decode_create(const pic_arch* arch, pic_decoder** out) {
+  if (!out) return PIC_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!arch) return PIC_ERR_INVALID_ARG;
+  if (arch->num_layers < 1 || arch->num_layers > pic::kMaxLayers) return PIC_ERR_INVALID_ARG;
+  if (arch->dims[0] != arch->num_levels * arch->channels_per_level ||
+      arch->dims[arch->num_layers] != 3)
+    return PIC_ERR_INVALID_ARG;
+  if (!arch_valid(arch)) return PIC_ERR_UNSUPPORTED;
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_UNSUPPORTED;
+  }
+  cudaDeviceProp prop;
+  if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  if (prop.major != 10 || prop.minor != 3) return PIC_ERR_UNSUPPORTED;  // built for sm_103a only
+
+  // Kernel selection: a compile-time specialisation of exactly this arch,
+  // else (fp32 only) the generic kernel.
+  KernelInfo table[32];
+  int n = arch->precision == PIC_PREC_FP32 ? pic::fp32_kernels(table, 32) : pic::tc_kernels(table, 32);
+  const KernelInfo* chosen = nullptr;
+  for (int i = 0; i < n && i < 32; ++i)
+    if (kernel_matches(table[i], arch)) {
+      chosen = &table[i];
+      break;
+    }
+  KernelInfo k{};
+  if (chosen) {
+    k = *chosen;
+  } else if (arch->precision == PIC_PREC_FP32) {
+    k = pic::fp32_generic_kernel_info();
+    k.smem_bytes = static_cast<int>(pic_param_count(arch) * 4);
+  } else {
+    return PIC_ERR_UNSUPPORTED;
+  }
+  if (k.smem_bytes > static_cast<int>(prop.sharedMemPerBlockOptin)) return PIC_ERR_UNSUPPORTED;
+  if (cudaFuncSetAttribute(k.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, k.smem_bytes) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k.fn, k.threads, k.smem_bytes) !=
+          cudaSuccess ||
+      per_sm < 1) {
+    cudaGetLastError();
+    return PIC_ERR_UNSUPPORTED;
+  }
+
+  pic_decoder* h = new (std::nothrow) pic_decoder();
+  if (!h) return PIC_ERR_ALLOC;
+  h->arch = *arch;
+  h->device = dev;
+  h->sm_count = prop.multiProcessorCount;
+  h->kern = k;
+  h->grid_cap = per_sm * prop.multiProcessorCount;
+  h->n_params = pic_param_count(arch);
+  if (cudaMalloc(&h->d_status, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    delete h;
+    return PIC_ERR_ALLOC;
+  }
+  if (cudaMemset(h->d_status, 0, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(h->d_status);
+    delete h;
+    return PIC_ERR_CUDA;
+  }
+  *out = h;
+  return PIC_OK;
+}
+
+int pic_decode_batch(pic_decoder* h, int B, const int32_t* latents, const float* steps,
+                     const void* weights, int H, int W, float* out_rgb, void* stream) {
+  int rc = check_decode_args(h, B, latents, steps, weights, H, W, out_rgb);
+  if (rc != PIC_OK) return rc;
+  DecodeParams p;
+  fill_params(h, p, B, latents, steps, weights, H, W, out_rgb);
+  return launch(h, p, static_cast<cudaStream_t>(stream));
+}
+
+int pic_decode(pic_decoder* h, const int32_t* latents, const float* steps, const void* weights,
+               int H, int W, float* out_rgb, void* stream) {
+  return pic_decode_batch(h, 1, latents, steps, weights, H, W, out_rgb, stream);
+}
+
+int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const float* steps,
+                          const void* weights, int H, int W, float* out_rgb, void* stream) {
+  if (!h || !latents || !steps || !weights || !out_rgb) return PIC_ERR_INVALID_ARG;
+  if (B < 1 || B > h->arch.max_batch || H < 1 || W < 1 || H > h->arch.max_H || W > h->arch.max_W)
+    return PIC_ERR_INVALID_ARG;
+  const pic_arch& a = h->arch;
+  const long long nb = a.max_batch;
+  if (!h->s_lat) {
+    const long long lat = pic_latent_count(a.max_H, a.max_W, a.num_levels, a.channels_per_level);
+    bool ok = cudaMalloc(&h->s_lat, nb * lat * sizeof(int32_t)) == cudaSuccess &&
+              cudaMalloc(&h->s_steps, nb * a.num_levels * sizeof(float)) == cudaSuccess &&
+              cudaMalloc(&h->s_w, nb * h->n_params * weight_elem_bytes(a)) == cudaSuccess &&
+              cudaMalloc(&h->s_out, nb * 3LL * a.max_H * a.max_W * sizeof(float)) == cudaSuccess;
+    if (!ok) {
+      cudaGetLastError();
+      cudaFree(h->s_lat);
+      cudaFree(h->s_steps);
+      cudaFree(h->s_w);
+      cudaFree(h->s_out);
+      h->s_lat = nullptr;
+      h->s_steps = nullptr;
+      h->s_w = nullptr;
+      h->s_out = nullptr;
+      return PIC_ERR_ALLOC;
+    }
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const long long lat_bytes = static_cast<long long>(B) *
+                              pic_latent_count(H, W, a.num_levels, a.channels_per_level) * 4;
+  const long long w_bytes = static_cast<long long>(B) * h->n_params * weight_elem_bytes(a);
+  const long long out_bytes = static_cast<long long>(B) * 3LL * H * W * 4;
+  if (cudaMemcpyAsync(h->s_lat, latents, lat_bytes, cudaMemcpyHostToDevice, s) != cudaSuccess ||
+      cudaMemcpyAsync(h->s_steps, steps, static_cast<size_t>(B) * a.num_levels * 4,
+                      cudaMemcpyHostToDevice, s) != cudaSuccess ||
+      cudaMemcpyAsync(h->s_w, weights, w_bytes, cudaMemcpyHostToDevice, s) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  int rc = pic_decode_batch(h, B, h->s_lat, h->s_steps, h->s_w, H, W, h->s_out, stream);
+  if (rc != PIC_OK) return rc;
+  if (cudaMemcpyAsync(out_rgb, h->s_out, out_bytes, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  return PIC_OK;
+}
+
+int pic_decode_check(pic_decoder* h, void* stream) {
+  if (!h) return PIC_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int flag = 0;
+  if (cudaMemcpyAsync(&flag, h->d_status, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  if (flag != 0) {
+    if (cudaMemsetAsync(h->d_status, 0, sizeof(int), s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess) {
+      cudaGetLastError();
+      return PIC_ERR_CUDA;
+    }
+    return PIC_ERR_TIMEOUT;
+  }
+  return PIC_OK;
+}
+
+void pic_decode_destroy(pic_decoder* h) {
+  if (!h) return;
+  cudaDeviceSynchronize();
+  cudaFree(h->d_status);
+  cudaFree(h->s_lat);
+  cudaFree(h->s_steps);
+  cudaFree(h->s_w);
+  cudaFree(h->s_out);
+  cudaGetLastError();
+  delete h;
+}
+
+const char* pic_decode_kernel_name(const pic_decoder* h) { return h ? h->kern.name : ""; }
+
+}  // extern "C"

@@ -1,0 +1,26 @@
+// pic_kernels.h -- internal registry of the decode kernels (not part of the
+// public C ABI).  Each kernel translation unit lists its instantiations here;
+// pic_decode.cu picks one at create time.
+#pragma once
+
+namespace pic {
+
+struct KernelInfo {
+  const char* name;
+  int precision;   // 0 = fp32 CUDA cores, 1 = fp16 tensor cores
+  int generic;     // 1: runtime dims (fallback), 0: dims fixed below
+  int C;
+  int n_layers;
+  int dims[7];
+  int act;
+  int threads;     // threads per CTA
+  int smem_bytes;  // dynamic shared memory per CTA
+  int tile_px;     // pixels per tile (one tile = a run of one image row)
+  const void* fn;  // __global__ function taking (DecodeParams)
+};
+
+int fp32_kernels(KernelInfo* out, int cap);
+KernelInfo fp32_generic_kernel_info();
+int tc_kernels(KernelInfo* out, int cap);
+
+}  // namespace pic

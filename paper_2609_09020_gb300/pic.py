@@ -1,0 +1,233 @@
+"""ctypes binding of the C ABI in include/pic_decode.h (libpic_gb300.so).
+
+Argument marshalling only: every step of the decode runs in the library's CUDA
+kernels.  The functions keep the C names; ``Decoder`` wraps a handle and
+accepts torch CUDA tensors (PyTorch supplies device memory and streams) or,
+for ``decode_batch_host``, host numpy arrays.
+
+Loading fails loudly (ImportError/OSError) when the library has not been
+built; there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+PIC_OK = 0
+PIC_ERR_INVALID_ARG = -1
+PIC_ERR_UNSUPPORTED = -2
+PIC_ERR_CUDA = -3
+PIC_ERR_ALLOC = -4
+PIC_ERR_TIMEOUT = -5
+
+PIC_ACT_RELU = 0
+PIC_ACT_GELU = 1
+PIC_PREC_FP32 = 0
+PIC_PREC_FP16_TC = 1
+
+ACTS = {"relu": PIC_ACT_RELU, "gelu": PIC_ACT_GELU}
+PRECS = {"fp32": PIC_PREC_FP32, "fp16_tc": PIC_PREC_FP16_TC}
+
+
+class pic_arch(ctypes.Structure):
+    _fields_ = [
+        ("num_levels", ctypes.c_int),
+        ("channels_per_level", ctypes.c_int),
+        ("num_layers", ctypes.c_int),
+        ("dims", ctypes.c_int * 7),
+        ("hidden_act", ctypes.c_int),
+        ("precision", ctypes.c_int),
+        ("clamp_output", ctypes.c_int),
+        ("max_H", ctypes.c_int),
+        ("max_W", ctypes.c_int),
+        ("max_batch", ctypes.c_int),
+    ]
+
+
+_P = ctypes.c_void_p
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load_library():
+    """Loads libpic_gb300.so (built by ``build.build()``); raises if missing."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = library_path()
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: run paper_2609_09020_gb300.build.build() first "
+                          "(there is no CPU fallback)")
+    lib = ctypes.CDLL(path)
+    i, i64 = ctypes.c_int, ctypes.c_int64
+    lib.pic_decode_create.argtypes = [ctypes.POINTER(pic_arch), ctypes.POINTER(_P)]
+    lib.pic_decode_create.restype = i
+    lib.pic_decode.argtypes = [_P, _P, _P, _P, i, i, _P, _P]
+    lib.pic_decode.restype = i
+    lib.pic_decode_batch.argtypes = [_P, i, _P, _P, _P, i, i, _P, _P]
+    lib.pic_decode_batch.restype = i
+    lib.pic_decode_batch_host.argtypes = [_P, i, _P, _P, _P, i, i, _P, _P]
+    lib.pic_decode_batch_host.restype = i
+    lib.pic_decode_check.argtypes = [_P, _P]
+    lib.pic_decode_check.restype = i
+    lib.pic_decode_destroy.argtypes = [_P]
+    lib.pic_decode_destroy.restype = None
+    lib.pic_decode_kernel_name.argtypes = [_P]
+    lib.pic_decode_kernel_name.restype = ctypes.c_char_p
+    lib.pic_latent_count.argtypes = [i, i, i, i]
+    lib.pic_latent_count.restype = i64
+    lib.pic_param_count.argtypes = [ctypes.POINTER(pic_arch)]
+    lib.pic_param_count.restype = i64
+    lib.pic_status_string.argtypes = [i]
+    lib.pic_status_string.restype = ctypes.c_char_p
+    _lib = lib
+    return lib
+
+
+class PicError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        lib = load_library()
+        super().__init__(f"{where}: {lib.pic_status_string(status).decode()} ({status})")
+        self.status = status
+
+
+def make_arch(L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1, max_W=1,
+              max_batch=1) -> pic_arch:
+    a = pic_arch()
+    a.num_levels, a.channels_per_level, a.num_layers = L, C, len(dims) - 1
+    for k, d in enumerate(dims):
+        a.dims[k] = int(d)
+    a.hidden_act = ACTS[act] if isinstance(act, str) else int(act)
+    a.precision = PRECS[precision] if isinstance(precision, str) else int(precision)
+    a.clamp_output = int(bool(clamp))
+    a.max_H, a.max_W, a.max_batch = max_H, max_W, max_batch
+    return a
+
+
+# ---- the C functions, same names -------------------------------------------
+def pic_decode_create(arch: pic_arch) -> int:
+    h = _P()
+    rc = load_library().pic_decode_create(ctypes.byref(arch), ctypes.byref(h))
+    if rc != PIC_OK:
+        raise PicError(rc, "pic_decode_create")
+    return h.value
+
+
+def pic_decode(h, latents, steps, weights, H, W, out_rgb, stream=None) -> int:
+    return load_library().pic_decode(h, latents, steps, weights, H, W, out_rgb, stream)
+
+
+def pic_decode_batch(h, B, latents, steps, weights, H, W, out_rgb, stream=None) -> int:
+    return load_library().pic_decode_batch(h, B, latents, steps, weights, H, W, out_rgb, stream)
+
+
+def pic_decode_batch_host(h, B, latents, steps, weights, H, W, out_rgb, stream=None) -> int:
+    return load_library().pic_decode_batch_host(h, B, latents, steps, weights, H, W, out_rgb,
+                                                stream)
+
+
+def pic_decode_check(h, stream=None) -> int:
+    return load_library().pic_decode_check(h, stream)
+
+
+def pic_decode_destroy(h) -> None:
+    load_library().pic_decode_destroy(h)
+
+
+def pic_decode_kernel_name(h) -> str:
+    return load_library().pic_decode_kernel_name(h).decode()
+
+
+def pic_latent_count(H, W, L, C) -> int:
+    return int(load_library().pic_latent_count(H, W, L, C))
+
+
+def pic_param_count(arch: pic_arch) -> int:
+    return int(load_library().pic_param_count(ctypes.byref(arch)))
+
+
+def pic_status_string(status: int) -> str:
+    return load_library().pic_status_string(status).decode()
+
+
+# ---- convenience wrapper over torch tensors --------------------------------
+def _stream_ptr(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return getattr(stream, "cuda_stream", stream)
+
+
+class Decoder:
+    """One decoder handle.  Tensors passed to the decode methods must be
+    contiguous CUDA tensors of the documented dtypes."""
+
+    def __init__(self, L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1,
+                 max_W=1, max_batch=1):
+        self.arch = make_arch(L, C, dims, act, precision, clamp, max_H, max_W, max_batch)
+        self.L, self.C, self.dims, self.precision = L, C, tuple(dims), precision
+        self.handle = pic_decode_create(self.arch)
+
+    @classmethod
+    def for_workload(cls, wl, precision: str, clamp=True, max_batch=None):
+        return cls(wl.L, wl.C, wl.dims, wl.act, precision, clamp, wl.H, wl.W,
+                   max_batch or wl.B)
+
+    @property
+    def kernel_name(self) -> str:
+        return pic_decode_kernel_name(self.handle)
+
+    def close(self):
+        if self.handle:
+            pic_decode_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @staticmethod
+    def _check(rc, where):
+        if rc != PIC_OK:
+            raise PicError(rc, where)
+
+    def decode_batch(self, latents, steps, weights, H, W, out, stream=None, B=None):
+        """Enqueues a batch decode; arguments are torch CUDA tensors."""
+        if B is None:
+            B = out.shape[0] if out.dim() == 4 else 1
+        rc = pic_decode_batch(self.handle, B, latents.data_ptr(), steps.data_ptr(),
+                              weights.data_ptr(), H, W, out.data_ptr(), _stream_ptr(stream))
+        self._check(rc, "pic_decode_batch")
+        return out
+
+    def decode(self, latents, steps, weights, H, W, out, stream=None):
+        rc = pic_decode(self.handle, latents.data_ptr(), steps.data_ptr(), weights.data_ptr(),
+                        H, W, out.data_ptr(), _stream_ptr(stream))
+        self._check(rc, "pic_decode")
+        return out
+
+    def decode_batch_host(self, latents: np.ndarray, steps: np.ndarray, weights: np.ndarray,
+                          H, W, out: np.ndarray, stream=None, B=None):
+        """Host buffers in, host RGB out (copies and decode inside the call)."""
+        if B is None:
+            B = latents.shape[0] if latents.ndim == 2 else 1
+        for a in (latents, steps, weights, out):
+            if not a.flags["C_CONTIGUOUS"]:
+                raise ValueError("host buffers must be C-contiguous")
+        ptr = lambda a: a.ctypes.data if isinstance(a, np.ndarray) else a.data_ptr()
+        rc = pic_decode_batch_host(self.handle, B, ptr(latents), ptr(steps), ptr(weights), H, W,
+                                   ptr(out), _stream_ptr(stream))
+        self._check(rc, "pic_decode_batch_host")
+        return out
+
+    def check(self, stream=None):
+        self._check(pic_decode_check(self.handle, _stream_ptr(stream)), "pic_decode_check")

@@ -1,0 +1,84 @@
+"""Host-side checks of the C-ABI library: it builds for sm_103a, loads, and
+exports every function include/pic_decode.h declares; size helpers and
+argument checks answer without touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_09020_gb300 import build, pic
+    build.build()
+    return pic.load_library()
+
+
+def declared_functions():
+    names = []
+    for fn in sorted(os.listdir(os.path.join(ROOT, "include"))):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names += re.findall(r"\b(pic_\w+)\s*\(", src)
+    return sorted(set(names))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("pic_decode_create", "pic_decode", "pic_decode_batch", "pic_decode_destroy",
+                     "pic_status_string"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert isinstance(getattr(lib, name), ctypes._CFuncPtr)
+
+
+def test_size_helpers(lib):
+    from paper_2609_09020_gb300 import pic, workloads as wk
+    for wl in wk.WORKLOADS.values():
+        assert pic.pic_latent_count(wl.H, wl.W, wl.L, wl.C) == wl.n_latents
+        arch = pic.make_arch(wl.L, wl.C, wl.dims, wl.act)
+        assert pic.pic_param_count(arch) == wl.n_params
+    assert pic.pic_latent_count(0, 5, 1, 1) == -1
+
+
+def test_status_strings(lib):
+    from paper_2609_09020_gb300 import pic
+    for s in (0, -1, -2, -3, -4, -5):
+        assert pic.pic_status_string(s) not in ("", "unknown status")
+    assert pic.pic_status_string(7) == "unknown status"
+
+
+def test_null_and_bad_arguments_are_rejected_without_a_gpu(lib):
+    from paper_2609_09020_gb300 import pic
+    assert lib.pic_decode(None, None, None, None, 4, 4, None, None) == pic.PIC_ERR_INVALID_ARG
+    assert lib.pic_decode_batch(None, 1, None, None, None, 4, 4, None, None) == pic.PIC_ERR_INVALID_ARG
+    assert lib.pic_decode_batch_host(None, 1, None, None, None, 4, 4, None, None) == pic.PIC_ERR_INVALID_ARG
+    assert lib.pic_decode_check(None, None) == pic.PIC_ERR_INVALID_ARG
+    lib.pic_decode_destroy(None)
+    assert pic.pic_decode_kernel_name(None) == ""
+    h = ctypes.c_void_p(123)
+    assert lib.pic_decode_create(None, ctypes.byref(h)) == pic.PIC_ERR_INVALID_ARG
+    assert h.value is None
+    bad = pic.make_arch(2, 1, (3, 8, 3))          # dims[0] != L*C
+    assert lib.pic_decode_create(ctypes.byref(bad), ctypes.byref(h)) == pic.PIC_ERR_INVALID_ARG
+    wide = pic.make_arch(2, 1, (2, 256, 3), max_H=4, max_W=4)   # width above the envelope
+    assert lib.pic_decode_create(ctypes.byref(wide), ctypes.byref(h)) == pic.PIC_ERR_UNSUPPORTED
+
+
+def test_create_without_gpu_fails_cleanly(lib):
+    torch = pytest.importorskip("torch")
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    from paper_2609_09020_gb300 import pic
+    arch = pic.make_arch(4, 1, (4, 16, 16, 3), max_H=8, max_W=8)
+    h = ctypes.c_void_p()
+    rc = lib.pic_decode_create(ctypes.byref(arch), ctypes.byref(h))
+    assert rc in (pic.PIC_ERR_UNSUPPORTED, pic.PIC_ERR_CUDA) and h.value is None
