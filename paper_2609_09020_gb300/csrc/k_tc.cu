@@ -1,11 +1,443 @@
-// k_tc.cu -- fused decode on the tensor cores (PIC_PREC_FP16_TC).
+// k_tc.cu -- fused decode on the 5th-generation tensor cores (PIC_PREC_FP16_TC).
+//
+// The synthesis MLP g_s (Sec. 4.1) runs as a chain of tcgen05 MMAs with the
+// accumulators in tensor memory; dequantisation, bilinear upsampling and
+// concatenation of the pyramid levels (Sec. 3.1, Eq. 1) produce the first
+// layer's operand directly in shared memory, and the clamped RGB leaves the
+// last accumulator straight for global memory.  Nothing between the latents
+// and the RGB planes touches HBM.
+//
+// Precision: weights are fp16 (used exactly as given).  Every activation
+// operand a (feature or hidden value, fp32) is split into two fp16 terms
+//   a_hi = a with its low 13 mantissa bits cleared (exact in fp16),
+//   a_lo = fp16(a - a_hi),
+// and each layer computes W a_hi + W a_lo + b with fp32 accumulation, so the
+// products carry ~22 significant bits instead of fp16's 11.  The bias rides
+// along as one more K column: A holds a constant 1, B holds b.
+//
+// Operand layout per 128-pixel tile (K-major, canonical no-swizzle layout):
+//   layer 0      A1 = [f_hi | f_lo | 1 | 0..]      K1 = round16(2 D0 + 1)
+//                B1 = [W_0  | W_0  | b | 0..]
+//   hidden k     A  = [h_hi | h_lo | 1 0..0]       KA = 2N + 16
+//                B  = [W_k | b 0..0]               KB = N + 16, read twice (hi, lo)
+//   output       B  = [W_out | b 0..0] (3 rows of 16)
+//
+// CTA organisation (one CTA per SM, persistent over a contiguous tile range):
+//   warps 0 .. 4*NWG-1 : NWG warpgroups; warpgroup w owns every NWG-th tile of
+//                        the range, a TMEM accumulator of N columns and its
+//                        own operand buffers.  Thread r of the group decodes
+//                        pixel r of the tile: features -> A1, then each
+//                        accumulator -> activation -> hi/lo -> next A, and
+//                        finally the clamped RGB store.
+//   warp 4*NWG         : one thread issues all MMAs (tcgen05.mma) in a fixed
+//                        round-robin over (tile round, layer, warpgroup) and
+//                        signals completion with tcgen05.commit.
+// Handshakes are mbarriers: a_full[w] (128 arrivals: operand written) and
+// acc_full[w] (commit: accumulator ready).  Every wait is bounded; on timeout
+// the kernel raises the handle's status word, skips the remaining work and
+// still frees its tensor memory.
+#include <cuda_fp16.h>
+
 #include "pic_common.cuh"
 #include "pic_kernels.h"
+#include "tc_ptx.cuh"
 
 namespace pic {
-int tc_kernels(KernelInfo* out, int cap) {
-  (void)out;
-  (void)cap;
-  return 0;
+namespace {
+
+using namespace tc;
+
+constexpr int kTile = 128;
+constexpr uint32_t kSpinLimit = 1u << 24;   // ~1 s of polling at most per wait
+
+__host__ __device__ constexpr int round_up(int v, int m) { return (v + m - 1) / m * m; }
+__host__ __device__ constexpr int pow2_at_least(int v) {
+  int p = 32;
+  while (p < v) p *= 2;
+  return p;
 }
+
+// Byte offset of element (row, k) in a [rows][K] fp16 tile stored K-major in
+// the canonical no-swizzle layout: core matrix (row/8, k/8) at
+// (row/8) * SBO + (k/8) * LBO with LBO = 128 B and SBO = 16 K bytes.
+__host__ __device__ constexpr uint32_t kmaj(int row, int k, int K) {
+  return static_cast<uint32_t>((row >> 3) * (K * 16) + (k >> 3) * 128 + (row & 7) * 16 + (k & 7) * 2);
+}
+
+template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_>
+struct TcNet {
+  static constexpr int C = C_, NL = NL_, D0 = D0_, N = N_, ACT = ACT_, NWG = NWG_;
+  static constexpr int L = D0 / C;
+  static constexpr int K1 = round_up(2 * D0 + 1, 16);
+  static constexpr int KA = 2 * N + 16;
+  static constexpr int KB = N + 16;
+  static constexpr int NOUT = 16;
+  static constexpr int THREADS = NWG * 128 + 32;
+  static constexpr int MMA_WARP = NWG * 4;
+  static constexpr int CTRL = 256;
+  static constexpr int B1_BYTES = N * K1 * 2;
+  static constexpr int BH_BYTES = N * KB * 2;
+  static constexpr int BO_BYTES = NOUT * KB * 2;
+  static constexpr int OFF_B1 = CTRL;
+  static constexpr int OFF_BH = OFF_B1 + B1_BYTES;
+  static constexpr int OFF_BO = OFF_BH + (NL - 2) * BH_BYTES;
+  static constexpr int OFF_WG = round_up(OFF_BO + BO_BYTES, 128);
+  static constexpr int A1_BYTES = kTile * K1 * 2;
+  static constexpr int A_BYTES = kTile * KA * 2;
+  static constexpr int WG_BYTES = A1_BYTES + A_BYTES;
+  static constexpr int SMEM = OFF_WG + NWG * WG_BYTES;
+  static constexpr int TMEM_COLS = pow2_at_least(NWG * N);
+  static_assert(N % 16 == 0 && N >= 16 && N <= 128, "hidden width must be 16..128, multiple of 16");
+  static_assert(NL >= 2, "the tensor-core path needs at least one hidden layer");
+  static_assert(TMEM_COLS <= 512, "tensor memory holds 512 columns");
+};
+
+// Bounded mbarrier wait.  Returns false (and raises the abort flag and the
+// handle's status word) if the phase does not complete in time, or if
+// another thread has already aborted.
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                             int* status) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 63u) {
+      if (*abort_flag) return false;
+      __nanosleep(32);
+    }
+  }
+  *abort_flag = 1;
+  atomicOr(status, 1);
+  return false;
+}
+
+__device__ __forceinline__ __half ldh(const __half* p) {
+  return __ushort_as_half(__ldg(reinterpret_cast<const unsigned short*>(p)));
+}
+
+// Fills the weight operands of one image into shared memory (all threads).
+template <class Net>
+__device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
+                                                const int (&dims)[Net::NL + 1]) {
+  constexpr int N = Net::N, D0 = Net::D0, K1 = Net::K1, KB = Net::KB, NL = Net::NL;
+  const __half zero = __float2half_rn(0.0f);
+  // layer 0: [W | W | b | 0]
+  {
+    const int d1 = dims[1];
+    const __half* W0 = w;
+    const __half* b0 = w + d1 * D0;
+    for (int e = threadIdx.x; e < N * K1; e += blockDim.x) {
+      const int n = e / K1, j = e - n * K1;
+      __half v = zero;
+      if (n < d1) {
+        if (j < D0) v = ldh(W0 + n * D0 + j);
+        else if (j < 2 * D0) v = ldh(W0 + n * D0 + (j - D0));
+        else if (j == 2 * D0) v = ldh(b0 + n);
+      }
+      *reinterpret_cast<__half*>(smem + Net::OFF_B1 + kmaj(n, j, K1)) = v;
+    }
+  }
+  // hidden layers and output: [W | b 0..0]
+  const __half* p = w + dims[1] * D0 + dims[1];
+#pragma unroll
+  for (int k = 1; k < NL; ++k) {
+    const int din = dims[k], dout = dims[k + 1];
+    const bool out_layer = (k == NL - 1);
+    const int rows = out_layer ? Net::NOUT : N;
+    uint8_t* base = smem + (out_layer ? Net::OFF_BO : Net::OFF_BH + (k - 1) * Net::BH_BYTES);
+    const __half* Wk = p;
+    const __half* bk = p + dout * din;
+    for (int e = threadIdx.x; e < rows * KB; e += blockDim.x) {
+      const int n = e / KB, j = e - n * KB;
+      __half v = zero;
+      if (n < dout) {
+        if (j < din) v = ldh(Wk + n * din + j);
+        else if (j == N) v = ldh(bk + n);
+      }
+      *reinterpret_cast<__half*>(base + kmaj(n, j, KB)) = v;
+    }
+    p = bk + dout;
+  }
+}
+
+// Splits v into (hi, lo) fp32 parts: hi = v with the low 13 mantissa bits
+// cleared (an fp16 value for |v| in fp16's normal range), lo = v - hi (exact).
+__device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
+  hi = __uint_as_float(__float_as_uint(v) & 0xFFFFE000u);
+  lo = v - hi;
+}
+
+template <class Net>
+__global__ void __launch_bounds__(Net::THREADS, 1) tc_decode_kernel(const DecodeParams p) {
+  constexpr int N = Net::N, NL = Net::NL, C = Net::C, L = Net::L, D0 = Net::D0, NWG = Net::NWG;
+  constexpr int K1 = Net::K1, KA = Net::KA, KB = Net::KB;
+  extern __shared__ __align__(1024) uint8_t smem[];
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t sbase = smem_addr(smem);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + 128);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + 136);
+  const uint32_t bar_a0 = sbase;              // a_full[w]   at sbase + 8 w
+  const uint32_t bar_c0 = sbase + 8 * NWG;    // acc_full[w] at sbase + 8 (NWG + w)
+  const uint32_t bar_drain = sbase + 16 * NWG; // final MMA completion before freeing TMEM
+
+  if (threadIdx.x == 0) {
+    for (int w = 0; w < NWG; ++w) {
+      mbar_init(bar_a0 + 8 * w, 128);
+      mbar_init(bar_c0 + 8 * w, 1);
+    }
+    mbar_init(bar_drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == Net::MMA_WARP) {
+    tmem_alloc(smem_addr(tmem_slot), Net::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  const long long chunk = (p.total_tiles + gridDim.x - 1) / gridDim.x;
+  const long long t_begin = blockIdx.x * chunk;
+  const long long t_end = min(t_begin + chunk, p.total_tiles);
+  const __half* wts = static_cast<const __half*>(p.weights);
+  const long long plane = static_cast<long long>(p.H) * p.W;
+
+  // Phase bits: epilogue threads track their group's acc_full; the MMA
+  // thread tracks every group's a_full.
+  uint32_t acc_phase = 0;
+  uint32_t a_phase = 0;  // bit w for group w
+
+  for (long long seg = t_begin; seg < t_end;) {
+    const int b = static_cast<int>(seg / p.tiles_per_image);
+    const long long seg_end = min(t_end, static_cast<long long>(b + 1) * p.tiles_per_image);
+    __syncthreads();  // all MMAs and reads of the previous image's weights are done
+    {
+      int dims[NL + 1];
+#pragma unroll
+      for (int k = 0; k <= NL; ++k) dims[k] = p.dims[k];
+      load_weights_tc<Net>(smem, wts + b * p.params_per_image, dims);
+    }
+    fence_async_smem();
+    __syncthreads();
+    const int n_tiles = static_cast<int>(seg_end - seg);
+
+    if (warp < 4 * NWG) {
+      // ------------------------------------------------------------ warpgroup
+      const int w = warp >> 2;
+      const int r = ((warp & 3) << 5) | lane;  // tile row = TMEM lane = pixel
+      uint8_t* a1 = smem + Net::OFF_WG + w * Net::WG_BYTES;
+      uint8_t* aa = a1 + Net::A1_BYTES;
+      const uint32_t a1_s = smem_addr(a1), aa_s = smem_addr(aa);
+      const uint32_t t_acc = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) +
+                             static_cast<uint32_t>(w * N);
+      const uint32_t bar_a = bar_a0 + 8 * w, bar_c = bar_c0 + 8 * w;
+      const int32_t* lat = p.latents + b * p.lat_per_image;
+      float step[L];
+#pragma unroll
+      for (int l = 0; l < L; ++l) step[l] = __ldg(p.steps + b * L + l);
+
+      for (int i = w; i < n_tiles; i += NWG) {
+        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+        const long long t = seg + i - static_cast<long long>(b) * p.tiles_per_image;
+        const int y = static_cast<int>(t / p.tiles_per_row);
+        const int x = static_cast<int>(t - static_cast<long long>(y) * p.tiles_per_row) * kTile + r;
+        const bool valid = x < p.W;
+        const int xc = valid ? x : p.W - 1;
+
+        // ---- features: dequantise + upsample + concatenate (Eq. 1) ----
+        float f[D0];
+#pragma unroll
+        for (int l = 0; l < L; ++l) {
+          const LevelGeom lg = p.lv[l];
+          if (l == 0) {
+#pragma unroll
+            for (int c = 0; c < C; ++c)
+              f[c] = step[0] * static_cast<float>(__ldg(lat + c * plane + static_cast<long long>(y) * p.W + xc));
+          } else {
+            const Tap tx = bilinear_tap(xc, lg.sx, lg.W);
+            const Tap ty = bilinear_tap(y, lg.sy, lg.H);
+#pragma unroll
+            for (int c = 0; c < C; ++c)
+              f[l * C + c] = step[l] * bilinear_sample(lat + lg.off + static_cast<long long>(c) * lg.H * lg.W,
+                                                       lg.W, tx, ty);
+          }
+        }
+        {
+          float v[K1];
+#pragma unroll
+          for (int j = 0; j < K1; ++j) v[j] = 0.0f;
+#pragma unroll
+          for (int j = 0; j < D0; ++j) split_hi_lo(f[j], v[j], v[D0 + j]);
+          v[2 * D0] = 1.0f;
+#pragma unroll
+          for (int kc = 0; kc < K1 / 8; ++kc)
+            sts128(a1_s + kmaj(r, kc * 8, K1), pack_f16x2(v[kc * 8 + 0], v[kc * 8 + 1]),
+                   pack_f16x2(v[kc * 8 + 2], v[kc * 8 + 3]), pack_f16x2(v[kc * 8 + 4], v[kc * 8 + 5]),
+                   pack_f16x2(v[kc * 8 + 6], v[kc * 8 + 7]));
+        }
+        fence_async_smem();
+        mbar_arrive(bar_a);
+
+        // ---- hidden layers: accumulator -> act -> hi/lo -> next operand ----
+        bool ok = true;
+#pragma unroll 1
+        for (int k = 0; k < NL - 1; ++k) {
+          if (!__all_sync(0xffffffffu, wait_bounded(bar_c, acc_phase, abort_flag, p.status))) {
+            ok = false;
+            break;
+          }
+          acc_phase ^= 1u;
+          tc_fence_after();
+          uint32_t acc[N];
+#pragma unroll
+          for (int c0 = 0; c0 < N; c0 += 16) tmem_ld16(t_acc + c0, acc + c0);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < N; j += 8) {
+            uint32_t hi[4], lo[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              float a = __uint_as_float(acc[j + 2 * q]);
+              float bb = __uint_as_float(acc[j + 2 * q + 1]);
+              if constexpr (Net::ACT == ACT_GELU) {
+                a = gelu_erf(a);
+                bb = gelu_erf(bb);
+              }
+              float ah, al, bh, bl;
+              split_hi_lo(a, ah, al);
+              split_hi_lo(bb, bh, bl);
+              if constexpr (Net::ACT == ACT_GELU) {
+                hi[q] = pack_f16x2(ah, bh);
+                lo[q] = pack_f16x2(al, bl);
+              } else {  // ReLU folded into the conversion (hi, lo share v's sign)
+                hi[q] = pack_f16x2_relu(ah, bh);
+                lo[q] = pack_f16x2_relu(al, bl);
+              }
+            }
+            sts128(aa_s + kmaj(r, j, KA), hi[0], hi[1], hi[2], hi[3]);
+            sts128(aa_s + kmaj(r, N + j, KA), lo[0], lo[1], lo[2], lo[3]);
+          }
+          sts128(aa_s + kmaj(r, 2 * N, KA), 0x00003C00u, 0u, 0u, 0u);  // the constant-1 bias column
+          sts128(aa_s + kmaj(r, 2 * N + 8, KA), 0u, 0u, 0u, 0u);
+          fence_async_smem();
+          tc_fence_before();
+          mbar_arrive(bar_a);
+        }
+        if (!ok) break;
+
+        // ---- output layer: clamp, planar coalesced store ----
+        if (!__all_sync(0xffffffffu, wait_bounded(bar_c, acc_phase, abort_flag, p.status))) break;
+        acc_phase ^= 1u;
+        tc_fence_after();
+        uint32_t o[4];
+        tmem_ld4(t_acc, o);
+        tmem_ld_wait();
+        tc_fence_before();
+        if (valid) {
+          float* dst = p.out + static_cast<long long>(b) * 3 * plane + static_cast<long long>(y) * p.W + x;
+#pragma unroll
+          for (int c = 0; c < 3; ++c) {
+            const float v = __uint_as_float(o[c]);
+            dst[c * plane] = p.clamp ? __saturatef(v) : v;
+          }
+        }
+      }
+    } else if (warp == Net::MMA_WARP && lane == 0) {
+      // --------------------------------------------------------------- MMA issuer
+      const uint32_t b1_s = sbase + Net::OFF_B1;
+      const uint32_t bh_s = sbase + Net::OFF_BH;
+      const uint32_t bo_s = sbase + Net::OFF_BO;
+      constexpr uint32_t id_hidden = idesc_f16(128, N);
+      constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
+      const int rounds = (n_tiles + NWG - 1) / NWG;
+      bool ok = true;
+      for (int rd = 0; rd < rounds && ok; ++rd) {
+        for (int k = 0; k < NL && ok; ++k) {
+          for (int w = 0; w < NWG; ++w) {
+            if (rd * NWG + w >= n_tiles) break;
+            if (!wait_bounded(bar_a0 + 8 * w, (a_phase >> w) & 1u, abort_flag, p.status)) {
+              ok = false;
+              break;
+            }
+            a_phase ^= (1u << w);
+            tc_fence_after();
+            const uint32_t d = tmem + static_cast<uint32_t>(w * N);
+            const uint32_t a1_s = sbase + Net::OFF_WG + w * Net::WG_BYTES;
+            const uint32_t aa_s = a1_s + Net::A1_BYTES;
+            if (k == 0) {
+#pragma unroll
+              for (int s = 0; s < K1 / 16; ++s)
+                mma_f16(d, smem_desc(a1_s + s * 256, 128, 16 * K1), smem_desc(b1_s + s * 256, 128, 16 * K1),
+                        id_hidden, s > 0);
+            } else {
+              const bool out_layer = (k == NL - 1);
+              const uint32_t bk = out_layer ? bo_s : bh_s + (k - 1) * Net::BH_BYTES;
+              const uint32_t id = out_layer ? id_out : id_hidden;
+#pragma unroll
+              for (int s = 0; s < N / 16; ++s)  // hi part
+                mma_f16(d, smem_desc(aa_s + s * 256, 128, 16 * KA), smem_desc(bk + s * 256, 128, 16 * KB), id,
+                        s > 0);
+#pragma unroll
+              for (int s = 0; s < N / 16; ++s)  // lo part, same weights
+                mma_f16(d, smem_desc(aa_s + (N / 16 + s) * 256, 128, 16 * KA),
+                        smem_desc(bk + s * 256, 128, 16 * KB), id, 1);
+              mma_f16(d, smem_desc(aa_s + (N / 8) * 256, 128, 16 * KA),  // bias column
+                      smem_desc(bk + (N / 16) * 256, 128, 16 * KB), id, 1);
+            }
+            mma_commit(bar_c0 + 8 * w);
+          }
+        }
+      }
+    }
+    __syncwarp();
+    seg = seg_end;
+  }
+
+  if (warp == Net::MMA_WARP && lane == 0) {
+    // Every MMA this thread issued must be complete before the memory goes.
+    mma_commit(bar_drain);
+    int dummy = 0;
+    wait_bounded(bar_drain, 0, reinterpret_cast<volatile int*>(&dummy), p.status);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == Net::MMA_WARP) {
+    tc_fence_after();
+    tmem_dealloc(tmem, Net::TMEM_COLS);
+  }
+}
+
+template <int C, int NL, int D0, int N, int ACT, int NWG>
+KernelInfo make_tc(const char* name, const int* dims) {
+  using Net = TcNet<C, NL, D0, N, ACT, NWG>;
+  KernelInfo k{};
+  k.name = name;
+  k.precision = 1;
+  k.C = C;
+  k.n_layers = NL;
+  for (int i = 0; i <= NL; ++i) k.dims[i] = dims[i];
+  k.act = ACT;
+  k.threads = Net::THREADS;
+  k.tile_px = kTile;
+  k.smem_bytes = Net::SMEM;
+  k.fn = reinterpret_cast<const void*>(&tc_decode_kernel<Net>);
+  return k;
+}
+
+}  // namespace
+
+int tc_kernels(KernelInfo* out, int cap) {
+  static const int d_c5[] = {7, 64, 64, 3};
+  static const int d_c4[] = {16, 64, 64, 64, 3};
+  const KernelInfo list[] = {
+      make_tc<1, 3, 7, 64, ACT_RELU, 3>("tc05_7x64x64x3_relu", d_c5),
+      make_tc<2, 4, 16, 64, ACT_GELU, 3>("tc05_16x64x64x64x3_gelu", d_c4),
+  };
+  const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
+  for (int i = 0; i < n && i < cap; ++i) out[i] = list[i];
+  return n;
+}
+
 }  // namespace pic
