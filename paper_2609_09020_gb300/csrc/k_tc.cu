@@ -48,7 +48,7 @@ namespace {
 using namespace tc;
 
 constexpr int kTile = 128;
-constexpr uint32_t kSpinLimit = 1u << 24;   // ~1 s of polling at most per wait
+constexpr uint32_t kSpinLimit = 1u << 22;   // a few seconds of polling at most per wait
 
 __host__ __device__ constexpr int round_up(int v, int m) { return (v + m - 1) / m * m; }
 __host__ __device__ constexpr int pow2_at_least(int v) {
