@@ -64,6 +64,12 @@ __host__ __device__ constexpr uint32_t kmaj(int row, int k, int K) {
   return static_cast<uint32_t>((row >> 3) * (K * 16) + (k >> 3) * 128 + (row & 7) * 16 + (k & 7) * 2);
 }
 
+__host__ __device__ constexpr int colbuf_floats(int L, int C) {
+  int n = 0;
+  for (int l = 1; l < L; ++l) n += C * ((kTile >> l) + 4);
+  return n;
+}
+
 template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_>
 struct TcNet {
   static constexpr int C = C_, NL = NL_, D0 = D0_, N = N_, ACT = ACT_, NWG = NWG_;
@@ -74,6 +80,9 @@ struct TcNet {
   static constexpr int NOUT = 16;
   static constexpr int THREADS = NWG * 128 + 32;
   static constexpr int MMA_WARP = NWG * 4;
+  // registers per thread that still let one CTA of THREADS threads fit an SM
+  static constexpr int MAXREG = (65536 / (((THREADS + 31) / 32) * 32)) / 8 * 8 > 255
+                                    ? 255 : (65536 / (((THREADS + 31) / 32) * 32)) / 8 * 8;
   static constexpr int CTRL = 256;
   static constexpr int B1_BYTES = N * K1 * 2;
   static constexpr int BH_BYTES = N * KB * 2;
@@ -84,7 +93,8 @@ struct TcNet {
   static constexpr int OFF_WG = round_up(OFF_BO + BO_BYTES, 128);
   static constexpr int A1_BYTES = kTile * K1 * 2;
   static constexpr int A_BYTES = kTile * KA * 2;
-  static constexpr int WG_BYTES = A1_BYTES + A_BYTES;
+  static constexpr int COL_BYTES = round_up(colbuf_floats(L, C) * 4, 128);
+  static constexpr int WG_BYTES = A1_BYTES + A_BYTES + COL_BYTES;
   static constexpr int SMEM = OFF_WG + NWG * WG_BYTES;
   static constexpr int TMEM_COLS = pow2_at_least(NWG * N);
   static_assert(N % 16 == 0 && N >= 16 && N <= 128, "hidden width must be 16..128, multiple of 16");
@@ -101,7 +111,7 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, vola
     if (mbar_try_wait(bar, parity)) return true;
     if ((i & 63u) == 63u) {
       if (*abort_flag) return false;
-      __nanosleep(32);
+      if (i > 4096) __nanosleep(64);
     }
   }
   *abort_flag = 1;
@@ -165,10 +175,43 @@ __device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
   lo = v - hi;
 }
 
+// Cooperative feature staging.  For level l >= 1 a 128-pixel row segment
+// needs at most NCOL(l) = 128/2^l + 4 source columns.  The warpgroup first
+// interpolates those columns vertically (rows v0, v1 of the level, weight
+// beta) into a small shared buffer -- one item per (level, channel, column),
+// spread over the 128 threads -- and every pixel then interpolates
+// horizontally between two buffer entries.  Column indices are clamped into
+// [0, W_l - 1] when the buffer is filled, which reproduces the edge clamp of
+// the bilinear definition.
+__host__ __device__ constexpr int ncol(int l) { return (kTile >> l) + 4; }
+
+template <int L, int C>
+struct ColLayout {
+  // float offset of (level l, channel c) inside the column buffer
+  static constexpr int off(int l, int c) {
+    int o = 0;
+    for (int k = 1; k < l; ++k) o += C * ncol(k);
+    return o + c * ncol(l);
+  }
+  static constexpr int total() { return off(L, 0); }
+};
+
+// Per-thread share of the column items of one tile: the raw texels (loaded
+// one tile ahead) and the vertical weight.
+template <int J>
+struct ColPrefetch {
+  int q0[J], q1[J];
+  float beta[J];
+};
+
 template <class Net>
-__global__ void __launch_bounds__(Net::THREADS, 1) tc_decode_kernel(const DecodeParams p) {
+__global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_decode_kernel(const DecodeParams p) {
   constexpr int N = Net::N, NL = Net::NL, C = Net::C, L = Net::L, D0 = Net::D0, NWG = Net::NWG;
   constexpr int K1 = Net::K1, KA = Net::KA, KB = Net::KB;
+  using CL = ColLayout<L, C>;
+  constexpr int NITEM = CL::total();
+  constexpr int J = (NITEM + kTile - 1) / kTile;  // column items per thread (0 if L == 1)
+  constexpr int JJ = J > 0 ? J : 1;
   extern __shared__ __align__(1024) uint8_t smem[];
 
   const int warp = threadIdx.x >> 5;
@@ -176,9 +219,11 @@ __global__ void __launch_bounds__(Net::THREADS, 1) tc_decode_kernel(const Decode
   const uint32_t sbase = smem_addr(smem);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + 128);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + 136);
-  const uint32_t bar_a0 = sbase;              // a_full[w]   at sbase + 8 w
-  const uint32_t bar_c0 = sbase + 8 * NWG;    // acc_full[w] at sbase + 8 (NWG + w)
+  const uint32_t bar_a0 = sbase;               // a_full[w]   at sbase + 8 w
+  const uint32_t bar_c0 = sbase + 8 * NWG;     // acc_full[w] at sbase + 8 (NWG + w)
   const uint32_t bar_drain = sbase + 16 * NWG; // final MMA completion before freeing TMEM
+  const uint32_t bar_col0 = sbase + 8 * (2 * NWG + 1);  // col_ready[w]: column buffer written
+  static_assert(8 * (3 * NWG + 1) <= 128, "control block holds the barriers");
 
   if (threadIdx.x == 0) {
     for (int w = 0; w < NWG; ++w) {
@@ -186,6 +231,7 @@ __global__ void __launch_bounds__(Net::THREADS, 1) tc_decode_kernel(const Decode
       mbar_init(bar_c0 + 8 * w, 1);
     }
     mbar_init(bar_drain, 1);
+    for (int w = 0; w < NWG; ++w) mbar_init(bar_col0 + 8 * w, 128);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -203,11 +249,13 @@ __global__ void __launch_bounds__(Net::THREADS, 1) tc_decode_kernel(const Decode
   const long long t_end = min(t_begin + chunk, p.total_tiles);
   const __half* wts = static_cast<const __half*>(p.weights);
   const long long plane = static_cast<long long>(p.H) * p.W;
+  // x-taps repeat from tile to tile when every level's width is exactly W / 2^l
+  // (and 2^l divides the 128-pixel tile origin, i.e. l <= 7)
+  const bool fast_x = (L - 1 <= 7) && (p.W % (1 << (L - 1))) == 0;
 
-  // Phase bits: epilogue threads track their group's acc_full; the MMA
-  // thread tracks every group's a_full.
-  uint32_t acc_phase = 0;
-  uint32_t a_phase = 0;  // bit w for group w
+  uint32_t acc_phase = 0;  // warpgroup threads: parity of their acc_full
+  uint32_t col_phase = 0;  // warpgroup threads: parity of their col_ready
+  uint32_t a_phase = 0;    // MMA thread: bit w = parity of a_full[w]
 
   for (long long seg = t_begin; seg < t_end;) {
     const int b = static_cast<int>(seg / p.tiles_per_image);
@@ -222,14 +270,15 @@ __global__ void __launch_bounds__(Net::THREADS, 1) tc_decode_kernel(const Decode
     fence_async_smem();
     __syncthreads();
     const int n_tiles = static_cast<int>(seg_end - seg);
+    const long long tile0 = seg - static_cast<long long>(b) * p.tiles_per_image;  // in-image index
 
     if (warp < 4 * NWG) {
       // ------------------------------------------------------------ warpgroup
       const int w = warp >> 2;
       const int r = ((warp & 3) << 5) | lane;  // tile row = TMEM lane = pixel
       uint8_t* a1 = smem + Net::OFF_WG + w * Net::WG_BYTES;
-      uint8_t* aa = a1 + Net::A1_BYTES;
-      const uint32_t a1_s = smem_addr(a1), aa_s = smem_addr(aa);
+      const uint32_t a1_s = smem_addr(a1), aa_s = a1_s + Net::A1_BYTES;
+      float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES + Net::A_BYTES);
       const uint32_t t_acc = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) +
                              static_cast<uint32_t>(w * N);
       const uint32_t bar_a = bar_a0 + 8 * w, bar_c = bar_c0 + 8 * w;
@@ -238,30 +287,127 @@ __global__ void __launch_bounds__(Net::THREADS, 1) tc_decode_kernel(const Decode
 #pragma unroll
       for (int l = 0; l < L; ++l) step[l] = __ldg(p.steps + b * L + l);
 
+      // This thread's column items: level, channel, column.
+      int it_l[JJ], it_c[JJ], it_i[JJ];
+#pragma unroll
+      for (int j = 0; j < J; ++j) {
+        int e = r + kTile * j, l = 0, c = 0, i = 0;
+        if (e < NITEM) {
+#pragma unroll
+          for (int lv = 1; lv < L; ++lv)
+#pragma unroll
+            for (int cc = 0; cc < C; ++cc)
+              if (e >= CL::off(lv, cc) && e < CL::off(lv, cc) + ncol(lv)) {
+                l = lv;
+                c = cc;
+                i = e - CL::off(lv, cc);
+              }
+        }
+        it_l[j] = l;  // l == 0 marks an idle slot
+        it_c[j] = c;
+        it_i[j] = i;
+      }
+      // Relative x-taps of pixel r for each level (used when fast_x): the
+      // source coordinate (r + 1/2) / 2^l - 1/2 relative to column x0/2^l - 1.
+      int rel[L];
+      float fx[L];
+#pragma unroll
+      for (int l = 1; l < L; ++l) {
+        const float sx = (static_cast<float>(r) + 0.5f) * (1.0f / static_cast<float>(1 << l)) - 0.5f;
+        const float fl = floorf(sx);
+        rel[l] = static_cast<int>(fl) + 1;
+        fx[l] = sx - fl;
+      }
+
+      // Loads of everything tile i needs from global memory: the level-0
+      // value of pixel r and the raw texel pairs of this thread's items.
+      auto prefetch = [&](int i, int (&q0)[C], ColPrefetch<JJ>& cp) {
+        const long long t = tile0 + i;
+        const int y = static_cast<int>(t / p.tiles_per_row);
+        const int x0 = static_cast<int>(t - static_cast<long long>(y) * p.tiles_per_row) * kTile;
+        const int xc = min(x0 + r, p.W - 1);
+#pragma unroll
+        for (int c = 0; c < C; ++c)
+          q0[c] = __ldg(lat + c * plane + static_cast<long long>(y) * p.W + xc);
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+          cp.q0[j] = 0;
+          cp.q1[j] = 0;
+          cp.beta[j] = 0.0f;
+          const int l = it_l[j];
+          if (l > 0) {
+            const LevelGeom lg = p.lv[l];
+            const Tap ty = bilinear_tap(y, lg.sy, lg.H);
+            const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, lg.sx, lg.W).i0;
+            const int u = min(max(u_start + it_i[j], 0), lg.W - 1);
+            const int32_t* pl = lat + lg.off + static_cast<long long>(it_c[j]) * lg.H * lg.W + u;
+            cp.q0[j] = __ldg(pl + static_cast<long long>(ty.i0) * lg.W);
+            cp.q1[j] = __ldg(pl + static_cast<long long>(ty.i1) * lg.W);
+            cp.beta[j] = ty.frac;
+          }
+        }
+      };
+
+      int q0c[C];
+      ColPrefetch<JJ> cpc;
+      if (w < n_tiles) prefetch(w, q0c, cpc);
+
       for (int i = w; i < n_tiles; i += NWG) {
         if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
-        const long long t = seg + i - static_cast<long long>(b) * p.tiles_per_image;
+        const long long t = tile0 + i;
         const int y = static_cast<int>(t / p.tiles_per_row);
-        const int x = static_cast<int>(t - static_cast<long long>(y) * p.tiles_per_row) * kTile + r;
+        const int x0 = static_cast<int>(t - static_cast<long long>(y) * p.tiles_per_row) * kTile;
+        const int x = x0 + r;
         const bool valid = x < p.W;
         const int xc = valid ? x : p.W - 1;
 
-        // ---- features: dequantise + upsample + concatenate (Eq. 1) ----
+        // prefetch the next tile of this warpgroup
+        int q0n[C];
+        ColPrefetch<JJ> cpn;
+        const bool has_next = i + NWG < n_tiles;
+        if (has_next) prefetch(i + NWG, q0n, cpn);
+
+        // ---- features: vertical pass into the column buffer ----
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+          const int l = it_l[j];
+          if (l > 0) {
+            const float a = static_cast<float>(cpc.q0[j]);
+            const float d = static_cast<float>(cpc.q1[j] - cpc.q0[j]);
+            colbuf[r + kTile * j] = step[l] * fmaf(cpc.beta[j], d, a);
+          }
+        }
+        // warpgroup-wide: the column buffer is complete (bounded wait)
+        mbar_arrive(bar_col0 + 8 * w);
+        if (!__all_sync(0xffffffffu, wait_bounded(bar_col0 + 8 * w, col_phase, abort_flag, p.status)))
+          break;
+        col_phase ^= 1u;
+
+        // ---- features: horizontal pass, level 0, hi/lo split -> A1 ----
         float f[D0];
 #pragma unroll
-        for (int l = 0; l < L; ++l) {
-          const LevelGeom lg = p.lv[l];
-          if (l == 0) {
+        for (int c = 0; c < C; ++c) f[c] = step[0] * static_cast<float>(q0c[c]);
 #pragma unroll
-            for (int c = 0; c < C; ++c)
-              f[c] = step[0] * static_cast<float>(__ldg(lat + c * plane + static_cast<long long>(y) * p.W + xc));
+        for (int l = 1; l < L; ++l) {
+          int i0, i1;
+          float a;
+          if (fast_x) {
+            i0 = rel[l];
+            i1 = rel[l] + 1;
+            a = fx[l];
           } else {
+            const LevelGeom lg = p.lv[l];
+            const int u_start = bilinear_tap(x0, lg.sx, lg.W).i0;
             const Tap tx = bilinear_tap(xc, lg.sx, lg.W);
-            const Tap ty = bilinear_tap(y, lg.sy, lg.H);
+            i0 = min(max(tx.i0 - u_start, 0), ncol(l) - 1);
+            i1 = min(max(tx.i1 - u_start, 0), ncol(l) - 1);
+            a = tx.frac;
+          }
 #pragma unroll
-            for (int c = 0; c < C; ++c)
-              f[l * C + c] = step[l] * bilinear_sample(lat + lg.off + static_cast<long long>(c) * lg.H * lg.W,
-                                                       lg.W, tx, ty);
+          for (int c = 0; c < C; ++c) {
+            const float* cb = colbuf + CL::off(l, c);
+            const float v0 = cb[i0], v1 = cb[i1];
+            f[l * C + c] = fmaf(a, v1 - v0, v0);
           }
         }
         {
@@ -343,51 +489,78 @@ __global__ void __launch_bounds__(Net::THREADS, 1) tc_decode_kernel(const Decode
             dst[c * plane] = p.clamp ? __saturatef(v) : v;
           }
         }
+        if (has_next) {
+#pragma unroll
+          for (int c = 0; c < C; ++c) q0c[c] = q0n[c];
+          cpc = cpn;
+        }
       }
     } else if (warp == Net::MMA_WARP && lane == 0) {
       // --------------------------------------------------------------- MMA issuer
+      // Serves whichever warpgroup has its next operand ready; per group the
+      // order is fixed (its tiles in turn, layers in turn).
       const uint32_t b1_s = sbase + Net::OFF_B1;
       const uint32_t bh_s = sbase + Net::OFF_BH;
       const uint32_t bo_s = sbase + Net::OFF_BO;
       constexpr uint32_t id_hidden = idesc_f16(128, N);
       constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
-      const int rounds = (n_tiles + NWG - 1) / NWG;
-      bool ok = true;
-      for (int rd = 0; rd < rounds && ok; ++rd) {
-        for (int k = 0; k < NL && ok; ++k) {
-          for (int w = 0; w < NWG; ++w) {
-            if (rd * NWG + w >= n_tiles) break;
-            if (!wait_bounded(bar_a0 + 8 * w, (a_phase >> w) & 1u, abort_flag, p.status)) {
-              ok = false;
-              break;
-            }
-            a_phase ^= (1u << w);
-            tc_fence_after();
-            const uint32_t d = tmem + static_cast<uint32_t>(w * N);
-            const uint32_t a1_s = sbase + Net::OFF_WG + w * Net::WG_BYTES;
-            const uint32_t aa_s = a1_s + Net::A1_BYTES;
-            if (k == 0) {
+      int tile_of[NWG], layer_of[NWG];
+      int remaining = 0;
 #pragma unroll
-              for (int s = 0; s < K1 / 16; ++s)
-                mma_f16(d, smem_desc(a1_s + s * 256, 128, 16 * K1), smem_desc(b1_s + s * 256, 128, 16 * K1),
-                        id_hidden, s > 0);
-            } else {
-              const bool out_layer = (k == NL - 1);
-              const uint32_t bk = out_layer ? bo_s : bh_s + (k - 1) * Net::BH_BYTES;
-              const uint32_t id = out_layer ? id_out : id_hidden;
+      for (int w = 0; w < NWG; ++w) {
+        tile_of[w] = w;
+        layer_of[w] = 0;
+        if (w < n_tiles) remaining += ((n_tiles - 1 - w) / NWG + 1) * NL;
+      }
+      uint32_t idle = 0;
+      while (remaining > 0) {
+        bool progressed = false;
 #pragma unroll
-              for (int s = 0; s < N / 16; ++s)  // hi part
-                mma_f16(d, smem_desc(aa_s + s * 256, 128, 16 * KA), smem_desc(bk + s * 256, 128, 16 * KB), id,
-                        s > 0);
+        for (int w = 0; w < NWG; ++w) {
+          if (tile_of[w] >= n_tiles) continue;
+          if (!mbar_test_wait(bar_a0 + 8 * w, (a_phase >> w) & 1u)) continue;
+          a_phase ^= (1u << w);
+          tc_fence_after();
+          const int k = layer_of[w];
+          const uint32_t d = tmem + static_cast<uint32_t>(w * N);
+          const uint32_t a1_s = sbase + Net::OFF_WG + w * Net::WG_BYTES;
+          const uint32_t aa_s = a1_s + Net::A1_BYTES;
+          if (k == 0) {
 #pragma unroll
-              for (int s = 0; s < N / 16; ++s)  // lo part, same weights
-                mma_f16(d, smem_desc(aa_s + (N / 16 + s) * 256, 128, 16 * KA),
-                        smem_desc(bk + s * 256, 128, 16 * KB), id, 1);
-              mma_f16(d, smem_desc(aa_s + (N / 8) * 256, 128, 16 * KA),  // bias column
-                      smem_desc(bk + (N / 16) * 256, 128, 16 * KB), id, 1);
-            }
-            mma_commit(bar_c0 + 8 * w);
+            for (int s = 0; s < K1 / 16; ++s)
+              mma_f16(d, smem_desc(a1_s + s * 256, 128, 16 * K1), smem_desc(b1_s + s * 256, 128, 16 * K1),
+                      id_hidden, s > 0);
+          } else {
+            const bool out_layer = (k == NL - 1);
+            const uint32_t bk = out_layer ? bo_s : bh_s + (k - 1) * Net::BH_BYTES;
+            const uint32_t id = out_layer ? id_out : id_hidden;
+#pragma unroll
+            for (int s = 0; s < N / 16; ++s)  // hi part
+              mma_f16(d, smem_desc(aa_s + s * 256, 128, 16 * KA), smem_desc(bk + s * 256, 128, 16 * KB), id,
+                      s > 0);
+#pragma unroll
+            for (int s = 0; s < N / 16; ++s)  // lo part, same weights
+              mma_f16(d, smem_desc(aa_s + (N / 16 + s) * 256, 128, 16 * KA),
+                      smem_desc(bk + s * 256, 128, 16 * KB), id, 1);
+            mma_f16(d, smem_desc(aa_s + (N / 8) * 256, 128, 16 * KA),  // bias column
+                    smem_desc(bk + (N / 16) * 256, 128, 16 * KB), id, 1);
           }
+          mma_commit(bar_c0 + 8 * w);
+          if (++layer_of[w] == NL) {
+            layer_of[w] = 0;
+            tile_of[w] += NWG;
+          }
+          --remaining;
+          progressed = true;
+        }
+        if (progressed) {
+          idle = 0;
+        } else if (++idle > kSpinLimit || *abort_flag) {
+          *abort_flag = 1;
+          atomicOr(p.status, 1);
+          break;
+        } else if (idle > 256) {
+          __nanosleep(20);
         }
       }
     }
@@ -432,7 +605,7 @@ int tc_kernels(KernelInfo* out, int cap) {
   static const int d_c5[] = {7, 64, 64, 3};
   static const int d_c4[] = {16, 64, 64, 64, 3};
   const KernelInfo list[] = {
-      make_tc<1, 3, 7, 64, ACT_RELU, 3>("tc05_7x64x64x3_relu", d_c5),
+      make_tc<1, 3, 7, 64, ACT_RELU, 4>("tc05_7x64x64x3_relu", d_c5),
       make_tc<2, 4, 16, 64, ACT_GELU, 3>("tc05_16x64x64x64x3_gelu", d_c4),
   };
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
