@@ -80,9 +80,11 @@ struct TcNet {
   static constexpr int NOUT = 16;
   static constexpr int THREADS = NWG * 128 + 32;
   static constexpr int MMA_WARP = NWG * 4;
-  // registers per thread that still let one CTA of THREADS threads fit an SM
-  static constexpr int MAXREG = (65536 / (((THREADS + 31) / 32) * 32)) / 8 * 8 > 255
-                                    ? 255 : (65536 / (((THREADS + 31) / 32) * 32)) / 8 * 8;
+  // Registers per thread that still let one CTA fit an SM: the warps are
+  // spread over the 4 sub-partitions, each with a 16K-register file.
+  static constexpr int WARPS_PER_SMSP = (THREADS / 32 + 3) / 4;
+  static constexpr int MAXREG_RAW = 16384 / (32 * WARPS_PER_SMSP) / 8 * 8;
+  static constexpr int MAXREG = MAXREG_RAW > 255 ? 255 : MAXREG_RAW;
   static constexpr int CTRL = 256;
   static constexpr int B1_BYTES = N * K1 * 2;
   static constexpr int BH_BYTES = N * KB * 2;
@@ -436,34 +438,39 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
           }
           acc_phase ^= 1u;
           tc_fence_after();
-          uint32_t acc[N];
 #pragma unroll
-          for (int c0 = 0; c0 < N; c0 += 16) tmem_ld16(t_acc + c0, acc + c0);
-          tmem_ld_wait();
+          for (int h0 = 0; h0 < N; h0 += 32) {  // two halves of 32 columns (fewer live registers)
+            const int hw = (N - h0) < 32 ? (N - h0) : 32;  // 16 or 32 (N is a multiple of 16)
+            uint32_t acc[32];
 #pragma unroll
-          for (int j = 0; j < N; j += 8) {
-            uint32_t hi[4], lo[4];
+            for (int c0 = 0; c0 < hw; c0 += 16) tmem_ld16(t_acc + h0 + c0, acc + c0);
+            tmem_ld_wait();
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              float a = __uint_as_float(acc[j + 2 * q]);
-              float bb = __uint_as_float(acc[j + 2 * q + 1]);
-              if constexpr (Net::ACT == ACT_GELU) {
-                a = gelu_erf(a);
-                bb = gelu_erf(bb);
+            for (int jj = 0; jj < hw; jj += 8) {
+              const int j = h0 + jj;
+              uint32_t hi[4], lo[4];
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                float a = __uint_as_float(acc[jj + 2 * q]);
+                float bb = __uint_as_float(acc[jj + 2 * q + 1]);
+                if constexpr (Net::ACT == ACT_GELU) {
+                  a = gelu_erf(a);
+                  bb = gelu_erf(bb);
+                }
+                float ah, al, bh, bl;
+                split_hi_lo(a, ah, al);
+                split_hi_lo(bb, bh, bl);
+                if constexpr (Net::ACT == ACT_GELU) {
+                  hi[q] = pack_f16x2(ah, bh);
+                  lo[q] = pack_f16x2(al, bl);
+                } else {  // ReLU folded into the conversion (hi, lo share v's sign)
+                  hi[q] = pack_f16x2_relu(ah, bh);
+                  lo[q] = pack_f16x2_relu(al, bl);
+                }
               }
-              float ah, al, bh, bl;
-              split_hi_lo(a, ah, al);
-              split_hi_lo(bb, bh, bl);
-              if constexpr (Net::ACT == ACT_GELU) {
-                hi[q] = pack_f16x2(ah, bh);
-                lo[q] = pack_f16x2(al, bl);
-              } else {  // ReLU folded into the conversion (hi, lo share v's sign)
-                hi[q] = pack_f16x2_relu(ah, bh);
-                lo[q] = pack_f16x2_relu(al, bl);
-              }
+              sts128(aa_s + kmaj(r, j, KA), hi[0], hi[1], hi[2], hi[3]);
+              sts128(aa_s + kmaj(r, N + j, KA), lo[0], lo[1], lo[2], lo[3]);
             }
-            sts128(aa_s + kmaj(r, j, KA), hi[0], hi[1], hi[2], hi[3]);
-            sts128(aa_s + kmaj(r, N + j, KA), lo[0], lo[1], lo[2], lo[3]);
           }
           sts128(aa_s + kmaj(r, 2 * N, KA), 0x00003C00u, 0u, 0u, 0u);  // the constant-1 bias column
           sts128(aa_s + kmaj(r, 2 * N + 8, KA), 0u, 0u, 0u, 0u);
