@@ -273,6 +273,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
     __syncthreads();
     const int n_tiles = static_cast<int>(seg_end - seg);
     const long long tile0 = seg - static_cast<long long>(b) * p.tiles_per_image;  // in-image index
+    (void)tile0;
 
     if (warp < 4 * NWG) {
       // ------------------------------------------------------------ warpgroup
@@ -309,6 +310,19 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
         it_c[j] = c;
         it_i[j] = i;
       }
+      // geometry of each item's level (fixed per thread)
+      int it_W[JJ], it_H[JJ];
+      long long it_off[JJ];
+      float it_sy[JJ], it_sx[JJ];
+#pragma unroll
+      for (int j = 0; j < J; ++j) {
+        const LevelGeom lg = p.lv[it_l[j]];
+        it_W[j] = lg.W;
+        it_H[j] = lg.H;
+        it_off[j] = lg.off + static_cast<long long>(it_c[j]) * lg.H * lg.W;
+        it_sy[j] = lg.sy;
+        it_sx[j] = lg.sx;
+      }
       // Relative x-taps of pixel r for each level (used when fast_x): the
       // source coordinate (r + 1/2) / 2^l - 1/2 relative to column x0/2^l - 1.
       int rel[L];
@@ -323,10 +337,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
 
       // Loads of everything tile i needs from global memory: the level-0
       // value of pixel r and the raw texel pairs of this thread's items.
-      auto prefetch = [&](int i, int (&q0)[C], ColPrefetch<JJ>& cp) {
-        const long long t = tile0 + i;
-        const int y = static_cast<int>(t / p.tiles_per_row);
-        const int x0 = static_cast<int>(t - static_cast<long long>(y) * p.tiles_per_row) * kTile;
+      auto prefetch = [&](int y, int x0, int (&q0)[C], ColPrefetch<JJ>& cp) {
         const int xc = min(x0 + r, p.W - 1);
 #pragma unroll
         for (int c = 0; c < C; ++c)
@@ -338,27 +349,39 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
           cp.beta[j] = 0.0f;
           const int l = it_l[j];
           if (l > 0) {
-            const LevelGeom lg = p.lv[l];
-            const Tap ty = bilinear_tap(y, lg.sy, lg.H);
-            const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, lg.sx, lg.W).i0;
-            const int u = min(max(u_start + it_i[j], 0), lg.W - 1);
-            const int32_t* pl = lat + lg.off + static_cast<long long>(it_c[j]) * lg.H * lg.W + u;
-            cp.q0[j] = __ldg(pl + static_cast<long long>(ty.i0) * lg.W);
-            cp.q1[j] = __ldg(pl + static_cast<long long>(ty.i1) * lg.W);
+            const Tap ty = bilinear_tap(y, it_sy[j], it_H[j]);
+            const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, it_sx[j], it_W[j]).i0;
+            const int u = min(max(u_start + it_i[j], 0), it_W[j] - 1);
+            const int32_t* pl = lat + it_off[j] + u;
+            cp.q0[j] = __ldg(pl + ty.i0 * it_W[j]);
+            cp.q1[j] = __ldg(pl + ty.i1 * it_W[j]);
             cp.beta[j] = ty.frac;
           }
         }
       };
 
+      // Tile cursor (row y, tile column tx) of this group's current tile and
+      // of the one after it, advanced by NWG tiles without divisions.
+      const int tpr = p.tiles_per_row;
+      int cy = static_cast<int>((tile0 + w) / tpr);
+      int ctx = static_cast<int>((tile0 + w) - static_cast<long long>(cy) * tpr);
+      auto advance = [&](int& yy, int& xx) {
+        xx += NWG;
+        while (xx >= tpr) {
+          xx -= tpr;
+          ++yy;
+        }
+      };
       int q0c[C];
       ColPrefetch<JJ> cpc;
-      if (w < n_tiles) prefetch(w, q0c, cpc);
+      if (w < n_tiles) prefetch(cy, ctx * kTile, q0c, cpc);
 
       for (int i = w; i < n_tiles; i += NWG) {
         if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
-        const long long t = tile0 + i;
-        const int y = static_cast<int>(t / p.tiles_per_row);
-        const int x0 = static_cast<int>(t - static_cast<long long>(y) * p.tiles_per_row) * kTile;
+        const int y = cy;
+        const int x0 = ctx * kTile;
+        int ny = cy, ntx = ctx;
+        advance(ny, ntx);
         const int x = x0 + r;
         const bool valid = x < p.W;
         const int xc = valid ? x : p.W - 1;
@@ -367,7 +390,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
         int q0n[C];
         ColPrefetch<JJ> cpn;
         const bool has_next = i + NWG < n_tiles;
-        if (has_next) prefetch(i + NWG, q0n, cpn);
+        if (has_next) prefetch(ny, ntx * kTile, q0n, cpn);
 
         // ---- features: vertical pass into the column buffer ----
 #pragma unroll
@@ -501,16 +524,26 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
           for (int c = 0; c < C; ++c) q0c[c] = q0n[c];
           cpc = cpn;
         }
+        cy = ny;
+        ctx = ntx;
       }
     } else if (warp == Net::MMA_WARP && lane == 0) {
       // --------------------------------------------------------------- MMA issuer
       // Serves whichever warpgroup has its next operand ready; per group the
       // order is fixed (its tiles in turn, layers in turn).
-      const uint32_t b1_s = sbase + Net::OFF_B1;
-      const uint32_t bh_s = sbase + Net::OFF_BH;
-      const uint32_t bo_s = sbase + Net::OFF_BO;
+      // Descriptors depend on the start address only through its low field,
+      // so each operand's descriptor is its base descriptor plus (offset >> 4).
       constexpr uint32_t id_hidden = idesc_f16(128, N);
       constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
+      const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG, 128, 16 * K1);
+      const uint64_t dA = smem_desc(sbase + Net::OFF_WG + Net::A1_BYTES, 128, 16 * KA);
+      const uint64_t dB1 = smem_desc(sbase + Net::OFF_B1, 128, 16 * K1);
+      const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * KB);
+      const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * KB);
+      constexpr uint64_t kStep = 256 >> 4;                 // one K-step (16 fp16) = 256 B
+      constexpr uint64_t kWg = Net::WG_BYTES >> 4;         // next warpgroup's buffers
+      constexpr uint64_t kLayer = Net::BH_BYTES >> 4;      // next hidden layer's weights
+      static_assert(Net::WG_BYTES % 16 == 0 && Net::BH_BYTES % 16 == 0, "16-byte aligned operands");
       int tile_of[NWG], layer_of[NWG];
       int remaining = 0;
 #pragma unroll
@@ -530,27 +563,21 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
           tc_fence_after();
           const int k = layer_of[w];
           const uint32_t d = tmem + static_cast<uint32_t>(w * N);
-          const uint32_t a1_s = sbase + Net::OFF_WG + w * Net::WG_BYTES;
-          const uint32_t aa_s = a1_s + Net::A1_BYTES;
           if (k == 0) {
+            const uint64_t da = dA1 + w * kWg;
 #pragma unroll
-            for (int s = 0; s < K1 / 16; ++s)
-              mma_f16(d, smem_desc(a1_s + s * 256, 128, 16 * K1), smem_desc(b1_s + s * 256, 128, 16 * K1),
-                      id_hidden, s > 0);
+            for (int s = 0; s < K1 / 16; ++s) mma_f16(d, da + s * kStep, dB1 + s * kStep, id_hidden, s > 0);
           } else {
             const bool out_layer = (k == NL - 1);
-            const uint32_t bk = out_layer ? bo_s : bh_s + (k - 1) * Net::BH_BYTES;
+            const uint64_t da = dA + w * kWg;
+            const uint64_t db = out_layer ? dBO : dBH + (k - 1) * kLayer;
             const uint32_t id = out_layer ? id_out : id_hidden;
 #pragma unroll
-            for (int s = 0; s < N / 16; ++s)  // hi part
-              mma_f16(d, smem_desc(aa_s + s * 256, 128, 16 * KA), smem_desc(bk + s * 256, 128, 16 * KB), id,
-                      s > 0);
+            for (int s = 0; s < N / 16; ++s) mma_f16(d, da + s * kStep, db + s * kStep, id, s > 0);  // hi
 #pragma unroll
             for (int s = 0; s < N / 16; ++s)  // lo part, same weights
-              mma_f16(d, smem_desc(aa_s + (N / 16 + s) * 256, 128, 16 * KA),
-                      smem_desc(bk + s * 256, 128, 16 * KB), id, 1);
-            mma_f16(d, smem_desc(aa_s + (N / 8) * 256, 128, 16 * KA),  // bias column
-                    smem_desc(bk + (N / 16) * 256, 128, 16 * KB), id, 1);
+              mma_f16(d, da + (N / 16 + s) * kStep, db + s * kStep, id, 1);
+            mma_f16(d, da + (N / 8) * kStep, db + (N / 16) * kStep, id, 1);  // bias column
           }
           mma_commit(bar_c0 + 8 * w);
           if (++layer_of[w] == NL) {
