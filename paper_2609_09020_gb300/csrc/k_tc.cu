@@ -527,10 +527,12 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
         cy = ny;
         ctx = ntx;
       }
-    } else if (warp == Net::MMA_WARP && lane == 0) {
+    } else if (warp == Net::MMA_WARP) {
       // --------------------------------------------------------------- MMA issuer
       // Serves whichever warpgroup has its next operand ready; per group the
-      // order is fixed (its tiles in turn, layers in turn).
+      // order is fixed (its tiles in turn, layers in turn).  The whole warp
+      // runs the control flow (so descriptors stay warp-uniform); one elected
+      // lane issues the MMAs and the commits.
       // Descriptors depend on the start address only through its low field,
       // so each operand's descriptor is its base descriptor plus (offset >> 4).
       constexpr uint32_t id_hidden = idesc_f16(128, N);
@@ -558,11 +560,13 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
 #pragma unroll
         for (int w = 0; w < NWG; ++w) {
           if (tile_of[w] >= n_tiles) continue;
-          if (!mbar_test_wait(bar_a0 + 8 * w, (a_phase >> w) & 1u)) continue;
+          const bool ready = __shfl_sync(0xffffffffu, mbar_test_wait(bar_a0 + 8 * w, (a_phase >> w) & 1u) ? 1 : 0, 0) != 0;
+          if (!ready) continue;
           a_phase ^= (1u << w);
-          tc_fence_after();
           const int k = layer_of[w];
           const uint32_t d = tmem + static_cast<uint32_t>(w * N);
+          if (elect_one()) {
+          tc_fence_after();
           if (k == 0) {
             const uint64_t da = dA1 + w * kWg;
 #pragma unroll
@@ -580,6 +584,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
             mma_f16(d, da + (N / 8) * kStep, db + (N / 16) * kStep, id, 1);  // bias column
           }
           mma_commit(bar_c0 + 8 * w);
+          }
+          __syncwarp();
           if (++layer_of[w] == NL) {
             layer_of[w] = 0;
             tile_of[w] += NWG;
@@ -589,9 +595,11 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
         }
         if (progressed) {
           idle = 0;
-        } else if (++idle > kSpinLimit || *abort_flag) {
-          *abort_flag = 1;
-          atomicOr(p.status, 1);
+        } else if (++idle > kSpinLimit || __shfl_sync(0xffffffffu, *abort_flag, 0) != 0) {
+          if (lane == 0) {
+            *abort_flag = 1;
+            atomicOr(p.status, 1);
+          }
           break;
         } else if (idle > 256) {
           __nanosleep(20);
