@@ -1,8 +1,8 @@
 // k_tc.cu -- fused decode on the 5th-generation tensor cores (PIC_PREC_FP16_TC).
 //
 // The synthesis MLP g_s (Sec. 4.1) runs as a chain of tcgen05 MMAs with the
-// accumulators in tensor memory; dequantisation, bilinear upsampling and
-// concatenation of the pyramid levels (Sec. 3.1, Eq. 1) produce the first
+// accumulators in tensor memory (TMEM); dequantisation, bilinear upsampling
+// and concatenation of the pyramid levels (Sec. 3.1, Eq. 1) produce the first
 // layer's operand directly in shared memory, and the clamped RGB leaves the
 // last accumulator straight for global memory.  Nothing between the latents
 // and the RGB planes touches HBM.
@@ -11,31 +11,30 @@
 // operand a (feature or hidden value, fp32) is split into two fp16 terms
 //   a_hi = a with its low 13 mantissa bits cleared (exact in fp16),
 //   a_lo = fp16(a - a_hi),
-// and each layer computes W a_hi + W a_lo + b with fp32 accumulation, so the
-// products carry ~22 significant bits instead of fp16's 11.  The bias rides
-// along as one more K column: A holds a constant 1, B holds b.
+// and each layer computes W a_hi + W a_lo with fp32 accumulation, so the
+// products carry ~22 significant bits instead of fp16's 11.
 //
-// Operand layout per 128-pixel tile (K-major, canonical no-swizzle layout):
-//   layer 0      A1 = [f_hi | f_lo | 1 | 0..]      K1 = round16(2 D0 + 1)
-//                B1 = [W_0  | W_0  | b | 0..]
-//   hidden k     A  = [h_hi | h_lo | 1 0..0]       KA = 2N + 16
-//                B  = [W_k | b 0..0]               KB = N + 16, read twice (hi, lo)
-//   output       B  = [W_out | b 0..0] (3 rows of 16)
+// Operands of one 128-pixel tile (row r = pixel r = TMEM lane r):
+//   layer 0  A1 = [f_hi | f_lo | 1 | 0..]  smem, K1 = round16(2 D0 + 1); the bias
+//            B1 = [W_0  | W_0  | b_0 | 0..] b_0 rides along as the constant-1 column
+//   hidden   A  = [h_hi | h_lo]            TMEM, N/2 + N/2 columns (2 fp16 per column)
+//            B  = W_k                       smem, used for the hi and the lo half;
+//                                           bias b_k added to the fp32 accumulator
+//   output   B  = W_out padded to 16 rows; bias added in the epilogue
 //
 // CTA organisation (one CTA per SM, persistent over a contiguous tile range):
-//   warps 0 .. 4*NWG-1 : NWG warpgroups; warpgroup w owns every NWG-th tile of
-//                        the range, a TMEM accumulator of N columns and its
-//                        own operand buffers.  Thread r of the group decodes
-//                        pixel r of the tile: features -> A1, then each
-//                        accumulator -> activation -> hi/lo -> next A, and
-//                        finally the clamped RGB store.
-//   warp 4*NWG         : one thread issues all MMAs (tcgen05.mma) in a fixed
-//                        round-robin over (tile round, layer, warpgroup) and
-//                        signals completion with tcgen05.commit.
-// Handshakes are mbarriers: a_full[w] (128 arrivals: operand written) and
-// acc_full[w] (commit: accumulator ready).  Every wait is bounded; on timeout
-// the kernel raises the handle's status word, skips the remaining work and
-// still frees its tensor memory.
+//   warps 0 .. 4*NWG-1 : NWG warpgroups; group w owns every NWG-th tile of the
+//                        range, TMEM columns [2Nw, 2Nw + 2N) (accumulator,
+//                        then operand A) and shared buffers (A1, column
+//                        buffer).  Thread r of the group decodes pixel r.
+//                        The features of the group's next tile are computed
+//                        while the tensor core runs the current tile's
+//                        second layer, and handed over once the current
+//                        accumulator has been read.
+//   warp 4*NWG         : issues every MMA (one elected lane) to whichever
+//                        group has its operand ready, then tcgen05.commit.
+// Handshakes are mbarriers; every wait is bounded (on timeout the kernel
+// raises the handle's status word, skips the rest and still frees TMEM).
 #include <cuda_fp16.h>
 
 #include "pic_common.cuh"
@@ -48,7 +47,7 @@ namespace {
 using namespace tc;
 
 constexpr int kTile = 128;
-constexpr uint32_t kSpinLimit = 1u << 22;   // a few seconds of polling at most per wait
+constexpr uint32_t kSpinLimit = 1u << 22;  // a few seconds of polling at most per wait
 
 __host__ __device__ constexpr int round_up(int v, int m) { return (v + m - 1) / m * m; }
 __host__ __device__ constexpr int pow2_at_least(int v) {
@@ -62,119 +61,6 @@ __host__ __device__ constexpr int pow2_at_least(int v) {
 // (row/8) * SBO + (k/8) * LBO with LBO = 128 B and SBO = 16 K bytes.
 __host__ __device__ constexpr uint32_t kmaj(int row, int k, int K) {
   return static_cast<uint32_t>((row >> 3) * (K * 16) + (k >> 3) * 128 + (row & 7) * 16 + (k & 7) * 2);
-}
-
-__host__ __device__ constexpr int colbuf_floats(int L, int C) {
-  int n = 0;
-  for (int l = 1; l < L; ++l) n += C * ((kTile >> l) + 4);
-  return n;
-}
-
-template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_>
-struct TcNet {
-  static constexpr int C = C_, NL = NL_, D0 = D0_, N = N_, ACT = ACT_, NWG = NWG_;
-  static constexpr int L = D0 / C;
-  static constexpr int K1 = round_up(2 * D0 + 1, 16);
-  static constexpr int KA = 2 * N + 16;
-  static constexpr int KB = N + 16;
-  static constexpr int NOUT = 16;
-  static constexpr int THREADS = NWG * 128 + 32;
-  static constexpr int MMA_WARP = NWG * 4;
-  // Registers per thread that still let one CTA fit an SM: the warps are
-  // spread over the 4 sub-partitions, each with a 16K-register file.
-  static constexpr int WARPS_PER_SMSP = (THREADS / 32 + 3) / 4;
-  static constexpr int MAXREG_RAW = 16384 / (32 * WARPS_PER_SMSP) / 8 * 8;
-  static constexpr int MAXREG = MAXREG_RAW > 255 ? 255 : MAXREG_RAW;
-  static constexpr int CTRL = 256;
-  static constexpr int B1_BYTES = N * K1 * 2;
-  static constexpr int BH_BYTES = N * KB * 2;
-  static constexpr int BO_BYTES = NOUT * KB * 2;
-  static constexpr int OFF_B1 = CTRL;
-  static constexpr int OFF_BH = OFF_B1 + B1_BYTES;
-  static constexpr int OFF_BO = OFF_BH + (NL - 2) * BH_BYTES;
-  static constexpr int OFF_WG = round_up(OFF_BO + BO_BYTES, 128);
-  static constexpr int A1_BYTES = kTile * K1 * 2;
-  static constexpr int A_BYTES = kTile * KA * 2;
-  static constexpr int COL_BYTES = round_up(colbuf_floats(L, C) * 4, 128);
-  static constexpr int WG_BYTES = A1_BYTES + A_BYTES + COL_BYTES;
-  static constexpr int SMEM = OFF_WG + NWG * WG_BYTES;
-  static constexpr int TMEM_COLS = pow2_at_least(NWG * N);
-  static_assert(N % 16 == 0 && N >= 16 && N <= 128, "hidden width must be 16..128, multiple of 16");
-  static_assert(NL >= 2, "the tensor-core path needs at least one hidden layer");
-  static_assert(TMEM_COLS <= 512, "tensor memory holds 512 columns");
-};
-
-// Bounded mbarrier wait.  Returns false (and raises the abort flag and the
-// handle's status word) if the phase does not complete in time, or if
-// another thread has already aborted.
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                             int* status) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 63u) == 63u) {
-      if (*abort_flag) return false;
-      if (i > 4096) __nanosleep(64);
-    }
-  }
-  *abort_flag = 1;
-  atomicOr(status, 1);
-  return false;
-}
-
-__device__ __forceinline__ __half ldh(const __half* p) {
-  return __ushort_as_half(__ldg(reinterpret_cast<const unsigned short*>(p)));
-}
-
-// Fills the weight operands of one image into shared memory (all threads).
-template <class Net>
-__device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
-                                                const int (&dims)[Net::NL + 1]) {
-  constexpr int N = Net::N, D0 = Net::D0, K1 = Net::K1, KB = Net::KB, NL = Net::NL;
-  const __half zero = __float2half_rn(0.0f);
-  // layer 0: [W | W | b | 0]
-  {
-    const int d1 = dims[1];
-    const __half* W0 = w;
-    const __half* b0 = w + d1 * D0;
-    for (int e = threadIdx.x; e < N * K1; e += blockDim.x) {
-      const int n = e / K1, j = e - n * K1;
-      __half v = zero;
-      if (n < d1) {
-        if (j < D0) v = ldh(W0 + n * D0 + j);
-        else if (j < 2 * D0) v = ldh(W0 + n * D0 + (j - D0));
-        else if (j == 2 * D0) v = ldh(b0 + n);
-      }
-      *reinterpret_cast<__half*>(smem + Net::OFF_B1 + kmaj(n, j, K1)) = v;
-    }
-  }
-  // hidden layers and output: [W | b 0..0]
-  const __half* p = w + dims[1] * D0 + dims[1];
-#pragma unroll
-  for (int k = 1; k < NL; ++k) {
-    const int din = dims[k], dout = dims[k + 1];
-    const bool out_layer = (k == NL - 1);
-    const int rows = out_layer ? Net::NOUT : N;
-    uint8_t* base = smem + (out_layer ? Net::OFF_BO : Net::OFF_BH + (k - 1) * Net::BH_BYTES);
-    const __half* Wk = p;
-    const __half* bk = p + dout * din;
-    for (int e = threadIdx.x; e < rows * KB; e += blockDim.x) {
-      const int n = e / KB, j = e - n * KB;
-      __half v = zero;
-      if (n < dout) {
-        if (j < din) v = ldh(Wk + n * din + j);
-        else if (j == N) v = ldh(bk + n);
-      }
-      *reinterpret_cast<__half*>(base + kmaj(n, j, KB)) = v;
-    }
-    p = bk + dout;
-  }
-}
-
-// Splits v into (hi, lo) fp32 parts: hi = v with the low 13 mantissa bits
-// cleared (an fp16 value for |v| in fp16's normal range), lo = v - hi (exact).
-__device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
-  hi = __uint_as_float(__float_as_uint(v) & 0xFFFFE000u);
-  lo = v - hi;
 }
 
 // Cooperative feature staging.  For level l >= 1 a 128-pixel row segment
@@ -198,8 +84,116 @@ struct ColLayout {
   static constexpr int total() { return off(L, 0); }
 };
 
-// Per-thread share of the column items of one tile: the raw texels (loaded
-// one tile ahead) and the vertical weight.
+template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_>
+struct TcNet {
+  static constexpr int C = C_, NL = NL_, D0 = D0_, N = N_, ACT = ACT_, NWG = NWG_;
+  static constexpr int L = D0 / C;
+  static constexpr int K1 = round_up(2 * D0 + 1, 16);
+  static constexpr int NOUT = 16;
+  static constexpr int THREADS = NWG * 128 + 32;
+  static constexpr int MMA_WARP = NWG * 4;
+  // Registers per thread that still let one CTA fit an SM: the warps are
+  // spread over the 4 sub-partitions, each with a 16K-register file.
+  static constexpr int WARPS_PER_SMSP = (THREADS / 32 + 3) / 4;
+  static constexpr int MAXREG_RAW = 16384 / (32 * WARPS_PER_SMSP) / 8 * 8;
+  static constexpr int MAXREG = MAXREG_RAW > 255 ? 255 : MAXREG_RAW;
+  static constexpr int CTRL = 256;
+  static constexpr int B1_BYTES = N * K1 * 2;
+  static constexpr int BH_BYTES = N * N * 2;
+  static constexpr int BO_BYTES = NOUT * N * 2;
+  static constexpr int BIAS_FLOATS = (NL - 2) * N + NOUT;  // hidden biases, then the output bias
+  static constexpr int OFF_B1 = CTRL;
+  static constexpr int OFF_BH = OFF_B1 + B1_BYTES;
+  static constexpr int OFF_BO = OFF_BH + (NL - 2) * BH_BYTES;
+  static constexpr int OFF_BIAS = round_up(OFF_BO + BO_BYTES, 16);
+  static constexpr int OFF_WG = round_up(OFF_BIAS + BIAS_FLOATS * 4, 128);
+  static constexpr int A1_BYTES = kTile * K1 * 2;
+  static constexpr int COL_BYTES = round_up(ColLayout<L, C>::total() * 4, 128);
+  static constexpr int WG_BYTES = A1_BYTES + COL_BYTES;
+  static constexpr int SMEM = OFF_WG + NWG * WG_BYTES;
+  static constexpr int TMEM_COLS = pow2_at_least(NWG * 2 * N);
+  static_assert(N == 16 || (N % 32 == 0 && N <= 128), "hidden width: 16, or a multiple of 32 up to 128");
+  static_assert(NL >= 2, "the tensor-core path needs at least one hidden layer");
+  static_assert(TMEM_COLS <= 512, "tensor memory holds 512 columns");
+  static_assert(8 * (4 * NWG + 1) <= 224, "control block holds the barriers");
+};
+
+// Bounded mbarrier wait.  Returns false (and raises the abort flag and the
+// handle's status word) if the phase does not complete in time, or if
+// another thread has already aborted.
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                             int* status) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 63u) {
+      if (*abort_flag) return false;
+      if (i > 4096) __nanosleep(64);
+    }
+  }
+  *abort_flag = 1;
+  atomicOr(status, 1);
+  return false;
+}
+
+__device__ __forceinline__ __half ldh(const __half* p) {
+  return __ushort_as_half(__ldg(reinterpret_cast<const unsigned short*>(p)));
+}
+
+// Fills the weight operands and biases of one image into shared memory (all threads).
+template <class Net>
+__device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
+                                                const int (&dims)[Net::NL + 1]) {
+  constexpr int N = Net::N, D0 = Net::D0, K1 = Net::K1, NL = Net::NL;
+  const __half zero = __float2half_rn(0.0f);
+  float* bias = reinterpret_cast<float*>(smem + Net::OFF_BIAS);
+  // layer 0: [W | W | b | 0]
+  {
+    const int d1 = dims[1];
+    const __half* W0 = w;
+    const __half* b0 = w + d1 * D0;
+    for (int e = threadIdx.x; e < N * K1; e += blockDim.x) {
+      const int n = e / K1, j = e - n * K1;
+      __half v = zero;
+      if (n < d1) {
+        if (j < D0) v = ldh(W0 + n * D0 + j);
+        else if (j < 2 * D0) v = ldh(W0 + n * D0 + (j - D0));
+        else if (j == 2 * D0) v = ldh(b0 + n);
+      }
+      *reinterpret_cast<__half*>(smem + Net::OFF_B1 + kmaj(n, j, K1)) = v;
+    }
+  }
+  // hidden layers and output: W (zero padded to N or 16 rows and N columns), bias in fp32
+  const __half* p = w + dims[1] * D0 + dims[1];
+#pragma unroll
+  for (int k = 1; k < NL; ++k) {
+    const int din = dims[k], dout = dims[k + 1];
+    const bool out_layer = (k == NL - 1);
+    const int rows = out_layer ? Net::NOUT : N;
+    uint8_t* base = smem + (out_layer ? Net::OFF_BO : Net::OFF_BH + (k - 1) * Net::BH_BYTES);
+    float* bk_s = bias + (k - 1) * N;
+    const __half* Wk = p;
+    const __half* bk = p + dout * din;
+    for (int e = threadIdx.x; e < rows * N; e += blockDim.x) {
+      const int n = e / N, j = e - n * N;
+      __half v = zero;
+      if (n < dout && j < din) v = ldh(Wk + n * din + j);
+      *reinterpret_cast<__half*>(base + kmaj(n, j, N)) = v;
+    }
+    for (int n = threadIdx.x; n < rows; n += blockDim.x)
+      bk_s[n] = n < dout ? __half2float(ldh(bk + n)) : 0.0f;
+    p = bk + dout;
+  }
+}
+
+// Splits v into (hi, lo) fp32 parts: hi = v with the low 13 mantissa bits
+// cleared (an fp16 value for |v| in fp16's normal range), lo = v - hi (exact).
+__device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
+  hi = __uint_as_float(__float_as_uint(v) & 0xFFFFE000u);
+  lo = v - hi;
+}
+
+// Per-thread share of the column items of one tile: the raw texel pairs
+// (loaded ahead of use) and the vertical weight.
 template <int J>
 struct ColPrefetch {
   int q0[J], q1[J];
@@ -207,9 +201,10 @@ struct ColPrefetch {
 };
 
 template <class Net>
-__global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_decode_kernel(const DecodeParams p) {
+__global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
+    tc_decode_kernel(const DecodeParams p) {
   constexpr int N = Net::N, NL = Net::NL, C = Net::C, L = Net::L, D0 = Net::D0, NWG = Net::NWG;
-  constexpr int K1 = Net::K1, KA = Net::KA, KB = Net::KB;
+  constexpr int K1 = Net::K1;
   using CL = ColLayout<L, C>;
   constexpr int NITEM = CL::total();
   constexpr int J = (NITEM + kTile - 1) / kTile;  // column items per thread (0 if L == 1)
@@ -219,21 +214,24 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const uint32_t sbase = smem_addr(smem);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + 128);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + 136);
-  const uint32_t bar_a0 = sbase;               // a_full[w]   at sbase + 8 w
-  const uint32_t bar_c0 = sbase + 8 * NWG;     // acc_full[w] at sbase + 8 (NWG + w)
-  const uint32_t bar_drain = sbase + 16 * NWG; // final MMA completion before freeing TMEM
-  const uint32_t bar_col0 = sbase + 8 * (2 * NWG + 1);  // col_ready[w]: column buffer written
-  static_assert(8 * (3 * NWG + 1) <= 128, "control block holds the barriers");
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + 224);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + 232);
+  // mbarriers, 8 bytes each: per group w a1_full (features written),
+  // a_full (hidden operand written), acc_full (MMAs done), col_ready; one drain.
+  const uint32_t bar_a1 = sbase;
+  const uint32_t bar_a = sbase + 8 * NWG;
+  const uint32_t bar_c = sbase + 16 * NWG;
+  const uint32_t bar_col = sbase + 24 * NWG;
+  const uint32_t bar_drain = sbase + 32 * NWG;
 
   if (threadIdx.x == 0) {
     for (int w = 0; w < NWG; ++w) {
-      mbar_init(bar_a0 + 8 * w, 128);
-      mbar_init(bar_c0 + 8 * w, 1);
+      mbar_init(bar_a1 + 8 * w, 128);
+      mbar_init(bar_a + 8 * w, 128);
+      mbar_init(bar_c + 8 * w, 1);
+      mbar_init(bar_col + 8 * w, 128);
     }
     mbar_init(bar_drain, 1);
-    for (int w = 0; w < NWG; ++w) mbar_init(bar_col0 + 8 * w, 128);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -257,7 +255,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
 
   uint32_t acc_phase = 0;  // warpgroup threads: parity of their acc_full
   uint32_t col_phase = 0;  // warpgroup threads: parity of their col_ready
-  uint32_t a_phase = 0;    // MMA thread: bit w = parity of a_full[w]
+  uint32_t a1_phase = 0;   // MMA warp: bit w = parity of a1_full[w]
+  uint32_t a_phase = 0;    // MMA warp: bit w = parity of a_full[w]
 
   for (long long seg = t_begin; seg < t_end;) {
     const int b = static_cast<int>(seg / p.tiles_per_image);
@@ -273,25 +272,29 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
     __syncthreads();
     const int n_tiles = static_cast<int>(seg_end - seg);
     const long long tile0 = seg - static_cast<long long>(b) * p.tiles_per_image;  // in-image index
-    (void)tile0;
 
     if (warp < 4 * NWG) {
       // ------------------------------------------------------------ warpgroup
       const int w = warp >> 2;
       const int r = ((warp & 3) << 5) | lane;  // tile row = TMEM lane = pixel
       uint8_t* a1 = smem + Net::OFF_WG + w * Net::WG_BYTES;
-      const uint32_t a1_s = smem_addr(a1), aa_s = a1_s + Net::A1_BYTES;
-      float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES + Net::A_BYTES);
-      const uint32_t t_acc = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) +
-                             static_cast<uint32_t>(w * N);
-      const uint32_t bar_a = bar_a0 + 8 * w, bar_c = bar_c0 + 8 * w;
+      const uint32_t a1_s = smem_addr(a1);
+      float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES);
+      const float* bias = reinterpret_cast<const float*>(smem + Net::OFF_BIAS);
+      const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
+      const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(w * 2 * N);
+      const uint32_t t_a = t_acc + N;  // hi in [0, N/2), lo in [N/2, N)
+      const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w,
+                     my_col = bar_col + 8 * w;
       const int32_t* lat = p.latents + b * p.lat_per_image;
       float step[L];
 #pragma unroll
       for (int l = 0; l < L; ++l) step[l] = __ldg(p.steps + b * L + l);
 
-      // This thread's column items: level, channel, column.
-      int it_l[JJ], it_c[JJ], it_i[JJ];
+      // This thread's column items: level, column, and the level's geometry.
+      int it_l[JJ], it_i[JJ], it_W[JJ], it_H[JJ];
+      long long it_off[JJ];
+      float it_sy[JJ], it_sx[JJ];
 #pragma unroll
       for (int j = 0; j < J; ++j) {
         int e = r + kTile * j, l = 0, c = 0, i = 0;
@@ -307,19 +310,11 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
               }
         }
         it_l[j] = l;  // l == 0 marks an idle slot
-        it_c[j] = c;
         it_i[j] = i;
-      }
-      // geometry of each item's level (fixed per thread)
-      int it_W[JJ], it_H[JJ];
-      long long it_off[JJ];
-      float it_sy[JJ], it_sx[JJ];
-#pragma unroll
-      for (int j = 0; j < J; ++j) {
-        const LevelGeom lg = p.lv[it_l[j]];
+        const LevelGeom lg = p.lv[l];
         it_W[j] = lg.W;
         it_H[j] = lg.H;
-        it_off[j] = lg.off + static_cast<long long>(it_c[j]) * lg.H * lg.W;
+        it_off[j] = lg.off + static_cast<long long>(c) * lg.H * lg.W;
         it_sy[j] = lg.sy;
         it_sx[j] = lg.sx;
       }
@@ -335,8 +330,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
         fx[l] = sx - fl;
       }
 
-      // Loads of everything tile i needs from global memory: the level-0
-      // value of pixel r and the raw texel pairs of this thread's items.
+      // Global loads tile (y, x0) needs: the level-0 values of pixel r and
+      // the raw texel pairs of this thread's column items.
       auto prefetch = [&](int y, int x0, int (&q0)[C], ColPrefetch<JJ>& cp) {
         const int xc = min(x0 + r, p.W - 1);
 #pragma unroll
@@ -360,58 +355,28 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
         }
       };
 
-      // Tile cursor (row y, tile column tx) of this group's current tile and
-      // of the one after it, advanced by NWG tiles without divisions.
-      const int tpr = p.tiles_per_row;
-      int cy = static_cast<int>((tile0 + w) / tpr);
-      int ctx = static_cast<int>((tile0 + w) - static_cast<long long>(cy) * tpr);
-      auto advance = [&](int& yy, int& xx) {
-        xx += NWG;
-        while (xx >= tpr) {
-          xx -= tpr;
-          ++yy;
-        }
-      };
-      int q0c[C];
-      ColPrefetch<JJ> cpc;
-      if (w < n_tiles) prefetch(cy, ctx * kTile, q0c, cpc);
-
-      for (int i = w; i < n_tiles; i += NWG) {
-        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
-        const int y = cy;
-        const int x0 = ctx * kTile;
-        int ny = cy, ntx = ctx;
-        advance(ny, ntx);
-        const int x = x0 + r;
-        const bool valid = x < p.W;
-        const int xc = valid ? x : p.W - 1;
-
-        // prefetch the next tile of this warpgroup
-        int q0n[C];
-        ColPrefetch<JJ> cpn;
-        const bool has_next = i + NWG < n_tiles;
-        if (has_next) prefetch(ny, ntx * kTile, q0n, cpn);
-
-        // ---- features: vertical pass into the column buffer ----
+      // Features of tile (y, x0) from its prefetched loads -> A1 (shared).
+      // Returns false if a wait gave up.
+      auto features = [&](int x0, const int (&q0)[C], const ColPrefetch<JJ>& cp) -> bool {
+        // vertical pass into the column buffer
 #pragma unroll
         for (int j = 0; j < J; ++j) {
           const int l = it_l[j];
           if (l > 0) {
-            const float a = static_cast<float>(cpc.q0[j]);
-            const float d = static_cast<float>(cpc.q1[j] - cpc.q0[j]);
-            colbuf[r + kTile * j] = step[l] * fmaf(cpc.beta[j], d, a);
+            const float a = static_cast<float>(cp.q0[j]);
+            const float d = static_cast<float>(cp.q1[j] - cp.q0[j]);
+            colbuf[r + kTile * j] = step[l] * fmaf(cp.beta[j], d, a);
           }
         }
-        // warpgroup-wide: the column buffer is complete (bounded wait)
-        mbar_arrive(bar_col0 + 8 * w);
-        if (!__all_sync(0xffffffffu, wait_bounded(bar_col0 + 8 * w, col_phase, abort_flag, p.status)))
-          break;
+        mbar_arrive(my_col);  // the group's column buffer is complete once all 128 arrived
+        if (!__all_sync(0xffffffffu, wait_bounded(my_col, col_phase, abort_flag, p.status)))
+          return false;
         col_phase ^= 1u;
-
-        // ---- features: horizontal pass, level 0, hi/lo split -> A1 ----
+        // horizontal pass + level 0
+        const int xc = min(x0 + r, p.W - 1);
         float f[D0];
 #pragma unroll
-        for (int c = 0; c < C; ++c) f[c] = step[0] * static_cast<float>(q0c[c]);
+        for (int c = 0; c < C; ++c) f[c] = step[0] * static_cast<float>(q0[c]);
 #pragma unroll
         for (int l = 1; l < L; ++l) {
           int i0, i1;
@@ -435,94 +400,132 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
             f[l * C + c] = fmaf(a, v1 - v0, v0);
           }
         }
-        {
-          float v[K1];
+        // hi/lo split, the constant-1 bias column, padding -> A1
+        float v[K1];
 #pragma unroll
-          for (int j = 0; j < K1; ++j) v[j] = 0.0f;
+        for (int j = 0; j < K1; ++j) v[j] = 0.0f;
 #pragma unroll
-          for (int j = 0; j < D0; ++j) split_hi_lo(f[j], v[j], v[D0 + j]);
-          v[2 * D0] = 1.0f;
+        for (int j = 0; j < D0; ++j) split_hi_lo(f[j], v[j], v[D0 + j]);
+        v[2 * D0] = 1.0f;
 #pragma unroll
-          for (int kc = 0; kc < K1 / 8; ++kc)
-            sts128(a1_s + kmaj(r, kc * 8, K1), pack_f16x2(v[kc * 8 + 0], v[kc * 8 + 1]),
-                   pack_f16x2(v[kc * 8 + 2], v[kc * 8 + 3]), pack_f16x2(v[kc * 8 + 4], v[kc * 8 + 5]),
-                   pack_f16x2(v[kc * 8 + 6], v[kc * 8 + 7]));
-        }
+        for (int kc = 0; kc < K1 / 8; ++kc)
+          sts128(a1_s + kmaj(r, kc * 8, K1), pack_f16x2(v[kc * 8 + 0], v[kc * 8 + 1]),
+                 pack_f16x2(v[kc * 8 + 2], v[kc * 8 + 3]), pack_f16x2(v[kc * 8 + 4], v[kc * 8 + 5]),
+                 pack_f16x2(v[kc * 8 + 6], v[kc * 8 + 7]));
         fence_async_smem();
-        mbar_arrive(bar_a);
+        return true;
+      };
 
-        // ---- hidden layers: accumulator -> act -> hi/lo -> next operand ----
-        bool ok = true;
-#pragma unroll 1
-        for (int k = 0; k < NL - 1; ++k) {
-          if (!__all_sync(0xffffffffu, wait_bounded(bar_c, acc_phase, abort_flag, p.status))) {
+      // Hidden epilogue: accumulator (+ bias) -> activation -> hi/lo -> TMEM operand.
+      auto hidden_epilogue = [&](const float* bk) {
+#pragma unroll
+        for (int h0 = 0; h0 < N; h0 += 32) {  // 32 columns at a time (fewer live registers)
+          constexpr int HW = N < 32 ? N : 32;   // N is a multiple of 32, or 16
+          uint32_t acc[HW];
+#pragma unroll
+          for (int c0 = 0; c0 < HW; c0 += 16) tmem_ld16(t_acc + h0 + c0, acc + c0);
+          tmem_ld_wait();
+          uint32_t hl[HW];  // [0, HW/2): hi pairs, [HW/2, HW): lo pairs
+#pragma unroll
+          for (int q = 0; q < HW / 2; ++q) {
+            float a = __uint_as_float(acc[2 * q]);
+            float bb = __uint_as_float(acc[2 * q + 1]);
+            if (bk != nullptr) {
+              const float2 bv = *reinterpret_cast<const float2*>(bk + h0 + 2 * q);
+              a += bv.x;
+              bb += bv.y;
+            }
+            if constexpr (Net::ACT == ACT_GELU) {
+              a = gelu_erf(a);
+              bb = gelu_erf(bb);
+            }
+            float ah, al, bh, bl;
+            split_hi_lo(a, ah, al);
+            split_hi_lo(bb, bh, bl);
+            if constexpr (Net::ACT == ACT_GELU) {
+              hl[q] = pack_f16x2(ah, bh);
+              hl[HW / 2 + q] = pack_f16x2(al, bl);
+            } else {  // ReLU folded into the conversion (hi, lo share v's sign)
+              hl[q] = pack_f16x2_relu(ah, bh);
+              hl[HW / 2 + q] = pack_f16x2_relu(al, bl);
+            }
+          }
+          // hi pair (h0/2 + q) -> column t_a + h0/2 + q; lo pair -> t_a + N/2 + h0/2 + q
+          if constexpr (HW == 32) {
+            tmem_st16(t_a + h0 / 2, hl);
+            tmem_st16(t_a + N / 2 + h0 / 2, hl + 16);
+          } else {
+            tmem_st8(t_a + h0 / 2, hl);
+            tmem_st8(t_a + N / 2 + h0 / 2, hl + 8);
+          }
+        }
+        tmem_st_wait();
+      };
+
+      // Tile cursor (row y, tile column tx) of this group's current tile and
+      // of the one after it, advanced by NWG tiles without divisions.
+      const int tpr = p.tiles_per_row;
+      int cy = static_cast<int>((tile0 + w) / tpr);
+      int ctx = static_cast<int>((tile0 + w) - static_cast<long long>(cy) * tpr);
+      auto advance = [&](int& yy, int& xx) {
+        xx += NWG;
+        while (xx >= tpr) {
+          xx -= tpr;
+          ++yy;
+        }
+      };
+
+      bool ok = true;
+      if (w < n_tiles) {
+        int q0[C];
+        ColPrefetch<JJ> cp;
+        prefetch(cy, ctx * kTile, q0, cp);
+        ok = features(ctx * kTile, q0, cp);
+        if (ok) mbar_arrive(my_a1);
+      }
+      for (int i = w; i < n_tiles && ok; i += NWG) {
+        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+        const int y = cy;
+        const int x0 = ctx * kTile;
+        int ny = cy, ntx = ctx;
+        advance(ny, ntx);
+        const bool has_next = i + NWG < n_tiles;
+        int q0n[C];
+        ColPrefetch<JJ> cpn;
+        if (has_next) prefetch(ny, ntx * kTile, q0n, cpn);  // in flight during the first epilogue
+
+        for (int k = 0; k < NL - 1 && ok; ++k) {
+          if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
             ok = false;
             break;
           }
           acc_phase ^= 1u;
           tc_fence_after();
-#pragma unroll
-          for (int h0 = 0; h0 < N; h0 += 32) {  // two halves of 32 columns (fewer live registers)
-            const int hw = (N - h0) < 32 ? (N - h0) : 32;  // 16 or 32 (N is a multiple of 16)
-            uint32_t acc[32];
-#pragma unroll
-            for (int c0 = 0; c0 < hw; c0 += 16) tmem_ld16(t_acc + h0 + c0, acc + c0);
-            tmem_ld_wait();
-#pragma unroll
-            for (int jj = 0; jj < hw; jj += 8) {
-              const int j = h0 + jj;
-              uint32_t hi[4], lo[4];
-#pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                float a = __uint_as_float(acc[jj + 2 * q]);
-                float bb = __uint_as_float(acc[jj + 2 * q + 1]);
-                if constexpr (Net::ACT == ACT_GELU) {
-                  a = gelu_erf(a);
-                  bb = gelu_erf(bb);
-                }
-                float ah, al, bh, bl;
-                split_hi_lo(a, ah, al);
-                split_hi_lo(bb, bh, bl);
-                if constexpr (Net::ACT == ACT_GELU) {
-                  hi[q] = pack_f16x2(ah, bh);
-                  lo[q] = pack_f16x2(al, bl);
-                } else {  // ReLU folded into the conversion (hi, lo share v's sign)
-                  hi[q] = pack_f16x2_relu(ah, bh);
-                  lo[q] = pack_f16x2_relu(al, bl);
-                }
-              }
-              sts128(aa_s + kmaj(r, j, KA), hi[0], hi[1], hi[2], hi[3]);
-              sts128(aa_s + kmaj(r, N + j, KA), lo[0], lo[1], lo[2], lo[3]);
-            }
-          }
-          sts128(aa_s + kmaj(r, 2 * N, KA), 0x00003C00u, 0u, 0u, 0u);  // the constant-1 bias column
-          sts128(aa_s + kmaj(r, 2 * N + 8, KA), 0u, 0u, 0u, 0u);
-          fence_async_smem();
+          hidden_epilogue(k == 0 ? nullptr : bias + (k - 1) * N);
           tc_fence_before();
-          mbar_arrive(bar_a);
+          mbar_arrive(my_a);
+          if (k == 0 && has_next) ok = features(ntx * kTile, q0n, cpn);  // overlaps layer 1
         }
         if (!ok) break;
 
-        // ---- output layer: clamp, planar coalesced store ----
-        if (!__all_sync(0xffffffffu, wait_bounded(bar_c, acc_phase, abort_flag, p.status))) break;
+        // ---- output layer: bias, clamp, planar coalesced store ----
+        if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
         acc_phase ^= 1u;
         tc_fence_after();
         uint32_t o[4];
         tmem_ld4(t_acc, o);
         tmem_ld_wait();
         tc_fence_before();
-        if (valid) {
+        if (has_next) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
+        const int x = x0 + r;
+        if (x < p.W) {
+          const float* bo = bias + (NL - 2) * N;
           float* dst = p.out + static_cast<long long>(b) * 3 * plane + static_cast<long long>(y) * p.W + x;
 #pragma unroll
           for (int c = 0; c < 3; ++c) {
-            const float v = __uint_as_float(o[c]);
+            const float v = __uint_as_float(o[c]) + bo[c];
             dst[c * plane] = p.clamp ? __saturatef(v) : v;
           }
-        }
-        if (has_next) {
-#pragma unroll
-          for (int c = 0; c < C; ++c) q0c[c] = q0n[c];
-          cpc = cpn;
         }
         cy = ny;
         ctx = ntx;
@@ -532,19 +535,17 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
       // Serves whichever warpgroup has its next operand ready; per group the
       // order is fixed (its tiles in turn, layers in turn).  The whole warp
       // runs the control flow (so descriptors stay warp-uniform); one elected
-      // lane issues the MMAs and the commits.
-      // Descriptors depend on the start address only through its low field,
-      // so each operand's descriptor is its base descriptor plus (offset >> 4).
+      // lane issues the MMAs and the commits.  Descriptors depend on the
+      // start address only through their low field: base + (offset >> 4).
       constexpr uint32_t id_hidden = idesc_f16(128, N);
       constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
       const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG, 128, 16 * K1);
-      const uint64_t dA = smem_desc(sbase + Net::OFF_WG + Net::A1_BYTES, 128, 16 * KA);
       const uint64_t dB1 = smem_desc(sbase + Net::OFF_B1, 128, 16 * K1);
-      const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * KB);
-      const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * KB);
-      constexpr uint64_t kStep = 256 >> 4;                 // one K-step (16 fp16) = 256 B
-      constexpr uint64_t kWg = Net::WG_BYTES >> 4;         // next warpgroup's buffers
-      constexpr uint64_t kLayer = Net::BH_BYTES >> 4;      // next hidden layer's weights
+      const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * N);
+      const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * N);
+      constexpr uint64_t kStep = 256 >> 4;              // one K-step (16 fp16) = 256 B
+      constexpr uint64_t kWg = Net::WG_BYTES >> 4;      // next warpgroup's A1
+      constexpr uint64_t kLayer = Net::BH_BYTES >> 4;   // next hidden layer's weights
       static_assert(Net::WG_BYTES % 16 == 0 && Net::BH_BYTES % 16 == 0, "16-byte aligned operands");
       int tile_of[NWG], layer_of[NWG];
       int remaining = 0;
@@ -560,30 +561,30 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG) tc_deco
 #pragma unroll
         for (int w = 0; w < NWG; ++w) {
           if (tile_of[w] >= n_tiles) continue;
-          const bool ready = __shfl_sync(0xffffffffu, mbar_test_wait(bar_a0 + 8 * w, (a_phase >> w) & 1u) ? 1 : 0, 0) != 0;
-          if (!ready) continue;
-          a_phase ^= (1u << w);
           const int k = layer_of[w];
-          const uint32_t d = tmem + static_cast<uint32_t>(w * N);
+          const uint32_t bar = (k == 0 ? bar_a1 : bar_a) + 8 * w;
+          const uint32_t par = ((k == 0 ? a1_phase : a_phase) >> w) & 1u;
+          if (__shfl_sync(0xffffffffu, mbar_test_wait(bar, par) ? 1 : 0, 0) == 0) continue;
+          if (k == 0) a1_phase ^= (1u << w);
+          else a_phase ^= (1u << w);
+          const uint32_t d = tmem + static_cast<uint32_t>(w * 2 * N);
           if (elect_one()) {
-          tc_fence_after();
-          if (k == 0) {
-            const uint64_t da = dA1 + w * kWg;
+            tc_fence_after();
+            if (k == 0) {
+              const uint64_t da = dA1 + w * kWg;
 #pragma unroll
-            for (int s = 0; s < K1 / 16; ++s) mma_f16(d, da + s * kStep, dB1 + s * kStep, id_hidden, s > 0);
-          } else {
-            const bool out_layer = (k == NL - 1);
-            const uint64_t da = dA + w * kWg;
-            const uint64_t db = out_layer ? dBO : dBH + (k - 1) * kLayer;
-            const uint32_t id = out_layer ? id_out : id_hidden;
+              for (int s = 0; s < K1 / 16; ++s) mma_f16(d, da + s * kStep, dB1 + s * kStep, id_hidden, s > 0);
+            } else {
+              const bool out_layer = (k == NL - 1);
+              const uint64_t db = out_layer ? dBO : dBH + (k - 1) * kLayer;
+              const uint32_t id = out_layer ? id_out : id_hidden;
+              const uint32_t ta = d + N;
 #pragma unroll
-            for (int s = 0; s < N / 16; ++s) mma_f16(d, da + s * kStep, db + s * kStep, id, s > 0);  // hi
+              for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + 8 * s, db + s * kStep, id, s > 0);  // hi
 #pragma unroll
-            for (int s = 0; s < N / 16; ++s)  // lo part, same weights
-              mma_f16(d, da + (N / 16 + s) * kStep, db + s * kStep, id, 1);
-            mma_f16(d, da + (N / 8) * kStep, db + (N / 16) * kStep, id, 1);  // bias column
-          }
-          mma_commit(bar_c0 + 8 * w);
+              for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
+            }
+            mma_commit(bar_c + 8 * w);
           }
           __syncwarp();
           if (++layer_of[w] == NL) {
@@ -648,7 +649,7 @@ int tc_kernels(KernelInfo* out, int cap) {
   static const int d_c4[] = {16, 64, 64, 64, 3};
   const KernelInfo list[] = {
       make_tc<1, 3, 7, 64, ACT_RELU, 4>("tc05_7x64x64x3_relu", d_c5),
-      make_tc<2, 4, 16, 64, ACT_GELU, 3>("tc05_16x64x64x64x3_gelu", d_c4),
+      make_tc<2, 4, 16, 64, ACT_GELU, 4>("tc05_16x64x64x64x3_gelu", d_c4),
   };
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
   for (int i = 0; i < n && i < cap; ++i) out[i] = list[i];
