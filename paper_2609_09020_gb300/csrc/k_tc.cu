@@ -37,6 +37,8 @@
 // raises the handle's status word, skips the rest and still frees TMEM).
 #include <cuda_fp16.h>
 
+#include <type_traits>
+
 #include "pic_common.cuh"
 #include "pic_kernels.h"
 #include "tc_ptx.cuh"
@@ -90,8 +92,9 @@ struct TcNet {
   static constexpr int L = D0 / C;
   static constexpr int K1 = round_up(2 * D0 + 1, 16);
   static constexpr int NOUT = 16;
-  static constexpr int THREADS = NWG * 128 + 32;
-  static constexpr int MMA_WARP = NWG * 4;
+  static constexpr int NISSUE = 2;                    // MMA-issuing warps
+  static constexpr int THREADS = NWG * 128 + 32 * NISSUE;
+  static constexpr int MMA_WARP = NWG * 4;            // first issuing warp (also owns TMEM)
   // Registers per thread that still let one CTA fit an SM: the warps are
   // spread over the 4 sub-partitions, each with a 16K-register file.
   static constexpr int WARPS_PER_SMSP = (THREADS / 32 + 3) / 4;
@@ -109,13 +112,16 @@ struct TcNet {
   static constexpr int OFF_WG = round_up(OFF_BIAS + BIAS_FLOATS * 4, 128);
   static constexpr int A1_BYTES = kTile * K1 * 2;
   static constexpr int COL_BYTES = round_up(ColLayout<L, C>::total() * 4, 128);
-  static constexpr int WG_BYTES = A1_BYTES + COL_BYTES;
+  static constexpr int NITEM_PER_THREAD = (ColLayout<L, C>::total() + kTile - 1) / kTile;
+  static constexpr int STAGE_SLOTS = C + 2 * NITEM_PER_THREAD;  // raw int32 loads per thread
+  static constexpr int STAGE_BYTES = STAGE_SLOTS * kTile * 4;
+  static constexpr int WG_BYTES = A1_BYTES + COL_BYTES + STAGE_BYTES;
   static constexpr int SMEM = OFF_WG + NWG * WG_BYTES;
   static constexpr int TMEM_COLS = pow2_at_least(NWG * 2 * N);
-  static_assert(N == 16 || (N % 32 == 0 && N <= 128), "hidden width: 16, or a multiple of 32 up to 128");
+  static_assert(N % 16 == 0 && N >= 16 && N <= 128, "hidden width must be 16..128, multiple of 16");
   static_assert(NL >= 2, "the tensor-core path needs at least one hidden layer");
   static_assert(TMEM_COLS <= 512, "tensor memory holds 512 columns");
-  static_assert(8 * (4 * NWG + 1) <= 224, "control block holds the barriers");
+  static_assert(8 * (4 * NWG + NISSUE) <= 224, "control block holds the barriers");
 };
 
 // Bounded mbarrier wait.  Returns false (and raises the abort flag and the
@@ -192,14 +198,6 @@ __device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
   lo = v - hi;
 }
 
-// Per-thread share of the column items of one tile: the raw texel pairs
-// (loaded ahead of use) and the vertical weight.
-template <int J>
-struct ColPrefetch {
-  int q0[J], q1[J];
-  float beta[J];
-};
-
 template <class Net>
 __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
     tc_decode_kernel(const DecodeParams p) {
@@ -222,7 +220,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
   const uint32_t bar_a = sbase + 8 * NWG;
   const uint32_t bar_c = sbase + 16 * NWG;
   const uint32_t bar_col = sbase + 24 * NWG;
-  const uint32_t bar_drain = sbase + 32 * NWG;
+  const uint32_t bar_drain = sbase + 32 * NWG;  // + 8 m for issuing warp m
 
   if (threadIdx.x == 0) {
     for (int w = 0; w < NWG; ++w) {
@@ -231,7 +229,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       mbar_init(bar_c + 8 * w, 1);
       mbar_init(bar_col + 8 * w, 128);
     }
-    mbar_init(bar_drain, 1);
+    for (int m = 0; m < Net::NISSUE; ++m) mbar_init(bar_drain + 8 * m, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -330,42 +328,45 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         fx[l] = sx - fl;
       }
 
-      // Global loads tile (y, x0) needs: the level-0 values of pixel r and
-      // the raw texel pairs of this thread's column items.
-      auto prefetch = [&](int y, int x0, int (&q0)[C], ColPrefetch<JJ>& cp) {
+      // Global loads tile (y, x0) needs -- the level-0 values of pixel r and
+      // the raw texel pairs of this thread's column items -- issued as
+      // asynchronous copies into this thread's column of the staging buffer
+      // (slot s of thread r at stage[s * 128 + r]); nothing waits on them
+      // until the features are computed.
+      const uint32_t stage_s = a1_s + Net::A1_BYTES + Net::COL_BYTES;
+      const int* stage = reinterpret_cast<const int*>(a1 + Net::A1_BYTES + Net::COL_BYTES);
+      auto prefetch = [&](int y, int x0) {
         const int xc = min(x0 + r, p.W - 1);
 #pragma unroll
         for (int c = 0; c < C; ++c)
-          q0[c] = __ldg(lat + c * plane + static_cast<long long>(y) * p.W + xc);
+          cp_async4(stage_s + (c * kTile + r) * 4, lat + c * plane + static_cast<long long>(y) * p.W + xc);
 #pragma unroll
         for (int j = 0; j < J; ++j) {
-          cp.q0[j] = 0;
-          cp.q1[j] = 0;
-          cp.beta[j] = 0.0f;
           const int l = it_l[j];
           if (l > 0) {
             const Tap ty = bilinear_tap(y, it_sy[j], it_H[j]);
             const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, it_sx[j], it_W[j]).i0;
             const int u = min(max(u_start + it_i[j], 0), it_W[j] - 1);
             const int32_t* pl = lat + it_off[j] + u;
-            cp.q0[j] = __ldg(pl + ty.i0 * it_W[j]);
-            cp.q1[j] = __ldg(pl + ty.i1 * it_W[j]);
-            cp.beta[j] = ty.frac;
+            cp_async4(stage_s + ((C + 2 * j) * kTile + r) * 4, pl + ty.i0 * it_W[j]);
+            cp_async4(stage_s + ((C + 2 * j + 1) * kTile + r) * 4, pl + ty.i1 * it_W[j]);
           }
         }
+        cp_async_commit();
       };
 
       // Features of tile (y, x0) from its prefetched loads -> A1 (shared).
       // Returns false if a wait gave up.
-      auto features = [&](int x0, const int (&q0)[C], const ColPrefetch<JJ>& cp) -> bool {
+      auto features = [&](int y, int x0) -> bool {
+        cp_async_wait_all();  // this thread's staged loads have landed
         // vertical pass into the column buffer
 #pragma unroll
         for (int j = 0; j < J; ++j) {
           const int l = it_l[j];
           if (l > 0) {
-            const float a = static_cast<float>(cp.q0[j]);
-            const float d = static_cast<float>(cp.q1[j] - cp.q0[j]);
-            colbuf[r + kTile * j] = step[l] * fmaf(cp.beta[j], d, a);
+            const float beta = bilinear_tap(y, it_sy[j], it_H[j]).frac;
+            const int t0 = stage[(C + 2 * j) * kTile + r], t1 = stage[(C + 2 * j + 1) * kTile + r];
+            colbuf[r + kTile * j] = step[l] * fmaf(beta, static_cast<float>(t1 - t0), static_cast<float>(t0));
           }
         }
         mbar_arrive(my_col);  // the group's column buffer is complete once all 128 arrived
@@ -376,7 +377,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         const int xc = min(x0 + r, p.W - 1);
         float f[D0];
 #pragma unroll
-        for (int c = 0; c < C; ++c) f[c] = step[0] * static_cast<float>(q0[c]);
+        for (int c = 0; c < C; ++c) f[c] = step[0] * static_cast<float>(stage[c * kTile + r]);
 #pragma unroll
         for (int l = 1; l < L; ++l) {
           int i0, i1;
@@ -417,10 +418,10 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       };
 
       // Hidden epilogue: accumulator (+ bias) -> activation -> hi/lo -> TMEM operand.
-      auto hidden_epilogue = [&](const float* bk) {
+      auto hidden_epilogue = [&](auto has_bias, const float* bk) {
 #pragma unroll
-        for (int h0 = 0; h0 < N; h0 += 32) {  // 32 columns at a time (fewer live registers)
-          constexpr int HW = N < 32 ? N : 32;   // N is a multiple of 32, or 16
+        for (int h0 = 0; h0 < N; h0 += 16) {  // 16 columns at a time (fewer live registers)
+          constexpr int HW = 16;
           uint32_t acc[HW];
 #pragma unroll
           for (int c0 = 0; c0 < HW; c0 += 16) tmem_ld16(t_acc + h0 + c0, acc + c0);
@@ -430,7 +431,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           for (int q = 0; q < HW / 2; ++q) {
             float a = __uint_as_float(acc[2 * q]);
             float bb = __uint_as_float(acc[2 * q + 1]);
-            if (bk != nullptr) {
+            if constexpr (decltype(has_bias)::value) {
               const float2 bv = *reinterpret_cast<const float2*>(bk + h0 + 2 * q);
               a += bv.x;
               bb += bv.y;
@@ -451,13 +452,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             }
           }
           // hi pair (h0/2 + q) -> column t_a + h0/2 + q; lo pair -> t_a + N/2 + h0/2 + q
-          if constexpr (HW == 32) {
-            tmem_st16(t_a + h0 / 2, hl);
-            tmem_st16(t_a + N / 2 + h0 / 2, hl + 16);
-          } else {
-            tmem_st8(t_a + h0 / 2, hl);
-            tmem_st8(t_a + N / 2 + h0 / 2, hl + 8);
-          }
+          tmem_st8(t_a + h0 / 2, hl);
+          tmem_st8(t_a + N / 2 + h0 / 2, hl + 8);
         }
         tmem_st_wait();
       };
@@ -477,10 +473,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
 
       bool ok = true;
       if (w < n_tiles) {
-        int q0[C];
-        ColPrefetch<JJ> cp;
-        prefetch(cy, ctx * kTile, q0, cp);
-        ok = features(ctx * kTile, q0, cp);
+        prefetch(cy, ctx * kTile);
+        ok = features(cy, ctx * kTile);
         if (ok) mbar_arrive(my_a1);
       }
       for (int i = w; i < n_tiles && ok; i += NWG) {
@@ -490,9 +484,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         int ny = cy, ntx = ctx;
         advance(ny, ntx);
         const bool has_next = i + NWG < n_tiles;
-        int q0n[C];
-        ColPrefetch<JJ> cpn;
-        if (has_next) prefetch(ny, ntx * kTile, q0n, cpn);  // in flight during the first epilogue
+        if (has_next) prefetch(ny, ntx * kTile);  // in flight during the first epilogue
 
         for (int k = 0; k < NL - 1 && ok; ++k) {
           if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
@@ -501,10 +493,11 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           }
           acc_phase ^= 1u;
           tc_fence_after();
-          hidden_epilogue(k == 0 ? nullptr : bias + (k - 1) * N);
+          if (k == 0) hidden_epilogue(std::false_type{}, bias);  // b_0 came in through A1
+          else hidden_epilogue(std::true_type{}, bias + (k - 1) * N);
           tc_fence_before();
           mbar_arrive(my_a);
-          if (k == 0 && has_next) ok = features(ntx * kTile, q0n, cpn);  // overlaps layer 1
+          if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
         }
         if (!ok) break;
 
@@ -530,7 +523,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         cy = ny;
         ctx = ntx;
       }
-    } else if (warp == Net::MMA_WARP) {
+    } else if (warp >= Net::MMA_WARP && warp < Net::MMA_WARP + Net::NISSUE) {
+      const int m = warp - Net::MMA_WARP;  // this warp issues for groups w = m, m + NISSUE, ...
       // --------------------------------------------------------------- MMA issuer
       // Serves whichever warpgroup has its next operand ready; per group the
       // order is fixed (its tiles in turn, layers in turn).  The whole warp
@@ -551,9 +545,9 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       int remaining = 0;
 #pragma unroll
       for (int w = 0; w < NWG; ++w) {
-        tile_of[w] = w;
+        tile_of[w] = (w % Net::NISSUE == m) ? w : n_tiles;  // other warp's groups: done
         layer_of[w] = 0;
-        if (w < n_tiles) remaining += ((n_tiles - 1 - w) / NWG + 1) * NL;
+        if (tile_of[w] < n_tiles) remaining += ((n_tiles - 1 - w) / NWG + 1) * NL;
       }
       uint32_t idle = 0;
       while (remaining > 0) {
@@ -611,11 +605,12 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
     seg = seg_end;
   }
 
-  if (warp == Net::MMA_WARP && lane == 0) {
+  if (warp >= Net::MMA_WARP && warp < Net::MMA_WARP + Net::NISSUE && elect_one()) {
     // Every MMA this thread issued must be complete before the memory goes.
-    mma_commit(bar_drain);
+    const uint32_t drain = bar_drain + 8 * (warp - Net::MMA_WARP);
+    mma_commit(drain);
     int dummy = 0;
-    wait_bounded(bar_drain, 0, reinterpret_cast<volatile int*>(&dummy), p.status);
+    wait_bounded(drain, 0, reinterpret_cast<volatile int*>(&dummy), p.status);
   }
   tc_fence_before();
   __syncthreads();
