@@ -18,9 +18,9 @@
 //   layer 0  A1 = [f_hi | f_lo | 1 | 0..]  smem, K1 = round16(2 D0 + 1); the bias
 //            B1 = [W_0  | W_0  | b_0 | 0..] b_0 rides along as the constant-1 column
 //   hidden   A  = [h_hi | h_lo]            TMEM, N/2 + N/2 columns (2 fp16 per column)
-//            B  = W_k                       smem, used for the hi and the lo half;
-//                                           bias b_k added to the fp32 accumulator
-//   output   B  = W_out padded to 16 rows; bias added in the epilogue
+//            B  = [W_k | b_k 0..0]          smem; W_k serves the hi and the lo half,
+//                                           b_k meets a shared constant tile [1 0..0]
+//   output   the same with W_out, b_out padded to 16 rows
 //
 // CTA organisation (one CTA per SM, persistent over a contiguous tile range):
 //   warps 0 .. 4*NWG-1 : NWG warpgroups; group w owns every NWG-th tile of the
@@ -102,14 +102,15 @@ struct TcNet {
   static constexpr int MAXREG = MAXREG_RAW > 255 ? 255 : MAXREG_RAW;
   static constexpr int CTRL = 256;
   static constexpr int B1_BYTES = N * K1 * 2;
-  static constexpr int BH_BYTES = N * N * 2;
-  static constexpr int BO_BYTES = NOUT * N * 2;
-  static constexpr int BIAS_FLOATS = (NL - 2) * N + NOUT;  // hidden biases, then the output bias
+  static constexpr int KB = N + 16;                      // [W | b 0..0]
+  static constexpr int BH_BYTES = N * KB * 2;
+  static constexpr int BO_BYTES = NOUT * KB * 2;
+  static constexpr int ONES_BYTES = kTile * 16 * 2;      // constant A tile [1 0..0] per row
   static constexpr int OFF_B1 = CTRL;
   static constexpr int OFF_BH = OFF_B1 + B1_BYTES;
   static constexpr int OFF_BO = OFF_BH + (NL - 2) * BH_BYTES;
-  static constexpr int OFF_BIAS = round_up(OFF_BO + BO_BYTES, 16);
-  static constexpr int OFF_WG = round_up(OFF_BIAS + BIAS_FLOATS * 4, 128);
+  static constexpr int OFF_ONES = round_up(OFF_BO + BO_BYTES, 128);
+  static constexpr int OFF_WG = round_up(OFF_ONES + ONES_BYTES, 128);
   static constexpr int A1_BYTES = kTile * K1 * 2;
   static constexpr int COL_BYTES = round_up(ColLayout<L, C>::total() * 4, 128);
   static constexpr int NITEM_PER_THREAD = (ColLayout<L, C>::total() + kTile - 1) / kTile;
@@ -149,9 +150,8 @@ __device__ __forceinline__ __half ldh(const __half* p) {
 template <class Net>
 __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
                                                 const int (&dims)[Net::NL + 1]) {
-  constexpr int N = Net::N, D0 = Net::D0, K1 = Net::K1, NL = Net::NL;
+  constexpr int N = Net::N, D0 = Net::D0, K1 = Net::K1, NL = Net::NL, KB = Net::KB;
   const __half zero = __float2half_rn(0.0f);
-  float* bias = reinterpret_cast<float*>(smem + Net::OFF_BIAS);
   // layer 0: [W | W | b | 0]
   {
     const int d1 = dims[1];
@@ -168,7 +168,7 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
       *reinterpret_cast<__half*>(smem + Net::OFF_B1 + kmaj(n, j, K1)) = v;
     }
   }
-  // hidden layers and output: W (zero padded to N or 16 rows and N columns), bias in fp32
+  // hidden layers and output: [W | b 0..0], zero padded to N (or 16) rows
   const __half* p = w + dims[1] * D0 + dims[1];
 #pragma unroll
   for (int k = 1; k < NL; ++k) {
@@ -176,17 +176,17 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
     const bool out_layer = (k == NL - 1);
     const int rows = out_layer ? Net::NOUT : N;
     uint8_t* base = smem + (out_layer ? Net::OFF_BO : Net::OFF_BH + (k - 1) * Net::BH_BYTES);
-    float* bk_s = bias + (k - 1) * N;
     const __half* Wk = p;
     const __half* bk = p + dout * din;
-    for (int e = threadIdx.x; e < rows * N; e += blockDim.x) {
-      const int n = e / N, j = e - n * N;
+    for (int e = threadIdx.x; e < rows * KB; e += blockDim.x) {
+      const int n = e / KB, j = e - n * KB;
       __half v = zero;
-      if (n < dout && j < din) v = ldh(Wk + n * din + j);
-      *reinterpret_cast<__half*>(base + kmaj(n, j, N)) = v;
+      if (n < dout) {
+        if (j < din) v = ldh(Wk + n * din + j);
+        else if (j == N) v = ldh(bk + n);
+      }
+      *reinterpret_cast<__half*>(base + kmaj(n, j, KB)) = v;
     }
-    for (int n = threadIdx.x; n < rows; n += blockDim.x)
-      bk_s[n] = n < dout ? __half2float(ldh(bk + n)) : 0.0f;
     p = bk + dout;
   }
 }
@@ -237,6 +237,11 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
     tmem_alloc(smem_addr(tmem_slot), Net::TMEM_COLS);
     tmem_relinquish();
   }
+  for (int e = threadIdx.x; e < kTile * 2; e += blockDim.x) {  // 16-byte chunks of the ones tile
+    const int row = e >> 1, kc = e & 1;
+    sts128(sbase + Net::OFF_ONES + kmaj(row, kc * 8, 16), kc == 0 ? 0x00003C00u : 0u, 0u, 0u, 0u);
+  }
+  fence_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -278,7 +283,6 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       uint8_t* a1 = smem + Net::OFF_WG + w * Net::WG_BYTES;
       const uint32_t a1_s = smem_addr(a1);
       float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES);
-      const float* bias = reinterpret_cast<const float*>(smem + Net::OFF_BIAS);
       const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
       const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(w * 2 * N);
       const uint32_t t_a = t_acc + N;  // hi in [0, N/2), lo in [N/2, N)
@@ -417,8 +421,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         return true;
       };
 
-      // Hidden epilogue: accumulator (+ bias) -> activation -> hi/lo -> TMEM operand.
-      auto hidden_epilogue = [&](auto has_bias, const float* bk) {
+      // Hidden epilogue: accumulator -> activation -> hi/lo -> TMEM operand.
+      auto hidden_epilogue = [&]() {
 #pragma unroll
         for (int h0 = 0; h0 < N; h0 += 16) {  // 16 columns at a time (fewer live registers)
           constexpr int HW = 16;
@@ -431,18 +435,15 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           for (int q = 0; q < HW / 2; ++q) {
             float a = __uint_as_float(acc[2 * q]);
             float bb = __uint_as_float(acc[2 * q + 1]);
-            if constexpr (decltype(has_bias)::value) {
-              const float2 bv = *reinterpret_cast<const float2*>(bk + h0 + 2 * q);
-              a += bv.x;
-              bb += bv.y;
-            }
             if constexpr (Net::ACT == ACT_GELU) {
               a = gelu_erf(a);
               bb = gelu_erf(bb);
             }
-            float ah, al, bh, bl;
-            split_hi_lo(a, ah, al);
-            split_hi_lo(bb, bh, bl);
+            // hi = v with 13 low mantissa bits cleared, lo = v - hi (one packed subtraction)
+            const float ah = __uint_as_float(__float_as_uint(a) & 0xFFFFE000u);
+            const float bh = __uint_as_float(__float_as_uint(bb) & 0xFFFFE000u);
+            const float2 l2 = unpack2(sub2(pack2(a, bb), pack2(ah, bh)));
+            const float al = l2.x, bl = l2.y;
             if constexpr (Net::ACT == ACT_GELU) {
               hl[q] = pack_f16x2(ah, bh);
               hl[HW / 2 + q] = pack_f16x2(al, bl);
@@ -493,8 +494,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           }
           acc_phase ^= 1u;
           tc_fence_after();
-          if (k == 0) hidden_epilogue(std::false_type{}, bias);  // b_0 came in through A1
-          else hidden_epilogue(std::true_type{}, bias + (k - 1) * N);
+          hidden_epilogue();
           tc_fence_before();
           mbar_arrive(my_a);
           if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
@@ -512,11 +512,10 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         if (has_next) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
         const int x = x0 + r;
         if (x < p.W) {
-          const float* bo = bias + (NL - 2) * N;
           float* dst = p.out + static_cast<long long>(b) * 3 * plane + static_cast<long long>(y) * p.W + x;
 #pragma unroll
           for (int c = 0; c < 3; ++c) {
-            const float v = __uint_as_float(o[c]) + bo[c];
+            const float v = __uint_as_float(o[c]);
             dst[c * plane] = p.clamp ? __saturatef(v) : v;
           }
         }
@@ -535,8 +534,9 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
       const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG, 128, 16 * K1);
       const uint64_t dB1 = smem_desc(sbase + Net::OFF_B1, 128, 16 * K1);
-      const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * N);
-      const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * N);
+      const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * Net::KB);
+      const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * Net::KB);
+      const uint64_t dONES = smem_desc(sbase + Net::OFF_ONES, 128, 16 * 16);
       constexpr uint64_t kStep = 256 >> 4;              // one K-step (16 fp16) = 256 B
       constexpr uint64_t kWg = Net::WG_BYTES >> 4;      // next warpgroup's A1
       constexpr uint64_t kLayer = Net::BH_BYTES >> 4;   // next hidden layer's weights
@@ -577,6 +577,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
               for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + 8 * s, db + s * kStep, id, s > 0);  // hi
 #pragma unroll
               for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
+              mma_f16(d, dONES, db + (N / 16) * kStep, id, 1);  // bias: [1 0..0] x [b 0..0]
             }
             mma_commit(bar_c + 8 * w);
           }

@@ -77,6 +77,13 @@ __device__ __forceinline__ unsigned long long fma2(unsigned long long a, unsigne
   return d;
 }
 
+// d = a - b on both halves.
+__device__ __forceinline__ unsigned long long sub2(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 // Bilinear source coordinate of output index x along one axis: the pixel
 // centre x + 1/2 maps to (x + 1/2) * ratio - 1/2, clamped below at 0; i0 is
 // its floor, i1 the next index clamped to n - 1, and frac the weight of i1.
