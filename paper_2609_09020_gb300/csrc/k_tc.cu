@@ -9,8 +9,9 @@
 //
 // Precision: weights are fp16 (used exactly as given).  Every activation
 // operand a (feature or hidden value, fp32) is split into two fp16 terms
-//   a_hi = a with its low 13 mantissa bits cleared (exact in fp16),
-//   a_lo = fp16(a - a_hi),
+//   a_hi = a rounded toward zero to fp16,
+//   a_lo = fp16(a - a_hi)      (a - a_hi is exact in fp32 and has a's sign,
+//                               so ReLU may be applied to each term alone),
 // and each layer computes W a_hi + W a_lo with fp32 accumulation, so the
 // products carry ~22 significant bits instead of fp16's 11.
 //
@@ -92,7 +93,7 @@ struct TcNet {
   static constexpr int L = D0 / C;
   static constexpr int K1 = round_up(2 * D0 + 1, 16);
   static constexpr int NOUT = 16;
-  static constexpr int NISSUE = 2;                    // MMA-issuing warps
+  static constexpr int NISSUE = NWG;                  // one MMA-issuing warp per group
   static constexpr int THREADS = NWG * 128 + 32 * NISSUE;
   static constexpr int MMA_WARP = NWG * 4;            // first issuing warp (also owns TMEM)
   // Registers per thread that still let one CTA fit an SM: the warps are
@@ -191,10 +192,10 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
   }
 }
 
-// Splits v into (hi, lo) fp32 parts: hi = v with the low 13 mantissa bits
-// cleared (an fp16 value for |v| in fp16's normal range), lo = v - hi (exact).
+// Splits v into (hi, lo) fp32 parts: hi = v rounded toward zero to fp16
+// (exactly representable), lo = v - hi (exact in fp32).
 __device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
-  hi = __uint_as_float(__float_as_uint(v) & 0xFFFFE000u);
+  hi = __half2float(__float2half_rz(v));
   lo = v - hi;
 }
 
@@ -439,18 +440,12 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
               a = gelu_erf(a);
               bb = gelu_erf(bb);
             }
-            // hi = v with 13 low mantissa bits cleared, lo = v - hi (one packed subtraction)
-            const float ah = __uint_as_float(__float_as_uint(a) & 0xFFFFE000u);
-            const float bh = __uint_as_float(__float_as_uint(bb) & 0xFFFFE000u);
-            const float2 l2 = unpack2(sub2(pack2(a, bb), pack2(ah, bh)));
-            const float al = l2.x, bl = l2.y;
-            if constexpr (Net::ACT == ACT_GELU) {
-              hl[q] = pack_f16x2(ah, bh);
-              hl[HW / 2 + q] = pack_f16x2(al, bl);
-            } else {  // ReLU folded into the conversion (hi, lo share v's sign)
-              hl[q] = pack_f16x2_relu(ah, bh);
-              hl[HW / 2 + q] = pack_f16x2_relu(al, bl);
-            }
+            // hi = fp16 truncation (ReLU folded in), lo = v - hi (packed subtraction)
+            const uint32_t h2 = (Net::ACT == ACT_GELU) ? pack_f16x2_rz(a, bb) : pack_f16x2_rz_relu(a, bb);
+            const float2 hf = unpack_f16x2(h2);
+            const float2 l2 = unpack2(sub2(pack2(a, bb), pack2(hf.x, hf.y)));
+            hl[q] = h2;
+            hl[HW / 2 + q] = (Net::ACT == ACT_GELU) ? pack_f16x2(l2.x, l2.y) : pack_f16x2_relu(l2.x, l2.y);
           }
           // hi pair (h0/2 + q) -> column t_a + h0/2 + q; lo pair -> t_a + N/2 + h0/2 + q
           tmem_st8(t_a + h0 / 2, hl);
@@ -523,82 +518,56 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         ctx = ntx;
       }
     } else if (warp >= Net::MMA_WARP && warp < Net::MMA_WARP + Net::NISSUE) {
-      const int m = warp - Net::MMA_WARP;  // this warp issues for groups w = m, m + NISSUE, ...
       // --------------------------------------------------------------- MMA issuer
-      // Serves whichever warpgroup has its next operand ready; per group the
-      // order is fixed (its tiles in turn, layers in turn).  The whole warp
-      // runs the control flow (so descriptors stay warp-uniform); one elected
-      // lane issues the MMAs and the commits.  Descriptors depend on the
-      // start address only through their low field: base + (offset >> 4).
+      // Warp MMA_WARP + w issues every MMA of group w, in the group's order
+      // (its tiles in turn, layers in turn), sleeping in the mbarrier wait
+      // in between.  The whole warp runs the control flow (descriptors stay
+      // warp-uniform); one elected lane issues the MMAs and the commit.
+      // Descriptors depend on the start address only through their low
+      // field: base + (offset >> 4).
+      const int w = warp - Net::MMA_WARP;
       constexpr uint32_t id_hidden = idesc_f16(128, N);
       constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
-      const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG, 128, 16 * K1);
+      const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG + w * Net::WG_BYTES, 128, 16 * K1);
       const uint64_t dB1 = smem_desc(sbase + Net::OFF_B1, 128, 16 * K1);
       const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * Net::KB);
       const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * Net::KB);
       const uint64_t dONES = smem_desc(sbase + Net::OFF_ONES, 128, 16 * 16);
       constexpr uint64_t kStep = 256 >> 4;              // one K-step (16 fp16) = 256 B
-      constexpr uint64_t kWg = Net::WG_BYTES >> 4;      // next warpgroup's A1
       constexpr uint64_t kLayer = Net::BH_BYTES >> 4;   // next hidden layer's weights
       static_assert(Net::WG_BYTES % 16 == 0 && Net::BH_BYTES % 16 == 0, "16-byte aligned operands");
-      int tile_of[NWG], layer_of[NWG];
-      int remaining = 0;
-#pragma unroll
-      for (int w = 0; w < NWG; ++w) {
-        tile_of[w] = (w % Net::NISSUE == m) ? w : n_tiles;  // other warp's groups: done
-        layer_of[w] = 0;
-        if (tile_of[w] < n_tiles) remaining += ((n_tiles - 1 - w) / NWG + 1) * NL;
-      }
-      uint32_t idle = 0;
-      while (remaining > 0) {
-        bool progressed = false;
-#pragma unroll
-        for (int w = 0; w < NWG; ++w) {
-          if (tile_of[w] >= n_tiles) continue;
-          const int k = layer_of[w];
-          const uint32_t bar = (k == 0 ? bar_a1 : bar_a) + 8 * w;
-          const uint32_t par = ((k == 0 ? a1_phase : a_phase) >> w) & 1u;
-          if (__shfl_sync(0xffffffffu, mbar_test_wait(bar, par) ? 1 : 0, 0) == 0) continue;
-          if (k == 0) a1_phase ^= (1u << w);
-          else a_phase ^= (1u << w);
-          const uint32_t d = tmem + static_cast<uint32_t>(w * 2 * N);
+      const uint32_t d = tmem + static_cast<uint32_t>(w * 2 * N);
+      const uint32_t ta = d + N;
+      const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w;
+      bool ok = true;
+      for (int i = w; i < n_tiles && ok; i += NWG) {
+        for (int k = 0; k < NL; ++k) {
+          const uint32_t bar = k == 0 ? my_a1 : my_a;
+          const uint32_t par = k == 0 ? (a1_phase & 1u) : (a_phase & 1u);
+          if (!__all_sync(0xffffffffu, wait_bounded(bar, par, abort_flag, p.status))) {
+            ok = false;
+            break;
+          }
+          if (k == 0) a1_phase ^= 1u;
+          else a_phase ^= 1u;
           if (elect_one()) {
             tc_fence_after();
             if (k == 0) {
-              const uint64_t da = dA1 + w * kWg;
 #pragma unroll
-              for (int s = 0; s < K1 / 16; ++s) mma_f16(d, da + s * kStep, dB1 + s * kStep, id_hidden, s > 0);
+              for (int s = 0; s < K1 / 16; ++s) mma_f16(d, dA1 + s * kStep, dB1 + s * kStep, id_hidden, s > 0);
             } else {
               const bool out_layer = (k == NL - 1);
               const uint64_t db = out_layer ? dBO : dBH + (k - 1) * kLayer;
               const uint32_t id = out_layer ? id_out : id_hidden;
-              const uint32_t ta = d + N;
 #pragma unroll
               for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + 8 * s, db + s * kStep, id, s > 0);  // hi
 #pragma unroll
               for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
               mma_f16(d, dONES, db + (N / 16) * kStep, id, 1);  // bias: [1 0..0] x [b 0..0]
             }
-            mma_commit(bar_c + 8 * w);
+            mma_commit(my_c);
           }
           __syncwarp();
-          if (++layer_of[w] == NL) {
-            layer_of[w] = 0;
-            tile_of[w] += NWG;
-          }
-          --remaining;
-          progressed = true;
-        }
-        if (progressed) {
-          idle = 0;
-        } else if (++idle > kSpinLimit || __shfl_sync(0xffffffffu, *abort_flag, 0) != 0) {
-          if (lane == 0) {
-            *abort_flag = 1;
-            atomicOr(p.status, 1);
-          }
-          break;
-        } else if (idle > 256) {
-          __nanosleep(20);
         }
       }
     }

@@ -195,6 +195,22 @@ __device__ __forceinline__ uint32_t pack_f16x2(float lo_elem, float hi_elem) {
   return d;
 }
 
+// Truncating (round-toward-zero) pack of (lo_elem, hi_elem), optionally with ReLU.
+__device__ __forceinline__ uint32_t pack_f16x2_rz_relu(float lo_elem, float hi_elem) {
+  uint32_t d;
+  asm("cvt.rz.relu.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi_elem), "f"(lo_elem));
+  return d;
+}
+__device__ __forceinline__ uint32_t pack_f16x2_rz(float lo_elem, float hi_elem) {
+  uint32_t d;
+  asm("cvt.rz.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi_elem), "f"(lo_elem));
+  return d;
+}
+// Widens both halves of an f16x2 to fp32.
+__device__ __forceinline__ float2 unpack_f16x2(uint32_t v) {
+  return __half22float2(*reinterpret_cast<const __half2*>(&v));
+}
+
 __device__ __forceinline__ void sts128(uint32_t saddr, uint32_t a, uint32_t b, uint32_t c,
                                        uint32_t d) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(saddr), "r"(a), "r"(b), "r"(c),
