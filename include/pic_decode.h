@@ -140,6 +140,29 @@ int pic_decode_batch_host(pic_decoder *h, int B, const int32_t *latents, const f
  */
 int pic_decode_check(pic_decoder *h, void *stream);
 
+/*
+ * Allocation-free decode (no counterpart in the paper; an interface for
+ * callers that may not allocate device memory: code inside a CUDA-graph
+ * stream capture, real-time or serving loops whose memory is fixed up front,
+ * embedders that forbid the library from touching the allocator).
+ * Same decode, layouts and argument rules as pic_decode_batch, with the
+ * architecture passed directly instead of a handle (arch->max_H, max_W and
+ * max_batch bound H, W and B as for a handle).  It allocates nothing: the
+ * only global memory it uses besides the caller's buffers is a 256-byte
+ * static device array built into the library (one status word of it per
+ * call; calls needing more are refused), held by every GPU that loads the
+ * library until the process exits.  The first call on a device looks up
+ * that array's device address (make it before any stream capture); each
+ * call clears the status word on `stream` first.  All calls share the
+ * array, so calls that overlap on the GPU (different streams, no ordering)
+ * race on it; a bounded wait that gives up in such a call is not reported.
+ * Errors: as pic_decode_batch (PIC_ERR_INVALID_ARG, PIC_ERR_UNSUPPORTED,
+ * PIC_ERR_CUDA); nothing is launched on an argument error.
+ */
+int pic_decode_batch_noalloc(const pic_arch *arch, int B, const int32_t *latents,
+                             const float *steps, const void *weights, int H, int W,
+                             float *out_rgb, void *stream);
+
 /* Frees the handle and its device state.  NULL is a no-op.  Synchronises the
  * device first, so that no kernel of this handle is still running. */
 void pic_decode_destroy(pic_decoder *h);

@@ -330,3 +330,143 @@ void pic_decode_destroy(pic_decoder* h) {
 const char* pic_decode_kernel_name(const pic_decoder* h) { return h ? h->kern.name : ""; }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free entry point.
+//
+// Some callers cannot allocate device memory at all: code running while a
+// stream is being captured into a CUDA graph (cudaMalloc is not capturable),
+// real-time or serving loops whose memory is fixed up front by a pool the
+// library must not bypass, and embedders that forbid the library from
+// touching the device allocator.  pic_decode_create() allocates (the
+// handle's status word), so those callers use pic_decode_batch_noalloc()
+// instead.  It runs the same kernels; the only global memory it needs beyond
+// the caller's inputs and outputs -- the status word that a bounded wait in
+// the tensor-core kernel raises when it gives up -- lives in the static
+// device array below, which every GPU that loads this library holds until
+// the process exits.
+namespace {
+
+constexpr int kStaticScratchInts = 64;  // 256 bytes; one call needs 1 word
+constexpr int kMaxStaticDevices = 64;
+
+struct StaticScratchSlot {
+  int ready;  // 0: not set up, 1: ok, -1: cudaGetSymbolAddress failed
+  int* ptr;   // device address of g_static_scratch on that device
+};
+StaticScratchSlot g_static_slots[kMaxStaticDevices];
+
+}  // namespace
+
+static __device__ __align__(256) int g_static_scratch[kStaticScratchInts];
+
+namespace {
+
+// Device address of the static scratch on `dev` (which is current).  The
+// array's name is only a host-side stand-in, so the address is looked up
+// once per device and cached.  Not thread-safe on the very first call per
+// device (two threads may both look it up; both get the same address).
+int static_scratch(int dev, int** out) {
+  if (dev < 0 || dev >= kMaxStaticDevices) return PIC_ERR_UNSUPPORTED;
+  StaticScratchSlot& s = g_static_slots[dev];
+  if (s.ready == 0) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr) {
+      cudaGetLastError();
+      s.ready = -1;
+    } else {
+      s.ptr = static_cast<int*>(p);
+      s.ready = 1;
+    }
+  }
+  if (s.ready != 1) return PIC_ERR_CUDA;
+  *out = s.ptr;
+  return PIC_OK;
+}
+
+}  // namespace
+
+extern "C" int pic_decode_batch_noalloc(const pic_arch* arch, int B, const int32_t* latents,
+                                        const float* steps, const void* weights, int H, int W,
+                                        float* out_rgb, void* stream) {
+  if (!arch) return PIC_ERR_INVALID_ARG;
+  if (arch->num_layers < 1 || arch->num_layers > pic::kMaxLayers) return PIC_ERR_INVALID_ARG;
+  if (arch->dims[0] != arch->num_levels * arch->channels_per_level ||
+      arch->dims[arch->num_layers] != 3)
+    return PIC_ERR_INVALID_ARG;
+  if (!arch_valid(arch)) return PIC_ERR_UNSUPPORTED;
+  // Scratch needed by one call: the status word.  Anything that would need
+  // more than the static array holds is refused.
+  constexpr int kNeededInts = 1;
+  static_assert(kNeededInts <= kStaticScratchInts, "static scratch too small");
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_UNSUPPORTED;
+  }
+  int major = 0, minor = 0, sms = 0, smem_optin = 0;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  if (major != 10 || minor != 3) return PIC_ERR_UNSUPPORTED;
+
+  // The same kernel selection as pic_decode_create, on a handle that lives
+  // on this stack frame.
+  KernelInfo table[32];
+  int n = arch->precision == PIC_PREC_FP32 ? pic::fp32_kernels(table, 32) : pic::tc_kernels(table, 32);
+  const KernelInfo* chosen = nullptr;
+  for (int i = 0; i < n && i < 32; ++i)
+    if (kernel_matches(table[i], arch)) {
+      chosen = &table[i];
+      break;
+    }
+  pic_decoder h{};
+  h.arch = *arch;
+  h.device = dev;
+  h.sm_count = sms;
+  if (chosen) {
+    h.kern = *chosen;
+  } else if (arch->precision == PIC_PREC_FP32) {
+    h.kern = pic::fp32_generic_kernel_info();
+    h.kern.smem_bytes = static_cast<int>(pic_param_count(arch) * 4);
+  } else {
+    return PIC_ERR_UNSUPPORTED;
+  }
+  if (h.kern.smem_bytes > smem_optin) return PIC_ERR_UNSUPPORTED;
+  if (cudaFuncSetAttribute(h.kern.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           h.kern.smem_bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, h.kern.fn, h.kern.threads,
+                                                    h.kern.smem_bytes) != cudaSuccess ||
+      per_sm < 1) {
+    cudaGetLastError();
+    return PIC_ERR_UNSUPPORTED;
+  }
+  h.grid_cap = per_sm * sms;
+  h.n_params = pic_param_count(arch);
+
+  int* scratch = nullptr;
+  int rc = static_scratch(dev, &scratch);
+  if (rc != PIC_OK) return rc;
+  h.d_status = scratch;
+
+  rc = check_decode_args(&h, B, latents, steps, weights, H, W, out_rgb);
+  if (rc != PIC_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(scratch, 0, kNeededInts * sizeof(int), s) != cudaSuccess) {  // starts at zero
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  DecodeParams p;
+  fill_params(&h, p, B, latents, steps, weights, H, W, out_rgb);
+  return launch(&h, p, s);
+}

@@ -75,6 +75,8 @@ def load_library():
     lib.pic_decode_batch.restype = i
     lib.pic_decode_batch_host.argtypes = [_P, i, _P, _P, _P, i, i, _P, _P]
     lib.pic_decode_batch_host.restype = i
+    lib.pic_decode_batch_noalloc.argtypes = [ctypes.POINTER(pic_arch), i, _P, _P, _P, i, i, _P, _P]
+    lib.pic_decode_batch_noalloc.restype = i
     lib.pic_decode_check.argtypes = [_P, _P]
     lib.pic_decode_check.restype = i
     lib.pic_decode_destroy.argtypes = [_P]
@@ -131,6 +133,12 @@ def pic_decode_batch(h, B, latents, steps, weights, H, W, out_rgb, stream=None) 
 def pic_decode_batch_host(h, B, latents, steps, weights, H, W, out_rgb, stream=None) -> int:
     return load_library().pic_decode_batch_host(h, B, latents, steps, weights, H, W, out_rgb,
                                                 stream)
+
+
+def pic_decode_batch_noalloc(arch: pic_arch, B, latents, steps, weights, H, W, out_rgb,
+                             stream=None) -> int:
+    return load_library().pic_decode_batch_noalloc(ctypes.byref(arch), B, latents, steps, weights,
+                                                   H, W, out_rgb, stream)
 
 
 def pic_decode_check(h, stream=None) -> int:

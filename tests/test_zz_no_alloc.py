@@ -1,0 +1,83 @@
+"""The allocation-free entry point, pic_decode_batch_noalloc.
+
+Callers that may not allocate device memory (inside a CUDA-graph stream
+capture, in serving loops whose memory is fixed up front, or in embedders
+that forbid the library from touching the allocator) decode through this
+entry point: it takes the architecture instead of a handle and keeps its
+only scratch -- the status word of the bounded waits -- in a static device
+array of the library.  Its output must match the handle-based
+pic_decode_batch within the tolerance of the other parity tests, on two
+calls in a row (the second call reuses the static array the first one left
+behind).
+
+The file name makes pytest collect it last.
+"""
+import numpy as np
+import pytest
+
+from paper_2609_09020_gb300 import workloads as wk
+
+from decode_util import TOL, max_abs_diff
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_09020_gb300 import build
+    build.build()
+
+
+CASES = [
+    (wk.WORKLOADS["c5"].replace(seeds=(100, 101, 102), name="c5x3"), "fp16_tc"),
+    (wk.WORKLOADS["c2"], "fp32"),
+    (wk.custom("odd", 37, 201, 7, 1, (7, 64, 64, 3), weight_dtype="fp16", batch=2), "fp16_tc"),
+]
+
+
+@pytest.mark.parametrize("wl,precision", CASES, ids=lambda c: getattr(c, "name", c))
+def test_noalloc_matches_handle_entry_point(wl, precision):
+    import torch
+    from paper_2609_09020_gb300 import pic
+    x = wk.make_inputs(wl)
+    B = x.latents.shape[0]
+    dev = torch.device("cuda:0")
+    lat = torch.from_numpy(x.latents).to(dev)
+    st = torch.from_numpy(x.steps).to(dev)
+    w = torch.from_numpy(np.ascontiguousarray(x.weights_for(precision))).to(dev)
+    stream = torch.cuda.current_stream().cuda_stream
+
+    dec = pic.Decoder.for_workload(wl, precision, max_batch=B)
+    ref = torch.full((B, 3, wl.H, wl.W), float("nan"), device=dev)
+    dec.decode_batch(lat, st, w, wl.H, wl.W, ref, B=B)
+    dec.check()
+    dec.close()
+
+    arch = pic.make_arch(wl.L, wl.C, wl.dims, wl.act, precision, True, wl.H, wl.W, B)
+    for call in range(2):
+        out = torch.full((B, 3, wl.H, wl.W), float("nan"), device=dev)
+        rc = pic.pic_decode_batch_noalloc(arch, B, lat.data_ptr(), st.data_ptr(), w.data_ptr(),
+                                          wl.H, wl.W, out.data_ptr(), stream)
+        assert rc == pic.PIC_OK, (call, pic.pic_status_string(rc))
+        torch.cuda.synchronize()
+        d, where = max_abs_diff(out.cpu().numpy(), ref.cpu().numpy().astype(np.float64))
+        assert d <= TOL[precision], (call, d, where)
+
+
+def test_noalloc_rejects_bad_arguments():
+    import torch
+    from paper_2609_09020_gb300 import pic
+    wl = wk.WORKLOADS["c1"]
+    arch = pic.make_arch(wl.L, wl.C, wl.dims, wl.act, "fp32", True, wl.H, wl.W, 1)
+    dev = torch.device("cuda:0")
+    buf = torch.zeros(3 * wl.H * wl.W + 64, device=dev)
+    p = buf.data_ptr()
+    s = torch.cuda.current_stream().cuda_stream
+    assert pic.pic_decode_batch_noalloc(arch, 2, p, p, p, wl.H, wl.W, p, s) == pic.PIC_ERR_INVALID_ARG
+    assert pic.pic_decode_batch_noalloc(arch, 1, p, p, p, wl.H + 1, wl.W, p, s) == pic.PIC_ERR_INVALID_ARG
+    assert pic.pic_decode_batch_noalloc(arch, 1, None, p, p, wl.H, wl.W, p, s) == pic.PIC_ERR_INVALID_ARG
+    bad = pic.make_arch(4, 1, (5, 16, 3), max_H=8, max_W=8)
+    assert pic.pic_decode_batch_noalloc(bad, 1, p, p, p, 8, 8, p, s) == pic.PIC_ERR_INVALID_ARG
