@@ -65,10 +65,18 @@ def algorithmic(wl: wk.Workload, batch: int):
     return flops, nbytes
 
 
-def kernel_source_hash():
+KERNEL_SOURCES = {
+    "tc": ["k_tc.cu", "tc_ptx.cuh", "pic_common.cuh", "pic_kernels.h"],
+    "fp32": ["k_fp32.cu", "pic_common.cuh", "pic_kernels.h"],
+}
+
+
+def kernel_source_hash(kernel_name: str) -> str:
+    """Hash of the source files a decode kernel is compiled from."""
+    files = KERNEL_SOURCES["tc" if kernel_name.startswith("tc") else "fp32"]
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_09020_gb300", "csrc")
-    for fn in sorted(os.listdir(csrc)):
+    for fn in files:
         with open(os.path.join(csrc, fn), "rb") as f:
             h.update(fn.encode() + f.read())
     return h.hexdigest()[:16]
@@ -84,7 +92,7 @@ def recorded_traffic(kernel_name: str, workload: str):
     except (OSError, ValueError):
         return None
     e = rec.get(f"{kernel_name}/{workload}")
-    if not e or e.get("source_hash") != kernel_source_hash():
+    if not e or e.get("source_hash") != kernel_source_hash(kernel_name):
         return None
     return e.get("dram_bytes_per_launch")
 
