@@ -132,7 +132,7 @@ struct TcNet {
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                              int* status) {
   for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait_sleep(bar, parity)) return true;
     if ((i & 63u) == 63u) {
       if (*abort_flag) return false;
       if (i > 4096) __nanosleep(64);
@@ -441,11 +441,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
               bb = gelu_erf(bb);
             }
             // hi = fp16 truncation (ReLU folded in), lo = v - hi (packed subtraction)
-            const uint32_t h2 = (Net::ACT == ACT_GELU) ? pack_f16x2_rz(a, bb) : pack_f16x2_rz_relu(a, bb);
-            const float2 hf = unpack_f16x2(h2);
-            const float2 l2 = unpack2(sub2(pack2(a, bb), pack2(hf.x, hf.y)));
-            hl[q] = h2;
-            hl[HW / 2 + q] = (Net::ACT == ACT_GELU) ? pack_f16x2(l2.x, l2.y) : pack_f16x2_relu(l2.x, l2.y);
+            split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[HW / 2 + q]);
           }
           // hi pair (h0/2 + q) -> column t_a + h0/2 + q; lo pair -> t_a + N/2 + h0/2 + q
           tmem_st8(t_a + h0 / 2, hl);

@@ -29,6 +29,19 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// Same, asking the hardware to suspend the thread up to ~1 ms while the
+// phase is incomplete (fewer polling iterations while a warp waits).
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(1000000u)
+      : "memory");
+  return ok != 0;
+}
 // Non-blocking probe of a phase.
 __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
@@ -209,6 +222,42 @@ __device__ __forceinline__ uint32_t pack_f16x2_rz(float lo_elem, float hi_elem) 
 // Widens both halves of an f16x2 to fp32.
 __device__ __forceinline__ float2 unpack_f16x2(uint32_t v) {
   return __half22float2(*reinterpret_cast<const __half2*>(&v));
+}
+
+// hi/lo split of a pair (a, b) of fp32 values for the split-operand MMA:
+// hi = RZ_fp16(x) (ReLU applied when RELU), lo = RN_fp16(x - hi) (ReLU too:
+// x - hi has x's sign).  Returns both as f16x2 with a in the low half.
+template <bool RELU>
+__device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi2, uint32_t& lo2) {
+  if constexpr (RELU) {
+    asm("{\n\t"
+        ".reg .b16 h0, h1;\n\t.reg .f32 ha, hb, la, lb;\n\t.reg .b64 v, hh, l;\n\t"
+        "cvt.rz.relu.f16x2.f32 %0, %3, %2;\n\t"
+        "mov.b32 {h0, h1}, %0;\n\t"
+        "cvt.f32.f16 ha, h0;\n\t"
+        "cvt.f32.f16 hb, h1;\n\t"
+        "mov.b64 v, {%2, %3};\n\t"
+        "mov.b64 hh, {ha, hb};\n\t"
+        "sub.rn.f32x2 l, v, hh;\n\t"
+        "mov.b64 {la, lb}, l;\n\t"
+        "cvt.rn.relu.f16x2.f32 %1, lb, la;\n\t}\n"
+        : "=r"(hi2), "=r"(lo2)
+        : "f"(a), "f"(b));
+  } else {
+    asm("{\n\t"
+        ".reg .b16 h0, h1;\n\t.reg .f32 ha, hb, la, lb;\n\t.reg .b64 v, hh, l;\n\t"
+        "cvt.rz.f16x2.f32 %0, %3, %2;\n\t"
+        "mov.b32 {h0, h1}, %0;\n\t"
+        "cvt.f32.f16 ha, h0;\n\t"
+        "cvt.f32.f16 hb, h1;\n\t"
+        "mov.b64 v, {%2, %3};\n\t"
+        "mov.b64 hh, {ha, hb};\n\t"
+        "sub.rn.f32x2 l, v, hh;\n\t"
+        "mov.b64 {la, lb}, l;\n\t"
+        "cvt.rn.f16x2.f32 %1, lb, la;\n\t}\n"
+        : "=r"(hi2), "=r"(lo2)
+        : "f"(a), "f"(b));
+  }
 }
 
 __device__ __forceinline__ void sts128(uint32_t saddr, uint32_t a, uint32_t b, uint32_t c,
