@@ -321,23 +321,6 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         it_sy[j] = lg.sy;
         it_sx[j] = lg.sx;
       }
-      // Lane l-1 of every warp holds the geometry of level l: per tile it
-      // computes that level's vertical tap once, and the lanes whose column
-      // items sit on level l fetch it with a shuffle.
-      static_assert(L - 1 <= 32, "one lane per coarse level");
-      int ln_H = 1, ln_W = 1;
-      float ln_sy = 1.0f, ln_sx = 1.0f;
-      if (lane + 1 < L) {
-        const LevelGeom lg = p.lv[lane + 1];
-        ln_H = lg.H;
-        ln_W = lg.W;
-        ln_sy = lg.sy;
-        ln_sx = lg.sx;
-      }
-      float it_beta[JJ];
-#pragma unroll
-      for (int j = 0; j < JJ; ++j) it_beta[j] = 0.0f;
-
       // Relative x-taps of pixel r for each level (used when fast_x): the
       // source coordinate (r + 1/2) / 2^l - 1/2 relative to column x0/2^l - 1.
       int rel[L];
@@ -362,25 +345,17 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
 #pragma unroll
         for (int c = 0; c < C; ++c)
           cp_async4(stage_s + (c * kTile + r) * 4, lat + c * plane + static_cast<long long>(y) * p.W + xc);
-        // this lane's level: rows v0, v1 (as element offsets), weight, first column
-        const Tap lt = bilinear_tap(y, ln_sy, ln_H);
-        const int ln_r0 = lt.i0 * ln_W, ln_r1 = lt.i1 * ln_W;
-        const int ln_u0 = fast_x ? (x0 >> (lane + 1)) - 1 : bilinear_tap(x0, ln_sx, ln_W).i0;
 #pragma unroll
         for (int j = 0; j < J; ++j) {
           const int l = it_l[j];
-          const int src = l > 0 ? l - 1 : 0;
-          const int r0 = __shfl_sync(0xffffffffu, ln_r0, src);
-          const int r1 = __shfl_sync(0xffffffffu, ln_r1, src);
-          const int u_start = __shfl_sync(0xffffffffu, ln_u0, src);
-          const float beta = __shfl_sync(0xffffffffu, lt.frac, src);
           if (l > 0) {
+            const Tap ty = bilinear_tap(y, it_sy[j], it_H[j]);
+            const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, it_sx[j], it_W[j]).i0;
             const int u = min(max(u_start + it_i[j], 0), it_W[j] - 1);
             const int32_t* pl = lat + it_off[j] + u;
-            cp_async4(stage_s + ((C + 2 * j) * kTile + r) * 4, pl + r0);
-            cp_async4(stage_s + ((C + 2 * j + 1) * kTile + r) * 4, pl + r1);
+            cp_async4(stage_s + ((C + 2 * j) * kTile + r) * 4, pl + ty.i0 * it_W[j]);
+            cp_async4(stage_s + ((C + 2 * j + 1) * kTile + r) * 4, pl + ty.i1 * it_W[j]);
           }
-          it_beta[j] = beta;
         }
         cp_async_commit();
       };
@@ -394,8 +369,9 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         for (int j = 0; j < J; ++j) {
           const int l = it_l[j];
           if (l > 0) {
+            const float beta = bilinear_tap(y, it_sy[j], it_H[j]).frac;
             const int t0 = stage[(C + 2 * j) * kTile + r], t1 = stage[(C + 2 * j + 1) * kTile + r];
-            colbuf[r + kTile * j] = step[l] * fmaf(it_beta[j], static_cast<float>(t1 - t0), static_cast<float>(t0));
+            colbuf[r + kTile * j] = step[l] * fmaf(beta, static_cast<float>(t1 - t0), static_cast<float>(t0));
           }
         }
         mbar_arrive(my_col);  // the group's column buffer is complete once all 128 arrived
@@ -448,26 +424,24 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
 
       // Hidden epilogue: accumulator -> activation -> hi/lo -> TMEM operand.
       auto hidden_epilogue = [&]() {
-        // 16 columns at a time; the load of the next chunk is in flight
-        // while the current one is converted.
-        uint32_t acc[2][16];
-        tmem_ld16(t_acc, acc[0]);
 #pragma unroll
-        for (int h0 = 0; h0 < N; h0 += 16) {
-          const int cur = (h0 / 16) & 1;
+        for (int h0 = 0; h0 < N; h0 += 16) {  // 16 columns at a time (fewer live registers)
+          constexpr int HW = 16;
+          uint32_t acc[HW];
+#pragma unroll
+          for (int c0 = 0; c0 < HW; c0 += 16) tmem_ld16(t_acc + h0 + c0, acc + c0);
           tmem_ld_wait();
-          if (h0 + 16 < N) tmem_ld16(t_acc + h0 + 16, acc[cur ^ 1]);
-          uint32_t hl[16];  // [0, 8): hi pairs, [8, 16): lo pairs
+          uint32_t hl[HW];  // [0, HW/2): hi pairs, [HW/2, HW): lo pairs
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            float a = __uint_as_float(acc[cur][2 * q]);
-            float bb = __uint_as_float(acc[cur][2 * q + 1]);
+          for (int q = 0; q < HW / 2; ++q) {
+            float a = __uint_as_float(acc[2 * q]);
+            float bb = __uint_as_float(acc[2 * q + 1]);
             if constexpr (Net::ACT == ACT_GELU) {
               a = gelu_erf(a);
               bb = gelu_erf(bb);
             }
             // hi = fp16 truncation (ReLU folded in), lo = v - hi (packed subtraction)
-            split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[8 + q]);
+            split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[HW / 2 + q]);
           }
           // hi pair (h0/2 + q) -> column t_a + h0/2 + q; lo pair -> t_a + N/2 + h0/2 + q
           tmem_st8(t_a + h0 / 2, hl);
