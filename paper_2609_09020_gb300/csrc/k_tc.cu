@@ -606,11 +606,17 @@ KernelInfo make_tc(const char* name, const int* dims) {
 }  // namespace
 
 int tc_kernels(KernelInfo* out, int cap) {
-  static const int d_c5[] = {7, 64, 64, 3};
+  static const int d_c1[] = {4, 16, 16, 3};
+  static const int d_c2[] = {7, 40, 40, 3};
+  static const int d_c3[] = {14, 64, 64, 3};
   static const int d_c4[] = {16, 64, 64, 64, 3};
+  static const int d_c5[] = {7, 64, 64, 3};
   const KernelInfo list[] = {
       make_tc<1, 3, 7, 64, ACT_RELU, 4>("tc05_7x64x64x3_relu", d_c5),
       make_tc<2, 4, 16, 64, ACT_GELU, 4>("tc05_16x64x64x64x3_gelu", d_c4),
+      make_tc<2, 3, 14, 64, ACT_RELU, 4>("tc05_14x64x64x3_relu", d_c3),
+      make_tc<1, 3, 7, 48, ACT_GELU, 4>("tc05_7x40x40x3_gelu", d_c2),
+      make_tc<1, 3, 4, 16, ACT_RELU, 4>("tc05_4x16x16x3_relu", d_c1),
   };
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
   for (int i = 0; i < n && i < cap; ++i) out[i] = list[i];

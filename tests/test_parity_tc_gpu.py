@@ -63,6 +63,14 @@ def test_c4_full_image(orc):
     _check(orc, wk.WORKLOADS["c4"])
 
 
+@pytest.mark.parametrize("name", ["c1", "c2", "c3"])
+def test_fp32_workloads_on_tensor_path(orc, name):
+    """The other workloads' architectures on the tensor path, with the fp16
+    copy of their fp32 weights (widths 16, 40 -> padded 48, and 64 with two
+    channels per level)."""
+    _check(orc, wk.WORKLOADS[name])
+
+
 def test_c5_unclamped(orc):
     wl = wk.WORKLOADS["c5"].replace(seeds=(100, 101), name="c5x2")
     _check(orc, wl, clamp=False)
@@ -85,7 +93,7 @@ def test_edge_shapes(orc, wl):
 
 def test_tc_kernels_are_selected():
     from paper_2609_09020_gb300.pic import Decoder
-    for name in ("c4", "c5"):
+    for name in ("c1", "c2", "c3", "c4", "c5"):
         dec = Decoder.for_workload(wk.WORKLOADS[name], P)
         assert dec.kernel_name.startswith("tc05_")
         dec.close()
