@@ -437,8 +437,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             float a = __uint_as_float(acc[2 * q]);
             float bb = __uint_as_float(acc[2 * q + 1]);
             if constexpr (Net::ACT == ACT_GELU) {
-              a = gelu_erf(a);
-              bb = gelu_erf(bb);
+              a = gelu_poly(a);
+              bb = gelu_poly(bb);
             }
             // hi = fp16 truncation (ReLU folded in), lo = v - hi (packed subtraction)
             split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[HW / 2 + q]);

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
 
+#include "pic_gelu.cuh"
+
 namespace pic {
 
 constexpr int kMaxLevels = 12;
@@ -43,19 +45,31 @@ struct DecodeParams {
 
 enum { ACT_RELU = 0, ACT_GELU = 1 };
 
-// GELU in its erf form, z * Phi(z), with CUDA's erff.
+// GELU in its erf form, z * Phi(z), with CUDA's erff (reference variant).
 __device__ __forceinline__ float gelu_erf(float z) {
   return 0.5f * z * (1.0f + erff(z * 0.70710678118654752f));
 }
 
+// GELU z * Phi(z) without special-function units or branches:
+// erf(x) ~= x P(u) with u = 2 min(x^2, X^2) / X^2 - 1, x = z / sqrt 2, P the
+// degree-14 least-squares fit of gen_gelu_poly.py; Phi = saturate(1/2 + x P / 2)
+// (the saturation is the |erf| <= 1 clamp).  Max abs error ~1.1e-6.
+__device__ __forceinline__ float gelu_poly(float z) {
+  const float t = fminf(0.5f * z * z, kGeluX2);
+  const float u = fmaf(t, kGeluUScale, -1.0f);
+  const float p = gelu_poly_p(u);
+  const float phi = __saturatef(fmaf(z * 0.35355339059327376f, p, 0.5f));  // z / (2 sqrt 2)
+  return z * phi;
+}
+
 template <int ACT>
 __device__ __forceinline__ float activate(float z) {
-  if constexpr (ACT == ACT_GELU) return gelu_erf(z);
+  if constexpr (ACT == ACT_GELU) return gelu_poly(z);
   else return fmaxf(z, 0.0f);
 }
 
 __device__ __forceinline__ float activate_rt(float z, int act) {
-  return act == ACT_GELU ? gelu_erf(z) : fmaxf(z, 0.0f);
+  return act == ACT_GELU ? gelu_poly(z) : fmaxf(z, 0.0f);
 }
 
 // ---- packed fp32 pairs (sm_100+ f32x2 instructions) ----------------------
