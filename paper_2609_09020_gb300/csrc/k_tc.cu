@@ -360,10 +360,9 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         cp_async_commit();
       };
 
-      // Features of tile (y, x0), first half: the upsampled, concatenated
-      // feature vector f of pixel r from the prefetched loads.  Returns false
-      // if a wait gave up.
-      auto feat_a = [&](int y, int x0, float (&f)[D0]) -> bool {
+      // Features of tile (y, x0) from its prefetched loads -> A1 (shared).
+      // Returns false if a wait gave up.
+      auto features = [&](int y, int x0) -> bool {
         cp_async_wait_all();  // this thread's staged loads have landed
         // vertical pass into the column buffer
 #pragma unroll
@@ -381,6 +380,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         col_phase ^= 1u;
         // horizontal pass + level 0
         const int xc = min(x0 + r, p.W - 1);
+        float f[D0];
 #pragma unroll
         for (int c = 0; c < C; ++c) f[c] = step[0] * static_cast<float>(stage[c * kTile + r]);
 #pragma unroll
@@ -406,10 +406,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             f[l * C + c] = fmaf(a, v1 - v0, v0);
           }
         }
-        return true;
-      };
-      // Second half: hi/lo split, the constant-1 bias column, padding -> A1.
-      auto feat_b = [&](const float (&f)[D0]) {
+        // hi/lo split, the constant-1 bias column, padding -> A1
         float v[K1];
 #pragma unroll
         for (int j = 0; j < K1; ++j) v[j] = 0.0f;
@@ -422,6 +419,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
                  pack_f16x2(v[kc * 8 + 2], v[kc * 8 + 3]), pack_f16x2(v[kc * 8 + 4], v[kc * 8 + 5]),
                  pack_f16x2(v[kc * 8 + 6], v[kc * 8 + 7]));
         fence_async_smem();
+        return true;
       };
 
       // Hidden epilogue: accumulator -> activation -> hi/lo -> TMEM operand.
@@ -465,36 +463,20 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         }
       };
 
-      // The next tile's features are computed in two halves inside the
-      // current tile's MMA waits (after the first and after the last hidden
-      // epilogue); the loads of the tile after that are issued once the
-      // staging buffer is free again.
       bool ok = true;
-      float f[D0];
       if (w < n_tiles) {
         prefetch(cy, ctx * kTile);
-        ok = feat_a(cy, ctx * kTile, f);
-        if (ok) {
-          feat_b(f);
-          mbar_arrive(my_a1);
-        }
+        ok = features(cy, ctx * kTile);
+        if (ok) mbar_arrive(my_a1);
       }
-      if (ok && w + NWG < n_tiles) {
-        int y1 = cy, x1 = ctx;
-        advance(y1, x1);
-        prefetch(y1, x1 * kTile);
-      }
-      constexpr int kFeatB = NL - 2 < 1 ? NL - 2 : 1;  // hidden epilogue after which feat_b runs
       for (int i = w; i < n_tiles && ok; i += NWG) {
         if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
         const int y = cy;
         const int x0 = ctx * kTile;
         int ny = cy, ntx = ctx;
         advance(ny, ntx);
-        int n2y = ny, n2tx = ntx;
-        advance(n2y, n2tx);
         const bool has_next = i + NWG < n_tiles;
-        const bool has_next2 = i + 2 * NWG < n_tiles;
+        if (has_next) prefetch(ny, ntx * kTile);  // in flight during the first epilogue
 
         for (int k = 0; k < NL - 1 && ok; ++k) {
           if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
@@ -506,11 +488,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           hidden_epilogue();
           tc_fence_before();
           mbar_arrive(my_a);
-          if (k == 0 && has_next) ok = ok && feat_a(ny, ntx * kTile, f);  // overlaps layer k+1
-          if (k == kFeatB && has_next && ok) {
-            feat_b(f);
-            if (has_next2) prefetch(n2y, n2tx * kTile);
-          }
+          if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
         }
         if (!ok) break;
 
