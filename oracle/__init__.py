@@ -81,6 +81,12 @@ def _declare(lib):
     lib.pic_oracle_decode_pixels.argtypes = [p, p, p, c_int, c_int, c_int, p, c_int, c_int,
                                              c_int, c_int, p, c_i64, p, p]
     lib.pic_oracle_decode_pixels.restype = c_int
+    lib.pic_oracle_zigzag.argtypes = [p]
+    lib.pic_oracle_zigzag.restype = None
+    lib.pic_oracle_zpr_encode.argtypes = [p, c_i64, ctypes.c_int32, p, c_i64]
+    lib.pic_oracle_zpr_encode.restype = c_i64
+    lib.pic_oracle_izpr.argtypes = [p, c_i64, ctypes.c_int32, p, c_i64]
+    lib.pic_oracle_izpr.restype = c_int
     return lib
 
 
@@ -190,6 +196,32 @@ class Oracle:
                                                _ptr(p), p.size, _ptr(out), _ptr(work))
         if rc != 0:
             raise ValueError("oracle decode_pixels rejected the arguments")
+        return out
+
+
+    # ---- ZpR / inverse ZpR (Sec. 3.3, Algorithm 1) ---------------------
+    def zigzag(self) -> np.ndarray:
+        order = np.empty(64, dtype=np.int32)
+        self.lib.pic_oracle_zigzag(_ptr(order))
+        return order
+
+    def zpr_encode(self, coeffs: np.ndarray, eob: int) -> np.ndarray:
+        """Forward ZpR of blocks [n][64] (raster order) -> int32 symbol stream."""
+        c = np.ascontiguousarray(coeffs, dtype=np.int32).reshape(-1, 64)
+        cap = c.shape[0] * 66 + 16
+        out = np.empty(cap, dtype=np.int32)
+        n = self.lib.pic_oracle_zpr_encode(_ptr(c), c.shape[0], int(eob), _ptr(out), cap)
+        if n < 0:
+            raise ValueError("zpr_encode: literal collides with the run codes, or overflow")
+        return out[:n].copy()
+
+    def izpr(self, symbols: np.ndarray, eob: int, n_blocks: int) -> np.ndarray:
+        """Inverse ZpR -> int32 blocks [n_blocks][64] in raster order."""
+        s = np.ascontiguousarray(symbols, dtype=np.int32)
+        out = np.empty((n_blocks, 64), dtype=np.int32)
+        rc = self.lib.pic_oracle_izpr(_ptr(s), s.size, int(eob), _ptr(out), n_blocks)
+        if rc != 0:
+            raise ValueError("izpr: malformed symbol stream")
         return out
 
 

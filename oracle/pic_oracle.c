@@ -259,3 +259,98 @@ int pic_oracle_decode_pixels(const int32_t *latents, const double *steps, const 
     }
     return 0;
 }
+
+/* ------------------------------------------------------------------------
+ * ZpR and its inverse (Sec. 3.3, Fig. 2; App. B, Algorithm 1).
+ *
+ * A block is 8 x 8 quantised DCT coefficients, row-major ("raster").  ZpR
+ * reorders a block in zigzag order, trims its trailing zeros and codes every
+ * run of zeros by run length ("partial RLE": only zeros are run-coded).
+ * The stream uses one end-of-block marker value eob, larger than every
+ * literal by at least 17: the 16 values eob-16 .. eob-1 code runs of 1..16
+ * zeros (code eob - 17 + n for a run of n), any smaller value is a literal
+ * coefficient, and eob itself ends a block.  Longer runs take several codes.
+ * ------------------------------------------------------------------------ */
+
+/* Zigzag order of an 8 x 8 block: order[k] is the raster index (row*8+col)
+ * of the k-th coefficient.  Anti-diagonal d = row + col is walked with the
+ * row falling for even d and rising for odd d, starting at (0, 0). */
+void pic_oracle_zigzag(int *order)
+{
+    int k = 0;
+    for (int d = 0; d <= 14; ++d) {
+        int lo = d < 8 ? 0 : d - 7, hi = d < 8 ? d : 7;
+        if (d % 2 == 0)
+            for (int row = hi; row >= lo; --row) order[k++] = row * 8 + (d - row);
+        else
+            for (int row = lo; row <= hi; ++row) order[k++] = row * 8 + (d - row);
+    }
+}
+
+/* Forward ZpR of n blocks (raster order) into symbols; returns the number of
+ * symbols written, or -1 if cap is too small or a literal collides with the
+ * run codes (coefficients must be < eob - 16). */
+int64_t pic_oracle_zpr_encode(const int32_t *coeffs, int64_t n_blocks, int32_t eob,
+                              int32_t *symbols, int64_t cap)
+{
+    int order[64];
+    pic_oracle_zigzag(order);
+    int64_t n = 0;
+    for (int64_t b = 0; b < n_blocks; ++b) {
+        const int32_t *blk = coeffs + 64 * b;
+        int zz[64];
+        for (int k = 0; k < 64; ++k) zz[k] = blk[order[k]];
+        int last = -1; /* trim trailing zeros */
+        for (int k = 0; k < 64; ++k)
+            if (zz[k] != 0) last = k;
+        int k = 0;
+        while (k <= last) {
+            if (zz[k] != 0) {
+                if (zz[k] >= eob - 16) return -1;
+                if (n >= cap) return -1;
+                symbols[n++] = zz[k++];
+            } else {
+                int run = 0;
+                while (k <= last && zz[k] == 0 && run < 16) { ++run; ++k; }
+                if (n >= cap) return -1;
+                symbols[n++] = eob - 17 + run;
+            }
+        }
+        if (n >= cap) return -1;
+        symbols[n++] = eob;
+    }
+    return n;
+}
+
+/* Inverse ZpR (Algorithm 1's expansion, done block after block): split the
+ * stream at the eob markers, write literals and zero runs at consecutive
+ * zigzag positions of the block, leave the trimmed tail zero.  Returns 0,
+ * or -1 for a malformed stream (a block overflowing 64 positions, a
+ * symbol >= eob other than the marker, or a marker count != n_blocks). */
+int pic_oracle_izpr(const int32_t *symbols, int64_t n_symbols, int32_t eob,
+                    int32_t *coeffs, int64_t n_blocks)
+{
+    int order[64];
+    pic_oracle_zigzag(order);
+    for (int64_t i = 0; i < 64 * n_blocks; ++i) coeffs[i] = 0;
+    int64_t b = 0, pos = 0;
+    for (int64_t i = 0; i < n_symbols; ++i) {
+        int32_t s = symbols[i];
+        if (s == eob) {
+            ++b;
+            pos = 0;
+            continue;
+        }
+        if (b >= n_blocks || s > eob) return -1;
+        int32_t *blk = coeffs + 64 * b;
+        if (s >= eob - 16) {
+            int run = s + 17 - eob;
+            if (pos + run > 64) return -1;
+            for (int r = 0; r < run; ++r) blk[order[pos++]] = 0;
+        } else {
+            if (pos + 1 > 64) return -1;
+            blk[order[pos++]] = s;
+        }
+    }
+    return b == n_blocks ? 0 : -1;
+}

@@ -295,4 +295,73 @@ def pin_decode_pixels_match(o):
     assert np.array_equal(part, full.reshape(3, -1)[:, pix].T)
 
 
+# ---------------------------------------------------------------- ZpR (Sec. 3.3, Alg. 1)
+def _golden_blocks(g):
+    n = int(g["nblocks"][0])
+    blocks = np.zeros((n, 64), dtype=np.int32)
+    for b in range(n):
+        for tok in g.get(f"block{b}", []):
+            pos, val = tok.split(":")
+            blocks[b, int(pos)] = int(val)
+    return blocks
+
+
+def pin_zigzag_order(o):
+    """The zigzag order is a permutation of 0..63 that walks the
+    anti-diagonals row + col = 0..14 in turn, alternating direction, starting
+    0, 1, 8, 16, 9, 2, 3, 10, 17, 24 (the JPEG order) and ending at 63."""
+    z = o.zigzag()
+    assert sorted(z.tolist()) == list(range(64))
+    assert z[:10].tolist() == [0, 1, 8, 16, 9, 2, 3, 10, 17, 24]
+    assert z[-3:].tolist() == [55, 62, 63]
+    diag = [int(r // 8 + r % 8) for r in z]
+    assert diag == sorted(diag)
+
+
+def pin_zpr_hand_stream(o):
+    """The hand-worked stream of tests/golden/zpr_blocks.txt, both ways."""
+    g = load_golden("zpr_blocks.txt")
+    eob = int(g["eob"][0])
+    blocks = _golden_blocks(g)
+    stream = np.array([int(v) for v in g["stream"]], dtype=np.int32)
+    assert np.array_equal(o.zpr_encode(blocks, eob), stream)
+    assert np.array_equal(o.izpr(stream, eob, blocks.shape[0]), blocks)
+
+
+def pin_zpr_round_trip(o):
+    """Inverse ZpR undoes ZpR on random sparse blocks, all-zero blocks, dense
+    blocks and long zero runs (> 16, split over several codes)."""
+    rng = np.random.Generator(np.random.PCG64(31))
+    b = rng.integers(-20, 21, (200, 64)).astype(np.int32)
+    b[rng.random((200, 64)) < 0.8] = 0
+    b[5] = 0
+    b[6] = rng.integers(1, 9, 64)
+    b[7] = 0
+    b[7, 63] = -3
+    b[8] = 0
+    b[8, 0] = 4
+    b[8, 62] = 2
+    eob = int(np.abs(b).max()) + 17
+    s = o.zpr_encode(b, eob)
+    assert (s == eob).sum() == 200
+    assert np.array_equal(o.izpr(s, eob, 200), b)
+    # trailing zeros are trimmed: an all-zero block is the marker alone
+    z = o.zpr_encode(np.zeros((3, 64), np.int32), 40)
+    assert z.tolist() == [40, 40, 40]
+
+
+def pin_izpr_rejects_malformed(o):
+    """A block longer than 64 positions, or the wrong number of markers, is
+    refused."""
+    eob = 30
+    over = np.array([29, 29, 29, 29, 29, 30], dtype=np.int32)  # 80 zeros
+    for s, n in [(over, 1), (np.array([1, 30, 2, 30], dtype=np.int32), 3),
+                 (np.array([1, 30, 2, 30], dtype=np.int32), 1)]:
+        try:
+            o.izpr(s, eob, n)
+        except ValueError:
+            continue
+        raise AssertionError(f"malformed stream accepted: {s.tolist()} n={n}")
+
+
 PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

@@ -85,6 +85,21 @@ MUTATIONS = {
     "channel_offset_dropped": (
         "f[d++] = pic_oracle_bilinear_at(y[l] + (int64_t)c * Hl * Wl, Hl, Wl, H, W, x, yy);",
         "f[d++] = pic_oracle_bilinear_at(y[l], Hl, Wl, H, W, x, yy);"),
+    "zigzag_direction_flipped": (
+        "if (d % 2 == 0)\n            for (int row = hi; row >= lo; --row)",
+        "if (d % 2 == 1)\n            for (int row = hi; row >= lo; --row)"),
+    "run_code_off_by_one": (
+        "symbols[n++] = eob - 17 + run;",
+        "symbols[n++] = eob - 16 + run - (run == 16);"),
+    "izpr_run_length_off_by_one": (
+        "int run = s + 17 - eob;",
+        "int run = s + 16 - eob;"),
+    "no_trailing_trim": (
+        "if (zz[k] != 0) last = k;",
+        "last = 63;"),
+    "izpr_raster_not_zigzag": (
+        "blk[order[pos++]] = s;",
+        "blk[pos++] = s;"),
 }
 
 
