@@ -87,6 +87,12 @@ def load_library():
     lib.pic_latent_count.restype = i64
     lib.pic_param_count.argtypes = [ctypes.POINTER(pic_arch)]
     lib.pic_param_count.restype = i64
+    lib.pic_izpr_workspace_bytes.argtypes = [i64]
+    lib.pic_izpr_workspace_bytes.restype = i64
+    lib.pic_izpr_decode.argtypes = [_P, i64, ctypes.c_int32, i64, _P, _P, _P, ctypes.c_size_t, _P]
+    lib.pic_izpr_decode.restype = i
+    lib.pic_izpr_status.argtypes = [_P, _P]
+    lib.pic_izpr_status.restype = i
     lib.pic_status_string.argtypes = [i]
     lib.pic_status_string.restype = ctypes.c_char_p
     _lib = lib
@@ -163,6 +169,43 @@ def pic_param_count(arch: pic_arch) -> int:
 
 def pic_status_string(status: int) -> str:
     return load_library().pic_status_string(status).decode()
+
+
+def pic_izpr_workspace_bytes(n_symbols) -> int:
+    return int(load_library().pic_izpr_workspace_bytes(n_symbols))
+
+
+def pic_izpr_decode(symbols, n_symbols, eob, n_blocks, coeffs, offsets, workspace,
+                    workspace_bytes, stream=None) -> int:
+    return load_library().pic_izpr_decode(symbols, n_symbols, eob, n_blocks, coeffs, offsets,
+                                          workspace, workspace_bytes, stream)
+
+
+def pic_izpr_status(workspace, stream=None) -> int:
+    return load_library().pic_izpr_status(workspace, stream)
+
+
+def izpr_decode(symbols, eob: int, n_blocks: int, stream=None):
+    """Inverse ZpR of a device int32 symbol tensor; returns (coeffs [n][64]
+    int32 raster order, offsets [n] int64) as torch CUDA tensors.  Raises if
+    the stream is malformed (this synchronises the stream)."""
+    import torch
+    dev = symbols.device
+    n = symbols.numel()
+    coeffs = torch.empty((max(n_blocks, 1), 64), dtype=torch.int32, device=dev)[:n_blocks]
+    offsets = torch.empty(max(n_blocks, 1), dtype=torch.int64, device=dev)[:n_blocks]
+    wb = pic_izpr_workspace_bytes(n)
+    ws = torch.empty(wb, dtype=torch.uint8, device=dev)
+    sp = _stream_ptr(stream)
+    rc = pic_izpr_decode(symbols.data_ptr() if n else None, n, int(eob), n_blocks,
+                         coeffs.data_ptr() if n_blocks else None,
+                         offsets.data_ptr() if n_blocks else None, ws.data_ptr(), wb, sp)
+    if rc != PIC_OK:
+        raise PicError(rc, "pic_izpr_decode")
+    rc = pic_izpr_status(ws.data_ptr(), sp)
+    if rc != PIC_OK:
+        raise PicError(rc, "pic_izpr_status")
+    return coeffs, offsets
 
 
 # ---- convenience wrapper over torch tensors --------------------------------

@@ -194,6 +194,20 @@ def custom(name: str, H: int, W: int, L: int, C: int, dims, act: str = "relu",
                     seeds=tuple(seed + i for i in range(batch)), precisions=tuple(precisions))
 
 
+def dct_blocks(n_blocks: int, seed: int, scale: float = 6.0, decay: float = 0.72,
+               clip: int = 255) -> np.ndarray:
+    """Synthetic quantised 8x8 DCT blocks, int32 [n][64] in raster order
+    (row * 8 + col): coefficient (row, col) is round(Laplace(0, scale *
+    decay^(row + col))) clipped to +-clip, so low frequencies are large and
+    high frequencies mostly zero -- the statistics the entropy stage of the
+    codec sees (Sec. 3.2 quantises DCT coefficients of the latents)."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    rc = np.add.outer(np.arange(8), np.arange(8)).ravel()
+    scales = scale * decay ** rc
+    q = np.rint(rng.laplace(0.0, 1.0, (n_blocks, 64)) * scales)
+    return np.clip(q, -clip, clip).astype(np.int32)
+
+
 def sample_pixels(H: int, W: int, n: int, seed: int) -> np.ndarray:
     """Flat pixel indices (y * W + x) to check at full size: the four corners,
     the middle of every border, and n seeded random positions."""

@@ -82,3 +82,15 @@ def test_create_without_gpu_fails_cleanly(lib):
     h = ctypes.c_void_p()
     rc = lib.pic_decode_create(ctypes.byref(arch), ctypes.byref(h))
     assert rc in (pic.PIC_ERR_UNSUPPORTED, pic.PIC_ERR_CUDA) and h.value is None
+
+
+def test_izpr_workspace_and_argument_checks(lib):
+    from paper_2609_09020_gb300 import pic
+    assert pic.pic_izpr_workspace_bytes(-1) == -1
+    assert pic.pic_izpr_workspace_bytes(0) == 32
+    assert pic.pic_izpr_workspace_bytes(1) >= 32 + 4 + 8
+    assert pic.pic_izpr_workspace_bytes(10 ** 8) > 10 ** 8 // 4096 * 12
+    # rejected before any CUDA call
+    assert pic.pic_izpr_decode(None, 10, 30, 1, None, None, None, 0, None) == pic.PIC_ERR_INVALID_ARG
+    assert pic.pic_izpr_decode(None, -1, 30, 1, None, None, None, 0, None) == pic.PIC_ERR_INVALID_ARG
+    assert pic.pic_izpr_status(None, None) == pic.PIC_ERR_INVALID_ARG
