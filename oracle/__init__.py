@@ -17,6 +17,13 @@ Parity status of each function (what pins it is in tests/test_oracle.py):
                       GELU closed forms)
   decode              pinned (hand-computed 4x4 image, reductions to the
                       pieces above, planted-mistake runs)
+  decode_values       pinned (equals decode on dequantised symbols)
+  dct8x8 / idct8x8    pinned (scipy's orthonormal DCT-II/III, DC-only and
+                      one-dimensional closed forms, Parseval, inverse pair)
+  patchify/unpatchify pinned (hand-placed DC patches on ragged planes,
+                      block counts of the decode workloads, round trip)
+  zigzag / ZpR / iZpR pinned (hand-worked stream, JPEG zigzag table start,
+                      round trips, malformed streams)
 """
 from __future__ import annotations
 
@@ -87,6 +94,19 @@ def _declare(lib):
     lib.pic_oracle_zpr_encode.restype = c_i64
     lib.pic_oracle_izpr.argtypes = [p, c_i64, ctypes.c_int32, p, c_i64]
     lib.pic_oracle_izpr.restype = c_int
+    lib.pic_oracle_decode_values.argtypes = [p, p, c_int, c_int, c_int, p, c_int, c_int, c_int,
+                                             c_int, p, c_int]
+    lib.pic_oracle_decode_values.restype = c_int
+    lib.pic_oracle_dct8x8.argtypes = [p, p]
+    lib.pic_oracle_dct8x8.restype = None
+    lib.pic_oracle_idct8x8.argtypes = [p, p]
+    lib.pic_oracle_idct8x8.restype = None
+    lib.pic_oracle_block_count.argtypes = [c_int, c_int, c_int, c_int]
+    lib.pic_oracle_block_count.restype = c_i64
+    lib.pic_oracle_patchify_dct.argtypes = [p, c_int, c_int, c_int, c_int, p]
+    lib.pic_oracle_patchify_dct.restype = c_int
+    lib.pic_oracle_unpatchify_idct.argtypes = [p, p, c_int, c_int, c_int, c_int, p]
+    lib.pic_oracle_unpatchify_idct.restype = c_int
     return lib
 
 
@@ -198,6 +218,60 @@ class Oracle:
             raise ValueError("oracle decode_pixels rejected the arguments")
         return out
 
+    def decode_values(self, latents, weights, H, W, L, C, dims, act, clamp=True,
+                      nthreads: int = 1) -> np.ndarray:
+        """Decodes one image from real-valued latents (the iDCT output);
+        returns planar fp64 [3][H][W]."""
+        y = np.ascontiguousarray(latents, dtype=np.float64).ravel()
+        w = np.ascontiguousarray(weights, dtype=np.float64).ravel()
+        d = np.ascontiguousarray(dims, dtype=np.int32)
+        if y.size != self.latent_count(H, W, L, C) or w.size != self.param_count(d):
+            raise ValueError("oracle decode_values: buffer sizes do not match the shapes")
+        out = np.empty((3, H, W), dtype=np.float64)
+        rc = self.lib.pic_oracle_decode_values(_ptr(y), _ptr(w), L, C, len(d) - 1, _ptr(d),
+                                               ACTS[act], int(bool(clamp)), H, W, _ptr(out),
+                                               int(nthreads))
+        if rc != 0:
+            raise ValueError("oracle decode_values rejected the arguments")
+        return out
+
+    # ---- Patchify / DCT and their inverses (Sec. 3.2, Eqs. 5-7) --------
+    def dct8x8(self, x: np.ndarray) -> np.ndarray:
+        x = np.ascontiguousarray(x, dtype=np.float64).reshape(8, 8)
+        S = np.empty((8, 8), dtype=np.float64)
+        self.lib.pic_oracle_dct8x8(_ptr(x), _ptr(S))
+        return S
+
+    def idct8x8(self, S: np.ndarray) -> np.ndarray:
+        S = np.ascontiguousarray(S, dtype=np.float64).reshape(8, 8)
+        x = np.empty((8, 8), dtype=np.float64)
+        self.lib.pic_oracle_idct8x8(_ptr(S), _ptr(x))
+        return x
+
+    def block_count(self, H: int, W: int, L: int, C: int) -> int:
+        return int(self.lib.pic_oracle_block_count(H, W, L, C))
+
+    def patchify_dct(self, latents, H, W, L, C) -> np.ndarray:
+        """Encoder side: real latents (pyramid layout) -> DCT coefficients [n][64]."""
+        y = np.ascontiguousarray(latents, dtype=np.float64).ravel()
+        if y.size != self.latent_count(H, W, L, C):
+            raise ValueError("patchify_dct: latent count does not match the shapes")
+        out = np.empty((self.block_count(H, W, L, C), 64), dtype=np.float64)
+        if self.lib.pic_oracle_patchify_dct(_ptr(y), H, W, L, C, _ptr(out)) != 0:
+            raise ValueError("patchify_dct rejected the shapes")
+        return out
+
+    def unpatchify_idct(self, symbols, steps, H, W, L, C) -> np.ndarray:
+        """Decoder side: int coefficients [n][64] x per-level step -> iDCT ->
+        real latents in the pyramid layout (fp64)."""
+        s = np.ascontiguousarray(symbols, dtype=np.int32).ravel()
+        st = np.ascontiguousarray(steps, dtype=np.float64).ravel()
+        if s.size != 64 * self.block_count(H, W, L, C) or st.size != L:
+            raise ValueError("unpatchify_idct: buffer sizes do not match the shapes")
+        out = np.empty(self.latent_count(H, W, L, C), dtype=np.float64)
+        if self.lib.pic_oracle_unpatchify_idct(_ptr(s), _ptr(st), H, W, L, C, _ptr(out)) != 0:
+            raise ValueError("unpatchify_idct rejected the shapes")
+        return out
 
     # ---- ZpR / inverse ZpR (Sec. 3.3, Algorithm 1) ---------------------
     def zigzag(self) -> np.ndarray:

@@ -208,18 +208,21 @@ static void dequant_pyramid(const int32_t *latents, const double *steps, int L, 
     }
 }
 
-/*
- * Full decode of one image.  `work` must hold pic_oracle_latent_count(H, W, L, C)
- * doubles.  nthreads > 1 splits the output rows over OpenMP threads (the
- * arithmetic of each pixel does not change).  Returns 0 or -1.
- */
-int pic_oracle_decode(const int32_t *latents, const double *steps, const double *weights,
-                      int L, int C, int n_layers, const int *dims, int act, int clamp,
-                      int H, int W, double *out_rgb, double *work, int nthreads)
+/* Points y[l] at the levels of a pyramid of real values (no dequantisation). */
+static void split_pyramid(const double *values, int L, int C, int H, int W, double **y)
 {
-    double *y[PIC_ORACLE_MAX_LEVELS];
-    if (check_args(H, W, L, C, n_layers, dims) != 0) return -1;
-    dequant_pyramid(latents, steps, L, C, H, W, work, y);
+    int64_t off = 0;
+    for (int l = 0; l < L; ++l) {
+        y[l] = (double *)(values + off);
+        off += (int64_t)C * level_size(H, l) * level_size(W, l);
+    }
+}
+
+/* Steps 2-5 over every pixel of one image, given its real-valued levels y[l]. */
+static int decode_levels(double *const *y, const double *weights, int L, int C, int n_layers,
+                         const int *dims, int act, int clamp, int H, int W, double *out_rgb,
+                         int nthreads)
+{
     int64_t plane = (int64_t)H * W;
     int bad = 0;
 #ifdef _OPENMP
@@ -237,6 +240,36 @@ int pic_oracle_decode(const int32_t *latents, const double *steps, const double 
     }
     (void)nthreads;
     return bad ? -1 : 0;
+}
+
+/*
+ * Full decode of one image.  `work` must hold pic_oracle_latent_count(H, W, L, C)
+ * doubles.  nthreads > 1 splits the output rows over OpenMP threads (the
+ * arithmetic of each pixel does not change).  Returns 0 or -1.
+ */
+int pic_oracle_decode(const int32_t *latents, const double *steps, const double *weights,
+                      int L, int C, int n_layers, const int *dims, int act, int clamp,
+                      int H, int W, double *out_rgb, double *work, int nthreads)
+{
+    double *y[PIC_ORACLE_MAX_LEVELS];
+    if (check_args(H, W, L, C, n_layers, dims) != 0) return -1;
+    dequant_pyramid(latents, steps, L, C, H, W, work, y);
+    return decode_levels(y, weights, L, C, n_layers, dims, act, clamp, H, W, out_rgb, nthreads);
+}
+
+/*
+ * Steps 2-5 of one image whose latents are already real values (the output
+ * of the iDCT stage below, Fig. 1: iDCT then g_r), same layout as the
+ * symbols of pic_oracle_decode.  Returns 0 or -1.
+ */
+int pic_oracle_decode_values(const double *latents, const double *weights, int L, int C,
+                             int n_layers, const int *dims, int act, int clamp, int H, int W,
+                             double *out_rgb, int nthreads)
+{
+    double *y[PIC_ORACLE_MAX_LEVELS];
+    if (check_args(H, W, L, C, n_layers, dims) != 0) return -1;
+    split_pyramid(latents, L, C, H, W, y);
+    return decode_levels(y, weights, L, C, n_layers, dims, act, clamp, H, W, out_rgb, nthreads);
 }
 
 /*
@@ -353,4 +386,132 @@ int pic_oracle_izpr(const int32_t *symbols, int64_t n_symbols, int32_t eob,
         }
     }
     return b == n_blocks ? 0 : -1;
+}
+
+/* ------------------------------------------------------------------------
+ * Patchify + DCT and their inverses (Fig. 1; Sec. 3.2, Eqs. 5-7).
+ *
+ * The encoder cuts every latent plane into 8 x 8 patches, concatenates them
+ * (z = Patchify(y), Eq. 6) and takes their DCT (s = DCT(z), Eq. 7); the
+ * quantised DCT coefficients are what ZpR codes.  The decoder runs the
+ * inverse: dequantise the coefficients, inverse DCT, put every patch back.
+ *
+ * Readings (the paper names the steps only):
+ *  - DCT is the orthonormal 2-D DCT-II of JPEG's transform,
+ *        S[u][v] = a(u) a(v) sum_m sum_n x[m][n] cos((2m+1) u pi / 16) cos((2n+1) v pi / 16)
+ *    with a(0) = sqrt(1/8), a(k > 0) = sqrt(2/8); its inverse (DCT-III) is
+ *        x[m][n] = sum_u sum_v a(u) a(v) S[u][v] cos((2m+1) u pi / 16) cos((2n+1) v pi / 16).
+ *    u, m index rows (vertical), v, n columns; a block is stored row-major,
+ *    coefficient (u, v) at u * 8 + v, the raster order iZpR produces.
+ *  - Patch order: levels l = 0..L-1 (finest first), then channel c, then
+ *    patch row by, then patch column bx.  A plane whose side is not a
+ *    multiple of 8 gets ceil(H_l / 8) x ceil(W_l / 8) patches; the encoder
+ *    fills positions past the edge with the nearest edge value and the
+ *    decoder drops them.
+ *  - Dequantisation multiplies every coefficient of a level-l patch by the
+ *    level's step (step = 1 is the paper's unit quantisation step).
+ * ------------------------------------------------------------------------ */
+
+static const double PIC_ORACLE_PI = 3.14159265358979323846;
+
+static double dct_alpha(int k)
+{
+    return k == 0 ? sqrt(1.0 / 8.0) : sqrt(2.0 / 8.0);
+}
+
+/* Forward orthonormal 8x8 DCT-II of x (row-major) into S (row-major). */
+void pic_oracle_dct8x8(const double *x, double *S)
+{
+    for (int u = 0; u < 8; ++u)
+        for (int v = 0; v < 8; ++v) {
+            double s = 0.0;
+            for (int m = 0; m < 8; ++m)
+                for (int n = 0; n < 8; ++n)
+                    s += x[m * 8 + n] * cos((2 * m + 1) * u * PIC_ORACLE_PI / 16.0) *
+                         cos((2 * n + 1) * v * PIC_ORACLE_PI / 16.0);
+            S[u * 8 + v] = dct_alpha(u) * dct_alpha(v) * s;
+        }
+}
+
+/* Inverse orthonormal 8x8 DCT (DCT-III) of S into x, both row-major. */
+void pic_oracle_idct8x8(const double *S, double *x)
+{
+    for (int m = 0; m < 8; ++m)
+        for (int n = 0; n < 8; ++n) {
+            double s = 0.0;
+            for (int u = 0; u < 8; ++u)
+                for (int v = 0; v < 8; ++v)
+                    s += dct_alpha(u) * dct_alpha(v) * S[u * 8 + v] *
+                         cos((2 * m + 1) * u * PIC_ORACLE_PI / 16.0) *
+                         cos((2 * n + 1) * v * PIC_ORACLE_PI / 16.0);
+            x[m * 8 + n] = s;
+        }
+}
+
+/* Number of 8x8 patches of one pyramid: sum_l C ceil(H_l / 8) ceil(W_l / 8). */
+int64_t pic_oracle_block_count(int H, int W, int L, int C)
+{
+    int64_t n = 0;
+    for (int l = 0; l < L; ++l)
+        n += (int64_t)C * ((level_size(H, l) + 7) / 8) * ((level_size(W, l) + 7) / 8);
+    return n;
+}
+
+/* Encoder side (for tests): Patchify (Eq. 6) then DCT (Eq. 7) of one
+ * pyramid of real latents into coeffs [block_count][64].  Returns 0 or -1. */
+int pic_oracle_patchify_dct(const double *latents, int H, int W, int L, int C, double *coeffs)
+{
+    if (H < 1 || W < 1 || L < 1 || L > PIC_ORACLE_MAX_LEVELS || C < 1) return -1;
+    int64_t off = 0, b = 0;
+    for (int l = 0; l < L; ++l) {
+        int Hl = level_size(H, l), Wl = level_size(W, l);
+        for (int c = 0; c < C; ++c) {
+            const double *g = latents + off + (int64_t)c * Hl * Wl;
+            for (int by = 0; by < (Hl + 7) / 8; ++by)
+                for (int bx = 0; bx < (Wl + 7) / 8; ++bx, ++b) {
+                    double x[64];
+                    for (int m = 0; m < 8; ++m)
+                        for (int n = 0; n < 8; ++n) {
+                            int r = 8 * by + m, q = 8 * bx + n;
+                            if (r > Hl - 1) r = Hl - 1;
+                            if (q > Wl - 1) q = Wl - 1;
+                            x[m * 8 + n] = g[(int64_t)r * Wl + q];
+                        }
+                    pic_oracle_dct8x8(x, coeffs + 64 * b);
+                }
+        }
+        off += (int64_t)C * Hl * Wl;
+    }
+    return 0;
+}
+
+/* Decoder side: dequantise the integer coefficients of every patch by its
+ * level's step, inverse DCT, and write the patch back into its plane,
+ * dropping the positions past the plane's edge.  symbols is
+ * [block_count][64], latents receives pic_oracle_latent_count values in the
+ * pyramid layout.  Returns 0 or -1. */
+int pic_oracle_unpatchify_idct(const int32_t *symbols, const double *steps, int H, int W, int L,
+                               int C, double *latents)
+{
+    if (H < 1 || W < 1 || L < 1 || L > PIC_ORACLE_MAX_LEVELS || C < 1) return -1;
+    int64_t off = 0, b = 0;
+    for (int l = 0; l < L; ++l) {
+        int Hl = level_size(H, l), Wl = level_size(W, l);
+        for (int c = 0; c < C; ++c) {
+            double *g = latents + off + (int64_t)c * Hl * Wl;
+            for (int by = 0; by < (Hl + 7) / 8; ++by)
+                for (int bx = 0; bx < (Wl + 7) / 8; ++bx, ++b) {
+                    double S[64], x[64];
+                    for (int k = 0; k < 64; ++k) S[k] = (double)symbols[64 * b + k] * steps[l];
+                    pic_oracle_idct8x8(S, x);
+                    for (int m = 0; m < 8; ++m)
+                        for (int n = 0; n < 8; ++n) {
+                            int r = 8 * by + m, q = 8 * bx + n;
+                            if (r < Hl && q < Wl) g[(int64_t)r * Wl + q] = x[m * 8 + n];
+                        }
+                }
+        }
+        off += (int64_t)C * Hl * Wl;
+    }
+    return 0;
 }

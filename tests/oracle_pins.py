@@ -364,4 +364,114 @@ def pin_izpr_rejects_malformed(o):
         raise AssertionError(f"malformed stream accepted: {s.tolist()} n={n}")
 
 
+# ------------------------------------------- patchify + DCT (Sec. 3.2, Eqs. 5-7)
+def pin_dct_matches_scipy(o):
+    """The orthonormal 8x8 DCT-II and its inverse are scipy's dctn / idctn
+    with norm="ortho" (type II / III)."""
+    import scipy.fft as F
+    rng = np.random.Generator(np.random.PCG64(41))
+    for _ in range(4):
+        S = rng.normal(0.0, 10.0, (8, 8))
+        assert np.abs(o.idct8x8(S) - F.idctn(S, type=2, norm="ortho")).max() < 1e-12
+        assert np.abs(o.dct8x8(S) - F.dctn(S, type=2, norm="ortho")).max() < 1e-12
+
+
+def pin_dct_closed_forms(o):
+    """DC only: S[0][0] = 8c gives the constant c.  S[0][4] = 1 (horizontal
+    frequency 4 only): cos((2n+1) pi / 4) = +-1/sqrt 2 and a(0) a(4) =
+    1/(4 sqrt 2), so every row is (1, -1, -1, 1, 1, -1, -1, 1) / 8; S[4][0]
+    is the same pattern down the columns.  Parseval holds and the two
+    transforms invert each other."""
+    S = np.zeros((8, 8))
+    S[0, 0] = 8 * 2.5
+    assert np.abs(o.idct8x8(S) - 2.5).max() < 1e-13
+    pat = np.array([1, -1, -1, 1, 1, -1, -1, 1]) / 8.0
+    S = np.zeros((8, 8))
+    S[0, 4] = 1.0
+    assert np.abs(o.idct8x8(S) - pat[None, :]).max() < 1e-14
+    S = np.zeros((8, 8))
+    S[4, 0] = 1.0
+    assert np.abs(o.idct8x8(S) - pat[:, None]).max() < 1e-14
+    rng = np.random.Generator(np.random.PCG64(43))
+    S = rng.normal(0.0, 5.0, (8, 8))
+    x = o.idct8x8(S)
+    assert abs((x ** 2).sum() - (S ** 2).sum()) < 1e-10 * (S ** 2).sum()
+    assert np.abs(o.dct8x8(x) - S).max() < 1e-12
+
+
+def pin_block_counts(o):
+    """sum_l C ceil(H_l/8) ceil(W_l/8), counted by hand for three pyramids."""
+    assert o.block_count(512, 768, 7, 1) == 6144 + 1536 + 384 + 96 + 24 + 6 + 2
+    assert o.block_count(256, 256, 4, 1) == 1024 + 256 + 64 + 16
+    # 1080 x 1920, 7 levels: 135x240, 68x120, 34x60, 17x30, 9x15, 5x8, 3x4 patches
+    assert o.block_count(1080, 1920, 7, 2) == 2 * (32400 + 8160 + 2040 + 510 + 135 + 40 + 12)
+
+
+def pin_unpatchify_hand(o):
+    """A 12 x 10 image, 2 levels, 1 channel, steps (1, 1/2): level 0 has 2 x 2
+    patches (the right and bottom ones ragged), level 1 (6 x 5) one.  With
+    DC-only patches of DC 8, 16, 24, 32 and 64 the level-0 plane is 1 in the
+    top-left 8 x 8, 2 in the top-right 8 x 2, 3 and 4 below; level 1 is
+    64 * 1/2 / 8 = 4.  A horizontal-frequency-4 patch in the bottom-left slot
+    gives its rows the pattern (1, -1, -1, 1, 1, -1, -1, 1) * S / 8."""
+    H, W, L, C = 12, 10, 2, 1
+    sym = np.zeros((5, 64), np.int32)
+    sym[:, 0] = [8, 16, 24, 32, 64]
+    y = o.unpatchify_idct(sym, [1.0, 0.5], H, W, L, C)
+    l0 = y[:120].reshape(12, 10)
+    want = np.zeros((12, 10))
+    want[:8, :8], want[:8, 8:], want[8:, :8], want[8:, 8:] = 1, 2, 3, 4
+    assert np.abs(l0 - want).max() < 1e-13
+    assert np.abs(y[120:] - 4.0).max() < 1e-13 and y.size == 120 + 30
+    sym[2] = 0
+    sym[2, 4] = 16
+    l0 = o.unpatchify_idct(sym, [1.0, 0.5], H, W, L, C)[:120].reshape(12, 10)
+    pat = np.array([1, -1, -1, 1, 1, -1, -1, 1]) * 2.0
+    assert np.abs(l0[8:, :8] - pat[None, :]).max() < 1e-13
+    assert np.abs(l0[8:, 8:] - 4).max() < 1e-13 and np.abs(l0[:8, :8] - 1).max() < 1e-13
+
+
+def pin_patchify_round_trip(o):
+    """On planes whose sides are multiples of 8 the encoder's Patchify + DCT
+    returns the integer coefficients the decoder started from, for every
+    patch of a 2-channel pyramid."""
+    H, W, L, C = 32, 64, 3, 2   # levels 32x64, 16x32, 8x16
+    n = o.block_count(H, W, L, C)
+    rng = np.random.Generator(np.random.PCG64(47))
+    sym = rng.integers(-40, 41, (n, 64)).astype(np.int32)
+    y = o.unpatchify_idct(sym, [1.0, 1.0, 1.0], H, W, L, C)
+    assert np.abs(o.patchify_dct(y, H, W, L, C) - sym).max() < 1e-10
+    # and the per-level step scales each level's latents exactly
+    y2 = o.unpatchify_idct(sym, [1.0, 0.5, 0.25], H, W, L, C)
+    off = 0
+    for l, st in enumerate([1.0, 0.5, 0.25]):
+        k = C * o.level_size(H, l) * o.level_size(W, l)
+        assert np.abs(y2[off:off + k] - st * y[off:off + k]).max() < 1e-12
+        off += k
+
+
+def pin_decode_values_matches_decode(o):
+    """Decoding real latents equal to the dequantised symbols is the integer
+    decode (2 channels, 3 levels, ragged sizes)."""
+    H, W, L, C = 11, 13, 3, 2
+    dims = [L * C, 8, 3]
+    rng = np.random.Generator(np.random.PCG64(53))
+    q = rng.integers(-9, 10, o.latent_count(H, W, L, C)).astype(np.int32)
+    steps = np.array([1.0, 0.5, 0.25])
+    w = rng.normal(0.0, 0.3, o.param_count(dims))
+    ref = o.decode(q, steps, w, H, W, L, C, dims, "relu", clamp=False)
+    y = np.concatenate([o.dequant(q[a:b], steps[l]) for l, (a, b) in enumerate(
+        _level_ranges(o, H, W, L, C))])
+    assert np.array_equal(o.decode_values(y, w, H, W, L, C, dims, "relu", clamp=False), ref)
+
+
+def _level_ranges(o, H, W, L, C):
+    out, off = [], 0
+    for l in range(L):
+        k = C * o.level_size(H, l) * o.level_size(W, l)
+        out.append((off, off + k))
+        off += k
+    return out
+
+
 PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

@@ -97,6 +97,30 @@ MUTATIONS = {
     "no_trailing_trim": (
         "if (zz[k] != 0) last = k;",
         "last = 63;"),
+    "idct_transposed_coefficients": (
+        "s += dct_alpha(u) * dct_alpha(v) * S[u * 8 + v] *",
+        "s += dct_alpha(u) * dct_alpha(v) * S[v * 8 + u] *"),
+    "dct_dc_weight_unnormalised": (
+        "return k == 0 ? sqrt(1.0 / 8.0) : sqrt(2.0 / 8.0);",
+        "return k == 0 ? 0.5 : sqrt(2.0 / 8.0);"),
+    "idct_no_half_sample": (
+        "S[u * 8 + v] *\n                         cos((2 * m + 1) * u * PIC_ORACLE_PI / 16.0)",
+        "S[u * 8 + v] *\n                         cos((2 * m) * u * PIC_ORACLE_PI / 16.0)"),
+    "patches_column_major": (
+        "for (int by = 0; by < (Hl + 7) / 8; ++by)\n                for (int bx = 0; bx < (Wl + 7) / 8; ++bx, ++b) {\n                    double S[64], x[64];",
+        "for (int bx = 0; bx < (Wl + 7) / 8; ++bx)\n                for (int by = 0; by < (Hl + 7) / 8; ++by, ++b) {\n                    double S[64], x[64];"),
+    "patch_step_ignored": (
+        "S[k] = (double)symbols[64 * b + k] * steps[l];",
+        "S[k] = (double)symbols[64 * b + k];"),
+    "patch_written_transposed": (
+        "if (r < Hl && q < Wl) g[(int64_t)r * Wl + q] = x[m * 8 + n];",
+        "if (r < Hl && q < Wl) g[(int64_t)r * Wl + q] = x[n * 8 + m];"),
+    "block_count_floor": (
+        "n += (int64_t)C * ((level_size(H, l) + 7) / 8) * ((level_size(W, l) + 7) / 8);",
+        "n += (int64_t)C * (level_size(H, l) / 8 + 1) * (level_size(W, l) / 8 + 1);"),
+    "value_levels_ignore_channels": (
+        "off += (int64_t)C * level_size(H, l) * level_size(W, l);\n    }\n}\n\n/* Steps 2-5",
+        "off += (int64_t)level_size(H, l) * level_size(W, l);\n    }\n}\n\n/* Steps 2-5"),
     "izpr_raster_not_zigzag": (
         "blk[order[pos++]] = s;",
         "blk[pos++] = s;"),
