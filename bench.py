@@ -66,7 +66,7 @@ def algorithmic(wl: wk.Workload, batch: int):
 
 
 KERNEL_SOURCES = {
-    "tc": ["k_tc.cu", "tc_ptx.cuh", "pic_common.cuh", "pic_gelu.cuh", "pic_kernels.h"],
+    "tc": ["k_tc.cuh", "tc_ptx.cuh", "pic_common.cuh", "pic_gelu.cuh", "pic_kernels.h"],
     "fp32": ["k_fp32.cu", "pic_common.cuh", "pic_gelu.cuh", "pic_kernels.h"],
 }
 

@@ -69,6 +69,15 @@ typedef enum {
     PIC_PREC_FP16_TC = 1
 } pic_prec;
 
+typedef enum {
+    /* int32 latent symbols q; the decode dequantises them, y_l = q * step_l. */
+    PIC_LATENT_INT32 = 0,
+    /* fp32 real latents, already dequantised -- the output of the inverse DCT
+     * stage of pic_idct.h (Fig. 1: iDCT then g_r).  `steps` is not read and
+     * may be NULL. */
+    PIC_LATENT_FP32 = 1
+} pic_latent_format;
+
 /* Architecture of one decoder instance (fixed at create). */
 typedef struct {
     int num_levels;         /* L, 1..12 */
@@ -80,6 +89,7 @@ typedef struct {
     int clamp_output;       /* 1: clamp to [0, 1] (the decode); 0: raw MLP output */
     int max_H, max_W;       /* largest image accepted by the decode calls */
     int max_batch;          /* largest B accepted by pic_decode_batch */
+    int latent_format;      /* pic_latent_format; same layout and size (4 B) either way */
 } pic_arch;
 
 /*
@@ -95,10 +105,13 @@ int pic_decode_create(const pic_arch *arch, pic_decoder **out);
 
 /*
  * Decodes one image (steps 1-5 above) on `stream`.
- *   latents : int32, device; levels l = 0..L-1 concatenated, each planar
+ *   latents : device; levels l = 0..L-1 concatenated, each planar
  *             [C][H_l][W_l] row-major, H_l = ceil(H / 2^l), W_l = ceil(W / 2^l);
- *             pic_latent_count(H, W, L, C) values.
- *   steps   : float, device; [L] dequantisation step of each level.
+ *             pic_latent_count(H, W, L, C) values: int32 symbols, or fp32
+ *             values (passed through the same pointer) when the arch's
+ *             latent_format is PIC_LATENT_FP32.
+ *   steps   : float, device; [L] dequantisation step of each level (not read,
+ *             and may be NULL, for PIC_LATENT_FP32).
  *   weights : device; for k = 0..n-1: W_k [dims[k+1]][dims[k]] row-major, then
  *             b_k [dims[k+1]]; pic_param_count(arch) values; float for
  *             PIC_PREC_FP32, IEEE half (uint16 bits) for PIC_PREC_FP16_TC.

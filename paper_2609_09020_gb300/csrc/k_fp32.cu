@@ -108,7 +108,7 @@ struct Fp32Net {
   }
 };
 
-template <int C, int NL, int D0, int D1, int D2, int D3, int D4, int ACT>
+template <int C, int NL, int D0, int D1, int D2, int D3, int D4, int ACT, bool FL>
 __global__ void __launch_bounds__(kThreads)
     fp32_decode_kernel(const DecodeParams p) {
   using Net = Fp32Net<C, NL, D0, D1, D2, D3, D4, ACT>;
@@ -135,7 +135,7 @@ __global__ void __launch_bounds__(kThreads)
       load_weights_fp32<NL, D0, D1, D2, D3, D4>(sm_w, wts + b * p.params_per_image);
       __syncthreads();
 #pragma unroll
-      for (int l = 0; l < L; ++l) step[l] = __ldg(p.steps + b * L + l);
+      for (int l = 0; l < L; ++l) step[l] = FL ? 1.0f : __ldg(p.steps + b * L + l);
       cur_b = b;
     }
     if (x >= p.W) continue;
@@ -149,13 +149,13 @@ __global__ void __launch_bounds__(kThreads)
       if (l == 0) {  // level 0 has the output size: the upsampling is the identity
 #pragma unroll
         for (int c = 0; c < C; ++c)
-          h[c] = step[0] * static_cast<float>(__ldg(lat + c * plane + static_cast<long long>(y) * p.W + x));
+          h[c] = step[0] * lat_value<FL>(__ldg(lat + c * plane + static_cast<long long>(y) * p.W + x));
       } else {
         const Tap tx = bilinear_tap(x, lg.sx, lg.W);
         const Tap ty = bilinear_tap(y, lg.sy, lg.H);
 #pragma unroll
         for (int c = 0; c < C; ++c)
-          h[l * C + c] = step[l] * bilinear_sample(lat + lg.off + static_cast<long long>(c) * lg.H * lg.W,
+          h[l * C + c] = step[l] * bilinear_sample<FL>(lat + lg.off + static_cast<long long>(c) * lg.H * lg.W,
                                                    lg.W, tx, ty);
       }
     }
@@ -198,6 +198,7 @@ __global__ void __launch_bounds__(kThreads)
 // Generic fallback: any dims up to kMaxDim, runtime loops, weights in shared
 // memory in the nn.Linear layout.  Slower (hidden values in local memory) but
 // covers every arch the C ABI accepts.
+template <bool FL>
 __global__ void __launch_bounds__(kThreads) fp32_generic_kernel(const DecodeParams p) {
   extern __shared__ __align__(16) float sm_w[];
   const long long chunk = (p.total_tiles + gridDim.x - 1) / gridDim.x;
@@ -224,11 +225,11 @@ __global__ void __launch_bounds__(kThreads) fp32_generic_kernel(const DecodePara
     float h[kMaxDim], g[kMaxDim];
     for (int l = 0; l < p.L; ++l) {
       const LevelGeom lg = p.lv[l];
-      const float s = __ldg(p.steps + b * p.L + l);
+      const float s = FL ? 1.0f : __ldg(p.steps + b * p.L + l);
       const Tap tx = bilinear_tap(x, lg.sx, lg.W);
       const Tap ty = bilinear_tap(y, lg.sy, lg.H);
       for (int c = 0; c < p.C; ++c)
-        h[l * p.C + c] = s * bilinear_sample(lat + lg.off + static_cast<long long>(c) * lg.H * lg.W,
+        h[l * p.C + c] = s * bilinear_sample<FL>(lat + lg.off + static_cast<long long>(c) * lg.H * lg.W,
                                              lg.W, tx, ty);
     }
     const float* wl = sm_w;
@@ -248,12 +249,13 @@ __global__ void __launch_bounds__(kThreads) fp32_generic_kernel(const DecodePara
   }
 }
 
-template <int C, int NL, int D0, int D1, int D2, int D3, int D4, int ACT>
+template <int C, int NL, int D0, int D1, int D2, int D3, int D4, int ACT, bool FL = false>
 KernelInfo make_fp32(const char* name) {
   using Net = Fp32Net<C, NL, D0, D1, D2, D3, D4, ACT>;
   KernelInfo k{};
   k.name = name;
   k.precision = 0;
+  k.latent_format = FL ? 1 : 0;
   k.C = C;
   k.n_layers = NL;
   const int d[5] = {D0, D1, D2, D3, D4};
@@ -262,7 +264,7 @@ KernelInfo make_fp32(const char* name) {
   k.threads = kThreads;
   k.tile_px = kThreads;
   k.smem_bytes = Net::smem_floats() * 4;
-  k.fn = reinterpret_cast<const void*>(&fp32_decode_kernel<C, NL, D0, D1, D2, D3, D4, ACT>);
+  k.fn = reinterpret_cast<const void*>(&fp32_decode_kernel<C, NL, D0, D1, D2, D3, D4, ACT, FL>);
   return k;
 }
 
@@ -277,21 +279,24 @@ int fp32_kernels(KernelInfo* out, int cap) {
       make_fp32<2, 3, 14, 64, 64, 3, 0, ACT_RELU>("fp32_14x64x64x3_relu"),
       make_fp32<2, 4, 16, 64, 64, 64, 3, ACT_GELU>("fp32_16x64x64x64x3_gelu"),
       make_fp32<1, 3, 7, 64, 64, 3, 0, ACT_RELU>("fp32_7x64x64x3_relu"),
+      make_fp32<1, 3, 7, 64, 64, 3, 0, ACT_RELU, true>("fp32_7x64x64x3_relu_f32lat"),
   };
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
   for (int i = 0; i < n && i < cap; ++i) out[i] = list[i];
   return n;
 }
 
-KernelInfo fp32_generic_kernel_info() {
+KernelInfo fp32_generic_kernel_info(int latent_format) {
   KernelInfo k{};
-  k.name = "fp32_generic";
+  k.name = latent_format ? "fp32_generic_f32lat" : "fp32_generic";
   k.precision = 0;
+  k.latent_format = latent_format ? 1 : 0;
   k.generic = 1;
   k.threads = kThreads;
   k.tile_px = kThreads;
   k.smem_bytes = 0;  // set per arch: params_per_image * 4
-  k.fn = reinterpret_cast<const void*>(&fp32_generic_kernel);
+  k.fn = latent_format ? reinterpret_cast<const void*>(&fp32_generic_kernel<true>)
+                      : reinterpret_cast<const void*>(&fp32_generic_kernel<false>);
   return k;
 }
 

@@ -1,626 +1,29 @@
-// k_tc.cu -- fused decode on the 5th-generation tensor cores (PIC_PREC_FP16_TC).
-//
-// The synthesis MLP g_s (Sec. 4.1) runs as a chain of tcgen05 MMAs with the
-// accumulators in tensor memory (TMEM); dequantisation, bilinear upsampling
-// and concatenation of the pyramid levels (Sec. 3.1, Eq. 1) produce the first
-// layer's operand directly in shared memory, and the clamped RGB leaves the
-// last accumulator straight for global memory.  Nothing between the latents
-// and the RGB planes touches HBM.
-//
-// Precision: weights are fp16 (used exactly as given).  Every activation
-// operand a (feature or hidden value, fp32) is split into two fp16 terms
-//   a_hi = a rounded toward zero to fp16,
-//   a_lo = fp16(a - a_hi)      (a - a_hi is exact in fp32 and has a's sign,
-//                               so ReLU may be applied to each term alone),
-// and each layer computes W a_hi + W a_lo with fp32 accumulation, so the
-// products carry ~22 significant bits instead of fp16's 11.
-//
-// Operands of one 128-pixel tile (row r = pixel r = TMEM lane r):
-//   layer 0  A1 = [f_hi | f_lo | 1 | 0..]  smem, K1 = round16(2 D0 + 1); the bias
-//            B1 = [W_0  | W_0  | b_0 | 0..] b_0 rides along as the constant-1 column
-//   hidden   A  = [h_hi | h_lo]            TMEM, N/2 + N/2 columns (2 fp16 per column)
-//            B  = [W_k | b_k 0..0]          smem; W_k serves the hi and the lo half,
-//                                           b_k meets a shared constant tile [1 0..0]
-//   output   the same with W_out, b_out padded to 16 rows
-//
-// CTA organisation (one CTA per SM, persistent over a contiguous tile range):
-//   warps 0 .. 4*NWG-1 : NWG warpgroups; group w owns every NWG-th tile of the
-//                        range, TMEM columns [2Nw, 2Nw + 2N) (accumulator,
-//                        then operand A) and shared buffers (A1, column
-//                        buffer).  Thread r of the group decodes pixel r.
-//                        The features of the group's next tile are computed
-//                        while the tensor core runs the current tile's
-//                        second layer, and handed over once the current
-//                        accumulator has been read.
-//   warp 4*NWG         : issues every MMA (one elected lane) to whichever
-//                        group has its operand ready, then tcgen05.commit.
-// Handshakes are mbarriers; every wait is bounded (on timeout the kernel
-// raises the handle's status word, skips the rest and still frees TMEM).
-#include <cuda_fp16.h>
-
-#include <type_traits>
-
-#include "pic_common.cuh"
-#include "pic_kernels.h"
-#include "tc_ptx.cuh"
+// k_tc.cu -- instantiations of the tensor-core decode kernel (k_tc.cuh) for
+// int32 latent symbols, one per decode workload architecture, and the
+// registry of both latent formats.
+#include "k_tc.cuh"
 
 namespace pic {
 namespace {
-
-using namespace tc;
-
-constexpr int kTile = 128;
-constexpr uint32_t kSpinLimit = 1u << 22;  // a few seconds of polling at most per wait
-
-__host__ __device__ constexpr int round_up(int v, int m) { return (v + m - 1) / m * m; }
-__host__ __device__ constexpr int pow2_at_least(int v) {
-  int p = 32;
-  while (p < v) p *= 2;
-  return p;
-}
-
-// Byte offset of element (row, k) in a [rows][K] fp16 tile stored K-major in
-// the canonical no-swizzle layout: core matrix (row/8, k/8) at
-// (row/8) * SBO + (k/8) * LBO with LBO = 128 B and SBO = 16 K bytes.
-__host__ __device__ constexpr uint32_t kmaj(int row, int k, int K) {
-  return static_cast<uint32_t>((row >> 3) * (K * 16) + (k >> 3) * 128 + (row & 7) * 16 + (k & 7) * 2);
-}
-
-// Cooperative feature staging.  For level l >= 1 a 128-pixel row segment
-// needs at most NCOL(l) = 128/2^l + 4 source columns.  The warpgroup first
-// interpolates those columns vertically (rows v0, v1 of the level, weight
-// beta) into a small shared buffer -- one item per (level, channel, column),
-// spread over the 128 threads -- and every pixel then interpolates
-// horizontally between two buffer entries.  Column indices are clamped into
-// [0, W_l - 1] when the buffer is filled, which reproduces the edge clamp of
-// the bilinear definition.
-__host__ __device__ constexpr int ncol(int l) { return (kTile >> l) + 4; }
-
-template <int L, int C>
-struct ColLayout {
-  // float offset of (level l, channel c) inside the column buffer
-  static constexpr int off(int l, int c) {
-    int o = 0;
-    for (int k = 1; k < l; ++k) o += C * ncol(k);
-    return o + c * ncol(l);
-  }
-  static constexpr int total() { return off(L, 0); }
-};
-
-template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_>
-struct TcNet {
-  static constexpr int C = C_, NL = NL_, D0 = D0_, N = N_, ACT = ACT_, NWG = NWG_;
-  static constexpr int L = D0 / C;
-  static constexpr int K1 = round_up(2 * D0 + 1, 16);
-  static constexpr int NOUT = 16;
-  static constexpr int NISSUE = NWG;                  // one MMA-issuing warp per group
-  static constexpr int THREADS = NWG * 128 + 32 * NISSUE;
-  static constexpr int MMA_WARP = NWG * 4;            // first issuing warp (also owns TMEM)
-  // Registers per thread that still let one CTA fit an SM: the warps are
-  // spread over the 4 sub-partitions, each with a 16K-register file.
-  static constexpr int WARPS_PER_SMSP = (THREADS / 32 + 3) / 4;
-  static constexpr int MAXREG_RAW = 16384 / (32 * WARPS_PER_SMSP) / 8 * 8;
-  static constexpr int MAXREG = MAXREG_RAW > 255 ? 255 : MAXREG_RAW;
-  static constexpr int CTRL = 256;
-  static constexpr int B1_BYTES = N * K1 * 2;
-  static constexpr int KB = N + 16;                      // [W | b 0..0]
-  static constexpr int BH_BYTES = N * KB * 2;
-  static constexpr int BO_BYTES = NOUT * KB * 2;
-  static constexpr int ONES_BYTES = kTile * 16 * 2;      // constant A tile [1 0..0] per row
-  static constexpr int OFF_B1 = CTRL;
-  static constexpr int OFF_BH = OFF_B1 + B1_BYTES;
-  static constexpr int OFF_BO = OFF_BH + (NL - 2) * BH_BYTES;
-  static constexpr int OFF_ONES = round_up(OFF_BO + BO_BYTES, 128);
-  static constexpr int OFF_WG = round_up(OFF_ONES + ONES_BYTES, 128);
-  static constexpr int A1_BYTES = kTile * K1 * 2;
-  static constexpr int COL_BYTES = round_up(ColLayout<L, C>::total() * 4, 128);
-  static constexpr int NITEM_PER_THREAD = (ColLayout<L, C>::total() + kTile - 1) / kTile;
-  static constexpr int STAGE_SLOTS = C + 2 * NITEM_PER_THREAD;  // raw int32 loads per thread
-  static constexpr int STAGE_BYTES = STAGE_SLOTS * kTile * 4;
-  static constexpr int WG_BYTES = A1_BYTES + COL_BYTES + STAGE_BYTES;
-  static constexpr int SMEM = OFF_WG + NWG * WG_BYTES;
-  static constexpr int TMEM_COLS = pow2_at_least(NWG * 2 * N);
-  static_assert(N % 16 == 0 && N >= 16 && N <= 128, "hidden width must be 16..128, multiple of 16");
-  static_assert(NL >= 2, "the tensor-core path needs at least one hidden layer");
-  static_assert(TMEM_COLS <= 512, "tensor memory holds 512 columns");
-  static_assert(8 * (4 * NWG + NISSUE) <= 224, "control block holds the barriers");
-};
-
-// Bounded mbarrier wait.  Returns false (and raises the abort flag and the
-// handle's status word) if the phase does not complete in time, or if
-// another thread has already aborted.
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                             int* status) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    if (mbar_try_wait_sleep(bar, parity)) return true;
-    if ((i & 63u) == 63u) {
-      if (*abort_flag) return false;
-      if (i > 4096) __nanosleep(64);
-    }
-  }
-  *abort_flag = 1;
-  atomicOr(status, 1);
-  return false;
-}
-
-__device__ __forceinline__ __half ldh(const __half* p) {
-  return __ushort_as_half(__ldg(reinterpret_cast<const unsigned short*>(p)));
-}
-
-// Fills the weight operands and biases of one image into shared memory (all threads).
-template <class Net>
-__device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
-                                                const int (&dims)[Net::NL + 1]) {
-  constexpr int N = Net::N, D0 = Net::D0, K1 = Net::K1, NL = Net::NL, KB = Net::KB;
-  const __half zero = __float2half_rn(0.0f);
-  // layer 0: [W | W | b | 0]
-  {
-    const int d1 = dims[1];
-    const __half* W0 = w;
-    const __half* b0 = w + d1 * D0;
-    for (int e = threadIdx.x; e < N * K1; e += blockDim.x) {
-      const int n = e / K1, j = e - n * K1;
-      __half v = zero;
-      if (n < d1) {
-        if (j < D0) v = ldh(W0 + n * D0 + j);
-        else if (j < 2 * D0) v = ldh(W0 + n * D0 + (j - D0));
-        else if (j == 2 * D0) v = ldh(b0 + n);
-      }
-      *reinterpret_cast<__half*>(smem + Net::OFF_B1 + kmaj(n, j, K1)) = v;
-    }
-  }
-  // hidden layers and output: [W | b 0..0], zero padded to N (or 16) rows
-  const __half* p = w + dims[1] * D0 + dims[1];
-#pragma unroll
-  for (int k = 1; k < NL; ++k) {
-    const int din = dims[k], dout = dims[k + 1];
-    const bool out_layer = (k == NL - 1);
-    const int rows = out_layer ? Net::NOUT : N;
-    uint8_t* base = smem + (out_layer ? Net::OFF_BO : Net::OFF_BH + (k - 1) * Net::BH_BYTES);
-    const __half* Wk = p;
-    const __half* bk = p + dout * din;
-    for (int e = threadIdx.x; e < rows * KB; e += blockDim.x) {
-      const int n = e / KB, j = e - n * KB;
-      __half v = zero;
-      if (n < dout) {
-        if (j < din) v = ldh(Wk + n * din + j);
-        else if (j == N) v = ldh(bk + n);
-      }
-      *reinterpret_cast<__half*>(base + kmaj(n, j, KB)) = v;
-    }
-    p = bk + dout;
-  }
-}
-
-// Splits v into (hi, lo) fp32 parts: hi = v rounded toward zero to fp16
-// (exactly representable), lo = v - hi (exact in fp32).
-__device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
-  hi = __half2float(__float2half_rz(v));
-  lo = v - hi;
-}
-
-template <class Net>
-__global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
-    tc_decode_kernel(const DecodeParams p) {
-  constexpr int N = Net::N, NL = Net::NL, C = Net::C, L = Net::L, D0 = Net::D0, NWG = Net::NWG;
-  constexpr int K1 = Net::K1;
-  using CL = ColLayout<L, C>;
-  constexpr int NITEM = CL::total();
-  constexpr int J = (NITEM + kTile - 1) / kTile;  // column items per thread (0 if L == 1)
-  constexpr int JJ = J > 0 ? J : 1;
-  extern __shared__ __align__(1024) uint8_t smem[];
-
-  const int warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  const uint32_t sbase = smem_addr(smem);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + 224);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + 232);
-  // mbarriers, 8 bytes each: per group w a1_full (features written),
-  // a_full (hidden operand written), acc_full (MMAs done), col_ready; one drain.
-  const uint32_t bar_a1 = sbase;
-  const uint32_t bar_a = sbase + 8 * NWG;
-  const uint32_t bar_c = sbase + 16 * NWG;
-  const uint32_t bar_col = sbase + 24 * NWG;
-  const uint32_t bar_drain = sbase + 32 * NWG;  // + 8 m for issuing warp m
-
-  if (threadIdx.x == 0) {
-    for (int w = 0; w < NWG; ++w) {
-      mbar_init(bar_a1 + 8 * w, 128);
-      mbar_init(bar_a + 8 * w, 128);
-      mbar_init(bar_c + 8 * w, 1);
-      mbar_init(bar_col + 8 * w, 128);
-    }
-    for (int m = 0; m < Net::NISSUE; ++m) mbar_init(bar_drain + 8 * m, 1);
-    *abort_flag = 0;
-    fence_mbar_init();
-  }
-  if (warp == Net::MMA_WARP) {
-    tmem_alloc(smem_addr(tmem_slot), Net::TMEM_COLS);
-    tmem_relinquish();
-  }
-  for (int e = threadIdx.x; e < kTile * 2; e += blockDim.x) {  // 16-byte chunks of the ones tile
-    const int row = e >> 1, kc = e & 1;
-    sts128(sbase + Net::OFF_ONES + kmaj(row, kc * 8, 16), kc == 0 ? 0x00003C00u : 0u, 0u, 0u, 0u);
-  }
-  fence_async_smem();
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-
-  const long long chunk = (p.total_tiles + gridDim.x - 1) / gridDim.x;
-  const long long t_begin = blockIdx.x * chunk;
-  const long long t_end = min(t_begin + chunk, p.total_tiles);
-  const __half* wts = static_cast<const __half*>(p.weights);
-  const long long plane = static_cast<long long>(p.H) * p.W;
-  // x-taps repeat from tile to tile when every level's width is exactly W / 2^l
-  // (and 2^l divides the 128-pixel tile origin, i.e. l <= 7)
-  const bool fast_x = (L - 1 <= 7) && (p.W % (1 << (L - 1))) == 0;
-
-  uint32_t acc_phase = 0;  // warpgroup threads: parity of their acc_full
-  uint32_t col_phase = 0;  // warpgroup threads: parity of their col_ready
-  uint32_t a1_phase = 0;   // MMA warp: bit w = parity of a1_full[w]
-  uint32_t a_phase = 0;    // MMA warp: bit w = parity of a_full[w]
-
-  for (long long seg = t_begin; seg < t_end;) {
-    const int b = static_cast<int>(seg / p.tiles_per_image);
-    const long long seg_end = min(t_end, static_cast<long long>(b + 1) * p.tiles_per_image);
-    __syncthreads();  // all MMAs and reads of the previous image's weights are done
-    {
-      int dims[NL + 1];
-#pragma unroll
-      for (int k = 0; k <= NL; ++k) dims[k] = p.dims[k];
-      load_weights_tc<Net>(smem, wts + b * p.params_per_image, dims);
-    }
-    fence_async_smem();
-    __syncthreads();
-    const int n_tiles = static_cast<int>(seg_end - seg);
-    const long long tile0 = seg - static_cast<long long>(b) * p.tiles_per_image;  // in-image index
-
-    if (warp < 4 * NWG) {
-      // ------------------------------------------------------------ warpgroup
-      const int w = warp >> 2;
-      const int r = ((warp & 3) << 5) | lane;  // tile row = TMEM lane = pixel
-      uint8_t* a1 = smem + Net::OFF_WG + w * Net::WG_BYTES;
-      const uint32_t a1_s = smem_addr(a1);
-      float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES);
-      const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
-      const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(w * 2 * N);
-      const uint32_t t_a = t_acc + N;  // hi in [0, N/2), lo in [N/2, N)
-      const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w,
-                     my_col = bar_col + 8 * w;
-      const int32_t* lat = p.latents + b * p.lat_per_image;
-      float step[L];
-#pragma unroll
-      for (int l = 0; l < L; ++l) step[l] = __ldg(p.steps + b * L + l);
-
-      // This thread's column items: level, column, and the level's geometry.
-      int it_l[JJ], it_i[JJ], it_W[JJ], it_H[JJ];
-      long long it_off[JJ];
-      float it_sy[JJ], it_sx[JJ];
-#pragma unroll
-      for (int j = 0; j < J; ++j) {
-        int e = r + kTile * j, l = 0, c = 0, i = 0;
-        if (e < NITEM) {
-#pragma unroll
-          for (int lv = 1; lv < L; ++lv)
-#pragma unroll
-            for (int cc = 0; cc < C; ++cc)
-              if (e >= CL::off(lv, cc) && e < CL::off(lv, cc) + ncol(lv)) {
-                l = lv;
-                c = cc;
-                i = e - CL::off(lv, cc);
-              }
-        }
-        it_l[j] = l;  // l == 0 marks an idle slot
-        it_i[j] = i;
-        const LevelGeom lg = p.lv[l];
-        it_W[j] = lg.W;
-        it_H[j] = lg.H;
-        it_off[j] = lg.off + static_cast<long long>(c) * lg.H * lg.W;
-        it_sy[j] = lg.sy;
-        it_sx[j] = lg.sx;
-      }
-      // Relative x-taps of pixel r for each level (used when fast_x): the
-      // source coordinate (r + 1/2) / 2^l - 1/2 relative to column x0/2^l - 1.
-      int rel[L];
-      float fx[L];
-#pragma unroll
-      for (int l = 1; l < L; ++l) {
-        const float sx = (static_cast<float>(r) + 0.5f) * (1.0f / static_cast<float>(1 << l)) - 0.5f;
-        const float fl = floorf(sx);
-        rel[l] = static_cast<int>(fl) + 1;
-        fx[l] = sx - fl;
-      }
-
-      // Global loads tile (y, x0) needs -- the level-0 values of pixel r and
-      // the raw texel pairs of this thread's column items -- issued as
-      // asynchronous copies into this thread's column of the staging buffer
-      // (slot s of thread r at stage[s * 128 + r]); nothing waits on them
-      // until the features are computed.
-      const uint32_t stage_s = a1_s + Net::A1_BYTES + Net::COL_BYTES;
-      const int* stage = reinterpret_cast<const int*>(a1 + Net::A1_BYTES + Net::COL_BYTES);
-      auto prefetch = [&](int y, int x0) {
-        const int xc = min(x0 + r, p.W - 1);
-#pragma unroll
-        for (int c = 0; c < C; ++c)
-          cp_async4(stage_s + (c * kTile + r) * 4, lat + c * plane + static_cast<long long>(y) * p.W + xc);
-#pragma unroll
-        for (int j = 0; j < J; ++j) {
-          const int l = it_l[j];
-          if (l > 0) {
-            const Tap ty = bilinear_tap(y, it_sy[j], it_H[j]);
-            const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, it_sx[j], it_W[j]).i0;
-            const int u = min(max(u_start + it_i[j], 0), it_W[j] - 1);
-            const int32_t* pl = lat + it_off[j] + u;
-            cp_async4(stage_s + ((C + 2 * j) * kTile + r) * 4, pl + ty.i0 * it_W[j]);
-            cp_async4(stage_s + ((C + 2 * j + 1) * kTile + r) * 4, pl + ty.i1 * it_W[j]);
-          }
-        }
-        cp_async_commit();
-      };
-
-      // Features of tile (y, x0) from its prefetched loads -> A1 (shared).
-      // Returns false if a wait gave up.
-      auto features = [&](int y, int x0) -> bool {
-        cp_async_wait_all();  // this thread's staged loads have landed
-        // vertical pass into the column buffer
-#pragma unroll
-        for (int j = 0; j < J; ++j) {
-          const int l = it_l[j];
-          if (l > 0) {
-            const float beta = bilinear_tap(y, it_sy[j], it_H[j]).frac;
-            const int t0 = stage[(C + 2 * j) * kTile + r], t1 = stage[(C + 2 * j + 1) * kTile + r];
-            colbuf[r + kTile * j] = step[l] * fmaf(beta, static_cast<float>(t1 - t0), static_cast<float>(t0));
-          }
-        }
-        mbar_arrive(my_col);  // the group's column buffer is complete once all 128 arrived
-        if (!__all_sync(0xffffffffu, wait_bounded(my_col, col_phase, abort_flag, p.status)))
-          return false;
-        col_phase ^= 1u;
-        // horizontal pass + level 0
-        const int xc = min(x0 + r, p.W - 1);
-        float f[D0];
-#pragma unroll
-        for (int c = 0; c < C; ++c) f[c] = step[0] * static_cast<float>(stage[c * kTile + r]);
-#pragma unroll
-        for (int l = 1; l < L; ++l) {
-          int i0, i1;
-          float a;
-          if (fast_x) {
-            i0 = rel[l];
-            i1 = rel[l] + 1;
-            a = fx[l];
-          } else {
-            const LevelGeom lg = p.lv[l];
-            const int u_start = bilinear_tap(x0, lg.sx, lg.W).i0;
-            const Tap tx = bilinear_tap(xc, lg.sx, lg.W);
-            i0 = min(max(tx.i0 - u_start, 0), ncol(l) - 1);
-            i1 = min(max(tx.i1 - u_start, 0), ncol(l) - 1);
-            a = tx.frac;
-          }
-#pragma unroll
-          for (int c = 0; c < C; ++c) {
-            const float* cb = colbuf + CL::off(l, c);
-            const float v0 = cb[i0], v1 = cb[i1];
-            f[l * C + c] = fmaf(a, v1 - v0, v0);
-          }
-        }
-        // hi/lo split, the constant-1 bias column, padding -> A1
-        float v[K1];
-#pragma unroll
-        for (int j = 0; j < K1; ++j) v[j] = 0.0f;
-#pragma unroll
-        for (int j = 0; j < D0; ++j) split_hi_lo(f[j], v[j], v[D0 + j]);
-        v[2 * D0] = 1.0f;
-#pragma unroll
-        for (int kc = 0; kc < K1 / 8; ++kc)
-          sts128(a1_s + kmaj(r, kc * 8, K1), pack_f16x2(v[kc * 8 + 0], v[kc * 8 + 1]),
-                 pack_f16x2(v[kc * 8 + 2], v[kc * 8 + 3]), pack_f16x2(v[kc * 8 + 4], v[kc * 8 + 5]),
-                 pack_f16x2(v[kc * 8 + 6], v[kc * 8 + 7]));
-        fence_async_smem();
-        return true;
-      };
-
-      // Hidden epilogue: accumulator -> activation -> hi/lo -> TMEM operand.
-      auto hidden_epilogue = [&]() {
-#pragma unroll
-        for (int h0 = 0; h0 < N; h0 += 16) {  // 16 columns at a time (fewer live registers)
-          constexpr int HW = 16;
-          uint32_t acc[HW];
-#pragma unroll
-          for (int c0 = 0; c0 < HW; c0 += 16) tmem_ld16(t_acc + h0 + c0, acc + c0);
-          tmem_ld_wait();
-          uint32_t hl[HW];  // [0, HW/2): hi pairs, [HW/2, HW): lo pairs
-#pragma unroll
-          for (int q = 0; q < HW / 2; ++q) {
-            float a = __uint_as_float(acc[2 * q]);
-            float bb = __uint_as_float(acc[2 * q + 1]);
-            if constexpr (Net::ACT == ACT_GELU) {
-              a = gelu_poly(a);
-              bb = gelu_poly(bb);
-            }
-            // hi = fp16 truncation (ReLU folded in), lo = v - hi (packed subtraction)
-            split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[HW / 2 + q]);
-          }
-          // hi pair (h0/2 + q) -> column t_a + h0/2 + q; lo pair -> t_a + N/2 + h0/2 + q
-          tmem_st8(t_a + h0 / 2, hl);
-          tmem_st8(t_a + N / 2 + h0 / 2, hl + 8);
-        }
-        tmem_st_wait();
-      };
-
-      // Tile cursor (row y, tile column tx) of this group's current tile and
-      // of the one after it, advanced by NWG tiles without divisions.
-      const int tpr = p.tiles_per_row;
-      int cy = static_cast<int>((tile0 + w) / tpr);
-      int ctx = static_cast<int>((tile0 + w) - static_cast<long long>(cy) * tpr);
-      auto advance = [&](int& yy, int& xx) {
-        xx += NWG;
-        while (xx >= tpr) {
-          xx -= tpr;
-          ++yy;
-        }
-      };
-
-      bool ok = true;
-      if (w < n_tiles) {
-        prefetch(cy, ctx * kTile);
-        ok = features(cy, ctx * kTile);
-        if (ok) mbar_arrive(my_a1);
-      }
-      for (int i = w; i < n_tiles && ok; i += NWG) {
-        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
-        const int y = cy;
-        const int x0 = ctx * kTile;
-        int ny = cy, ntx = ctx;
-        advance(ny, ntx);
-        const bool has_next = i + NWG < n_tiles;
-        if (has_next) prefetch(ny, ntx * kTile);  // in flight during the first epilogue
-
-        for (int k = 0; k < NL - 1 && ok; ++k) {
-          if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
-            ok = false;
-            break;
-          }
-          acc_phase ^= 1u;
-          tc_fence_after();
-          hidden_epilogue();
-          tc_fence_before();
-          mbar_arrive(my_a);
-          if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
-        }
-        if (!ok) break;
-
-        // ---- output layer: bias, clamp, planar coalesced store ----
-        if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
-        acc_phase ^= 1u;
-        tc_fence_after();
-        uint32_t o[4];
-        tmem_ld4(t_acc, o);
-        tmem_ld_wait();
-        tc_fence_before();
-        if (has_next) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
-        const int x = x0 + r;
-        if (x < p.W) {
-          float* dst = p.out + static_cast<long long>(b) * 3 * plane + static_cast<long long>(y) * p.W + x;
-#pragma unroll
-          for (int c = 0; c < 3; ++c) {
-            const float v = __uint_as_float(o[c]);
-            dst[c * plane] = p.clamp ? __saturatef(v) : v;
-          }
-        }
-        cy = ny;
-        ctx = ntx;
-      }
-    } else if (warp >= Net::MMA_WARP && warp < Net::MMA_WARP + Net::NISSUE) {
-      // --------------------------------------------------------------- MMA issuer
-      // Warp MMA_WARP + w issues every MMA of group w, in the group's order
-      // (its tiles in turn, layers in turn), sleeping in the mbarrier wait
-      // in between.  The whole warp runs the control flow (descriptors stay
-      // warp-uniform); one elected lane issues the MMAs and the commit.
-      // Descriptors depend on the start address only through their low
-      // field: base + (offset >> 4).
-      const int w = warp - Net::MMA_WARP;
-      constexpr uint32_t id_hidden = idesc_f16(128, N);
-      constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
-      const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG + w * Net::WG_BYTES, 128, 16 * K1);
-      const uint64_t dB1 = smem_desc(sbase + Net::OFF_B1, 128, 16 * K1);
-      const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * Net::KB);
-      const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * Net::KB);
-      const uint64_t dONES = smem_desc(sbase + Net::OFF_ONES, 128, 16 * 16);
-      constexpr uint64_t kStep = 256 >> 4;              // one K-step (16 fp16) = 256 B
-      constexpr uint64_t kLayer = Net::BH_BYTES >> 4;   // next hidden layer's weights
-      static_assert(Net::WG_BYTES % 16 == 0 && Net::BH_BYTES % 16 == 0, "16-byte aligned operands");
-      const uint32_t d = tmem + static_cast<uint32_t>(w * 2 * N);
-      const uint32_t ta = d + N;
-      const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w;
-      bool ok = true;
-      for (int i = w; i < n_tiles && ok; i += NWG) {
-        for (int k = 0; k < NL; ++k) {
-          const uint32_t bar = k == 0 ? my_a1 : my_a;
-          const uint32_t par = k == 0 ? (a1_phase & 1u) : (a_phase & 1u);
-          if (!__all_sync(0xffffffffu, wait_bounded(bar, par, abort_flag, p.status))) {
-            ok = false;
-            break;
-          }
-          if (k == 0) a1_phase ^= 1u;
-          else a_phase ^= 1u;
-          if (elect_one()) {
-            tc_fence_after();
-            if (k == 0) {
-#pragma unroll
-              for (int s = 0; s < K1 / 16; ++s) mma_f16(d, dA1 + s * kStep, dB1 + s * kStep, id_hidden, s > 0);
-            } else {
-              const bool out_layer = (k == NL - 1);
-              const uint64_t db = out_layer ? dBO : dBH + (k - 1) * kLayer;
-              const uint32_t id = out_layer ? id_out : id_hidden;
-#pragma unroll
-              for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + 8 * s, db + s * kStep, id, s > 0);  // hi
-#pragma unroll
-              for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
-              mma_f16(d, dONES, db + (N / 16) * kStep, id, 1);  // bias: [1 0..0] x [b 0..0]
-            }
-            mma_commit(my_c);
-          }
-          __syncwarp();
-        }
-      }
-    }
-    __syncwarp();
-    seg = seg_end;
-  }
-
-  if (warp >= Net::MMA_WARP && warp < Net::MMA_WARP + Net::NISSUE && elect_one()) {
-    // Every MMA this thread issued must be complete before the memory goes.
-    const uint32_t drain = bar_drain + 8 * (warp - Net::MMA_WARP);
-    mma_commit(drain);
-    int dummy = 0;
-    wait_bounded(drain, 0, reinterpret_cast<volatile int*>(&dummy), p.status);
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == Net::MMA_WARP) {
-    tc_fence_after();
-    tmem_dealloc(tmem, Net::TMEM_COLS);
-  }
-}
-
-template <int C, int NL, int D0, int N, int ACT, int NWG>
-KernelInfo make_tc(const char* name, const int* dims) {
-  using Net = TcNet<C, NL, D0, N, ACT, NWG>;
-  KernelInfo k{};
-  k.name = name;
-  k.precision = 1;
-  k.C = C;
-  k.n_layers = NL;
-  for (int i = 0; i <= NL; ++i) k.dims[i] = dims[i];
-  k.act = ACT;
-  k.threads = Net::THREADS;
-  k.tile_px = kTile;
-  k.smem_bytes = Net::SMEM;
-  k.fn = reinterpret_cast<const void*>(&tc_decode_kernel<Net>);
-  return k;
-}
-
+const int d_c1[] = {4, 16, 16, 3};
+const int d_c2[] = {7, 40, 40, 3};
+const int d_c3[] = {14, 64, 64, 3};
+const int d_c4[] = {16, 64, 64, 64, 3};
+const int d_c5[] = {7, 64, 64, 3};
 }  // namespace
 
 int tc_kernels(KernelInfo* out, int cap) {
-  static const int d_c1[] = {4, 16, 16, 3};
-  static const int d_c2[] = {7, 40, 40, 3};
-  static const int d_c3[] = {14, 64, 64, 3};
-  static const int d_c4[] = {16, 64, 64, 64, 3};
-  static const int d_c5[] = {7, 64, 64, 3};
   const KernelInfo list[] = {
-      make_tc<1, 3, 7, 64, ACT_RELU, 4>("tc05_7x64x64x3_relu", d_c5),
-      make_tc<2, 4, 16, 64, ACT_GELU, 4>("tc05_16x64x64x64x3_gelu", d_c4),
-      make_tc<2, 3, 14, 64, ACT_RELU, 4>("tc05_14x64x64x3_relu", d_c3),
-      make_tc<1, 3, 7, 48, ACT_GELU, 4>("tc05_7x40x40x3_gelu", d_c2),
-      make_tc<1, 3, 4, 16, ACT_RELU, 4>("tc05_4x16x16x3_relu", d_c1),
+      make_tc<1, 3, 7, 64, ACT_RELU, 4, false>("tc05_7x64x64x3_relu", d_c5),
+      make_tc<2, 4, 16, 64, ACT_GELU, 4, false>("tc05_16x64x64x64x3_gelu", d_c4),
+      make_tc<2, 3, 14, 64, ACT_RELU, 4, false>("tc05_14x64x64x3_relu", d_c3),
+      make_tc<1, 3, 7, 48, ACT_GELU, 4, false>("tc05_7x40x40x3_gelu", d_c2),
+      make_tc<1, 3, 4, 16, ACT_RELU, 4, false>("tc05_4x16x16x3_relu", d_c1),
   };
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
-  for (int i = 0; i < n && i < cap; ++i) out[i] = list[i];
-  return n;
+  int k = 0;
+  for (; k < n && k < cap; ++k) out[k] = list[k];
+  return k + (k < cap ? tc_kernels_fp32lat(out + k, cap - k) : 0);
 }
 
 }  // namespace pic

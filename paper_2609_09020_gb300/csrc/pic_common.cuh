@@ -25,7 +25,7 @@ struct LevelGeom {
 
 // Everything a decode launch needs; passed by value (kernel parameter space).
 struct DecodeParams {
-  const int32_t* latents;
+  const int32_t* latents;      // int32 symbols, or fp32 values (PIC_LATENT_FP32) as 32-bit words
   const float* steps;
   const void* weights;
   float* out;
@@ -115,16 +115,37 @@ __device__ __forceinline__ Tap bilinear_tap(int x, float ratio, int n) {
   return t;
 }
 
-// One bilinear sample of integer grid `q` (row stride w), in fp32: the two
-// horizontal lerps use exact integer differences, then one vertical lerp.
+// Latent words: int32 symbols, or fp32 values carried in the same 32 bits
+// (FL = true, PIC_LATENT_FP32).
+template <bool FL>
+__device__ __forceinline__ float lat_value(int w) {
+  if constexpr (FL)
+    return __int_as_float(w);
+  else
+    return static_cast<float>(w);
+}
+// a + t (b - a); for symbols the difference b - a is exact in integers.
+template <bool FL>
+__device__ __forceinline__ float lat_lerp(int a, int b, float t) {
+  if constexpr (FL) {
+    const float fa = __int_as_float(a);
+    return fmaf(t, __int_as_float(b) - fa, fa);
+  } else {
+    return fmaf(t, static_cast<float>(b - a), static_cast<float>(a));
+  }
+}
+
+// One bilinear sample of latent grid `q` (row stride w), in fp32: two
+// horizontal lerps, then one vertical lerp.
+template <bool FL>
 __device__ __forceinline__ float bilinear_sample(const int32_t* __restrict__ q, int w, Tap tx,
                                                  Tap ty) {
   const int32_t* r0 = q + static_cast<long long>(ty.i0) * w;
   const int32_t* r1 = q + static_cast<long long>(ty.i1) * w;
   int a = __ldg(r0 + tx.i0), b = __ldg(r0 + tx.i1);
   int c = __ldg(r1 + tx.i0), d = __ldg(r1 + tx.i1);
-  float top = fmaf(tx.frac, static_cast<float>(b - a), static_cast<float>(a));
-  float bot = fmaf(tx.frac, static_cast<float>(d - c), static_cast<float>(c));
+  float top = lat_lerp<FL>(a, b, tx.frac);
+  float bot = lat_lerp<FL>(c, d, tx.frac);
   return fmaf(ty.frac, bot - top, top);
 }
 

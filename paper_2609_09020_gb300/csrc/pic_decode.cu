@@ -47,11 +47,13 @@ bool arch_valid(const pic_arch* a) {
   if (a->clamp_output != 0 && a->clamp_output != 1) return false;
   if (a->max_H < 1 || a->max_W < 1 || a->max_batch < 1) return false;
   if (a->max_H > 65536 || a->max_W > 65536 || a->max_batch > 65536) return false;
+  if (a->latent_format != PIC_LATENT_INT32 && a->latent_format != PIC_LATENT_FP32) return false;
   return true;
 }
 
 bool kernel_matches(const KernelInfo& k, const pic_arch* a) {
-  if (k.generic || k.precision != a->precision || k.C != a->channels_per_level ||
+  if (k.generic || k.precision != a->precision || k.latent_format != a->latent_format ||
+      k.C != a->channels_per_level ||
       k.n_layers != a->num_layers || k.act != a->hidden_act)
     return false;
   for (int i = 0; i <= a->num_layers; ++i)
@@ -63,7 +65,8 @@ bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p
 
 int check_decode_args(const pic_decoder* h, int B, const int32_t* latents, const float* steps,
                       const void* weights, int H, int W, const float* out) {
-  if (!h || !latents || !steps || !weights || !out) return PIC_ERR_INVALID_ARG;
+  const bool need_steps = h && h->arch.latent_format == PIC_LATENT_INT32;
+  if (!h || !latents || (need_steps && !steps) || !weights || !out) return PIC_ERR_INVALID_ARG;
   if (B < 1 || B > h->arch.max_batch) return PIC_ERR_INVALID_ARG;
   if (H < 1 || W < 1 || H > h->arch.max_H || W > h->arch.max_W) return PIC_ERR_INVALID_ARG;
   if (!aligned(latents, 16) || !aligned(weights, 16) || !aligned(out, 16) || !aligned(steps, 4))
@@ -191,7 +194,7 @@ int pic_decode_create(const pic_arch* arch, pic_decoder** out) {
   if (chosen) {
     k = *chosen;
   } else if (arch->precision == PIC_PREC_FP32) {
-    k = pic::fp32_generic_kernel_info();
+    k = pic::fp32_generic_kernel_info(arch->latent_format);
     k.smem_bytes = static_cast<int>(pic_param_count(arch) * 4);
   } else {
     return PIC_ERR_UNSUPPORTED;
@@ -249,7 +252,9 @@ int pic_decode(pic_decoder* h, const int32_t* latents, const float* steps, const
 
 int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const float* steps,
                           const void* weights, int H, int W, float* out_rgb, void* stream) {
-  if (!h || !latents || !steps || !weights || !out_rgb) return PIC_ERR_INVALID_ARG;
+  if (!h || !latents || (h->arch.latent_format == PIC_LATENT_INT32 && !steps) || !weights ||
+      !out_rgb)
+    return PIC_ERR_INVALID_ARG;
   if (B < 1 || B > h->arch.max_batch || H < 1 || W < 1 || H > h->arch.max_H || W > h->arch.max_W)
     return PIC_ERR_INVALID_ARG;
   const pic_arch& a = h->arch;
@@ -279,8 +284,8 @@ int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const f
   const long long w_bytes = static_cast<long long>(B) * h->n_params * weight_elem_bytes(a);
   const long long out_bytes = static_cast<long long>(B) * 3LL * H * W * 4;
   if (cudaMemcpyAsync(h->s_lat, latents, lat_bytes, cudaMemcpyHostToDevice, s) != cudaSuccess ||
-      cudaMemcpyAsync(h->s_steps, steps, static_cast<size_t>(B) * a.num_levels * 4,
-                      cudaMemcpyHostToDevice, s) != cudaSuccess ||
+      (steps && cudaMemcpyAsync(h->s_steps, steps, static_cast<size_t>(B) * a.num_levels * 4,
+                                cudaMemcpyHostToDevice, s) != cudaSuccess) ||
       cudaMemcpyAsync(h->s_w, weights, w_bytes, cudaMemcpyHostToDevice, s) != cudaSuccess) {
     cudaGetLastError();
     return PIC_ERR_CUDA;
@@ -433,7 +438,7 @@ extern "C" int pic_decode_batch_noalloc(const pic_arch* arch, int B, const int32
   if (chosen) {
     h.kern = *chosen;
   } else if (arch->precision == PIC_PREC_FP32) {
-    h.kern = pic::fp32_generic_kernel_info();
+    h.kern = pic::fp32_generic_kernel_info(arch->latent_format);
     h.kern.smem_bytes = static_cast<int>(pic_param_count(arch) * 4);
   } else {
     return PIC_ERR_UNSUPPORTED;

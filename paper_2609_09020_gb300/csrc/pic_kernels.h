@@ -8,6 +8,7 @@ namespace pic {
 struct KernelInfo {
   const char* name;
   int precision;   // 0 = fp32 CUDA cores, 1 = fp16 tensor cores
+  int latent_format;  // 0 = int32 symbols, 1 = fp32 values
   int generic;     // 1: runtime dims (fallback), 0: dims fixed below
   int C;
   int n_layers;
@@ -20,7 +21,8 @@ struct KernelInfo {
 };
 
 int fp32_kernels(KernelInfo* out, int cap);
-KernelInfo fp32_generic_kernel_info();
-int tc_kernels(KernelInfo* out, int cap);
+KernelInfo fp32_generic_kernel_info(int latent_format);
+int tc_kernels(KernelInfo* out, int cap);     // both latent formats
+int tc_kernels_fp32lat(KernelInfo* out, int cap);  // the fp32-latent ones (own translation unit)
 
 }  // namespace pic

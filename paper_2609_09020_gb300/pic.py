@@ -28,9 +28,12 @@ PIC_ACT_RELU = 0
 PIC_ACT_GELU = 1
 PIC_PREC_FP32 = 0
 PIC_PREC_FP16_TC = 1
+PIC_LATENT_INT32 = 0
+PIC_LATENT_FP32 = 1
 
 ACTS = {"relu": PIC_ACT_RELU, "gelu": PIC_ACT_GELU}
 PRECS = {"fp32": PIC_PREC_FP32, "fp16_tc": PIC_PREC_FP16_TC}
+LATENTS = {"int32": PIC_LATENT_INT32, "fp32": PIC_LATENT_FP32}
 
 
 class pic_arch(ctypes.Structure):
@@ -45,6 +48,7 @@ class pic_arch(ctypes.Structure):
         ("max_H", ctypes.c_int),
         ("max_W", ctypes.c_int),
         ("max_batch", ctypes.c_int),
+        ("latent_format", ctypes.c_int),
     ]
 
 
@@ -93,6 +97,10 @@ def load_library():
     lib.pic_izpr_decode.restype = i
     lib.pic_izpr_status.argtypes = [_P, _P]
     lib.pic_izpr_status.restype = i
+    lib.pic_idct_block_count.argtypes = [i, i, i, i]
+    lib.pic_idct_block_count.restype = i64
+    lib.pic_idct_unpatchify.argtypes = [_P, _P, i, i, i, i, i, _P, _P]
+    lib.pic_idct_unpatchify.restype = i
     lib.pic_status_string.argtypes = [i]
     lib.pic_status_string.restype = ctypes.c_char_p
     _lib = lib
@@ -107,7 +115,7 @@ class PicError(RuntimeError):
 
 
 def make_arch(L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1, max_W=1,
-              max_batch=1) -> pic_arch:
+              max_batch=1, latent="int32") -> pic_arch:
     a = pic_arch()
     a.num_levels, a.channels_per_level, a.num_layers = L, C, len(dims) - 1
     for k, d in enumerate(dims):
@@ -116,6 +124,7 @@ def make_arch(L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1, max
     a.precision = PRECS[precision] if isinstance(precision, str) else int(precision)
     a.clamp_output = int(bool(clamp))
     a.max_H, a.max_W, a.max_batch = max_H, max_W, max_batch
+    a.latent_format = LATENTS[latent] if isinstance(latent, str) else int(latent)
     return a
 
 
@@ -208,6 +217,33 @@ def izpr_decode(symbols, eob: int, n_blocks: int, stream=None):
     return coeffs, offsets
 
 
+def pic_idct_block_count(H, W, L, C) -> int:
+    return int(load_library().pic_idct_block_count(H, W, L, C))
+
+
+def pic_idct_unpatchify(coeffs, steps, B, H, W, L, C, latents, stream=None) -> int:
+    return load_library().pic_idct_unpatchify(coeffs, steps, B, H, W, L, C, latents, stream)
+
+
+def idct_unpatchify(coeffs, steps, H, W, L, C, out=None, stream=None):
+    """Inverse DCT stage on torch CUDA tensors: coeffs int32 [B][n_blocks][64]
+    (or [n_blocks][64] for one image), steps fp32 [B][L]; returns fp32
+    latents [B][pic_latent_count] (enqueued on the stream, not synchronised)."""
+    import torch
+    n_blk = pic_idct_block_count(H, W, L, C)
+    B = coeffs.numel() // (64 * n_blk) if n_blk > 0 else 0
+    if B < 1 or coeffs.numel() != B * 64 * n_blk or steps.numel() != B * L:
+        raise ValueError("idct_unpatchify: tensor sizes do not match the shapes")
+    if out is None:
+        out = torch.empty((B, pic_latent_count(H, W, L, C)), dtype=torch.float32,
+                          device=coeffs.device)
+    rc = pic_idct_unpatchify(coeffs.data_ptr(), steps.data_ptr(), B, H, W, L, C, out.data_ptr(),
+                             _stream_ptr(stream))
+    if rc != PIC_OK:
+        raise PicError(rc, "pic_idct_unpatchify")
+    return out
+
+
 # ---- convenience wrapper over torch tensors --------------------------------
 def _stream_ptr(stream):
     if stream is None:
@@ -221,15 +257,16 @@ class Decoder:
     contiguous CUDA tensors of the documented dtypes."""
 
     def __init__(self, L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1,
-                 max_W=1, max_batch=1):
-        self.arch = make_arch(L, C, dims, act, precision, clamp, max_H, max_W, max_batch)
+                 max_W=1, max_batch=1, latent="int32"):
+        self.arch = make_arch(L, C, dims, act, precision, clamp, max_H, max_W, max_batch, latent)
+        self.latent = latent
         self.L, self.C, self.dims, self.precision = L, C, tuple(dims), precision
         self.handle = pic_decode_create(self.arch)
 
     @classmethod
-    def for_workload(cls, wl, precision: str, clamp=True, max_batch=None):
+    def for_workload(cls, wl, precision: str, clamp=True, max_batch=None, latent="int32"):
         return cls(wl.L, wl.C, wl.dims, wl.act, precision, clamp, wl.H, wl.W,
-                   max_batch or wl.B)
+                   max_batch or wl.B, latent)
 
     @property
     def kernel_name(self) -> str:
@@ -255,7 +292,8 @@ class Decoder:
         """Enqueues a batch decode; arguments are torch CUDA tensors."""
         if B is None:
             B = out.shape[0] if out.dim() == 4 else 1
-        rc = pic_decode_batch(self.handle, B, latents.data_ptr(), steps.data_ptr(),
+        sp = steps.data_ptr() if steps is not None else None
+        rc = pic_decode_batch(self.handle, B, latents.data_ptr(), sp,
                               weights.data_ptr(), H, W, out.data_ptr(), _stream_ptr(stream))
         self._check(rc, "pic_decode_batch")
         return out

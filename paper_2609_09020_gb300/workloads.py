@@ -157,6 +157,10 @@ def _draw_image(rng: np.random.Generator, H, W, L, C, dims, lap_scale, clip, wei
         for _c in range(C):
             q = np.clip(np.rint(rng.laplace(0.0, lap_scale, (h, w))), -clip, clip).astype(np.int32)
             levels.append(q.ravel())
+    return np.concatenate(levels), _draw_weights(rng, dims, weight_dtype)
+
+
+def _draw_weights(rng: np.random.Generator, dims, weight_dtype):
     params = []
     for k in range(len(dims) - 1):
         din, dout = dims[k], dims[k + 1]
@@ -165,8 +169,7 @@ def _draw_image(rng: np.random.Generator, H, W, L, C, dims, lap_scale, clip, wei
         params.append(Wk.ravel())
         params.append(bk)
     p64 = np.concatenate(params)
-    weights = p64.astype(np.float16) if weight_dtype == "fp16" else p64.astype(np.float32)
-    return np.concatenate(levels), weights
+    return p64.astype(np.float16) if weight_dtype == "fp16" else p64.astype(np.float32)
 
 
 def make_inputs(wl: Workload | str, batch: int | None = None) -> Inputs:
@@ -206,6 +209,60 @@ def dct_blocks(n_blocks: int, seed: int, scale: float = 6.0, decay: float = 0.72
     scales = scale * decay ** rc
     q = np.rint(rng.laplace(0.0, 1.0, (n_blocks, 64)) * scales)
     return np.clip(q, -clip, clip).astype(np.int32)
+
+
+def block_count(H: int, W: int, L: int, C: int) -> int:
+    """Number of 8x8 patches of one pyramid, sum_l C ceil(H_l/8) ceil(W_l/8)
+    (Sec. 3.2, Eq. 6: every latent plane is cut into 8x8 patches)."""
+    return sum(C * ((h + 7) // 8) * ((w + 7) // 8) for h, w in level_shapes(H, W, L))
+
+
+# Quantised DCT coefficients in place of integer latents (the input of the
+# inverse DCT stage, Fig. 1).  Coefficient (u, v) of every patch is
+# round(Laplace(0, DCT_GAIN * lap_scale * DCT_DECAY^(u+v))) clipped to
+# +-DCT_CLIP: large at low frequencies, mostly zero at high ones, as in a
+# JPEG-like coder.  DCT_GAIN = 4 gives decoded latents about the spread of
+# the workload's integer latents (an orthonormal 8x8 transform keeps the
+# energy: latent variance = sum_uv 2 (4 b 0.72^(u+v))^2 / 64 ~= 2.1 b^2,
+# against 2 b^2 for Laplace(b) symbols).
+DCT_GAIN = 4.0
+DCT_DECAY = 0.72
+DCT_CLIP = 255
+
+
+@dataclass
+class DctInputs:
+    """Host arrays for B images whose latents arrive as DCT coefficients."""
+
+    wl: Workload
+    coeffs: np.ndarray       # int32 [B, n_blocks, 64], patch-major, raster within a patch
+    steps: np.ndarray        # float32 [B, L]
+    weights: np.ndarray      # as Inputs.weights
+
+    def weights_for(self, precision: str) -> np.ndarray:
+        if precision == "fp32" or self.weights.dtype == np.float16:
+            return self.weights.astype(np.float32) if precision == "fp32" else self.weights
+        return self.weights.astype(np.float16)
+
+
+def make_dct_inputs(wl: Workload | str, batch: int | None = None) -> DctInputs:
+    """Draws, per image, the DCT coefficients of every patch and then the MLP
+    weights, from PCG64 seeded with (seed, 7) -- a stream apart from
+    make_inputs' latents."""
+    if isinstance(wl, str):
+        wl = WORKLOADS[wl]
+    seeds = wl.seeds if batch is None else wl.seeds[:batch]
+    n = block_count(wl.H, wl.W, wl.L, wl.C)
+    rc = np.add.outer(np.arange(8), np.arange(8)).ravel()
+    scales = DCT_GAIN * wl.lap_scale * DCT_DECAY ** rc
+    cs, ws = [], []
+    for s in seeds:
+        rng = np.random.Generator(np.random.PCG64([s, 7]))
+        q = np.rint(rng.laplace(0.0, 1.0, (n, 64)) * scales)
+        cs.append(np.clip(q, -DCT_CLIP, DCT_CLIP).astype(np.int32))
+        ws.append(_draw_weights(rng, wl.dims, wl.weight_dtype))
+    steps = np.array([[2.0 ** -l for l in range(wl.L)]] * len(seeds), dtype=np.float32)
+    return DctInputs(wl=wl, coeffs=np.stack(cs), steps=steps, weights=np.stack(ws))
 
 
 def sample_pixels(H: int, W: int, n: int, seed: int) -> np.ndarray:

@@ -94,3 +94,28 @@ def test_izpr_workspace_and_argument_checks(lib):
     assert pic.pic_izpr_decode(None, 10, 30, 1, None, None, None, 0, None) == pic.PIC_ERR_INVALID_ARG
     assert pic.pic_izpr_decode(None, -1, 30, 1, None, None, None, 0, None) == pic.PIC_ERR_INVALID_ARG
     assert pic.pic_izpr_status(None, None) == pic.PIC_ERR_INVALID_ARG
+
+
+def test_idct_block_count_and_argument_checks(lib, orc):
+    from paper_2609_09020_gb300 import pic
+    from paper_2609_09020_gb300 import workloads as wk
+    for H, W, L, C in [(512, 768, 7, 1), (1080, 1920, 7, 2), (5, 3, 4, 4), (1, 1, 1, 1),
+                       (2160, 3840, 8, 2)]:
+        n = pic.pic_idct_block_count(H, W, L, C)
+        assert n == orc.block_count(H, W, L, C) == wk.block_count(H, W, L, C)
+    assert pic.pic_idct_block_count(0, 5, 1, 1) == -1
+    assert pic.pic_idct_block_count(5, 5, 13, 1) == -1
+    assert pic.pic_idct_block_count(5, 5, 1, 5) == -1
+    # rejected before any CUDA call
+    assert pic.pic_idct_unpatchify(None, None, 1, 8, 8, 1, 1, None, None) == pic.PIC_ERR_INVALID_ARG
+    assert pic.pic_idct_unpatchify(16, 16, 0, 8, 8, 1, 1, 16, None) == pic.PIC_ERR_INVALID_ARG
+    assert pic.pic_idct_unpatchify(8, 16, 1, 8, 8, 1, 1, 16, None) == pic.PIC_ERR_INVALID_ARG
+
+
+def test_fp32_latent_arch_is_validated(lib):
+    """latent_format outside the enum is refused at create (no device needed
+    to reach that check)."""
+    from paper_2609_09020_gb300 import pic
+    a = pic.make_arch(2, 1, [2, 8, 3], max_H=8, max_W=8, latent=2)
+    h = pic._P()
+    assert lib.pic_decode_create(pic.ctypes.byref(a), pic.ctypes.byref(h)) == pic.PIC_ERR_UNSUPPORTED
