@@ -7,6 +7,7 @@ throughput workload (64 independent 768x512 images, 7 levels x 1 channel,
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c5]
                     [--precision fp16_tc|fp32] [--impl ours|reference]
+                    [--stage decode|izpr|idct|pipeline] [--chunk 16]
 
 Prints one JSON line (rank 0).  ``value`` is decoded megapixels/s over all
 ranks (weak scaling: each rank decodes its own batch; no collective on the
@@ -212,6 +213,251 @@ def run_reference(args, wl, precision, rank):
     print(json.dumps(line), flush=True)
 
 
+# ---------------------------------------------------------------------------
+# Stage benchmarks: the decoder's stages before the synthesis (Fig. 1: iZpR,
+# then dequantisation + iDCT + un-patchify), alone and chained with it, on
+# the 64-image workload's 524,288 patches.  One step = one pass over the
+# whole batch.
+STAGE_METRIC = {
+    "izpr": ("inverse ZpR (Algorithm 1): 8x8 blocks/s at 1 GB300; % of HBM roofline", "Mblocks/s"),
+    "idct": ("dequantise + 8x8 iDCT + un-patchify: 8x8 blocks/s at 1 GB300; % of HBM roofline",
+             "Mblocks/s"),
+    "pipeline": ("decoded megapixels/s from ZpR symbols (iZpR + iDCT + synthesis) at 1 GB300",
+                 "MP/s"),
+}
+
+
+def _event_time(fn, steps, stream, torch):
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for _ in range(steps):
+        fn()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    return ev0.elapsed_time(ev1) / steps
+
+
+def _stage_cpu(stage, wl, sym_h, counts, n_blk, eob, dx, budget_s):
+    """The oracle, as it stands, on a bounded sample: whole images, one after
+    another, until about budget_s seconds have passed."""
+    import oracle
+    orc = oracle.load()
+    cores = os.cpu_count() or 1
+    starts = np.r_[0, np.cumsum(counts)[:-1]]
+    n, t0 = 0, time.perf_counter()
+    while True:
+        b = n % wl.B
+        if stage == "izpr":
+            orc.izpr(sym_h[starts[b]:starts[b] + counts[b]], eob, n_blk)
+        elif stage == "idct":
+            orc.unpatchify_idct(dx.coeffs[b], dx.steps[b].astype(np.float64), wl.H, wl.W, wl.L,
+                                wl.C)
+        else:
+            c = orc.izpr(sym_h[starts[b]:starts[b] + counts[b]], eob, n_blk)
+            y = orc.unpatchify_idct(c, dx.steps[b].astype(np.float64), wl.H, wl.W, wl.L, wl.C)
+            orc.decode_values(y, dx.weights[b].astype(np.float64), wl.H, wl.W, wl.L, wl.C,
+                              wl.dims, wl.act, nthreads=cores)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s:
+            break
+    if stage == "pipeline":
+        v, unit = n * wl.H * wl.W / 1e6 / el, "MP/s"
+    else:
+        v, unit = n * n_blk / 1e6 / el, "Mblocks/s"
+    threads = cores if stage == "pipeline" else 1
+    return {"value": v, "unit": unit, "cores": threads, "kind": "oracle",
+            "sample": f"{n} whole image(s) of workload {wl.name} in {el:.1f} s "
+                      f"({'fp64 C oracle, decode on ' + str(cores) + ' OpenMP threads' if stage == 'pipeline' else 'fp64 C oracle, one thread'})"}
+
+
+def run_stage(args):
+    import torch
+    from paper_2609_09020_gb300 import build, pic
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    build.build()
+    stage = args.stage
+    wl = wk.WORKLOADS["c5"]
+    B = wl.B
+    sym_h, counts, n_blk, eob = wk.zpr_streams(wl)
+    dx = wk.make_dct_inputs(wl)
+    stream = torch.cuda.current_stream(dev)
+    sp = stream.cuda_stream
+    n_lat = wl.n_latents
+    starts = np.r_[0, np.cumsum(counts)]
+    chunk = max(1, min(args.chunk, B))
+    peaks = load_peaks()
+
+    sym = torch.from_numpy(sym_h).to(dev)
+    coeffs_in = torch.from_numpy(dx.coeffs).to(dev)
+    steps_t = torch.from_numpy(dx.steps).to(dev)
+    w_host = np.ascontiguousarray(dx.weights_for("fp16_tc"))
+    wts = torch.from_numpy(w_host).to(dev)
+    rows = chunk if stage == "pipeline" else B
+    coeffs = torch.empty((rows * n_blk, 64), dtype=torch.int32, device=dev)
+    offsets = torch.empty(rows * n_blk, dtype=torch.int64, device=dev)
+    lat = torch.empty((rows, n_lat), dtype=torch.float32, device=dev)
+    out = torch.empty((B, 3, wl.H, wl.W), dtype=torch.float32, device=dev)
+    wsb = pic.pic_izpr_workspace_bytes(int(counts.max()) * rows if stage == "pipeline"
+                                       else sym.numel())
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    dec = pic.Decoder.for_workload(wl, "fp16_tc", max_batch=chunk, latent="fp32") \
+        if stage == "pipeline" else None
+
+    def izpr(s_ptr, n_sym, nb):
+        rc = pic.pic_izpr_decode(s_ptr, n_sym, eob, nb, coeffs.data_ptr(), offsets.data_ptr(),
+                                 ws.data_ptr(), wsb, sp)
+        if rc != pic.PIC_OK:
+            raise pic.PicError(rc, "pic_izpr_decode")
+
+    def idct(c_ptr, s_ptr, nb_img):
+        rc = pic.pic_idct_unpatchify(c_ptr, s_ptr, nb_img, wl.H, wl.W, wl.L, wl.C,
+                                     lat.data_ptr(), sp)
+        if rc != pic.PIC_OK:
+            raise pic.PicError(rc, "pic_idct_unpatchify")
+
+    def one_step():
+        if stage == "izpr":
+            izpr(sym.data_ptr(), sym.numel(), B * n_blk)
+        elif stage == "idct":
+            idct(coeffs_in.data_ptr(), steps_t.data_ptr(), B)
+        else:
+            for b0 in range(0, B, chunk):
+                nb = min(chunk, B - b0)
+                izpr(sym.data_ptr() + 4 * int(starts[b0]), int(starts[b0 + nb] - starts[b0]),
+                     nb * n_blk)
+                idct(coeffs.data_ptr(), steps_t.data_ptr() + 4 * b0 * wl.L, nb)
+                dec.decode_batch(lat, None, wts[b0:b0 + nb], wl.H, wl.W, out[b0:b0 + nb],
+                                 stream=stream, B=nb)
+
+    for _ in range(max(args.warmup, 3)):
+        one_step()
+    torch.cuda.synchronize()
+    if stage in ("izpr", "pipeline"):
+        rc = pic.pic_izpr_status(ws.data_ptr(), sp)
+        if rc != pic.PIC_OK:
+            raise pic.PicError(rc, "pic_izpr_status")
+    if dec is not None:
+        dec.check(stream)
+    with ClockSampler(0) as clk:
+        ms = _event_time(one_step, args.steps, stream, torch)
+    if dec is not None:
+        dec.check(stream)
+
+    # per-stage launch times (the same calls, timed one stage at a time)
+    n_sym = sym.numel()
+    stage_ms = {}
+    if stage == "pipeline":
+        def part(which):
+            def f():
+                for b0 in range(0, B, chunk):
+                    nb = min(chunk, B - b0)
+                    if which == "izpr":
+                        izpr(sym.data_ptr() + 4 * int(starts[b0]),
+                             int(starts[b0 + nb] - starts[b0]), nb * n_blk)
+                    elif which == "idct":
+                        idct(coeffs.data_ptr(), steps_t.data_ptr() + 4 * b0 * wl.L, nb)
+                    else:
+                        dec.decode_batch(lat, None, wts[b0:b0 + nb], wl.H, wl.W,
+                                         out[b0:b0 + nb], stream=stream, B=nb)
+            return f
+        for which in ("izpr", "idct", "decode"):
+            stage_ms[which] = _event_time(part(which), args.steps, stream, torch)
+
+    blocks = B * n_blk
+    n_chunks = (B + chunk - 1) // chunk
+    if stage == "izpr":
+        nbytes = 4 * n_sym + (256 + 8) * blocks
+        value = blocks / (ms * 1e-3) / 1e6
+        launches = 4
+    elif stage == "idct":
+        nbytes = 256 * blocks + 4 * B * n_lat + 4 * B * wl.L
+        value = blocks / (ms * 1e-3) / 1e6
+        launches = 1
+    else:
+        nbytes = (4 * n_sym + 2 * B * wl.n_params + 4 * B * wl.L + 12 * B * wl.H * wl.W)
+        value = B * wl.H * wl.W / (ms * 1e-3) / 1e6
+        launches = n_chunks * 6
+    metric, unit = STAGE_METRIC[stage]
+    if stage == "pipeline":
+        flops = 2.0 * wl.macs_per_pixel * B * wl.H * wl.W
+        t_dec = stage_ms["decode"] * 1e-3
+        roof = {"bound": "tensor", "achieved": flops / t_dec / 1e12,
+                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "peak_source": f"bf16 dense burst, {peaks['source']}",
+                "kernel": "tc05_7x64x64x3_relu_f32lat (the dominant stage)",
+                "avg_launch_us": 1e3 * stage_ms["decode"] / n_chunks,
+                "whole_step_hbm_gbs": nbytes / (ms * 1e-3) / 1e9}
+    else:
+        roof = {"bound": "hbm", "achieved": nbytes / (ms * 1e-3) / 1e9, "peak": peaks["hbm_gbs"],
+                "unit": "GB/s", "peak_source": f"copy bandwidth, {peaks['source']}",
+                "kernel": "izpr_count+izpr_scan+izpr_compact+izpr_expand (one call)"
+                if stage == "izpr" else "idct_unpatchify_kernel",
+                "avg_launch_us": ms * 1e3}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = None
+    roof["algorithmic_bytes_per_launch"] = nbytes
+
+    # end to end with host buffers: H2D of the step's input, the stage, D2H of its result
+    e2e = None
+    if not args.no_e2e:
+        if stage == "izpr":
+            src_h, dst_d = torch.from_numpy(sym_h).pin_memory(), sym
+            res_d = coeffs
+        elif stage == "idct":
+            src_h, dst_d = torch.from_numpy(dx.coeffs).pin_memory(), coeffs_in
+            res_d = lat
+        else:
+            src_h, dst_d = torch.from_numpy(sym_h).pin_memory(), sym
+            res_d = out
+        res_h = torch.empty(res_d.shape, dtype=res_d.dtype).pin_memory()
+
+        def e2e_step():
+            dst_d.copy_(src_h, non_blocking=True)
+            one_step()
+            res_h.copy_(res_d, non_blocking=True)
+            torch.cuda.current_stream().synchronize()
+
+        e2e_step()
+        k = max(3, min(args.steps, 10))
+        t0 = time.perf_counter()
+        for _ in range(k):
+            e2e_step()
+        el = (time.perf_counter() - t0) / k
+        units = blocks / 1e6 if stage != "pipeline" else B * wl.H * wl.W / 1e6
+        e2e = {"value": units / el, "unit": unit,
+               "h2d_bytes_per_step": int(src_h.numel() * src_h.element_size()),
+               "d2h_bytes_per_step": int(res_h.numel() * res_h.element_size()),
+               "ms_per_step": 1e3 * el}
+
+    cpu = None if args.no_cpu_baseline else _stage_cpu(stage, wl, sym_h, counts, n_blk, eob, dx,
+                                                       min(args.cpu_budget_s, 12.0))
+    line = {"metric": metric, "value": value, "unit": unit, "n_gpus": 1, "steps": args.steps,
+            "warmup": max(args.warmup, 3), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None,
+            "dtype": {"izpr": "int32", "idct": "int32 in, f32 arithmetic and out",
+                      "pipeline": "int32 symbols; f32 iDCT; f16 operands (hi+lo), f32 accumulate"}[stage],
+            "data": "synthetic (seeded DCT coefficients / ZpR streams shaped like the 64-image workload)",
+            "config": {"workload": f"{stage}: {B} x {wl.W}x{wl.H}, {wl.L} levels x {wl.C} ch, "
+                                   f"{n_blk} 8x8 patches per image",
+                       "images": B, "patches": blocks, "symbols": int(n_sym),
+                       "symbols_per_patch": n_sym / blocks, "eob": eob,
+                       "chunk_images": chunk if stage == "pipeline" else None,
+                       "l2": "inputs larger than L2 (no flush needed)",
+                       "parallelism": "dp1"},
+            "roofline": roof, "clocks": clk.summary(), "e2e": e2e, "gpu_launches": launches * args.steps,
+            "cpu_baseline": cpu, "stage": stage}
+    if stage_ms:
+        line["stage_ms"] = stage_ms
+    if stage == "pipeline":
+        line["images_per_s"] = B / (ms * 1e-3)
+    print(json.dumps(line), flush=True)
+    if dec is not None:
+        dec.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -224,7 +470,19 @@ def main():
     ap.add_argument("--ref-step-s", type=float, default=5.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--stage", default="decode", choices=["decode", "izpr", "idct", "pipeline"],
+                    help="decode (default): the synthesis; the others time the stages before "
+                         "it, alone or chained, on one GPU")
+    ap.add_argument("--chunk", type=int, default=16,
+                    help="pipeline stage: images per iZpR/iDCT/decode round")
     args = ap.parse_args()
+    if args.stage != "decode":
+        if args.impl == "reference" or int(os.environ.get("WORLD_SIZE", "1")) > 1:
+            print(json.dumps({"stage": args.stage, "unavailable":
+                              "stage benchmarks run our arm on one GPU only"}))
+            return
+        run_stage(args)
+        return
 
     wl = wk.WORKLOADS[args.workload]
     precision = args.precision or wl.precisions[-1]

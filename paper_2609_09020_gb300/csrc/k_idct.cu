@@ -9,15 +9,19 @@
 // per patch (the 8 threads of a patch sit in one warp, so the exchanges
 // between the two 1-D passes need only __syncwarp):
 //   load    thread j reads 16 B at coefficient 4j and 32 + 4j of its patch
-//           (a warp reads 4 whole patches, 1 KB contiguous), scales them by
-//           the level's step and stores them into the patch's shared slot;
+//           (a warp reads 4 whole patches, 1 KB contiguous) one pass ahead,
+//           scales them by the level's step and stores them into the
+//           patch's shared slot;
 //   pass 1  thread j transforms column j: T[m][j] = sum_u c[u][m] S[u][j];
 //   pass 2  thread j transforms row j:    x[j][n] = sum_v c[v][n] T[j][v];
-//   store   thread j writes row j of the patch (32 B, two float4 when the
-//           row is whole and aligned) into its plane.
-// c[k][n] = a(k) cos((2n + 1) k pi / 16) is built once per CTA in shared
-// memory from CUDA's cospi in double precision.  The patch slot is padded to
-// 72 floats so the column accesses of pass 1 hit 32 distinct banks.
+//   store   lanes 2i and 2i+1 trade row halves so that each store
+//           instruction writes whole 32-byte rows: row 2i in the first,
+//           row 2i+1 in the second.
+// c[k][n] = a(k) cos((2n + 1) k pi / 16) lives in constant memory; every
+// index into it is warp-uniform, so each FMA reads its coefficient straight
+// from the constant bank.  The patch slot is padded to 72 floats so the
+// column accesses of pass 1 hit 32 distinct banks.
+#include <cmath>
 #include <cstdint>
 
 #include <cuda_runtime.h>
@@ -35,9 +39,10 @@ constexpr int kPatches = kThreads / 8;  // patches per CTA pass
 constexpr int kSlot = 72;               // floats per patch slot (64 + 8 bank pad)
 
 struct Plane {
-  long long blk0;     // first patch of the plane, counted within one image
-  long long lat_off;  // offset of the plane within one image's latents
-  int bw;             // patches per row: ceil(W_l / 8)
+  int blk0;                     // first patch of the plane, counted within one image
+  int bw;                       // patches per row: ceil(W_l / 8)
+  unsigned long long bw_inv;    // division by bw (see udiv)
+  long long lat_off;            // offset of the plane within one image's latents
   int Hl, Wl;
   int level;
 };
@@ -46,51 +51,68 @@ struct IdctParams {
   const int32_t* coeffs;
   const float* steps;
   float* latents;
-  long long blocks_per_image;
+  int blocks_per_image;
+  unsigned long long bpi_inv;   // division by blocks_per_image
   long long lat_per_image;
-  long long total_blocks;
+  int total_blocks;             // < 2^31
   int L, n_planes;
   Plane pl[kPlanesMax];
 };
 
+__constant__ float kBasis[64];  // c[k][n] at k * 8 + n
+
+// floor(n / d) for 32-bit n and d by one multiply-high with inv = ceil(2^64 / d)
+// (division by invariant integers, Granlund & Montgomery 1994: the error term
+// n (inv d - 2^64) / (d 2^64) stays below 1/d); d == 1 is stored as inv == 0.
+__host__ unsigned long long udiv_inv(unsigned d) { return d > 1 ? ~0ULL / d + 1 : 0; }
+__device__ __forceinline__ unsigned udiv(unsigned n, unsigned d, unsigned long long inv) {
+  (void)d;
+  return inv ? static_cast<unsigned>(__umul64hi(n, inv)) : n;
+}
+
 int level_size(int n, int l) { return static_cast<int>((static_cast<long long>(n) + (1LL << l) - 1) >> l); }
 
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 6)
     idct_unpatchify_kernel(const __grid_constant__ IdctParams p) {
-  __shared__ __align__(16) float basis[64];  // basis[k * 8 + n] = a(k) cos((2n+1) k pi / 16)
   __shared__ __align__(16) float tile[kPatches * kSlot];
   const int t = threadIdx.x;
-  if (t < 64) {
-    const int k = t >> 3, n = t & 7;
-    const double a = k == 0 ? rsqrt(8.0) : 0.5;
-    basis[t] = static_cast<float>(a * cospi(static_cast<double>((2 * n + 1) * k) / 16.0));
-  }
-  __syncthreads();
   const int slot = t >> 3;
   const int j = t & 7;
+  const int odd = j & 1;
   float* my = tile + slot * kSlot;
-  const float4* basis4 = reinterpret_cast<const float4*>(basis);
 
-  for (long long g0 = static_cast<long long>(blockIdx.x) * kPatches; g0 < p.total_blocks;
-       g0 += static_cast<long long>(gridDim.x) * kPatches) {
-    const long long g = g0 + slot;
+  const int stride = static_cast<int>(gridDim.x) * kPatches;
+  int g = static_cast<int>(blockIdx.x) * kPatches + slot;
+  int4 v0 = make_int4(0, 0, 0, 0), v1 = v0;
+  if (g < p.total_blocks) {
+    const int4* src = reinterpret_cast<const int4*>(p.coeffs + static_cast<long long>(g) * 64);
+    v0 = __ldcs(src + j);
+    v1 = __ldcs(src + 8 + j);
+  }
+  for (int g0 = static_cast<int>(blockIdx.x) * kPatches; g0 < p.total_blocks;
+       g0 += stride, g += stride) {
     const bool live = g < p.total_blocks;
-    int b = 0, pi = 0;
-    long long k = 0;
+    int4 n0 = make_int4(0, 0, 0, 0), n1 = n0;
+    if (g + stride < p.total_blocks) {  // next pass's coefficients
+      const int4* src = reinterpret_cast<const int4*>(p.coeffs + static_cast<long long>(g + stride) * 64);
+      n0 = __ldcs(src + j);
+      n1 = __ldcs(src + 8 + j);
+    }
+    int b = 0, k = 0, pi = 0;
     float step = 0.0f;
     if (live) {
-      b = static_cast<int>(g / p.blocks_per_image);
-      k = g - static_cast<long long>(b) * p.blocks_per_image;
+      b = static_cast<int>(udiv(g, p.blocks_per_image, p.bpi_inv));
+      k = g - b * p.blocks_per_image;
       for (int q = 1; q < p.n_planes; ++q)
         if (k >= p.pl[q].blk0) pi = q;
       step = __ldg(p.steps + b * p.L + p.pl[pi].level);
-      const int4* src = reinterpret_cast<const int4*>(p.coeffs + g * 64);
-      const int4 v0 = __ldcs(src + j), v1 = __ldcs(src + 8 + j);
-      reinterpret_cast<float4*>(my)[j] =
-          make_float4(v0.x * step, v0.y * step, v0.z * step, v0.w * step);
-      reinterpret_cast<float4*>(my + 32)[j] =
-          make_float4(v1.x * step, v1.y * step, v1.z * step, v1.w * step);
     }
+    reinterpret_cast<float4*>(my)[j] =
+        make_float4(v0.x * step, v0.y * step, v0.z * step, v0.w * step);
+    reinterpret_cast<float4*>(my + 32)[j] =
+        make_float4(v1.x * step, v1.y * step, v1.z * step, v1.w * step);
+    v0 = n0;
+    v1 = n1;
     __syncwarp();
 
     // pass 1: column j, vertical inverse transform
@@ -98,18 +120,11 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
     for (int u = 0; u < 8; ++u) col[u] = my[u * 8 + j];
 #pragma unroll
-    for (int m = 0; m < 8; ++m) tr[m] = 0.0f;
+    for (int m = 0; m < 8; ++m) {
+      float acc = 0.0f;
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const float4 c0 = basis4[2 * u], c1 = basis4[2 * u + 1];
-      tr[0] = fmaf(c0.x, col[u], tr[0]);
-      tr[1] = fmaf(c0.y, col[u], tr[1]);
-      tr[2] = fmaf(c0.z, col[u], tr[2]);
-      tr[3] = fmaf(c0.w, col[u], tr[3]);
-      tr[4] = fmaf(c1.x, col[u], tr[4]);
-      tr[5] = fmaf(c1.y, col[u], tr[5]);
-      tr[6] = fmaf(c1.z, col[u], tr[6]);
-      tr[7] = fmaf(c1.w, col[u], tr[7]);
+      for (int u = 0; u < 8; ++u) acc = fmaf(kBasis[u * 8 + m], col[u], acc);
+      tr[m] = acc;
     }
     __syncwarp();
 #pragma unroll
@@ -122,41 +137,75 @@ __global__ void __launch_bounds__(kThreads)
     const float row[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
     float x[8];
 #pragma unroll
-    for (int n = 0; n < 8; ++n) x[n] = 0.0f;
+    for (int n = 0; n < 8; ++n) {
+      float acc = 0.0f;
 #pragma unroll
-    for (int v = 0; v < 8; ++v) {
-      const float4 c0 = basis4[2 * v], c1 = basis4[2 * v + 1];
-      x[0] = fmaf(c0.x, row[v], x[0]);
-      x[1] = fmaf(c0.y, row[v], x[1]);
-      x[2] = fmaf(c0.z, row[v], x[2]);
-      x[3] = fmaf(c0.w, row[v], x[3]);
-      x[4] = fmaf(c1.x, row[v], x[4]);
-      x[5] = fmaf(c1.y, row[v], x[5]);
-      x[6] = fmaf(c1.z, row[v], x[6]);
-      x[7] = fmaf(c1.w, row[v], x[7]);
+      for (int v = 0; v < 8; ++v) acc = fmaf(kBasis[v * 8 + n], row[v], acc);
+      x[n] = acc;
     }
     __syncwarp();  // the slot is refilled by the next pass
 
+    // lanes 2i, 2i+1: the even lane sends its right half, the odd lane its left
+    float recv[4];
+#pragma unroll
+    for (int n = 0; n < 4; ++n) recv[n] = __shfl_xor_sync(0xffffffffu, odd ? x[n] : x[4 + n], 1);
+    // store 0 writes row j & ~1 (even lane: columns 0-3 of its own row; odd
+    // lane: columns 4-7 received), store 1 row j | 1 (even lane: columns 0-3
+    // received; odd lane: columns 4-7 of its own row)
+    const float4 s0 = odd ? make_float4(recv[0], recv[1], recv[2], recv[3])
+                          : make_float4(x[0], x[1], x[2], x[3]);
+    const float4 s1 = odd ? make_float4(x[4], x[5], x[6], x[7])
+                          : make_float4(recv[0], recv[1], recv[2], recv[3]);
     if (live) {
       const Plane& P = p.pl[pi];
-      const int pr = static_cast<int>(k - P.blk0);
-      const int by = pr / P.bw, bx = pr - by * P.bw;
-      const int r = 8 * by + j;
-      if (r < P.Hl) {
-        const int q0 = 8 * bx;
-        float* dst = p.latents + b * p.lat_per_image + P.lat_off + static_cast<long long>(r) * P.Wl + q0;
-        const int nv = min(8, P.Wl - q0);
-        if (nv == 8 && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
-          reinterpret_cast<float4*>(dst)[0] = make_float4(x[0], x[1], x[2], x[3]);
-          reinterpret_cast<float4*>(dst)[1] = make_float4(x[4], x[5], x[6], x[7]);
-        } else {
+      const int pr = k - P.blk0;
+      const int by = static_cast<int>(udiv(pr, P.bw, P.bw_inv)), bx = pr - by * P.bw;
+      const int q0 = 8 * bx + 4 * odd;
+      const int nv = min(4, P.Wl - q0);  // valid columns of this half (may be <= 0)
+      float* plane = p.latents + b * p.lat_per_image + P.lat_off + q0;
 #pragma unroll
-          for (int n = 0; n < 8; ++n)
-            if (n < nv) dst[n] = x[n];
+      for (int e = 0; e < 2; ++e) {
+        const int r = 8 * by + (e ? (j | 1) : (j & ~1));
+        const float4 sv = e ? s1 : s0;
+        if (r < P.Hl && nv > 0) {
+          float* dst = plane + static_cast<long long>(r) * P.Wl;
+          if (nv == 4 && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+            *reinterpret_cast<float4*>(dst) = sv;
+          } else {
+            const float vv[4] = {sv.x, sv.y, sv.z, sv.w};
+#pragma unroll
+            for (int n = 0; n < 4; ++n)
+              if (n < nv) dst[n] = vv[n];
+          }
         }
       }
     }
   }
+}
+
+// The basis table of the current device, written once per device.
+int ensure_basis() {
+  constexpr int kMaxDev = 64;
+  static bool done[kMaxDev];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  if (!done[dev]) {
+    float h[64];
+    const double pi = 3.14159265358979323846;
+    for (int k = 0; k < 8; ++k)
+      for (int n = 0; n < 8; ++n)
+        h[k * 8 + n] = static_cast<float>((k == 0 ? std::sqrt(0.125) : 0.5) *
+                                          std::cos((2 * n + 1) * k * pi / 16.0));
+    if (cudaMemcpyToSymbol(kBasis, h, sizeof(h)) != cudaSuccess) {
+      cudaGetLastError();
+      return PIC_ERR_CUDA;
+    }
+    done[dev] = true;
+  }
+  return PIC_OK;
 }
 
 bool sizes_ok(int H, int W, int L, int C) {
@@ -193,9 +242,10 @@ extern "C" int pic_idct_unpatchify(const int32_t* coeffs, const float* steps, in
     const int Hl = level_size(H, l), Wl = level_size(W, l);
     for (int c = 0; c < C; ++c, ++q) {
       Plane& P = p.pl[q];
-      P.blk0 = blk;
+      P.blk0 = static_cast<int>(blk);
       P.lat_off = off + static_cast<long long>(c) * Hl * Wl;
       P.bw = (Wl + 7) / 8;
+      P.bw_inv = udiv_inv(static_cast<unsigned>(P.bw));
       P.Hl = Hl;
       P.Wl = Wl;
       P.level = l;
@@ -203,10 +253,13 @@ extern "C" int pic_idct_unpatchify(const int32_t* coeffs, const float* steps, in
     }
     off += static_cast<long long>(C) * Hl * Wl;
   }
+  if (blk * B >= (1LL << 31) - (1LL << 24)) return PIC_ERR_INVALID_ARG;  // 32-bit patch indices (+ one stride)
   p.n_planes = q;
-  p.blocks_per_image = blk;
+  p.blocks_per_image = static_cast<int>(blk);
+  p.bpi_inv = udiv_inv(static_cast<unsigned>(blk));
   p.lat_per_image = off;
-  p.total_blocks = blk * B;
+  p.total_blocks = static_cast<int>(blk * B);
+  if (ensure_basis() != PIC_OK) return PIC_ERR_CUDA;
 
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||

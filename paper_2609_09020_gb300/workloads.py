@@ -265,6 +265,59 @@ def make_dct_inputs(wl: Workload | str, batch: int | None = None) -> DctInputs:
     return DctInputs(wl=wl, coeffs=np.stack(cs), steps=steps, weights=np.stack(ws))
 
 
+def zigzag_diagonals() -> np.ndarray:
+    """Anti-diagonal u + v of each zigzag position 0..63: the diagonals of an
+    8x8 block hold 1, 2, .., 8, 7, .., 1 positions, walked in turn."""
+    return np.repeat(np.arange(15), [min(d + 1, 15 - d) for d in range(15)])
+
+
+def zpr_streams(wl: Workload | str, batch: int | None = None, eob: int | None = None):
+    """Seeded symbol streams in the ZpR format (Sec. 3.3, Fig. 2), one per
+    image, for timing the inverse ZpR without an encoder: the coefficients of
+    each patch are drawn directly in zigzag order -- position k with the
+    Laplace scale of its frequency diagonal, as make_dct_inputs draws them --
+    and written as the stream format reads: literals as themselves, every
+    run of zeros before a literal as codes eob - 17 + n (n <= 16 zeros each),
+    nothing after the last literal, then eob.  Returns (symbols int32 [total],
+    per-image symbol counts int64 [B], n_blocks per image, eob)."""
+    if isinstance(wl, str):
+        wl = WORKLOADS[wl]
+    eob = DCT_CLIP + 17 if eob is None else eob
+    seeds = wl.seeds if batch is None else wl.seeds[:batch]
+    n = block_count(wl.H, wl.W, wl.L, wl.C)
+    scales = DCT_GAIN * wl.lap_scale * DCT_DECAY ** zigzag_diagonals()
+    out, counts = [], []
+    for s in seeds:
+        rng = np.random.Generator(np.random.PCG64([s, 11]))
+        z = np.clip(np.rint(rng.laplace(0.0, 1.0, (n, 64)) * scales), -DCT_CLIP, DCT_CLIP)
+        z = z.astype(np.int32)
+        blk, pos = np.nonzero(z)                          # literals, block-major, in position order
+        first = np.r_[True, blk[1:] != blk[:-1]]
+        prev = np.where(first, -1, np.r_[-1, pos[:-1]])
+        run = pos - prev - 1                              # zeros before each literal
+        ncode = (run + 15) // 16
+        per_lit = ncode + 1                               # symbols each literal brings
+        lits_per_blk = np.bincount(blk, minlength=n)
+        sym_per_blk = np.bincount(blk, weights=per_lit, minlength=n).astype(np.int64) + 1
+        blk_start = np.r_[0, np.cumsum(sym_per_blk)[:-1]]
+        total = int(sym_per_blk.sum())
+        stream = np.full(total, eob, dtype=np.int32)      # every slot not written below is a marker
+        cum = np.cumsum(per_lit)                          # over all literals, block-major
+        first_lit = np.r_[0, np.cumsum(lits_per_blk)[:-1]]
+        lit_end = blk_start[blk] + cum - np.r_[0, cum][first_lit][blk]  # one past each literal
+        stream[lit_end - 1] = z[blk, pos]                 # the literal, after its run codes
+        # run codes: ncode slots before the literal, full runs of 16 then the remainder
+        has = ncode > 0
+        idx = np.repeat(np.nonzero(has)[0], ncode[has])
+        j = np.arange(idx.size) - np.r_[0, np.cumsum(ncode[has])[:-1]].repeat(ncode[has])
+        slot = lit_end[idx] - 1 - ncode[idx] + j
+        left = run[idx] - 16 * j
+        stream[slot] = eob - 17 + np.minimum(left, 16)
+        out.append(stream)
+        counts.append(total)
+    return np.concatenate(out), np.array(counts, dtype=np.int64), n, eob
+
+
 def sample_pixels(H: int, W: int, n: int, seed: int) -> np.ndarray:
     """Flat pixel indices (y * W + x) to check at full size: the four corners,
     the middle of every border, and n seeded random positions."""

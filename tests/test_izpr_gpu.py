@@ -83,6 +83,10 @@ def test_malformed_streams_are_flagged():
         (np.array([1, 30, 2, 30], np.int32), 3),             # fewer markers than blocks
         (np.array([1, 30, 2, 30, 30], np.int32), 2),         # more markers than blocks
         (np.array([31, 30], np.int32), 1),                   # value above eob
+        (np.array([1, 30, 5], np.int32), 1),                 # symbols after the last marker
+        (np.zeros(0, np.int32), 2),                          # no symbols, two blocks expected
+        (np.r_[np.full(70, 3), 30].astype(np.int32), 1),     # 70 literals in one block
+        (np.r_[np.full(5000, 3), 30].astype(np.int32), 1),   # a block across a whole chunk
     ]
     for s, n in cases:
         with pytest.raises(pic.PicError):

@@ -53,3 +53,28 @@ def test_sample_pixels_include_corners():
     for idx in (0, 6, 63, 69):
         assert idx in p
     assert p.min() >= 0 and p.max() < 70
+
+
+def test_zpr_streams_are_the_oracle_encoding(orc):
+    """The direct stream generator writes exactly what the oracle's ZpR
+    encoder makes of the same coefficients (redrawn here in zigzag order and
+    scattered to raster order with the oracle's zigzag table)."""
+    wl = wk.custom("z", H=40, W=72, L=3, C=2, dims=(6, 8, 3), batch=3, lap_scale=3.0)
+    s, counts, n, eob = wk.zpr_streams(wl)
+    assert n == orc.block_count(40, 72, 3, 2) and eob == wk.DCT_CLIP + 17
+    assert counts.sum() == s.size
+    order = orc.zigzag()
+    scales = wk.DCT_GAIN * wl.lap_scale * wk.DCT_DECAY ** wk.zigzag_diagonals()
+    off = 0
+    for b in range(3):
+        rng = np.random.Generator(np.random.PCG64([wl.seeds[b], 11]))
+        z = np.clip(np.rint(rng.laplace(0.0, 1.0, (n, 64)) * scales), -255, 255).astype(np.int32)
+        raster = np.zeros_like(z)
+        raster[:, order] = z
+        assert np.array_equal(orc.zpr_encode(raster, eob), s[off:off + counts[b]])
+        off += counts[b]
+
+
+def test_zigzag_diagonals(orc):
+    order = orc.zigzag()
+    assert np.array_equal(wk.zigzag_diagonals(), order // 8 + order % 8)
