@@ -67,6 +67,8 @@ def algorithmic(wl: wk.Workload, batch: int):
 
 
 KERNEL_SOURCES = {
+    "idct": ["k_idct.cu"],
+    "izpr": ["k_izpr.cu"],
     "tc": ["k_tc.cuh", "tc_ptx.cuh", "pic_common.cuh", "pic_gelu.cuh", "pic_kernels.h"],
     "fp32": ["k_fp32.cu", "pic_common.cuh", "pic_gelu.cuh", "pic_kernels.h"],
 }
@@ -74,7 +76,8 @@ KERNEL_SOURCES = {
 
 def kernel_source_hash(kernel_name: str) -> str:
     """Hash of the source files a decode kernel is compiled from."""
-    files = KERNEL_SOURCES["tc" if kernel_name.startswith("tc") else "fp32"]
+    key = next((k for k in ("tc", "idct", "izpr") if kernel_name.startswith(k)), "fp32")
+    files = KERNEL_SOURCES[key]
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_09020_gb300", "csrc")
     for fn in files:
@@ -397,7 +400,11 @@ def run_stage(args):
                 if stage == "izpr" else "idct_unpatchify_kernel",
                 "avg_launch_us": ms * 1e3}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = None
+    roof["traffic"] = recorded_traffic("idct_unpatchify_kernel", "c5x64") if stage == "idct" \
+        else None
+    if stage == "izpr":
+        roof["traffic_note"] = ("one call is 3 kernels; ncu measured izpr_expand alone at "
+                                "104.4 MB read + 79.5 MB written (profiles/izpr__c5x64_launches_and_full.md)")
     roof["algorithmic_bytes_per_launch"] = nbytes
 
     # end to end with host buffers: H2D of the step's input, the stage, D2H of its result
