@@ -24,6 +24,9 @@ Parity status of each function (what pins it is in tests/test_oracle.py):
                       block counts of the decode workloads, round trip)
   zigzag / ZpR / iZpR pinned (hand-worked stream, JPEG zigzag table start,
                       round trips, malformed streams)
+  modulation fusion   pinned (closed-form statistics, normalised moments,
+                      fused == un-fused on random data and on whole decodes,
+                      the identity special case, brute-force statistics)
 """
 from __future__ import annotations
 
@@ -107,6 +110,18 @@ def _declare(lib):
     lib.pic_oracle_patchify_dct.restype = c_int
     lib.pic_oracle_unpatchify_idct.argtypes = [p, p, c_int, c_int, c_int, c_int, p]
     lib.pic_oracle_unpatchify_idct.restype = c_int
+    lib.pic_oracle_channel_stats.argtypes = [p, c_int, c_i64, p, p]
+    lib.pic_oracle_channel_stats.restype = None
+    lib.pic_oracle_norm_modulate.argtypes = [p, c_int, c_i64, p, p, p, p, p]
+    lib.pic_oracle_norm_modulate.restype = None
+    lib.pic_oracle_fuse_modulation.argtypes = [p, p, c_int, c_int, p, p, p, p, p, p]
+    lib.pic_oracle_fuse_modulation.restype = None
+    lib.pic_oracle_mlps_stats.argtypes = [p, p, p, c_int, c_int, c_int, p, c_int, c_int, c_int,
+                                          p, p, p]
+    lib.pic_oracle_mlps_stats.restype = c_int
+    lib.pic_oracle_decode_modulated.argtypes = [p, p, p, c_int, c_int, c_int, p, c_int, c_int,
+                                                p, p, p, p, c_int, c_int, p, p, c_int]
+    lib.pic_oracle_decode_modulated.restype = c_int
     return lib
 
 
@@ -271,6 +286,68 @@ class Oracle:
         out = np.empty(self.latent_count(H, W, L, C), dtype=np.float64)
         if self.lib.pic_oracle_unpatchify_idct(_ptr(s), _ptr(st), H, W, L, C, _ptr(out)) != 0:
             raise ValueError("unpatchify_idct rejected the shapes")
+        return out
+
+    # ---- modulation fusion (Sec. 3.1 Eqs. 2-3, App. A) -----------------
+    def channel_stats(self, f):
+        """Population mean and std per channel of f [C][N]."""
+        f = np.ascontiguousarray(f, dtype=np.float64)
+        C, N = f.shape
+        mu, sd = np.empty(C), np.empty(C)
+        self.lib.pic_oracle_channel_stats(_ptr(f), C, N, _ptr(mu), _ptr(sd))
+        return mu, sd
+
+    def norm_modulate(self, f, mu, sigma, gamma, beta):
+        f = np.ascontiguousarray(f, dtype=np.float64)
+        C, N = f.shape
+        a = [np.ascontiguousarray(v, dtype=np.float64) for v in (mu, sigma, gamma, beta)]
+        out = np.empty_like(f)
+        self.lib.pic_oracle_norm_modulate(_ptr(f), C, N, *[_ptr(v) for v in a], _ptr(out))
+        return out
+
+    def fuse_modulation(self, w, b, gamma, beta, mu, sigma):
+        """App. A: (w', b') of the fused MLP^i layer; w [dout][C]."""
+        w = np.ascontiguousarray(w, dtype=np.float64)
+        dout, C = w.shape
+        a = [np.ascontiguousarray(v, dtype=np.float64) for v in (b, gamma, beta, mu, sigma)]
+        wo, bo = np.empty_like(w), np.empty(dout)
+        self.lib.pic_oracle_fuse_modulation(_ptr(w), _ptr(a[0]), dout, C, *[_ptr(v) for v in a[1:]],
+                                            _ptr(wo), _ptr(bo))
+        return wo, bo
+
+    def mlps_stats(self, latents, steps, weights, H, W, L, C, dims, act):
+        """mu, sigma of the MLP^s output of one image over its pixels."""
+        q = np.ascontiguousarray(latents, dtype=np.int32).ravel()
+        s = np.ascontiguousarray(steps, dtype=np.float64).ravel()
+        w = np.ascontiguousarray(weights, dtype=np.float64).ravel()
+        d = np.ascontiguousarray(dims, dtype=np.int32)
+        cf = int(d[-2])
+        mu, sd = np.empty(cf), np.empty(cf)
+        work = np.empty(max(q.size, 1))
+        rc = self.lib.pic_oracle_mlps_stats(_ptr(q), _ptr(s), _ptr(w), L, C, len(d) - 1, _ptr(d),
+                                            ACTS[act], H, W, _ptr(mu), _ptr(sd), _ptr(work))
+        if rc != 0:
+            raise ValueError("mlps_stats rejected the arguments")
+        return mu, sd
+
+    def decode_modulated(self, latents, steps, weights, H, W, L, C, dims, act, gamma, beta, mu,
+                         sigma, clamp=True, nthreads: int = 1):
+        """Un-fused decode: MLP^s, normalise, modulate, MLP^i, clamp -> [3][H][W]."""
+        q = np.ascontiguousarray(latents, dtype=np.int32).ravel()
+        s = np.ascontiguousarray(steps, dtype=np.float64).ravel()
+        w = np.ascontiguousarray(weights, dtype=np.float64).ravel()
+        d = np.ascontiguousarray(dims, dtype=np.int32)
+        a = [np.ascontiguousarray(v, dtype=np.float64) for v in (gamma, beta, mu, sigma)]
+        if q.size != self.latent_count(H, W, L, C) or w.size != self.param_count(d):
+            raise ValueError("decode_modulated: buffer sizes do not match the shapes")
+        out = np.empty((3, H, W))
+        work = np.empty(max(q.size, 1))
+        rc = self.lib.pic_oracle_decode_modulated(_ptr(q), _ptr(s), _ptr(w), L, C, len(d) - 1,
+                                                  _ptr(d), ACTS[act], int(bool(clamp)),
+                                                  *[_ptr(v) for v in a], H, W, _ptr(out),
+                                                  _ptr(work), int(nthreads))
+        if rc != 0:
+            raise ValueError("decode_modulated rejected the arguments")
         return out
 
     # ---- ZpR / inverse ZpR (Sec. 3.3, Algorithm 1) ---------------------

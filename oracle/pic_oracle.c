@@ -175,6 +175,17 @@ static int check_args(int H, int W, int L, int C, int n_layers, const int *dims)
     return 0;
 }
 
+/* The upsampled feature vector of pixel (x, yy) (steps 2-3). */
+static void features_at(double *const *y, int L, int C, int H, int W, int x, int yy, double *f)
+{
+    int d = 0;
+    for (int l = 0; l < L; ++l) {
+        int Hl = level_size(H, l), Wl = level_size(W, l);
+        for (int c = 0; c < C; ++c)
+            f[d++] = pic_oracle_bilinear_at(y[l] + (int64_t)c * Hl * Wl, Hl, Wl, H, W, x, yy);
+    }
+}
+
 /*
  * Steps 1-5 at one pixel, given the dequantised levels y[l] (planar [C][H_l][W_l]).
  */
@@ -183,12 +194,7 @@ static int decode_pixel(double *const *y, int L, int C, const double *weights,
                         int H, int W, int x, int yy, double *rgb)
 {
     double f[PIC_ORACLE_MAX_WIDTH];
-    int d = 0;
-    for (int l = 0; l < L; ++l) {
-        int Hl = level_size(H, l), Wl = level_size(W, l);
-        for (int c = 0; c < C; ++c)
-            f[d++] = pic_oracle_bilinear_at(y[l] + (int64_t)c * Hl * Wl, Hl, Wl, H, W, x, yy);
-    }
+    features_at(y, L, C, H, W, x, yy, f);
     if (pic_oracle_mlp(f, weights, n_layers, dims, act, rgb) != 0) return -1;
     if (clamp)
         for (int c = 0; c < 3; ++c) rgb[c] = pic_oracle_clamp01(rgb[c]);
@@ -513,5 +519,152 @@ int pic_oracle_unpatchify_idct(const int32_t *symbols, const double *steps, int 
         }
         off += (int64_t)C * Hl * Wl;
     }
+    return 0;
+}
+
+/* ------------------------------------------------------------------------
+ * Modulation fusion (Sec. 3.1, Eqs. 2-3; App. A).
+ *
+ * g_s is MLP^s (every layer but the last, with its activations; shared by all
+ * images) followed by MLP^i (the last, linear layer).  For one image the
+ * encoder normalises the MLP^s output features f per channel over the H x W
+ * pixels, fbar = (f - mu) / sigma, modulates them, ftilde = gamma fbar +
+ * beta, and feeds ftilde to MLP^i.  App. A folds normalisation and
+ * modulation into MLP^i's weights, so the decoder needs only
+ *     w'[i][c] = w[i][c] gamma_c / sigma_c,
+ *     b'[i]    = b[i] + sum_c w[i][c] (beta_c - gamma_c mu_c / sigma_c).
+ * Reading: mean(f) and std(f) are the population mean and standard deviation
+ * over the image's pixels (divide by N, no epsilon).
+ * ------------------------------------------------------------------------ */
+
+/* Per-channel population mean and standard deviation of f [C][N] (two passes). */
+void pic_oracle_channel_stats(const double *f, int C, int64_t N, double *mu, double *sigma)
+{
+    for (int c = 0; c < C; ++c) {
+        const double *x = f + (int64_t)c * N;
+        double s = 0.0;
+        for (int64_t i = 0; i < N; ++i) s += x[i];
+        double m = s / (double)N, v = 0.0;
+        for (int64_t i = 0; i < N; ++i) v += (x[i] - m) * (x[i] - m);
+        mu[c] = m;
+        sigma[c] = sqrt(v / (double)N);
+    }
+}
+
+/* ftilde = gamma (f - mu) / sigma + beta, per channel, f and out [C][N]. */
+void pic_oracle_norm_modulate(const double *f, int C, int64_t N, const double *mu,
+                              const double *sigma, const double *gamma, const double *beta,
+                              double *out)
+{
+    for (int c = 0; c < C; ++c)
+        for (int64_t i = 0; i < N; ++i)
+            out[(int64_t)c * N + i] =
+                gamma[c] * ((f[(int64_t)c * N + i] - mu[c]) / sigma[c]) + beta[c];
+}
+
+/* App. A: the fused MLP^i layer w' [dout][C], b' [dout] from w, b, gamma, beta, mu, sigma. */
+void pic_oracle_fuse_modulation(const double *w, const double *b, int dout, int C,
+                                const double *gamma, const double *beta, const double *mu,
+                                const double *sigma, double *w_out, double *b_out)
+{
+    for (int i = 0; i < dout; ++i) {
+        double s = b[i];
+        for (int c = 0; c < C; ++c) {
+            w_out[(int64_t)i * C + c] = w[(int64_t)i * C + c] * gamma[c] / sigma[c];
+            s += w[(int64_t)i * C + c] * (beta[c] - gamma[c] * mu[c] / sigma[c]);
+        }
+        b_out[i] = s;
+    }
+}
+
+/* MLP^s at one pixel: the first n_layers - 1 layers, each followed by act;
+ * f receives dims[n_layers - 1] values. */
+static void mlps_at(const double *in, const double *weights, int n_layers, const int *dims,
+                    int act, double *f)
+{
+    double h[PIC_ORACLE_MAX_WIDTH], z[PIC_ORACLE_MAX_WIDTH];
+    for (int j = 0; j < dims[0]; ++j) h[j] = in[j];
+    const double *p = weights;
+    for (int k = 0; k < n_layers - 1; ++k) {
+        int din = dims[k], dout = dims[k + 1];
+        const double *Wk = p, *bk = p + (int64_t)dout * din;
+        for (int i = 0; i < dout; ++i) {
+            double acc = 0.0;
+            for (int j = 0; j < din; ++j) acc += Wk[(int64_t)i * din + j] * h[j];
+            z[i] = pic_oracle_act(acc + bk[i], act);
+        }
+        for (int i = 0; i < dout; ++i) h[i] = z[i];
+        p = bk + dout;
+    }
+    for (int i = 0; i < dims[n_layers - 1]; ++i) f[i] = h[i];
+}
+
+/* mu and sigma of the MLP^s output of one image over all its pixels (the
+ * encoder's statistics); `work` holds pic_oracle_latent_count doubles.
+ * Needs n_layers >= 2.  Returns 0 or -1. */
+int pic_oracle_mlps_stats(const int32_t *latents, const double *steps, const double *weights,
+                          int L, int C, int n_layers, const int *dims, int act, int H, int W,
+                          double *mu, double *sigma, double *work)
+{
+    double *y[PIC_ORACLE_MAX_LEVELS];
+    if (check_args(H, W, L, C, n_layers, dims) != 0 || n_layers < 2) return -1;
+    dequant_pyramid(latents, steps, L, C, H, W, work, y);
+    int Cf = dims[n_layers - 1];
+    double feat[PIC_ORACLE_MAX_WIDTH], f[PIC_ORACLE_MAX_WIDTH];
+    double s[PIC_ORACLE_MAX_WIDTH], v[PIC_ORACLE_MAX_WIDTH];
+    int64_t N = (int64_t)H * W;
+    for (int c = 0; c < Cf; ++c) s[c] = v[c] = 0.0;
+    for (int yy = 0; yy < H; ++yy)
+        for (int x = 0; x < W; ++x) {
+            features_at(y, L, C, H, W, x, yy, feat);
+            mlps_at(feat, weights, n_layers, dims, act, f);
+            for (int c = 0; c < Cf; ++c) s[c] += f[c];
+        }
+    for (int c = 0; c < Cf; ++c) mu[c] = s[c] / (double)N;
+    for (int yy = 0; yy < H; ++yy)
+        for (int x = 0; x < W; ++x) {
+            features_at(y, L, C, H, W, x, yy, feat);
+            mlps_at(feat, weights, n_layers, dims, act, f);
+            for (int c = 0; c < Cf; ++c) v[c] += (f[c] - mu[c]) * (f[c] - mu[c]);
+        }
+    for (int c = 0; c < Cf; ++c) sigma[c] = sqrt(v[c] / (double)N);
+    return 0;
+}
+
+/* The un-fused decode: per pixel MLP^s, then normalise and modulate with the
+ * given mu, sigma, gamma, beta, then MLP^i (the last layer of `weights`),
+ * then clamp.  Returns 0 or -1. */
+int pic_oracle_decode_modulated(const int32_t *latents, const double *steps, const double *weights,
+                                int L, int C, int n_layers, const int *dims, int act, int clamp,
+                                const double *gamma, const double *beta, const double *mu,
+                                const double *sigma, int H, int W, double *out_rgb, double *work,
+                                int nthreads)
+{
+    double *y[PIC_ORACLE_MAX_LEVELS];
+    if (check_args(H, W, L, C, n_layers, dims) != 0 || n_layers < 2) return -1;
+    dequant_pyramid(latents, steps, L, C, H, W, work, y);
+    int Cf = dims[n_layers - 1];
+    const double *wl = weights;  /* the last layer's W and b */
+    for (int k = 0; k < n_layers - 1; ++k) wl += (int64_t)dims[k + 1] * (dims[k] + 1);
+    const double *bl = wl + (int64_t)3 * Cf;
+    int64_t plane = (int64_t)H * W;
+#ifdef _OPENMP
+#pragma omp parallel for num_threads(nthreads > 0 ? nthreads : 1) schedule(static)
+#endif
+    for (int yy = 0; yy < H; ++yy) {
+        double feat[PIC_ORACLE_MAX_WIDTH], f[PIC_ORACLE_MAX_WIDTH];
+        for (int x = 0; x < W; ++x) {
+            features_at(y, L, C, H, W, x, yy, feat);
+            mlps_at(feat, weights, n_layers, dims, act, f);
+            for (int c = 0; c < Cf; ++c) f[c] = gamma[c] * ((f[c] - mu[c]) / sigma[c]) + beta[c];
+            for (int i = 0; i < 3; ++i) {
+                double s = 0.0;
+                for (int c = 0; c < Cf; ++c) s += wl[(int64_t)i * Cf + c] * f[c];
+                s += bl[i];
+                out_rgb[i * plane + (int64_t)yy * W + x] = clamp ? pic_oracle_clamp01(s) : s;
+            }
+        }
+    }
+    (void)nthreads;
     return 0;
 }

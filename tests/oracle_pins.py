@@ -474,4 +474,92 @@ def _level_ranges(o, H, W, L, C):
     return out
 
 
+# --------------------------------------- modulation fusion (Sec. 3.1, App. A)
+def pin_channel_stats_closed_form(o):
+    """Population mean / std: (1, 2, 3, 4) -> 2.5, sqrt(5/4); (-1, 1, -1, 1)
+    -> 0, 1 (dividing by N, not N - 1)."""
+    mu, sd = o.channel_stats(np.array([[1.0, 2, 3, 4], [-1, 1, -1, 1]]))
+    assert np.allclose(mu, [2.5, 0.0], atol=1e-15)
+    assert np.allclose(sd, [np.sqrt(1.25), 1.0], atol=1e-15)
+
+
+def pin_norm_modulate_moments(o):
+    """Normalised features have mean 0 and population std 1 per channel;
+    modulated ones have mean beta and std |gamma|."""
+    rng = np.random.Generator(np.random.PCG64(61))
+    f = rng.normal(3.0, 2.0, (5, 1000)) * rng.uniform(0.5, 4, (5, 1))
+    mu, sd = o.channel_stats(f)
+    z = o.norm_modulate(f, mu, sd, np.ones(5), np.zeros(5))
+    assert np.abs(z.mean(axis=1)).max() < 1e-12 and np.abs(z.std(axis=1) - 1).max() < 1e-12
+    g, b = rng.uniform(-2, 2, 5), rng.normal(0, 1, 5)
+    z = o.norm_modulate(f, mu, sd, g, b)
+    assert np.abs(z.mean(axis=1) - b).max() < 1e-12
+    assert np.abs(z.std(axis=1) - np.abs(g)).max() < 1e-12
+
+
+def pin_fusion_identity(o):
+    """App. A: the linear layer on normalised, modulated features equals the
+    fused layer (w', b') on the raw features, pixel by pixel; with
+    gamma = sigma and beta = mu the fusion leaves (w, b) unchanged."""
+    rng = np.random.Generator(np.random.PCG64(67))
+    C, N, dout = 16, 300, 3
+    f = rng.normal(1.0, 3.0, (C, N))
+    w, b = rng.normal(0, 0.3, (dout, C)), rng.normal(0, 0.1, dout)
+    g, be = rng.uniform(0.5, 1.5, C), rng.normal(0, 0.5, C)
+    mu, sd = o.channel_stats(f)
+    ref = w @ o.norm_modulate(f, mu, sd, g, be) + b[:, None]
+    wf, bf = o.fuse_modulation(w, b, g, be, mu, sd)
+    assert np.abs(wf @ f + bf[:, None] - ref).max() < 1e-12
+    wi, bi = o.fuse_modulation(w, b, sd, mu, mu, sd)
+    assert np.abs(wi - w).max() < 1e-15 and np.abs(bi - b).max() < 1e-15
+
+
+def _fuse_last_layer(o, weights, dims, g, be, mu, sd):
+    w = np.array(weights, dtype=np.float64)
+    off = sum(dims[k + 1] * (dims[k] + 1) for k in range(len(dims) - 2))
+    cf = dims[-2]
+    wl = w[off:off + 3 * cf].reshape(3, cf)
+    bl = w[off + 3 * cf: off + 3 * cf + 3]
+    wf, bf = o.fuse_modulation(wl, bl, g, be, mu, sd)
+    w[off:off + 3 * cf] = wf.ravel()
+    w[off + 3 * cf: off + 3 * cf + 3] = bf
+    return w
+
+
+def pin_decode_modulated_equals_fused(o):
+    """A whole decode: MLP^s -> normalise (the image's own mu, sigma) ->
+    modulate -> MLP^i equals the plain decode with the fused last layer
+    (unclamped, 2 channels, ragged sizes, both activations)."""
+    H, W, L, C = 13, 17, 3, 2
+    rng = np.random.Generator(np.random.PCG64(71))
+    for act, dims in (("relu", [6, 12, 8, 3]), ("gelu", [6, 10, 3])):
+        q = rng.integers(-9, 10, o.latent_count(H, W, L, C)).astype(np.int32)
+        st = np.array([1.0, 0.5, 0.25])
+        w = rng.normal(0, 0.4, o.param_count(dims))
+        mu, sd = o.mlps_stats(q, st, w, H, W, L, C, dims, act)
+        g, be = rng.uniform(0.5, 1.5, dims[-2]), rng.normal(0, 0.5, dims[-2])
+        ref = o.decode_modulated(q, st, w, H, W, L, C, dims, act, g, be, mu, sd, clamp=False)
+        got = o.decode(q, st, _fuse_last_layer(o, w, dims, g, be, mu, sd), H, W, L, C, dims, act,
+                       clamp=False)
+        assert np.abs(got - ref).max() < 1e-11 * max(1.0, np.abs(ref).max())
+
+
+def pin_mlps_stats_bruteforce(o):
+    """With MLP^s a single identity layer (W = I, b = 0, ReLU), its output is
+    ReLU of the upsampled latents, whose per-channel moments numpy computes
+    from the (pinned) upsampler directly."""
+    H, W, L, C = 12, 20, 2, 1
+    rng = np.random.Generator(np.random.PCG64(73))
+    q = rng.integers(-7, 8, o.latent_count(H, W, L, C)).astype(np.int32)
+    st = np.array([1.0, 0.5])
+    dims = [2, 2, 3]
+    w = np.concatenate([np.eye(2).ravel(), np.zeros(2), rng.normal(0, 1, 9)])
+    mu, sd = o.mlps_stats(q, st, w, H, W, L, C, dims, "relu")
+    l0 = q[:H * W].reshape(H, W) * 1.0
+    l1 = o.upsample(q[H * W:].reshape(6, 10) * 0.5, H, W)
+    f = np.maximum(np.stack([l0.ravel(), l1.ravel()]), 0.0)
+    assert np.abs(mu - f.mean(axis=1)).max() < 1e-13
+    assert np.abs(sd - f.std(axis=1)).max() < 1e-13
+
+
 PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

@@ -121,6 +121,27 @@ MUTATIONS = {
     "value_levels_ignore_channels": (
         "off += (int64_t)C * level_size(H, l) * level_size(W, l);\n    }\n}\n\n/* Steps 2-5",
         "off += (int64_t)level_size(H, l) * level_size(W, l);\n    }\n}\n\n/* Steps 2-5"),
+    "sample_std_not_population": (
+        "sigma[c] = sqrt(v / (double)N);\n    }\n}",
+        "sigma[c] = sqrt(v / (double)(N - 1));\n    }\n}"),
+    "fused_bias_sign": (
+        "s += w[(int64_t)i * C + c] * (beta[c] - gamma[c] * mu[c] / sigma[c]);",
+        "s += w[(int64_t)i * C + c] * (beta[c] + gamma[c] * mu[c] / sigma[c]);"),
+    "fused_weight_times_sigma": (
+        "w_out[(int64_t)i * C + c] = w[(int64_t)i * C + c] * gamma[c] / sigma[c];",
+        "w_out[(int64_t)i * C + c] = w[(int64_t)i * C + c] * gamma[c] * sigma[c];"),
+    "fused_bias_drops_beta": (
+        "s += w[(int64_t)i * C + c] * (beta[c] - gamma[c] * mu[c] / sigma[c]);",
+        "s += w[(int64_t)i * C + c] * (0.0 - gamma[c] * mu[c] / sigma[c]);"),
+    "mlps_without_last_activation": (
+        "z[i] = pic_oracle_act(acc + bk[i], act);",
+        "z[i] = (k == n_layers - 2) ? acc + bk[i] : pic_oracle_act(acc + bk[i], act);"),
+    "modulate_before_normalise": (
+        "for (int c = 0; c < Cf; ++c) f[c] = gamma[c] * ((f[c] - mu[c]) / sigma[c]) + beta[c];",
+        "for (int c = 0; c < Cf; ++c) f[c] = (gamma[c] * f[c] + beta[c] - mu[c]) / sigma[c];"),
+    "stats_second_pass_unshifted": (
+        "for (int c = 0; c < Cf; ++c) v[c] += (f[c] - mu[c]) * (f[c] - mu[c]);",
+        "for (int c = 0; c < Cf; ++c) v[c] += f[c] * f[c];"),
     "izpr_raster_not_zigzag": (
         "blk[order[pos++]] = s;",
         "blk[pos++] = s;"),
