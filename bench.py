@@ -227,7 +227,88 @@ STAGE_METRIC = {
              "Mblocks/s"),
     "pipeline": ("decoded megapixels/s from ZpR symbols (iZpR + iDCT + synthesis) at 1 GB300",
                  "MP/s"),
+    "fuse": ("modulation fusion (App. A): per-image decoder weight blobs/s at 1 GB300", "images/s"),
 }
+
+
+def run_fuse_stage(args):
+    """64 images' decoder weights (7-64-64-3, fp16 blobs for the tensor path)
+    from the shared g_s weights and each image's gamma, beta, mu, sigma."""
+    import torch
+    from paper_2609_09020_gb300 import build, pic
+    torch.cuda.set_device(0)
+    build.build()
+    wl = wk.WORKLOADS["c5"]
+    B, dims = wl.B, list(wl.dims)
+    shared_h = wk.make_inputs(wl, batch=1).weights[0].astype(np.float32)
+    cf = dims[-2]
+    mod_h = wk.make_modulation(B, cf, 0)
+    arch = pic.make_arch(wl.L, wl.C, dims, wl.act, "fp16_tc", max_H=wl.H, max_W=wl.W, max_batch=B)
+    shared, mod = torch.from_numpy(shared_h).cuda(), torch.from_numpy(mod_h).cuda()
+    out = torch.empty((B, shared_h.size), dtype=torch.float16, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step():
+        pic.fuse_modulation(arch, shared, mod, out=out, stream=stream)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    with ClockSampler(0) as clk:
+        ms = _event_time(step, args.steps, stream, torch)
+    peaks = load_peaks()
+    nbytes = 4 * shared_h.size + 4 * mod_h.size + 2 * B * shared_h.size
+    roof = {"bound": "hbm", "achieved": nbytes / (ms * 1e-3) / 1e9, "peak": peaks["hbm_gbs"],
+            "unit": "GB/s", "peak_source": f"copy bandwidth, {peaks['source']}",
+            "kernel": "fuse_kernel<half>", "avg_launch_us": ms * 1e3, "traffic": None,
+            "algorithmic_bytes_per_launch": nbytes,
+            "note": f"{nbytes / 1e6:.2f} MB per launch: launch-latency bound, far from any roofline"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    e2e = None
+    if not args.no_e2e:
+        mod_p = torch.from_numpy(mod_h).pin_memory()
+        out_p = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+
+        def e2e_step():
+            mod.copy_(mod_p, non_blocking=True)
+            step()
+            out_p.copy_(out, non_blocking=True)
+            torch.cuda.current_stream().synchronize()
+
+        e2e_step()
+        k = max(3, min(args.steps, 10))
+        t0 = time.perf_counter()
+        for _ in range(k):
+            e2e_step()
+        el = (time.perf_counter() - t0) / k
+        e2e = {"value": B / el, "unit": "images/s", "h2d_bytes_per_step": int(mod_h.nbytes),
+               "d2h_bytes_per_step": int(out_p.numel() * 2), "ms_per_step": 1e3 * el}
+    cpu = None
+    if not args.no_cpu_baseline:
+        import oracle
+        orc = oracle.load()
+        off = sum(dims[k + 1] * (dims[k] + 1) for k in range(len(dims) - 2))
+        w = shared_h[off:off + 3 * cf].astype(np.float64).reshape(3, cf)
+        bb = shared_h[off + 3 * cf:].astype(np.float64)
+        n, t0 = 0, time.perf_counter()
+        while time.perf_counter() - t0 < min(args.cpu_budget_s, 5.0):
+            g, be, mu, sd = mod_h[n % B].astype(np.float64)
+            orc.fuse_modulation(w, bb, g, be, mu, sd)
+            n += 1
+        el = time.perf_counter() - t0
+        cpu = {"value": n / el, "unit": "images/s", "cores": 1, "kind": "oracle",
+               "sample": f"{n} fusions of one image's last layer in {el:.1f} s (fp64 C oracle, "
+                         "one thread; the copy of the shared layers not included)"}
+    line = {"metric": STAGE_METRIC["fuse"][0], "value": B / (ms * 1e-3), "unit": "images/s",
+            "n_gpus": 1, "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32 arithmetic, f16 out",
+            "data": "synthetic (seeded weights; gamma, beta, mu, sigma stand-ins)",
+            "config": {"workload": f"fuse: {B} images, MLP {'-'.join(map(str, dims))}",
+                       "images": B, "params_per_image": int(shared_h.size),
+                       "l2": "inputs smaller than L2; back-to-back calls", "parallelism": "dp1"},
+            "roofline": roof, "clocks": clk.summary(), "e2e": e2e, "gpu_launches": args.steps,
+            "cpu_baseline": cpu, "stage": "fuse"}
+    print(json.dumps(line), flush=True)
 
 
 def _event_time(fn, steps, stream, torch):
@@ -477,7 +558,8 @@ def main():
     ap.add_argument("--ref-step-s", type=float, default=5.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--stage", default="decode", choices=["decode", "izpr", "idct", "pipeline"],
+    ap.add_argument("--stage", default="decode",
+                    choices=["decode", "izpr", "idct", "pipeline", "fuse"],
                     help="decode (default): the synthesis; the others time the stages before "
                          "it, alone or chained, on one GPU")
     ap.add_argument("--chunk", type=int, default=16,
@@ -488,7 +570,7 @@ def main():
             print(json.dumps({"stage": args.stage, "unavailable":
                               "stage benchmarks run our arm on one GPU only"}))
             return
-        run_stage(args)
+        run_fuse_stage(args) if args.stage == "fuse" else run_stage(args)
         return
 
     wl = wk.WORKLOADS[args.workload]

@@ -101,6 +101,8 @@ def load_library():
     lib.pic_idct_block_count.restype = i64
     lib.pic_idct_unpatchify.argtypes = [_P, _P, i, i, i, i, i, _P, _P]
     lib.pic_idct_unpatchify.restype = i
+    lib.pic_fuse_modulation.argtypes = [ctypes.POINTER(pic_arch), i, _P, _P, _P, _P]
+    lib.pic_fuse_modulation.restype = i
     lib.pic_status_string.argtypes = [i]
     lib.pic_status_string.restype = ctypes.c_char_p
     _lib = lib
@@ -241,6 +243,28 @@ def idct_unpatchify(coeffs, steps, H, W, L, C, out=None, stream=None):
                              _stream_ptr(stream))
     if rc != PIC_OK:
         raise PicError(rc, "pic_idct_unpatchify")
+    return out
+
+
+def pic_fuse_modulation(arch: pic_arch, B, shared, mod, weights_out, stream=None) -> int:
+    return load_library().pic_fuse_modulation(ctypes.byref(arch), B, shared, mod, weights_out,
+                                              stream)
+
+
+def fuse_modulation(arch: pic_arch, shared, mod, out=None, stream=None):
+    """App. A fusion on torch CUDA tensors: shared fp32 [P], mod fp32
+    [B][4][C'] (gamma, beta, mu, sigma); returns the per-image weight blobs
+    [B][P] (fp32, or fp16 for the tensor-core arch), enqueued on the stream."""
+    import torch
+    B = mod.shape[0]
+    P = pic_param_count(arch)
+    dt = torch.float16 if arch.precision == PIC_PREC_FP16_TC else torch.float32
+    if out is None:
+        out = torch.empty((B, P), dtype=dt, device=mod.device)
+    rc = pic_fuse_modulation(arch, B, shared.data_ptr(), mod.data_ptr(), out.data_ptr(),
+                             _stream_ptr(stream))
+    if rc != PIC_OK:
+        raise PicError(rc, "pic_fuse_modulation")
     return out
 
 

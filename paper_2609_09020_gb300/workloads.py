@@ -318,6 +318,20 @@ def zpr_streams(wl: Workload | str, batch: int | None = None, eob: int | None = 
     return np.concatenate(out), np.array(counts, dtype=np.int64), n, eob
 
 
+def make_modulation(B: int, cf: int, seed: int) -> np.ndarray:
+    """Seeded stand-ins for g_m's modulation vectors and an image's feature
+    statistics (g_m is a trained network, not available): float32 [B][4][cf]
+    rows gamma ~ U(0.5, 1.5), beta ~ N(0, 0.5^2), mu ~ U(0, 2),
+    sigma ~ U(0.3, 2)."""
+    rng = np.random.Generator(np.random.PCG64([seed, 13]))
+    m = np.empty((B, 4, cf))
+    m[:, 0] = rng.uniform(0.5, 1.5, (B, cf))
+    m[:, 1] = rng.normal(0.0, 0.5, (B, cf))
+    m[:, 2] = rng.uniform(0.0, 2.0, (B, cf))
+    m[:, 3] = rng.uniform(0.3, 2.0, (B, cf))
+    return m.astype(np.float32)
+
+
 def sample_pixels(H: int, W: int, n: int, seed: int) -> np.ndarray:
     """Flat pixel indices (y * W + x) to check at full size: the four corners,
     the middle of every border, and n seeded random positions."""

@@ -119,3 +119,13 @@ def test_fp32_latent_arch_is_validated(lib):
     a = pic.make_arch(2, 1, [2, 8, 3], max_H=8, max_W=8, latent=2)
     h = pic._P()
     assert lib.pic_decode_create(pic.ctypes.byref(a), pic.ctypes.byref(h)) == pic.PIC_ERR_UNSUPPORTED
+
+
+def test_fuse_modulation_argument_checks(lib):
+    from paper_2609_09020_gb300 import pic
+    a = pic.make_arch(7, 1, [7, 64, 64, 3], max_H=8, max_W=8)
+    assert pic.pic_fuse_modulation(a, 1, None, None, None) == pic.PIC_ERR_INVALID_ARG
+    assert pic.pic_fuse_modulation(a, 0, 16, 16, 16) == pic.PIC_ERR_INVALID_ARG
+    assert pic.pic_fuse_modulation(a, 1, 16, 16, 8) == pic.PIC_ERR_INVALID_ARG  # misaligned out
+    one = pic.make_arch(7, 1, [7, 3], max_H=8, max_W=8)  # no MLP^s to fuse after
+    assert pic.pic_fuse_modulation(one, 1, 16, 16, 16) == pic.PIC_ERR_INVALID_ARG
