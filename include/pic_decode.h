@@ -78,6 +78,12 @@ typedef enum {
     PIC_LATENT_FP32 = 1
 } pic_latent_format;
 
+typedef enum {
+    PIC_OUT_F32_CHW = 0, /* fp32 planar [3][H][W] (R, G, B planes) -- the default */
+    PIC_OUT_F32_HWC = 1, /* fp32 interleaved [H][W][3] */
+    PIC_OUT_U8_HWC = 2   /* uint8 interleaved [H][W][3]: round-half-even(255 clamp(v, 0, 1)) */
+} pic_output_format;
+
 /* Architecture of one decoder instance (fixed at create). */
 typedef struct {
     int num_levels;         /* L, 1..12 */
@@ -90,6 +96,7 @@ typedef struct {
     int max_H, max_W;       /* largest image accepted by the decode calls */
     int max_batch;          /* largest B accepted by pic_decode_batch */
     int latent_format;      /* pic_latent_format; same layout and size (4 B) either way */
+    int output_format;      /* pic_output_format (uint8 output always clamps) */
 } pic_arch;
 
 /*
@@ -116,22 +123,25 @@ int pic_decode_create(const pic_arch *arch, pic_decoder **out);
  *             b_k [dims[k+1]]; pic_param_count(arch) values; float for
  *             PIC_PREC_FP32, IEEE half (uint16 bits) for PIC_PREC_FP16_TC.
  *   H, W    : image size, 1..max_H, 1..max_W.
- *   out_rgb : float, device; planar [3][H][W] (R, G, B planes).
+ *   out_rgb : device, 16-byte aligned, in the arch's output_format: fp32
+ *             planar [3][H][W] (R, G, B planes), fp32 [H][W][3], or uint8
+ *             [H][W][3].
  * Errors: PIC_ERR_INVALID_ARG (NULL handle/pointer, misaligned pointer, H or W
  * out of range) with nothing launched; PIC_ERR_CUDA if the launch failed.
  */
 int pic_decode(pic_decoder *h, const int32_t *latents, const float *steps, const void *weights,
-               int H, int W, float *out_rgb, void *stream);
+               int H, int W, void *out_rgb, void *stream);
 
 /*
  * Decodes B independent images of the same size in one launch.  Image b uses
  * latents + b * pic_latent_count(H, W, L, C), steps + b * L,
- * weights + b * pic_param_count(arch) and writes out_rgb + b * 3 * H * W
+ * weights + b * pic_param_count(arch) and writes the image's 3 * H * W
+ * outputs at out_rgb + b * 3 * H * W elements
  * (all images' buffers are contiguous, image-major).  B in 1..max_batch;
  * other arguments and errors as pic_decode.
  */
 int pic_decode_batch(pic_decoder *h, int B, const int32_t *latents, const float *steps,
-                     const void *weights, int H, int W, float *out_rgb, void *stream);
+                     const void *weights, int H, int W, void *out_rgb, void *stream);
 
 /*
  * End-to-end convenience for callers holding HOST buffers (same layouts as
@@ -143,7 +153,7 @@ int pic_decode_batch(pic_decoder *h, int B, const int32_t *latents, const float 
  * Errors: as pic_decode_batch, plus PIC_ERR_ALLOC.
  */
 int pic_decode_batch_host(pic_decoder *h, int B, const int32_t *latents, const float *steps,
-                          const void *weights, int H, int W, float *out_rgb, void *stream);
+                          const void *weights, int H, int W, void *out_rgb, void *stream);
 
 /*
  * Synchronises `stream` and reports whether any kernel of this handle
@@ -174,7 +184,7 @@ int pic_decode_check(pic_decoder *h, void *stream);
  */
 int pic_decode_batch_noalloc(const pic_arch *arch, int B, const int32_t *latents,
                              const float *steps, const void *weights, int H, int W,
-                             float *out_rgb, void *stream);
+                             void *out_rgb, void *stream);
 
 /* Frees the handle and its device state.  NULL is a no-op.  Synchronises the
  * device first, so that no kernel of this handle is still running. */

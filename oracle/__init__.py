@@ -85,6 +85,8 @@ def _declare(lib):
     lib.pic_oracle_mlp.restype = c_int
     lib.pic_oracle_clamp01.argtypes = [c_dbl]
     lib.pic_oracle_clamp01.restype = c_dbl
+    lib.pic_oracle_to_u8.argtypes = [c_dbl]
+    lib.pic_oracle_to_u8.restype = c_int
     lib.pic_oracle_decode.argtypes = [p, p, p, c_int, c_int, c_int, p, c_int, c_int,
                                       c_int, c_int, p, p, c_int]
     lib.pic_oracle_decode.restype = c_int
@@ -194,6 +196,9 @@ class Oracle:
 
     def clamp01(self, v: float) -> float:
         return float(self.lib.pic_oracle_clamp01(float(v)))
+
+    def to_u8(self, v: float) -> int:
+        return int(self.lib.pic_oracle_to_u8(float(v)))
 
     # ---- whole decode --------------------------------------------------
     def decode(self, latents, steps, weights, H, W, L, C, dims, act, clamp=True,

@@ -165,6 +165,13 @@ double pic_oracle_clamp01(double v)
     return v;
 }
 
+/* The 8-bit output variant: round-half-even(255 clamp(v, 0, 1)) (the decode
+ * statement's clamp to [0, 1], scaled to the byte range). */
+int pic_oracle_to_u8(double v)
+{
+    return (int)nearbyint(255.0 * pic_oracle_clamp01(v));
+}
+
 /* Checks shared by the two decode entry points. */
 static int check_args(int H, int W, int L, int C, int n_layers, const int *dims)
 {

@@ -187,10 +187,8 @@ __global__ void __launch_bounds__(kThreads)
       rgb[0] = h[0]; rgb[1] = h[1]; rgb[2] = h[2];
     }
 
-    // ---- step 5: clamp, planar coalesced stores ----
-    float* o = p.out + static_cast<long long>(b) * 3 * plane + static_cast<long long>(y) * p.W + x;
-#pragma unroll
-    for (int c = 0; c < 3; ++c) o[c * plane] = p.clamp ? __saturatef(rgb[c]) : rgb[c];
+    // ---- step 5: clamp and store (planar rows are coalesced) ----
+    store_rgb(p, b, y, x, rgb[0], rgb[1], rgb[2]);
   }
 }
 
@@ -244,8 +242,7 @@ __global__ void __launch_bounds__(kThreads) fp32_generic_kernel(const DecodePara
       for (int i = 0; i < dout; ++i) h[i] = g[i];
       wl += dout * din + dout;
     }
-    float* o = p.out + static_cast<long long>(b) * 3 * plane + static_cast<long long>(y) * p.W + x;
-    for (int c = 0; c < 3; ++c) o[c * plane] = p.clamp ? __saturatef(h[c]) : h[c];
+    store_rgb(p, b, y, x, h[0], h[1], h[2]);
   }
 }
 
@@ -280,6 +277,11 @@ int fp32_kernels(KernelInfo* out, int cap) {
       make_fp32<2, 4, 16, 64, 64, 64, 3, ACT_GELU>("fp32_16x64x64x64x3_gelu"),
       make_fp32<1, 3, 7, 64, 64, 3, 0, ACT_RELU>("fp32_7x64x64x3_relu"),
       make_fp32<1, 3, 7, 64, 64, 3, 0, ACT_RELU, true>("fp32_7x64x64x3_relu_f32lat"),
+      // the width ablation's architectures
+      make_fp32<1, 4, 8, 8, 8, 8, 3, ACT_RELU>("fp32_8x8x8x8x3_relu"),
+      make_fp32<1, 4, 8, 16, 16, 16, 3, ACT_RELU>("fp32_8x16x16x16x3_relu"),
+      make_fp32<1, 4, 8, 32, 32, 32, 3, ACT_RELU>("fp32_8x32x32x32x3_relu"),
+      make_fp32<1, 4, 8, 64, 64, 64, 3, ACT_RELU>("fp32_8x64x64x64x3_relu"),
   };
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
   for (int i = 0; i < n && i < cap; ++i) out[i] = list[i];

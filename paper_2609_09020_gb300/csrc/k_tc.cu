@@ -23,7 +23,9 @@ int tc_kernels(KernelInfo* out, int cap) {
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
   int k = 0;
   for (; k < n && k < cap; ++k) out[k] = list[k];
-  return k + (k < cap ? tc_kernels_fp32lat(out + k, cap - k) : 0);
+  if (k < cap) k += tc_kernels_fp32lat(out + k, cap - k);
+  if (k < cap) k += tc_kernels_sweep(out + k, cap - k);
+  return k;
 }
 
 }  // namespace pic

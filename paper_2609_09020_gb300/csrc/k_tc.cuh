@@ -496,7 +496,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         }
         if (!ok) break;
 
-        // ---- output layer: bias, clamp, planar coalesced store ----
+        // ---- output layer: bias, clamp, store ----
         if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
         acc_phase ^= 1u;
         tc_fence_after();
@@ -506,14 +506,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         tc_fence_before();
         if (has_next) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
         const int x = x0 + r;
-        if (x < p.W) {
-          float* dst = p.out + static_cast<long long>(b) * 3 * plane + static_cast<long long>(y) * p.W + x;
-#pragma unroll
-          for (int c = 0; c < 3; ++c) {
-            const float v = __uint_as_float(o[c]);
-            dst[c * plane] = p.clamp ? __saturatef(v) : v;
-          }
-        }
+        if (x < p.W)
+          store_rgb(p, b, y, x, __uint_as_float(o[0]), __uint_as_float(o[1]), __uint_as_float(o[2]));
         cy = ny;
         ctx = ntx;
       }

@@ -28,9 +28,10 @@ struct DecodeParams {
   const int32_t* latents;      // int32 symbols, or fp32 values (PIC_LATENT_FP32) as 32-bit words
   const float* steps;
   const void* weights;
-  float* out;
+  void* out;                   // fp32 [B][3][H][W], fp32 [B][H][W][3] or uint8 [B][H][W][3]
   int H, W, B, L, C;
   int clamp;
+  int out_format;              // OUT_F32_CHW, OUT_F32_HWC or OUT_U8_HWC
   long long lat_per_image;     // sum_l C H_l W_l
   long long params_per_image;  // sum_k d_{k+1} (d_k + 1)
   int tiles_per_row;
@@ -44,6 +45,39 @@ struct DecodeParams {
 };
 
 enum { ACT_RELU = 0, ACT_GELU = 1 };
+enum { OUT_F32_CHW = 0, OUT_F32_HWC = 1, OUT_U8_HWC = 2 };
+
+// Step 5 for pixel (x, y) of image b: clamp (unless the handle asks for raw
+// values) and store in the handle's output format.  uint8 is
+// round-half-even(255 clamp(v, 0, 1)) and always clamps.
+__device__ __forceinline__ void store_rgb(const DecodeParams& p, int b, int y, int x, float r, float g,
+                                          float bl) {
+  const long long plane = static_cast<long long>(p.H) * p.W;
+  const long long pix = static_cast<long long>(y) * p.W + x;
+  if (p.out_format == OUT_U8_HWC) {
+    uint8_t* o = static_cast<uint8_t*>(p.out) + (static_cast<long long>(b) * plane + pix) * 3;
+    o[0] = static_cast<uint8_t>(__float2int_rn(__saturatef(r) * 255.0f));
+    o[1] = static_cast<uint8_t>(__float2int_rn(__saturatef(g) * 255.0f));
+    o[2] = static_cast<uint8_t>(__float2int_rn(__saturatef(bl) * 255.0f));
+    return;
+  }
+  if (p.clamp) {
+    r = __saturatef(r);
+    g = __saturatef(g);
+    bl = __saturatef(bl);
+  }
+  if (p.out_format == OUT_F32_HWC) {
+    float* o = static_cast<float*>(p.out) + (static_cast<long long>(b) * plane + pix) * 3;
+    o[0] = r;
+    o[1] = g;
+    o[2] = bl;
+  } else {
+    float* o = static_cast<float*>(p.out) + static_cast<long long>(b) * 3 * plane + pix;
+    o[0] = r;
+    o[plane] = g;
+    o[2 * plane] = bl;
+  }
+}
 
 // GELU in its erf form, z * Phi(z), with CUDA's erff (reference variant).
 __device__ __forceinline__ float gelu_erf(float z) {

@@ -48,6 +48,7 @@ bool arch_valid(const pic_arch* a) {
   if (a->max_H < 1 || a->max_W < 1 || a->max_batch < 1) return false;
   if (a->max_H > 65536 || a->max_W > 65536 || a->max_batch > 65536) return false;
   if (a->latent_format != PIC_LATENT_INT32 && a->latent_format != PIC_LATENT_FP32) return false;
+  if (a->output_format < PIC_OUT_F32_CHW || a->output_format > PIC_OUT_U8_HWC) return false;
   return true;
 }
 
@@ -64,7 +65,7 @@ bool kernel_matches(const KernelInfo& k, const pic_arch* a) {
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 int check_decode_args(const pic_decoder* h, int B, const int32_t* latents, const float* steps,
-                      const void* weights, int H, int W, const float* out) {
+                      const void* weights, int H, int W, const void* out) {
   const bool need_steps = h && h->arch.latent_format == PIC_LATENT_INT32;
   if (!h || !latents || (need_steps && !steps) || !weights || !out) return PIC_ERR_INVALID_ARG;
   if (B < 1 || B > h->arch.max_batch) return PIC_ERR_INVALID_ARG;
@@ -75,7 +76,7 @@ int check_decode_args(const pic_decoder* h, int B, const int32_t* latents, const
 }
 
 void fill_params(const pic_decoder* h, DecodeParams& p, int B, const int32_t* latents,
-                 const float* steps, const void* weights, int H, int W, float* out) {
+                 const float* steps, const void* weights, int H, int W, void* out) {
   std::memset(&p, 0, sizeof(p));
   const pic_arch& a = h->arch;
   p.latents = latents;
@@ -88,6 +89,7 @@ void fill_params(const pic_decoder* h, DecodeParams& p, int B, const int32_t* la
   p.L = a.num_levels;
   p.C = a.channels_per_level;
   p.clamp = a.clamp_output;
+  p.out_format = a.output_format;
   p.status = h->d_status;
   p.n_layers = a.num_layers;
   for (int k = 0; k <= a.num_layers; ++k) p.dims[k] = a.dims[k];
@@ -237,7 +239,7 @@ int pic_decode_create(const pic_arch* arch, pic_decoder** out) {
 }
 
 int pic_decode_batch(pic_decoder* h, int B, const int32_t* latents, const float* steps,
-                     const void* weights, int H, int W, float* out_rgb, void* stream) {
+                     const void* weights, int H, int W, void* out_rgb, void* stream) {
   int rc = check_decode_args(h, B, latents, steps, weights, H, W, out_rgb);
   if (rc != PIC_OK) return rc;
   DecodeParams p;
@@ -246,12 +248,12 @@ int pic_decode_batch(pic_decoder* h, int B, const int32_t* latents, const float*
 }
 
 int pic_decode(pic_decoder* h, const int32_t* latents, const float* steps, const void* weights,
-               int H, int W, float* out_rgb, void* stream) {
+               int H, int W, void* out_rgb, void* stream) {
   return pic_decode_batch(h, 1, latents, steps, weights, H, W, out_rgb, stream);
 }
 
 int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const float* steps,
-                          const void* weights, int H, int W, float* out_rgb, void* stream) {
+                          const void* weights, int H, int W, void* out_rgb, void* stream) {
   if (!h || !latents || (h->arch.latent_format == PIC_LATENT_INT32 && !steps) || !weights ||
       !out_rgb)
     return PIC_ERR_INVALID_ARG;
@@ -282,7 +284,8 @@ int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const f
   const long long lat_bytes = static_cast<long long>(B) *
                               pic_latent_count(H, W, a.num_levels, a.channels_per_level) * 4;
   const long long w_bytes = static_cast<long long>(B) * h->n_params * weight_elem_bytes(a);
-  const long long out_bytes = static_cast<long long>(B) * 3LL * H * W * 4;
+  const long long out_bytes = static_cast<long long>(B) * 3LL * H * W *
+                              (a.output_format == PIC_OUT_U8_HWC ? 1 : 4);
   if (cudaMemcpyAsync(h->s_lat, latents, lat_bytes, cudaMemcpyHostToDevice, s) != cudaSuccess ||
       (steps && cudaMemcpyAsync(h->s_steps, steps, static_cast<size_t>(B) * a.num_levels * 4,
                                 cudaMemcpyHostToDevice, s) != cudaSuccess) ||
@@ -393,7 +396,7 @@ int static_scratch(int dev, int** out) {
 
 extern "C" int pic_decode_batch_noalloc(const pic_arch* arch, int B, const int32_t* latents,
                                         const float* steps, const void* weights, int H, int W,
-                                        float* out_rgb, void* stream) {
+                                        void* out_rgb, void* stream) {
   if (!arch) return PIC_ERR_INVALID_ARG;
   if (arch->num_layers < 1 || arch->num_layers > pic::kMaxLayers) return PIC_ERR_INVALID_ARG;
   if (arch->dims[0] != arch->num_levels * arch->channels_per_level ||

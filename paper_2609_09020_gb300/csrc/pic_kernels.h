@@ -24,5 +24,6 @@ int fp32_kernels(KernelInfo* out, int cap);
 KernelInfo fp32_generic_kernel_info(int latent_format);
 int tc_kernels(KernelInfo* out, int cap);     // both latent formats
 int tc_kernels_fp32lat(KernelInfo* out, int cap);  // the fp32-latent ones (own translation unit)
+int tc_kernels_sweep(KernelInfo* out, int cap);    // the width ablation's (own translation unit)
 
 }  // namespace pic

@@ -34,6 +34,10 @@ PIC_LATENT_FP32 = 1
 ACTS = {"relu": PIC_ACT_RELU, "gelu": PIC_ACT_GELU}
 PRECS = {"fp32": PIC_PREC_FP32, "fp16_tc": PIC_PREC_FP16_TC}
 LATENTS = {"int32": PIC_LATENT_INT32, "fp32": PIC_LATENT_FP32}
+PIC_OUT_F32_CHW = 0
+PIC_OUT_F32_HWC = 1
+PIC_OUT_U8_HWC = 2
+OUTPUTS = {"f32_chw": PIC_OUT_F32_CHW, "f32_hwc": PIC_OUT_F32_HWC, "u8_hwc": PIC_OUT_U8_HWC}
 
 
 class pic_arch(ctypes.Structure):
@@ -49,6 +53,7 @@ class pic_arch(ctypes.Structure):
         ("max_W", ctypes.c_int),
         ("max_batch", ctypes.c_int),
         ("latent_format", ctypes.c_int),
+        ("output_format", ctypes.c_int),
     ]
 
 
@@ -117,7 +122,7 @@ class PicError(RuntimeError):
 
 
 def make_arch(L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1, max_W=1,
-              max_batch=1, latent="int32") -> pic_arch:
+              max_batch=1, latent="int32", output="f32_chw") -> pic_arch:
     a = pic_arch()
     a.num_levels, a.channels_per_level, a.num_layers = L, C, len(dims) - 1
     for k, d in enumerate(dims):
@@ -127,6 +132,7 @@ def make_arch(L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1, max
     a.clamp_output = int(bool(clamp))
     a.max_H, a.max_W, a.max_batch = max_H, max_W, max_batch
     a.latent_format = LATENTS[latent] if isinstance(latent, str) else int(latent)
+    a.output_format = OUTPUTS[output] if isinstance(output, str) else int(output)
     return a
 
 
@@ -281,16 +287,18 @@ class Decoder:
     contiguous CUDA tensors of the documented dtypes."""
 
     def __init__(self, L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1,
-                 max_W=1, max_batch=1, latent="int32"):
-        self.arch = make_arch(L, C, dims, act, precision, clamp, max_H, max_W, max_batch, latent)
+                 max_W=1, max_batch=1, latent="int32", output="f32_chw"):
+        self.arch = make_arch(L, C, dims, act, precision, clamp, max_H, max_W, max_batch, latent,
+                              output)
         self.latent = latent
         self.L, self.C, self.dims, self.precision = L, C, tuple(dims), precision
         self.handle = pic_decode_create(self.arch)
 
     @classmethod
-    def for_workload(cls, wl, precision: str, clamp=True, max_batch=None, latent="int32"):
+    def for_workload(cls, wl, precision: str, clamp=True, max_batch=None, latent="int32",
+                     output="f32_chw"):
         return cls(wl.L, wl.C, wl.dims, wl.act, precision, clamp, wl.H, wl.W,
-                   max_batch or wl.B, latent)
+                   max_batch or wl.B, latent, output)
 
     @property
     def kernel_name(self) -> str:

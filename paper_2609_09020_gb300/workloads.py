@@ -121,6 +121,18 @@ WORKLOADS = {
                    note="batch of 64 Kodak-sized images, 7-64-64-3 ReLU, fp16 weights"),
 }
 
+# The decoding-speed ablation over the synthesis network's width (Sec. 4.3,
+# "Decoding speed for different width"): the paper's own g_s -- L = 8
+# single-channel latents, a 4-layer MLP with ReLU -- at widths 8, 16 (the
+# paper's choice), 32 and 64, on batches of 64 Kodak-sized images.
+for _w in (8, 16, 32, 64):
+    WORKLOADS[f"w{_w}"] = Workload(
+        f"w{_w}", H=512, W=768, L=8, C=1, dims=(8, _w, _w, _w, 3), act="relu",
+        weight_dtype="fp16", lap_scale=3.0, clip=31, seeds=tuple(range(200, 264)),
+        precisions=("fp32", "fp16_tc"),
+        note=f"batch of 64 Kodak-sized images, 8 levels x 1 ch, 8-{_w}-{_w}-{_w}-3 ReLU, fp16 weights")
+del _w
+
 
 @dataclass
 class Inputs:

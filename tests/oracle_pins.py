@@ -220,6 +220,14 @@ def pin_clamp(o):
 
 
 # ---------------------------------------------------------------- decode
+def pin_to_u8(o):
+    """round-half-even(255 clamp(v)): 0.25 -> 63.75 -> 64, 0.75 -> 191.25 ->
+    191, 0.5 -> 127.5 -> 128 (the even neighbour), saturation at both ends."""
+    for v, want in ((0.0, 0), (1.0, 255), (-3.0, 0), (7.0, 255), (0.25, 64), (0.75, 191),
+                    (0.5, 128), (1.0 / 255.0, 1), (254.4 / 255.0, 254)):
+        assert o.to_u8(v) == want, (v, o.to_u8(v), want)
+
+
 def pin_decode_hand_4x4(o):
     """The hand-computed 4x4 image (tests/golden/hand_4x4.txt)."""
     g = load_golden("hand_4x4.txt")

@@ -129,3 +129,10 @@ def test_fuse_modulation_argument_checks(lib):
     assert pic.pic_fuse_modulation(a, 1, 16, 16, 8) == pic.PIC_ERR_INVALID_ARG  # misaligned out
     one = pic.make_arch(7, 1, [7, 3], max_H=8, max_W=8)  # no MLP^s to fuse after
     assert pic.pic_fuse_modulation(one, 1, 16, 16, 16) == pic.PIC_ERR_INVALID_ARG
+
+
+def test_output_format_is_validated(lib):
+    from paper_2609_09020_gb300 import pic
+    a = pic.make_arch(2, 1, [2, 8, 3], max_H=8, max_W=8, output=3)
+    h = pic._P()
+    assert lib.pic_decode_create(pic.ctypes.byref(a), pic.ctypes.byref(h)) == pic.PIC_ERR_UNSUPPORTED

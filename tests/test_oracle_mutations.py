@@ -142,6 +142,12 @@ MUTATIONS = {
     "stats_second_pass_unshifted": (
         "for (int c = 0; c < Cf; ++c) v[c] += (f[c] - mu[c]) * (f[c] - mu[c]);",
         "for (int c = 0; c < Cf; ++c) v[c] += f[c] * f[c];"),
+    "u8_truncates": (
+        "return (int)nearbyint(255.0 * pic_oracle_clamp01(v));",
+        "return (int)floor(255.0 * pic_oracle_clamp01(v));"),
+    "u8_scale_256": (
+        "return (int)nearbyint(255.0 * pic_oracle_clamp01(v));",
+        "return (int)nearbyint(256.0 * pic_oracle_clamp01(v)) > 255 ? 255 : (int)nearbyint(256.0 * pic_oracle_clamp01(v));"),
     "izpr_raster_not_zigzag": (
         "blk[order[pos++]] = s;",
         "blk[pos++] = s;"),
