@@ -701,13 +701,18 @@ def main():
     roof["algorithmic_flops_per_launch"] = flops
     if precision == "fp16_tc":
         # MACs the tensor cores execute per pixel: layer 0 (K = round16(2 D0 + 1),
-        # N = round16 of the width), hidden layers and the output layer (N = 16)
-        # with the hi and lo halves of K plus one K = 16 bias step each.
+        # N = round16 of the width), hidden layers and (for wide, shallow nets)
+        # the output layer (N = 16), with the hi and lo halves of K plus one
+        # K = 16 bias step each.
         def r16(v):
             return (v + 15) // 16 * 16
         n_pad = r16(max(wl.dims[1:-1]))
         mac = r16(2 * wl.dims[0] + 1) * n_pad
-        mac += (len(wl.dims) - 3) * (2 * n_pad + 16) * n_pad + (2 * n_pad + 16) * 16
+        mac += (len(wl.dims) - 3) * (2 * n_pad + 16) * n_pad
+        # the output layer runs on the tensor cores only for wide, shallow
+        # nets (N > 32 and fewer than 4 layers); else on the CUDA cores
+        if n_pad > 32 and len(wl.dims) - 1 < 4:
+            mac += (2 * n_pad + 16) * 16
         roof["executed_tensor_flops_per_launch"] = 2.0 * mac * B * wl.H * wl.W
     roof["algorithmic_bytes_per_launch"] = nbytes
     roof["binding_time_us"] = max(t_pipe, t_hbm) * 1e6

@@ -23,7 +23,9 @@
 //   hidden   A  = [h_hi | h_lo]            TMEM, N/2 + N/2 columns (2 fp16 per column)
 //            B  = [W_k | b_k 0..0]          smem; W_k serves the hi and the lo half,
 //                                           b_k meets a shared constant tile [1 0..0]
-//   output   the same with W_out, b_out padded to 16 rows
+//   output   the same with W_out, b_out padded to 16 rows -- or, for narrow
+//            or deep nets (Net::OUTCC), on the CUDA cores in fp32 inside the
+//            last hidden layer's epilogue, which saves an MMA round trip
 //
 // CTA organisation (one CTA per SM, persistent over a contiguous tile range):
 //   warps 0 .. 4*NWG-1 : NWG warpgroups; group w owns every NWG-th tile of the
@@ -96,6 +98,12 @@ struct TcNet {
   static constexpr int C = C_, NL = NL_, D0 = D0_, N = N_, ACT = ACT_, NWG = NWG_;
   static constexpr int L = D0 / C;
   static constexpr int K1 = round_up(2 * D0 + 1, 16);
+  // Output layer on the CUDA cores (fp32, one MMA round trip less per tile)
+  // when the hidden width is small or the net deep enough that the saved
+  // round trip outweighs the extra FMAs; else on the tensor cores (N = 16
+  // tile, split operands).  Measured: faster for 8-16-16-16-3 and
+  // 16-64-64-64-3, slower for 7-64-64-3.
+  static constexpr bool OUTCC = (N <= 32) || (NL >= 4);
   static constexpr int NOUT = 16;
   static constexpr int NISSUE = NWG;                  // one MMA-issuing warp per group
   static constexpr int THREADS = NWG * 128 + 32 * NISSUE;
@@ -109,7 +117,10 @@ struct TcNet {
   static constexpr int B1_BYTES = N * K1 * 2;
   static constexpr int KB = N + 16;                      // [W | b 0..0]
   static constexpr int BH_BYTES = N * KB * 2;
-  static constexpr int BO_BYTES = NOUT * KB * 2;
+  // output layer: [W | b 0..0] padded to NOUT rows for the tensor cores; on
+  // the CUDA cores fp32, per pair q of inputs 8 floats (w0 w0 | w1 w1 |
+  // w2 w2 | 0 0 at inputs 2q, 2q+1), then the 3 biases
+  static constexpr int BO_BYTES = OUTCC ? (N / 2) * 32 + 16 : NOUT * KB * 2;
   static constexpr int ONES_BYTES = kTile * 16 * 2;      // constant A tile [1 0..0] per row
   static constexpr int OFF_B1 = CTRL;
   static constexpr int OFF_BH = OFF_B1 + B1_BYTES;
@@ -179,6 +190,18 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
   for (int k = 1; k < NL; ++k) {
     const int din = dims[k], dout = dims[k + 1];
     const bool out_layer = (k == NL - 1);
+    if constexpr (Net::OUTCC) {
+      if (out_layer) {  // 3 x din, fp16 -> fp32 (exact), in the pair layout of BO_BYTES
+        float* wo = reinterpret_cast<float*>(smem + Net::OFF_BO);
+        for (int e = threadIdx.x; e < (N / 2) * 8; e += blockDim.x) {
+          const int q = e >> 3, o = (e >> 1) & 3, j = 2 * q + (e & 1);
+          wo[e] = (o < 3 && j < din) ? __half2float(ldh(p + o * din + j)) : 0.0f;
+        }
+        if (threadIdx.x < 4)
+          wo[4 * N + threadIdx.x] = threadIdx.x < 3 ? __half2float(ldh(p + 3 * din + threadIdx.x)) : 0.0f;
+        break;
+      }
+    }
     const int rows = out_layer ? Net::NOUT : N;
     uint8_t* base = smem + (out_layer ? Net::OFF_BO : Net::OFF_BH + (k - 1) * Net::BH_BYTES);
     const __half* Wk = p;
@@ -201,6 +224,45 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
 __device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
   hi = __half2float(__float2half_rz(v));
   lo = v - hi;
+}
+
+// The last hidden layer's epilogue fused with the output layer on the CUDA
+// cores (Net::OUTCC): activation, then rgb = W_out h + b_out in fp32 (packed
+// FMAs on pairs of hidden values; the weights are the fp16 values held
+// exactly in fp32, layout of Net::BO_BYTES).
+template <class Net>
+__device__ __forceinline__ void output_layer_cc(const uint8_t* smem, uint32_t t_acc, float (&rgb)[3]) {
+  constexpr int N = Net::N;
+  const float* wo = reinterpret_cast<const float*>(smem + Net::OFF_BO);
+  unsigned long long s0 = 0ull, s1 = 0ull, s2 = 0ull;  // (+0, +0) pairs
+#pragma unroll
+  for (int h0 = 0; h0 < N; h0 += 16) {
+    uint32_t acc[16];
+    tmem_ld16(t_acc + h0, acc);
+    tmem_ld_wait();
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      float a = __uint_as_float(acc[2 * q]);
+      float bb = __uint_as_float(acc[2 * q + 1]);
+      if constexpr (Net::ACT == ACT_GELU) {
+        a = gelu_poly(a);
+        bb = gelu_poly(bb);
+      } else {
+        a = fmaxf(a, 0.0f);
+        bb = fmaxf(bb, 0.0f);
+      }
+      const unsigned long long hv = pack2(a, bb);
+      const float4 wa = *reinterpret_cast<const float4*>(wo + 8 * (h0 / 2 + q));
+      const float4 wb = *reinterpret_cast<const float4*>(wo + 8 * (h0 / 2 + q) + 4);
+      s0 = fma2(pack2(wa.x, wa.y), hv, s0);
+      s1 = fma2(pack2(wa.z, wa.w), hv, s1);
+      s2 = fma2(pack2(wb.x, wb.y), hv, s2);
+    }
+  }
+  const float2 r0 = unpack2(s0), r1 = unpack2(s1), r2 = unpack2(s2);
+  rgb[0] = r0.x + r0.y + wo[4 * N + 0];
+  rgb[1] = r1.x + r1.y + wo[4 * N + 1];
+  rgb[2] = r2.x + r2.y + wo[4 * N + 2];
 }
 
 template <class Net, bool FL>
@@ -482,6 +544,36 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         const bool has_next = i + NWG < n_tiles;
         if (has_next) prefetch(ny, ntx * kTile);  // in flight during the first epilogue
 
+        if constexpr (Net::OUTCC) {
+          // hidden epilogues up to the last one, which runs the output layer
+          for (int k = 0; k < NL - 2 && ok; ++k) {
+            if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
+              ok = false;
+              break;
+            }
+            acc_phase ^= 1u;
+            tc_fence_after();
+            hidden_epilogue();
+            tc_fence_before();
+            mbar_arrive(my_a);
+            if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
+          }
+          if (!ok) break;
+          if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
+          acc_phase ^= 1u;
+          tc_fence_after();
+          float rgb[3];
+          output_layer_cc<Net>(smem, t_acc, rgb);
+          tc_fence_before();
+          if (NL == 2 && has_next) ok = features(ny, ntx * kTile);  // no hidden layer to overlap
+          if (has_next && ok) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
+          const int x = x0 + r;
+          if (x < p.W) store_rgb(p, b, y, x, rgb[0], rgb[1], rgb[2]);
+          cy = ny;
+          ctx = ntx;
+          if (!ok) break;
+          continue;
+        }
         for (int k = 0; k < NL - 1 && ok; ++k) {
           if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
             ok = false;
@@ -535,7 +627,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w;
       bool ok = true;
       for (int i = w; i < n_tiles && ok; i += NWG) {
-        for (int k = 0; k < NL; ++k) {
+        for (int k = 0; k < (Net::OUTCC ? NL - 1 : NL); ++k) {  // OUTCC: no output-layer MMA
           const uint32_t bar = k == 0 ? my_a1 : my_a;
           const uint32_t par = k == 0 ? (a1_phase & 1u) : (a_phase & 1u);
           if (!__all_sync(0xffffffffu, wait_bounded(bar, par, abort_flag, p.status))) {
