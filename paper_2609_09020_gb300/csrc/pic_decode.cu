@@ -23,11 +23,16 @@ struct pic_decoder {
   int grid_cap;          // resident CTAs over all SMs
   int* d_status;         // bounded-wait failure flag (device word)
   long long n_params;    // per image
-  // staging for pic_decode_batch_host (allocated on first use)
-  int32_t* s_lat;
-  float* s_steps;
-  void* s_w;
-  float* s_out;
+  // staging for pic_decode_batch_host (allocated on first use): one region
+  // per chunk of images, each starting on a 256-byte boundary
+  unsigned char* s_lat;
+  unsigned char* s_steps;
+  unsigned char* s_w;
+  unsigned char* s_out;
+  // its copy-in / decode / copy-out pipeline (created on first use)
+  cudaStream_t p_in, p_run, p_out;
+  cudaEvent_t p_ev[3 * 16 + 1];
+  bool p_ready;
 };
 
 namespace {
@@ -252,6 +257,45 @@ int pic_decode(pic_decoder* h, const int32_t* latents, const float* steps, const
   return pic_decode_batch(h, 1, latents, steps, weights, H, W, out_rgb, stream);
 }
 
+}  // extern "C"
+
+namespace {
+
+constexpr int kHostChunks = 16;  // pipeline depth of pic_decode_batch_host
+constexpr long long kChunkAlign = 256;
+
+long long align_up(long long v, long long a) { return (v + a - 1) / a * a; }
+
+// Per-chunk stride of a staging buffer holding `per_image` bytes per image
+// for up to `imgs` images of a chunk.
+long long chunk_stride(long long per_image, int imgs) { return align_up(per_image * imgs, kChunkAlign); }
+
+void free_host_pipeline(pic_decoder* h) {
+  cudaFree(h->s_lat);
+  cudaFree(h->s_steps);
+  cudaFree(h->s_w);
+  cudaFree(h->s_out);
+  h->s_lat = h->s_steps = h->s_w = h->s_out = nullptr;
+  if (h->p_ready) {
+    cudaStreamDestroy(h->p_in);
+    cudaStreamDestroy(h->p_run);
+    cudaStreamDestroy(h->p_out);
+    for (cudaEvent_t& e : h->p_ev) cudaEventDestroy(e);
+    h->p_ready = false;
+  }
+  cudaGetLastError();
+}
+
+}  // namespace
+
+extern "C" {
+
+/*
+ * Host-buffer decode as a three-stage pipeline over chunks of images: the
+ * inputs of chunk c go to the device on one stream while chunk c - 1 decodes
+ * on a second and chunk c - 2's RGB returns on a third, so the host<->device
+ * copies overlap each other and the kernels instead of adding up.
+ */
 int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const float* steps,
                           const void* weights, int H, int W, void* out_rgb, void* stream) {
   if (!h || !latents || (h->arch.latent_format == PIC_LATENT_INT32 && !steps) || !weights ||
@@ -260,46 +304,82 @@ int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const f
   if (B < 1 || B > h->arch.max_batch || H < 1 || W < 1 || H > h->arch.max_H || W > h->arch.max_W)
     return PIC_ERR_INVALID_ARG;
   const pic_arch& a = h->arch;
-  const long long nb = a.max_batch;
+  const int per_chunk_max = (a.max_batch + kHostChunks - 1) / kHostChunks;
+  const long long out_elem = a.output_format == PIC_OUT_U8_HWC ? 1 : 4;
   if (!h->s_lat) {
     const long long lat = pic_latent_count(a.max_H, a.max_W, a.num_levels, a.channels_per_level);
-    bool ok = cudaMalloc(&h->s_lat, nb * lat * sizeof(int32_t)) == cudaSuccess &&
-              cudaMalloc(&h->s_steps, nb * a.num_levels * sizeof(float)) == cudaSuccess &&
-              cudaMalloc(&h->s_w, nb * h->n_params * weight_elem_bytes(a)) == cudaSuccess &&
-              cudaMalloc(&h->s_out, nb * 3LL * a.max_H * a.max_W * sizeof(float)) == cudaSuccess;
+    bool ok =
+        cudaMalloc(&h->s_lat, kHostChunks * chunk_stride(lat * 4, per_chunk_max)) == cudaSuccess &&
+        cudaMalloc(&h->s_steps, kHostChunks * chunk_stride(a.num_levels * 4LL, per_chunk_max)) ==
+            cudaSuccess &&
+        cudaMalloc(&h->s_w, kHostChunks * chunk_stride(h->n_params * static_cast<long long>(weight_elem_bytes(a)),
+                                                       per_chunk_max)) == cudaSuccess &&
+        cudaMalloc(&h->s_out, kHostChunks * chunk_stride(3LL * a.max_H * a.max_W * 4, per_chunk_max)) ==
+            cudaSuccess;
+    if (ok && !h->p_ready) {
+      ok = cudaStreamCreateWithFlags(&h->p_in, cudaStreamNonBlocking) == cudaSuccess &&
+           cudaStreamCreateWithFlags(&h->p_run, cudaStreamNonBlocking) == cudaSuccess &&
+           cudaStreamCreateWithFlags(&h->p_out, cudaStreamNonBlocking) == cudaSuccess;
+      for (cudaEvent_t& e : h->p_ev)
+        ok = ok && cudaEventCreateWithFlags(&e, cudaEventDisableTiming) == cudaSuccess;
+      h->p_ready = ok;
+    }
     if (!ok) {
-      cudaGetLastError();
-      cudaFree(h->s_lat);
-      cudaFree(h->s_steps);
-      cudaFree(h->s_w);
-      cudaFree(h->s_out);
-      h->s_lat = nullptr;
-      h->s_steps = nullptr;
-      h->s_w = nullptr;
-      h->s_out = nullptr;
+      free_host_pipeline(h);
       return PIC_ERR_ALLOC;
     }
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const long long lat_bytes = static_cast<long long>(B) *
-                              pic_latent_count(H, W, a.num_levels, a.channels_per_level) * 4;
-  const long long w_bytes = static_cast<long long>(B) * h->n_params * weight_elem_bytes(a);
-  const long long out_bytes = static_cast<long long>(B) * 3LL * H * W *
-                              (a.output_format == PIC_OUT_U8_HWC ? 1 : 4);
-  if (cudaMemcpyAsync(h->s_lat, latents, lat_bytes, cudaMemcpyHostToDevice, s) != cudaSuccess ||
-      (steps && cudaMemcpyAsync(h->s_steps, steps, static_cast<size_t>(B) * a.num_levels * 4,
-                                cudaMemcpyHostToDevice, s) != cudaSuccess) ||
-      cudaMemcpyAsync(h->s_w, weights, w_bytes, cudaMemcpyHostToDevice, s) != cudaSuccess) {
+  const long long lat_img = pic_latent_count(H, W, a.num_levels, a.channels_per_level) * 4;
+  const long long st_img = a.num_levels * 4LL;
+  const long long w_img = h->n_params * static_cast<long long>(weight_elem_bytes(a));
+  const long long out_img = 3LL * H * W * out_elem;
+  const long long lat_max = pic_latent_count(a.max_H, a.max_W, a.num_levels, a.channels_per_level) * 4;
+  const long long s_lat_stride = chunk_stride(lat_max, per_chunk_max);
+  const long long s_st_stride = chunk_stride(st_img, per_chunk_max);
+  const long long s_w_stride = chunk_stride(w_img, per_chunk_max);
+  const long long s_out_stride = chunk_stride(3LL * a.max_H * a.max_W * 4, per_chunk_max);
+  const int per_chunk = (B + kHostChunks - 1) / kHostChunks;
+  const bool have_steps = steps != nullptr;
+  cudaEvent_t* ev = h->p_ev;  // [0]: start; then (in, run, out) per chunk
+
+  auto cuda_fail = [&]() {
     cudaGetLastError();
     return PIC_ERR_CUDA;
+  };
+  if (cudaEventRecord(ev[0], s) != cudaSuccess || cudaStreamWaitEvent(h->p_in, ev[0], 0) != cudaSuccess)
+    return cuda_fail();
+  int c = 0;
+  for (int b0 = 0; b0 < B; b0 += per_chunk, ++c) {
+    const int nb = B - b0 < per_chunk ? B - b0 : per_chunk;
+    unsigned char* d_lat = h->s_lat + c * s_lat_stride;
+    unsigned char* d_st = h->s_steps + c * s_st_stride;
+    unsigned char* d_w = h->s_w + c * s_w_stride;
+    unsigned char* d_out = h->s_out + c * s_out_stride;
+    cudaEvent_t e_in = ev[1 + 3 * c], e_run = ev[2 + 3 * c], e_out = ev[3 + 3 * c];
+    if (cudaMemcpyAsync(d_lat, reinterpret_cast<const unsigned char*>(latents) + b0 * lat_img, nb * lat_img,
+                        cudaMemcpyHostToDevice, h->p_in) != cudaSuccess ||
+        (have_steps && cudaMemcpyAsync(d_st, reinterpret_cast<const unsigned char*>(steps) + b0 * st_img,
+                                       nb * st_img, cudaMemcpyHostToDevice, h->p_in) != cudaSuccess) ||
+        cudaMemcpyAsync(d_w, static_cast<const unsigned char*>(weights) + b0 * w_img, nb * w_img,
+                        cudaMemcpyHostToDevice, h->p_in) != cudaSuccess ||
+        cudaEventRecord(e_in, h->p_in) != cudaSuccess ||
+        cudaStreamWaitEvent(h->p_run, e_in, 0) != cudaSuccess)
+      return cuda_fail();
+    const int rc = pic_decode_batch(h, nb, reinterpret_cast<const int32_t*>(d_lat),
+                                    have_steps ? reinterpret_cast<const float*>(d_st) : nullptr, d_w, H,
+                                    W, d_out, h->p_run);
+    if (rc != PIC_OK) return rc;
+    if (cudaEventRecord(e_run, h->p_run) != cudaSuccess ||
+        cudaStreamWaitEvent(h->p_out, e_run, 0) != cudaSuccess ||
+        cudaMemcpyAsync(static_cast<unsigned char*>(out_rgb) + b0 * out_img, d_out, nb * out_img,
+                        cudaMemcpyDeviceToHost, h->p_out) != cudaSuccess ||
+        cudaEventRecord(e_out, h->p_out) != cudaSuccess)
+      return cuda_fail();
   }
-  int rc = pic_decode_batch(h, B, h->s_lat, h->s_steps, h->s_w, H, W, h->s_out, stream);
-  if (rc != PIC_OK) return rc;
-  if (cudaMemcpyAsync(out_rgb, h->s_out, out_bytes, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
-      cudaStreamSynchronize(s) != cudaSuccess) {
-    cudaGetLastError();
-    return PIC_ERR_CUDA;
-  }
+  // every copy-out is on p_out in order: the caller's stream waits for the last
+  if (cudaStreamWaitEvent(s, ev[3 * c], 0) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess)
+    return cuda_fail();
   return PIC_OK;
 }
 
@@ -327,11 +407,7 @@ void pic_decode_destroy(pic_decoder* h) {
   if (!h) return;
   cudaDeviceSynchronize();
   cudaFree(h->d_status);
-  cudaFree(h->s_lat);
-  cudaFree(h->s_steps);
-  cudaFree(h->s_w);
-  cudaFree(h->s_out);
-  cudaGetLastError();
+  free_host_pipeline(h);
   delete h;
 }
 

@@ -338,11 +338,14 @@ class Decoder:
 
     def decode_batch_host(self, latents: np.ndarray, steps: np.ndarray, weights: np.ndarray,
                           H, W, out: np.ndarray, stream=None, B=None):
-        """Host buffers in, host RGB out (copies and decode inside the call)."""
+        """Host buffers in (numpy arrays or CPU tensors, preferably pinned),
+        host RGB out; copies and decodes inside the call, pipelined over
+        chunks of images."""
         if B is None:
             B = latents.shape[0] if latents.ndim == 2 else 1
         for a in (latents, steps, weights, out):
-            if not a.flags["C_CONTIGUOUS"]:
+            ok = a.flags["C_CONTIGUOUS"] if isinstance(a, np.ndarray) else a.is_contiguous()
+            if not ok:
                 raise ValueError("host buffers must be C-contiguous")
         ptr = lambda a: a.ctypes.data if isinstance(a, np.ndarray) else a.data_ptr()
         rc = pic_decode_batch_host(self.handle, B, ptr(latents), ptr(steps), ptr(weights), H, W,
