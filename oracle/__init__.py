@@ -24,6 +24,9 @@ Parity status of each function (what pins it is in tests/test_oracle.py):
                       block counts of the decode workloads, round trip)
   zigzag / ZpR / iZpR pinned (hand-worked stream, JPEG zigzag table start,
                       round trips, malformed streams)
+  Huffman code        pinned (textbook example lengths, Kraft equality,
+                      optimal cost against a heap-built Huffman tree,
+                      length limit, hand-worked bits, round trips)
   modulation fusion   pinned (closed-form statistics, normalised moments,
                       fused == un-fused on random data and on whole decodes,
                       the identity special case, brute-force statistics)
@@ -124,6 +127,14 @@ def _declare(lib):
     lib.pic_oracle_decode_modulated.argtypes = [p, p, p, c_int, c_int, c_int, p, c_int, c_int,
                                                 p, p, p, p, c_int, c_int, p, p, c_int]
     lib.pic_oracle_decode_modulated.restype = c_int
+    lib.pic_oracle_huffman_lengths.argtypes = [p, c_int, c_int, p]
+    lib.pic_oracle_huffman_lengths.restype = c_int
+    lib.pic_oracle_huffman_table.argtypes = [p, p, c_int, p, p]
+    lib.pic_oracle_huffman_table.restype = c_int
+    lib.pic_oracle_huffman_encode.argtypes = [p, c_i64, p, p, c_int, p, c_i64]
+    lib.pic_oracle_huffman_encode.restype = c_i64
+    lib.pic_oracle_huffman_decode.argtypes = [p, c_i64, p, p, c_int, p, c_i64]
+    lib.pic_oracle_huffman_decode.restype = c_int
     return lib
 
 
@@ -353,6 +364,47 @@ class Oracle:
                                                   _ptr(work), int(nthreads))
         if rc != 0:
             raise ValueError("decode_modulated rejected the arguments")
+        return out
+
+    # ---- Huffman coding (Sec. 3.3) -------------------------------------
+    def huffman_lengths(self, freq, max_len: int) -> np.ndarray:
+        f = np.ascontiguousarray(freq, dtype=np.int64)
+        out = np.empty(f.size, dtype=np.int32)
+        if self.lib.pic_oracle_huffman_lengths(_ptr(f), f.size, int(max_len), _ptr(out)) != 0:
+            raise ValueError("huffman_lengths: no code under that length limit")
+        return out
+
+    def huffman_table(self, values, lengths):
+        """(values, lengths) of the coded symbols in canonical order."""
+        v = np.ascontiguousarray(values, dtype=np.int32)
+        ln = np.ascontiguousarray(lengths, dtype=np.int32)
+        tv, tl = np.empty(v.size, np.int32), np.empty(v.size, np.int32)
+        m = self.lib.pic_oracle_huffman_table(_ptr(v), _ptr(ln), v.size, _ptr(tv), _ptr(tl))
+        if m < 0:
+            raise ValueError("huffman_table rejected the arguments")
+        return tv[:m].copy(), tl[:m].copy()
+
+    def huffman_encode(self, syms, tab_value, tab_len):
+        """-> (uint32 words, number of bits)."""
+        s = np.ascontiguousarray(syms, dtype=np.int32)
+        tv = np.ascontiguousarray(tab_value, dtype=np.int32)
+        tl = np.ascontiguousarray(tab_len, dtype=np.int32)
+        cap = (s.size * int(tl.max(initial=1)) + 31) // 32 + 1
+        words = np.empty(cap, dtype=np.uint32)
+        nb = self.lib.pic_oracle_huffman_encode(_ptr(s), s.size, _ptr(tv), _ptr(tl), tv.size,
+                                                _ptr(words), cap)
+        if nb < 0:
+            raise ValueError("huffman_encode: symbol not in the table")
+        return words[:(nb + 31) // 32].copy(), int(nb)
+
+    def huffman_decode(self, words, n_bits, tab_value, tab_len, n_out):
+        w = np.ascontiguousarray(words, dtype=np.uint32)
+        tv = np.ascontiguousarray(tab_value, dtype=np.int32)
+        tl = np.ascontiguousarray(tab_len, dtype=np.int32)
+        out = np.empty(n_out, dtype=np.int32)
+        if self.lib.pic_oracle_huffman_decode(_ptr(w), int(n_bits), _ptr(tv), _ptr(tl), tv.size,
+                                              _ptr(out), int(n_out)) != 0:
+            raise ValueError("huffman_decode: malformed bit stream")
         return out
 
     # ---- ZpR / inverse ZpR (Sec. 3.3, Algorithm 1) ---------------------

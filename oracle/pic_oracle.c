@@ -675,3 +675,196 @@ int pic_oracle_decode_modulated(const int32_t *latents, const double *steps, con
     (void)nthreads;
     return 0;
 }
+
+/* ------------------------------------------------------------------------
+ * Huffman coding of the ZpR symbol stream (Sec. 3.3: image-specific Huffman
+ * tables; O(1) decoding per symbol from a table of 2^p entries, p the code
+ * precision, i.e. the longest code; the table stored run-length compressed,
+ * one entry per coded symbol).
+ *
+ * Readings:
+ *  - the code is a canonical prefix code with lengths <= p, the optimal one
+ *    under that limit (package-merge, Larmore & Hirschberg 1990);
+ *  - canonical order: symbols sorted by (code length, symbol value); codes
+ *    are assigned in that order, each the previous plus one, shifted left
+ *    when the length grows.  The stored table is that list of (value,
+ *    length); in the 2^p-entry lookup table the k-th symbol covers
+ *    2^(p - length) consecutive entries (its run), so the list is the
+ *    table's run-length code;
+ *  - bits are written most significant first into 32-bit words.
+ * The decoder here reads bit by bit against the canonical code (the
+ * textbook method), not through the lookup table.
+ * ------------------------------------------------------------------------ */
+
+#define PIC_HUFF_MAX_SYMS 4096
+#define PIC_HUFF_MAX_LEN 24
+
+/* Optimal code lengths under max_len for n symbols with weights freq (0
+ * weight: not coded, length 0).  Package-merge: at each of max_len levels
+ * the list is the leaves merged with the pairs (packages) of the previous
+ * level's list; a leaf's code length is the number of times it occurs in the
+ * first 2m - 2 items of the last list (m coded symbols).  Returns 0, or -1
+ * if 2^max_len < m or the arguments are out of range. */
+int pic_oracle_huffman_lengths(const int64_t *freq, int n, int max_len, int *len)
+{
+    if (n < 1 || n > PIC_HUFF_MAX_SYMS || max_len < 1 || max_len > PIC_HUFF_MAX_LEN) return -1;
+    int idx[PIC_HUFF_MAX_SYMS], m = 0;
+    for (int i = 0; i < n; ++i) {
+        len[i] = 0;
+        if (freq[i] > 0) idx[m++] = i;
+    }
+    if (m == 0) return 0;
+    if (m == 1) {
+        len[idx[0]] = 1;
+        return 0;
+    }
+    if (max_len < 31 && (1LL << max_len) < m) return -1;
+    /* leaves sorted by weight (insertion sort; ties by symbol index) */
+    for (int a = 1; a < m; ++a) {
+        int v = idx[a], b = a - 1;
+        while (b >= 0 && (freq[idx[b]] > freq[v] || (freq[idx[b]] == freq[v] && idx[b] > v))) {
+            idx[b + 1] = idx[b];
+            --b;
+        }
+        idx[b + 1] = v;
+    }
+    /* items: weight and either a leaf (child_a < 0, leaf = -child_a - 1) or
+     * a package of two items of the previous level */
+    static int64_t wt[PIC_HUFF_MAX_LEN + 1][2 * PIC_HUFF_MAX_SYMS];
+    static int ca[PIC_HUFF_MAX_LEN + 1][2 * PIC_HUFF_MAX_SYMS];
+    static int cnt_lvl[PIC_HUFF_MAX_LEN + 1];
+    /* level 1: the leaves */
+    for (int a = 0; a < m; ++a) {
+        wt[1][a] = freq[idx[a]];
+        ca[1][a] = -idx[a] - 1;
+    }
+    cnt_lvl[1] = m;
+    for (int lv = 2; lv <= max_len; ++lv) {
+        int np = cnt_lvl[lv - 1] / 2, a = 0, p = 0, k = 0;
+        while (a < m || p < np) {
+            int64_t wp = p < np ? wt[lv - 1][2 * p] + wt[lv - 1][2 * p + 1] : 0;
+            if (p >= np || (a < m && freq[idx[a]] <= wp)) {
+                wt[lv][k] = freq[idx[a]];
+                ca[lv][k] = -idx[a] - 1;
+                ++a;
+            } else {
+                wt[lv][k] = wp;
+                ca[lv][k] = 2 * p; /* children 2p, 2p+1 of level lv - 1 */
+                ++p;
+            }
+            ++k;
+        }
+        cnt_lvl[lv] = k;
+    }
+    /* count leaf occurrences in the first 2m - 2 items of the last level */
+    static int take[PIC_HUFF_MAX_LEN + 1];
+    take[max_len] = 2 * m - 2;
+    for (int lv = max_len; lv >= 1; --lv) {
+        int packs = 0;
+        for (int k = 0; k < take[lv]; ++k) {
+            if (ca[lv][k] < 0) len[-ca[lv][k] - 1] += 1;
+            else packs += 1;
+        }
+        if (lv > 1) take[lv - 1] = 2 * packs;
+    }
+    return 0;
+}
+
+/* Canonical order of the coded symbols: order[] receives the indices i with
+ * len[i] > 0 sorted by (len, value[i]); returns their number. */
+static int canonical_order(const int32_t *value, const int *len, int n, int *order)
+{
+    int m = 0;
+    for (int i = 0; i < n; ++i)
+        if (len[i] > 0) order[m++] = i;
+    for (int a = 1; a < m; ++a) {
+        int v = order[a], b = a - 1;
+        while (b >= 0 && (len[order[b]] > len[v] ||
+                          (len[order[b]] == len[v] && value[order[b]] > value[v]))) {
+            order[b + 1] = order[b];
+            --b;
+        }
+        order[b + 1] = v;
+    }
+    return m;
+}
+
+/* The stored (run-length) table: the coded symbols' values and lengths in
+ * canonical order.  Returns the number of entries. */
+int pic_oracle_huffman_table(const int32_t *value, const int *len, int n, int32_t *tab_value,
+                             int *tab_len)
+{
+    int order[PIC_HUFF_MAX_SYMS];
+    if (n < 1 || n > PIC_HUFF_MAX_SYMS) return -1;
+    int m = canonical_order(value, len, n, order);
+    for (int k = 0; k < m; ++k) {
+        tab_value[k] = value[order[k]];
+        tab_len[k] = len[order[k]];
+    }
+    return m;
+}
+
+/* Codes of the table entries in canonical order: code_k = (code_{k-1} + 1)
+ * << (len_k - len_{k-1}), code_0 = 0. */
+static void canonical_codes(const int *tab_len, int m, uint32_t *code)
+{
+    uint32_t c = 0;
+    for (int k = 0; k < m; ++k) {
+        if (k > 0) c = (c + 1) << (tab_len[k] - tab_len[k - 1]);
+        code[k] = c;
+    }
+}
+
+/* Encodes n symbols (values that must be in the table) MSB-first into
+ * 32-bit words; returns the number of bits, or -1 (a value not in the
+ * table, or cap_words too small). */
+int64_t pic_oracle_huffman_encode(const int32_t *syms, int64_t n, const int32_t *tab_value,
+                                  const int *tab_len, int m, uint32_t *words, int64_t cap_words)
+{
+    uint32_t code[PIC_HUFF_MAX_SYMS];
+    if (m < 1 || m > PIC_HUFF_MAX_SYMS) return -1;
+    canonical_codes(tab_len, m, code);
+    for (int64_t w = 0; w < cap_words; ++w) words[w] = 0;
+    int64_t bit = 0;
+    for (int64_t i = 0; i < n; ++i) {
+        int k = 0;
+        while (k < m && tab_value[k] != syms[i]) ++k;
+        if (k == m) return -1;
+        for (int b = tab_len[k] - 1; b >= 0; --b) {
+            if ((bit >> 5) >= cap_words) return -1;
+            if ((code[k] >> b) & 1u) words[bit >> 5] |= 0x80000000u >> (bit & 31);
+            ++bit;
+        }
+    }
+    return bit;
+}
+
+/* Decodes n_out symbols from n_bits bits: reads one bit at a time, and
+ * after every bit checks whether the code read so far is a codeword of the
+ * current length (canonical decoding).  Returns 0, or -1 if the bits run out
+ * or end inside a codeword that is not complete. */
+int pic_oracle_huffman_decode(const uint32_t *words, int64_t n_bits, const int32_t *tab_value,
+                              const int *tab_len, int m, int32_t *out, int64_t n_out)
+{
+    uint32_t code[PIC_HUFF_MAX_SYMS];
+    if (m < 1 || m > PIC_HUFF_MAX_SYMS) return -1;
+    canonical_codes(tab_len, m, code);
+    int64_t bit = 0;
+    for (int64_t i = 0; i < n_out; ++i) {
+        uint32_t c = 0;
+        int l = 0, found = -1;
+        while (found < 0) {
+            if (bit >= n_bits || l >= PIC_HUFF_MAX_LEN) return -1;
+            c = (c << 1) | ((words[bit >> 5] >> (31 - (bit & 31))) & 1u);
+            ++bit;
+            ++l;
+            for (int k = 0; k < m; ++k)
+                if (tab_len[k] == l && code[k] == c) {
+                    found = k;
+                    break;
+                }
+        }
+        out[i] = tab_value[found];
+    }
+    return bit == n_bits ? 0 : -1;
+}

@@ -570,4 +570,98 @@ def pin_mlps_stats_bruteforce(o):
     assert np.abs(sd - f.std(axis=1)).max() < 1e-13
 
 
+# --------------------------------------------------- Huffman coding (Sec. 3.3)
+def _heap_huffman_cost(freq):
+    """Cost (sum of weight x length) of an optimal prefix code, as the sum of
+    the internal-node weights of Huffman's merge tree (heapq)."""
+    import heapq
+    h = [int(f) for f in freq if f > 0]
+    heapq.heapify(h)
+    cost = 0
+    while len(h) > 1:
+        a, b = heapq.heappop(h), heapq.heappop(h)
+        cost += a + b
+        heapq.heappush(h, a + b)
+    return cost
+
+
+def pin_huffman_textbook_example(o):
+    """The classic six-symbol example (frequencies 45, 13, 12, 16, 9, 5 -- a:1
+    b:3 c:3 d:3 e:4 f:4, cost 224)."""
+    ln = o.huffman_lengths([45, 13, 12, 16, 9, 5], 15)
+    assert ln.tolist() == [1, 3, 3, 3, 4, 4]
+    assert int(np.dot(ln, [45, 13, 12, 16, 9, 5])) == 224
+
+
+def pin_huffman_optimal_and_complete(o):
+    """Without an effective length limit the lengths are optimal (cost of a
+    heap-built Huffman tree) and complete (Kraft sum exactly 1); zero weights
+    get no code; a single symbol gets length 1."""
+    rng = np.random.Generator(np.random.PCG64(79))
+    for n in (2, 3, 17, 200):
+        f = rng.integers(1, 10 ** rng.integers(1, 6), n)
+        f[rng.random(n) < 0.1] = 0
+        if (f > 0).sum() < 2:
+            f[:2] = [3, 5]
+        ln = o.huffman_lengths(f, 24)
+        assert int(np.dot(ln, f)) == _heap_huffman_cost(f)
+        assert np.all((ln == 0) == (f == 0))
+        assert sum(2.0 ** -l for l in ln if l > 0) == 1.0
+    assert o.huffman_lengths([0, 7, 0], 5).tolist() == [0, 1, 0]
+
+
+def pin_huffman_length_limited_optimal(o):
+    """Fibonacci weights make an unlimited code 9 levels deep; with a limit of
+    4 the lengths respect it, stay complete, and reach the least cost of all
+    length vectors under the limit that satisfy Kraft's inequality (brute
+    force over the non-increasing assignments, heavier symbols shorter)."""
+    import itertools
+    f = [1, 1, 2, 3, 5, 8, 13, 21, 34, 55]
+    assert o.huffman_lengths(f, 24).max() == 9
+    ln = o.huffman_lengths(f, 4)
+    assert ln.max() <= 4 and sum(2.0 ** -l for l in ln) == 1.0
+    best = None
+    for combo in itertools.combinations_with_replacement(range(1, 5), len(f)):
+        lens = sorted(combo, reverse=True)  # lightest symbol gets the longest code
+        if sum(2.0 ** -l for l in lens) <= 1.0:
+            c = sum(a * b for a, b in zip(f, lens))
+            best = c if best is None or c < best else best
+    assert int(np.dot(ln, f)) == best
+
+
+def pin_huffman_hand_bits(o):
+    """Lengths (1, 2, 2) give canonical codes 0, 10, 11: the stream
+    (A, B, C, A) is the 6 bits 010110, MSB first: word 0x58000000."""
+    tv, tl = o.huffman_table([7, -3, 12], [1, 2, 2])
+    assert tv.tolist() == [7, -3, 12] and tl.tolist() == [1, 2, 2]
+    w, nb = o.huffman_encode([7, -3, 12, 7], tv, tl)
+    assert nb == 6 and w.tolist() == [0x58000000]
+    assert o.huffman_decode(w, nb, tv, tl, 4).tolist() == [7, -3, 12, 7]
+    # canonical order is (length, value): value 12 before 20 at equal length
+    tv, tl = o.huffman_table([20, 5, 12], [2, 1, 2])
+    assert tv.tolist() == [5, 12, 20] and tl.tolist() == [1, 2, 2]
+
+
+def pin_huffman_round_trip(o):
+    """ZpR-like streams (a few frequent values, a long tail) under a 12-bit
+    limit decode back exactly; the bit count is sum(length); decoding past
+    the end is refused."""
+    rng = np.random.Generator(np.random.PCG64(83))
+    syms = np.rint(rng.laplace(0, 3, 5000)).astype(np.int32)
+    syms[rng.random(5000) < 0.1] = 300
+    vals, counts = np.unique(syms, return_counts=True)
+    ln = o.huffman_lengths(counts, 12)
+    assert ln.max() <= 12
+    tv, tl = o.huffman_table(vals, ln)
+    w, nb = o.huffman_encode(syms, tv, tl)
+    assert nb == int(np.dot(counts, ln))
+    assert np.array_equal(o.huffman_decode(w, nb, tv, tl, syms.size), syms)
+    try:
+        o.huffman_decode(w, nb, tv, tl, syms.size + 1)
+    except ValueError:
+        pass
+    else:
+        raise AssertionError("decoding past the end was accepted")
+
+
 PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

@@ -148,6 +148,21 @@ MUTATIONS = {
     "u8_scale_256": (
         "return (int)nearbyint(255.0 * pic_oracle_clamp01(v));",
         "return (int)nearbyint(256.0 * pic_oracle_clamp01(v)) > 255 ? 255 : (int)nearbyint(256.0 * pic_oracle_clamp01(v));"),
+    "canonical_code_shift_order": (
+        "if (k > 0) c = (c + 1) << (tab_len[k] - tab_len[k - 1]);",
+        "if (k > 0) c = (c << (tab_len[k] - tab_len[k - 1])) + 1;"),
+    "huffman_lsb_first": (
+        "if ((code[k] >> b) & 1u) words[bit >> 5] |= 0x80000000u >> (bit & 31);",
+        "if ((code[k] >> b) & 1u) words[bit >> 5] |= 1u << (bit & 31);"),
+    "package_merge_takes_one_more": (
+        "take[max_len] = 2 * m - 2;",
+        "take[max_len] = 2 * m - 1;"),
+    "canonical_ties_descending": (
+        "(len[order[b]] == len[v] && value[order[b]] > value[v]))) {",
+        "(len[order[b]] == len[v] && value[order[b]] < value[v]))) {"),
+    "package_merge_no_packages": (
+        "if (lv > 1) take[lv - 1] = 2 * packs;",
+        "if (lv > 1) take[lv - 1] = packs;"),
     "izpr_raster_not_zigzag": (
         "blk[order[pos++]] = s;",
         "blk[pos++] = s;"),
