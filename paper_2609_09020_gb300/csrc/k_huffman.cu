@@ -1,0 +1,396 @@
+// k_huffman.cu -- Huffman decoding of B image-specific streams on the GPU
+// (include/pic_huffman.h; Sec. 3.3 and Sec. 4.1 of the paper, which adapts
+// GPUHD, Weissenberger & Schmidt 2018: self-synchronising parallel decoding).
+//
+// 1. huff_lut (one CTA per image): the stored table -- values and lengths in
+//    canonical order -- is the run-length code of the 2^p-entry lookup table:
+//    symbol k covers 2^(p - len_k) consecutive entries.  Expanding the runs
+//    gives the table (entry = length << 24 | value), so one lookup of the
+//    next p bits decodes a symbol.  Kraft's inequality is checked here.
+// 2. huff_decode (one cooperative launch; every CTA resident, grid-wide
+//    barriers between the phases):
+//    a. each thread decodes its 256-bit subsequences speculatively from their
+//       first bit, which may lie inside a codeword, until it passes the
+//       subsequence's end; it records the first codeword boundary at or
+//       after the end (the exit) and the number of codewords started;
+//    b. synchronisation passes: a subsequence whose start differs from its
+//       predecessor's exit is decoded again from that exit.  Prefix codes
+//       resynchronise within a few codewords, so the passes stop changing
+//       after one or two; pass i has made subsequence i exact, and after 64
+//       passes without convergence the status word says so;
+//    c. an exclusive scan of the codeword counts gives every subsequence's
+//       output position (each image's must equal its symbol offset);
+//    d. every subsequence is decoded from its final start, writing values.
+// Each thread keeps a 64-bit window of the stream in registers and reloads
+// one word when its position crosses a word boundary (codes are at most 12
+// bits, so at most one word per codeword).
+#include <cstdint>
+
+#include <cooperative_groups.h>
+#include <cuda_runtime.h>
+
+#include "pic_decode.h"
+#include "pic_huffman.h"
+
+namespace cg = cooperative_groups;
+
+namespace {
+
+constexpr int kQ = PIC_HUFF_WORDS_PER_SUBSEQ;  // words per subsequence
+constexpr int kS = 32 * kQ;                     // bits per subsequence
+constexpr int kThreads = 256;
+constexpr int kMaxPasses = 64;
+constexpr int kMaxTable = 4096;
+constexpr int kMaxGrid = 8192;
+enum : int { kBadCode = 1, kBadCount = 2, kNoSync = 4, kBadTable = 8 };
+
+struct Ws {
+  int* status;           // [4]
+  int* changed;          // [kMaxPasses]
+  long long* block_sum;  // [kMaxGrid]
+  uint32_t* lut;         // [B][2^p]
+  long long* exit0;      // [n_sub]
+  long long* exit1;      // [n_sub]
+  long long* start;      // [n_sub]
+  long long* off;        // [n_sub]
+  int* cnt;              // [n_sub]
+};
+
+long long ws_size(long long n_sub, int B, int p) {
+  long long b = 16 + kMaxPasses * 4 + kMaxGrid * 8;
+  b += (static_cast<long long>(B) << p) * 4;
+  b = (b + 15) / 16 * 16;
+  b += n_sub * (8 * 4 + 4);
+  return (b + 15) / 16 * 16;
+}
+
+__host__ __device__ inline Ws ws_view(void* w, long long n_sub, int B, int p) {
+  char* c = static_cast<char*>(w);
+  Ws v;
+  v.status = reinterpret_cast<int*>(c);
+  v.changed = reinterpret_cast<int*>(c + 16);
+  v.block_sum = reinterpret_cast<long long*>(c + 16 + kMaxPasses * 4);
+  v.lut = reinterpret_cast<uint32_t*>(c + 16 + kMaxPasses * 4 + kMaxGrid * 8);
+  long long o = 16 + kMaxPasses * 4 + kMaxGrid * 8 + (static_cast<long long>(B) << p) * 4;
+  o = (o + 15) / 16 * 16;
+  v.exit0 = reinterpret_cast<long long*>(c + o);
+  v.exit1 = v.exit0 + n_sub;
+  v.start = v.exit1 + n_sub;
+  v.off = v.start + n_sub;
+  v.cnt = reinterpret_cast<int*>(v.off + n_sub);
+  return v;
+}
+
+// ---------------------------------------------------------------- 1. tables
+__global__ void __launch_bounds__(kThreads)
+    huff_lut(const int32_t* __restrict__ tab_value, const int32_t* __restrict__ tab_len,
+             int max_table, int p, uint32_t* lut, int* status) {
+  __shared__ int s_start[kMaxTable + 1];
+  __shared__ int s_m, s_fill;
+  const int b = blockIdx.x;
+  const int32_t* tv = tab_value + static_cast<long long>(b) * max_table;
+  const int32_t* tl = tab_len + static_cast<long long>(b) * max_table;
+  uint32_t* out = lut + (static_cast<long long>(b) << p);
+  if (threadIdx.x == 0) {  // run starts: prefix sums of 2^(p - len)
+    int m = 0, bad = 0;
+    long long pos = 0;
+    for (; m < max_table; ++m) {
+      const int l = tl[m];
+      if (l == 0) break;
+      if (l < 1 || l > p) {
+        bad = 1;
+        break;
+      }
+      s_start[m] = static_cast<int>(pos);
+      pos += 1LL << (p - l);
+      if (pos > (1LL << p)) {  // Kraft's inequality violated
+        bad = 1;
+        break;
+      }
+    }
+    s_start[m] = static_cast<int>(pos > (1LL << p) ? (1LL << p) : pos);
+    s_m = bad ? 0 : m;
+    s_fill = bad ? 0 : s_start[m];  // a bad table decodes nothing: every entry "no codeword"
+    if (bad) atomicOr(status, kBadTable);
+  }
+  __syncthreads();
+  const int m = s_m;
+  for (int k = threadIdx.x; k < m; k += blockDim.x) {
+    const uint32_t e = (static_cast<uint32_t>(tl[k]) << 24) | (static_cast<uint32_t>(tv[k]) & 0xFFFFFFu);
+    for (int i = s_start[k]; i < s_start[k + 1]; ++i) out[i] = e;
+  }
+  for (int i = s_fill + threadIdx.x; i < (1 << p); i += blockDim.x) out[i] = 0;  // no codeword
+}
+
+// --------------------------------------------------------------- 2. decode
+struct DecodeParams {
+  const uint32_t* words;
+  long long n_words;
+  const long long* word_off;
+  const long long* n_bits;
+  int B;
+  int p;
+  const long long* sym_off;
+  int32_t* out;
+  Ws ws;
+  long long n_sub;
+};
+
+__device__ __forceinline__ int image_of(const DecodeParams& P, long long word) {
+  int lo = 0, hi = P.B - 1;  // last b with word_off[b] <= word
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (__ldg(P.word_off + mid) <= word) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+__device__ __forceinline__ int32_t value_of(uint32_t e) {
+  return static_cast<int32_t>(e << 8) >> 8;  // sign-extend the 24-bit value
+}
+
+// Decodes codewords of image b starting at bit `pos` while pos < ke; returns
+// the position after the last one.  With out != nullptr writes the values
+// (at most lim of them).  *bad is raised on a bit pattern that is no codeword.
+__device__ long long decode_span(const DecodeParams& P, const uint32_t* __restrict__ lut,
+                                 long long wbase, long long pos, long long ke, int* count,
+                                 int32_t* out, long long lim, bool* bad) {
+  int c = 0;
+  if (pos < ke) {
+    long long wp = wbase + (pos >> 5);
+    uint64_t cur = (static_cast<uint64_t>(__ldg(P.words + wp)) << 32) |
+                   (wp + 1 < P.n_words ? __ldg(P.words + wp + 1) : 0u);
+    const int shr = 64 - P.p;
+    while (pos < ke) {
+      const long long w = wbase + (pos >> 5);
+      if (w != wp) {  // crossed into the next word (codes are shorter than 32 bits)
+        wp = w;
+        cur = (cur << 32) | (wp + 1 < P.n_words ? __ldg(P.words + wp + 1) : 0u);
+      }
+      const uint32_t e = __ldg(lut + static_cast<uint32_t>((cur << (pos & 31)) >> shr));
+      int len = static_cast<int>(e >> 24);
+      if (len == 0) {
+        *bad = true;
+        len = 1;
+      }
+      if (out != nullptr && c < lim) out[c] = value_of(e);
+      ++c;
+      pos += len;
+    }
+  }
+  *count = c;
+  return pos;
+}
+
+__device__ long long block_sum_ll(long long v, long long* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  long long t = 0;
+  for (int i = 0; i < kThreads / 32; ++i) t += red[i];
+  return t;
+}
+
+__global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
+  cg::grid_group grid = cg::this_grid();
+  __shared__ long long red[kThreads / 32];
+  __shared__ long long scan[kThreads];
+  const Ws& ws = P.ws;
+  const long long per_block = (P.n_sub + gridDim.x - 1) / gridDim.x;
+  const long long k_begin = static_cast<long long>(blockIdx.x) * per_block;
+  const long long k_end = min(k_begin + per_block, P.n_sub);
+  bool bad = false;
+
+  // a. speculative decode of every subsequence from its first bit
+  for (long long k = k_begin + threadIdx.x; k < k_end; k += blockDim.x) {
+    const int b = image_of(P, k * kQ);
+    const long long wbase = __ldg(P.word_off + b), nb = __ldg(P.n_bits + b);
+    const long long ks = (k * kQ - wbase) * 32, ke = min(ks + kS, nb);
+    int c = 0;
+    bool junk = false;
+    const long long ex = decode_span(P, ws.lut + (static_cast<long long>(b) << P.p), wbase, ks, ke, &c,
+                                     nullptr, 0, &junk);
+    ws.exit0[k] = ex;
+    ws.start[k] = ks;
+    ws.cnt[k] = c;
+  }
+  grid.sync();
+
+  // b. synchronisation passes (exits double-buffered)
+  int pass = 0;
+  bool stable = false;
+  for (; pass < kMaxPasses; ++pass) {
+    const long long* ex_in = (pass & 1) ? ws.exit1 : ws.exit0;
+    long long* ex_out = (pass & 1) ? ws.exit0 : ws.exit1;
+    long long ch = 0;
+    for (long long k = k_begin + threadIdx.x; k < k_end; k += blockDim.x) {
+      const int b = image_of(P, k * kQ);
+      const long long wbase = __ldg(P.word_off + b), nb = __ldg(P.n_bits + b);
+      const long long ks = (k * kQ - wbase) * 32;
+      const long long st = ks == 0 || ks >= nb ? ws.start[k] : ex_in[k - 1];
+      if (st == ws.start[k]) {
+        ex_out[k] = ex_in[k];
+      } else {
+        int c = 0;
+        bool junk = false;
+        ex_out[k] = decode_span(P, ws.lut + (static_cast<long long>(b) << P.p), wbase, st,
+                                min(ks + kS, nb), &c, nullptr, 0, &junk);
+        ws.start[k] = st;
+        ws.cnt[k] = c;
+        ++ch;
+      }
+    }
+    ch = block_sum_ll(ch, red);
+    if (threadIdx.x == 0 && ch) atomicAdd(ws.changed + pass, 1);
+    grid.sync();
+    if (*reinterpret_cast<volatile int*>(ws.changed + pass) == 0) {
+      stable = true;
+      break;
+    }
+  }
+  if (!stable && blockIdx.x == 0 && threadIdx.x == 0) atomicOr(ws.status, kNoSync);
+
+  // c. output positions: exclusive scan of the counts in subsequence order
+  long long mine = 0;
+  for (long long k = k_begin + threadIdx.x; k < k_end; k += blockDim.x) mine += ws.cnt[k];
+  mine = block_sum_ll(mine, red);
+  if (threadIdx.x == 0) ws.block_sum[blockIdx.x] = mine;
+  grid.sync();
+  long long base = 0;
+  for (int j = threadIdx.x; j < static_cast<int>(blockIdx.x); j += blockDim.x) base += ws.block_sum[j];
+  base = block_sum_ll(base, red);
+  long long carry = base;
+  for (long long k0 = k_begin; k0 < k_end; k0 += blockDim.x) {
+    const long long k = k0 + threadIdx.x;
+    const long long v = k < k_end ? ws.cnt[k] : 0;
+    __syncthreads();
+    scan[threadIdx.x] = v;
+    __syncthreads();
+    for (int o = 1; o < kThreads; o <<= 1) {  // inclusive scan (Hillis-Steele)
+      const long long y = threadIdx.x >= o ? scan[threadIdx.x - o] : 0;
+      __syncthreads();
+      scan[threadIdx.x] += y;
+      __syncthreads();
+    }
+    if (k < k_end) ws.off[k] = carry + scan[threadIdx.x] - v;
+    carry += scan[kThreads - 1];
+  }
+  if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0 && carry != __ldg(P.sym_off + P.B))
+    atomicOr(ws.status, kBadCount);
+  __syncthreads();
+
+  // d. final decode from the synchronised starts
+  for (long long k = k_begin + threadIdx.x; k < k_end; k += blockDim.x) {
+    const int b = image_of(P, k * kQ);
+    const long long wbase = __ldg(P.word_off + b), nb = __ldg(P.n_bits + b);
+    const long long ks = (k * kQ - wbase) * 32;
+    const long long o = ws.off[k];
+    const long long img_end = __ldg(P.sym_off + b + 1);
+    if (ks == 0 && o != __ldg(P.sym_off + b)) atomicOr(ws.status, kBadCount);
+    if (ks >= nb) continue;
+    int c = 0;
+    const long long room = o < img_end ? img_end - o : 0;
+    const long long ex = decode_span(P, ws.lut + (static_cast<long long>(b) << P.p), wbase, ws.start[k],
+                                     min(ks + kS, nb), &c, P.out + o, room, &bad);
+    if (c > room) atomicOr(ws.status, kBadCount);
+    if (ks + kS >= nb && ex != nb) atomicOr(ws.status, kBadCode);  // the last codeword overruns
+  }
+  if (bad) atomicOr(ws.status, kBadCode);
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Resident CTAs of huff_decode on the current device (the cooperative grid).
+int decode_grid(int* grid) {
+  constexpr int kMaxDev = 64;
+  static int cached[kMaxDev];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  if (cached[dev] == 0) {
+    int coop = 0, sms = 0, per_sm = 0;
+    if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, huff_decode, kThreads, 0) != cudaSuccess) {
+      cudaGetLastError();
+      return PIC_ERR_CUDA;
+    }
+    if (!coop || per_sm < 1) return PIC_ERR_UNSUPPORTED;
+    cached[dev] = sms * per_sm < kMaxGrid ? sms * per_sm : kMaxGrid;
+  }
+  *grid = cached[dev];
+  return PIC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int64_t pic_huffman_workspace_bytes(int64_t n_words, int B, int p) {
+  if (n_words < 0 || n_words % kQ != 0 || B < 1 || p < 1 || p > PIC_HUFF_MAX_PRECISION) return -1;
+  return ws_size(n_words / kQ, B, p);
+}
+
+int pic_huffman_decode(const uint32_t* words, int64_t n_words, const int64_t* word_off,
+                       const int64_t* n_bits, int B, const int32_t* tab_value, const int32_t* tab_len,
+                       int max_table, int p, const int64_t* sym_off, int32_t* out, void* workspace,
+                       size_t workspace_bytes, void* stream) {
+  if (n_words < 1 || n_words % kQ != 0 || B < 1 || B > 65536 || p < 1 || p > PIC_HUFF_MAX_PRECISION ||
+      max_table < 1 || max_table > kMaxTable)
+    return PIC_ERR_INVALID_ARG;
+  if (!words || !word_off || !n_bits || !tab_value || !tab_len || !sym_off || !out || !workspace ||
+      !aligned(words, 16) || !aligned(workspace, 16) || !aligned(word_off, 8) || !aligned(n_bits, 8) ||
+      !aligned(sym_off, 8) || !aligned(tab_value, 4) || !aligned(tab_len, 4) || !aligned(out, 4))
+    return PIC_ERR_INVALID_ARG;
+  const long long n_sub = n_words / kQ;
+  if (static_cast<long long>(workspace_bytes) < ws_size(n_sub, B, p)) return PIC_ERR_INVALID_ARG;
+  int grid = 0;
+  int rc = decode_grid(&grid);
+  if (rc != PIC_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  DecodeParams P{};
+  P.words = words;
+  P.n_words = n_words;
+  P.word_off = reinterpret_cast<const long long*>(word_off);
+  P.n_bits = reinterpret_cast<const long long*>(n_bits);
+  P.B = B;
+  P.p = p;
+  P.sym_off = reinterpret_cast<const long long*>(sym_off);
+  P.out = out;
+  P.ws = ws_view(workspace, n_sub, B, p);
+  P.n_sub = n_sub;
+  if (cudaMemsetAsync(workspace, 0, 16 + kMaxPasses * 4, s) != cudaSuccess) {  // status, pass counters
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  huff_lut<<<B, kThreads, 0, s>>>(tab_value, tab_len, max_table, p, P.ws.lut, P.ws.status);
+  const long long g = n_sub < grid ? n_sub : grid;
+  void* args[] = {&P};
+  if (cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(huff_decode), dim3(static_cast<unsigned>(g)),
+                                  dim3(kThreads), args, 0, s) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  if (cudaGetLastError() != cudaSuccess) return PIC_ERR_CUDA;
+  return PIC_OK;
+}
+
+int pic_huffman_status(const void* workspace, void* stream) {
+  if (!workspace) return PIC_ERR_INVALID_ARG;
+  int st = 0;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&st, workspace, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  return st == 0 ? PIC_OK : PIC_ERR_INVALID_ARG;
+}
+
+}  // extern "C"

@@ -108,6 +108,13 @@ def load_library():
     lib.pic_idct_unpatchify.restype = i
     lib.pic_fuse_modulation.argtypes = [ctypes.POINTER(pic_arch), i, _P, _P, _P, _P]
     lib.pic_fuse_modulation.restype = i
+    lib.pic_huffman_workspace_bytes.argtypes = [i64, i, i]
+    lib.pic_huffman_workspace_bytes.restype = i64
+    lib.pic_huffman_decode.argtypes = [_P, i64, _P, _P, i, _P, _P, i, i, _P, _P, _P,
+                                       ctypes.c_size_t, _P]
+    lib.pic_huffman_decode.restype = i
+    lib.pic_huffman_status.argtypes = [_P, _P]
+    lib.pic_huffman_status.restype = i
     lib.pic_status_string.argtypes = [i]
     lib.pic_status_string.restype = ctypes.c_char_p
     _lib = lib
@@ -271,6 +278,50 @@ def fuse_modulation(arch: pic_arch, shared, mod, out=None, stream=None):
                              _stream_ptr(stream))
     if rc != PIC_OK:
         raise PicError(rc, "pic_fuse_modulation")
+    return out
+
+
+def pic_huffman_workspace_bytes(n_words, B, p) -> int:
+    return int(load_library().pic_huffman_workspace_bytes(n_words, B, p))
+
+
+def pic_huffman_decode(words, n_words, word_off, n_bits, B, tab_value, tab_len, max_table, p,
+                       sym_off, out, workspace, workspace_bytes, stream=None) -> int:
+    return load_library().pic_huffman_decode(words, n_words, word_off, n_bits, B, tab_value, tab_len,
+                                             max_table, p, sym_off, out, workspace,
+                                             workspace_bytes, stream)
+
+
+def pic_huffman_status(workspace, stream=None) -> int:
+    return load_library().pic_huffman_status(workspace, stream)
+
+
+def huffman_decode(words, word_off, n_bits, tab_value, tab_len, p, sym_off, stream=None,
+                   check=True):
+    """Decodes B Huffman streams given as torch CUDA tensors (uint32 words as
+    int32, int64 word_off [B+1], n_bits [B], int32 tables [B][max_table],
+    int64 sym_off [B+1]); returns the int32 symbols [sym_off[B]].  With
+    check, synchronises and raises if a stream is malformed."""
+    import torch
+    B = n_bits.numel()
+    n_words = words.numel()
+    total = int(sym_off[-1].item())
+    out = torch.empty(max(total, 1), dtype=torch.int32, device=words.device)[:total]
+    wb = pic_huffman_workspace_bytes(n_words, B, p)
+    if wb < 0:
+        raise ValueError("huffman_decode: arguments out of range")
+    ws = torch.empty(wb, dtype=torch.uint8, device=words.device)
+    sp = _stream_ptr(stream)
+    rc = pic_huffman_decode(words.data_ptr(), n_words, word_off.data_ptr(), n_bits.data_ptr(), B,
+                            tab_value.data_ptr(), tab_len.data_ptr(), tab_value.shape[-1], p,
+                            sym_off.data_ptr(), out.data_ptr() if total else ws.data_ptr(),
+                            ws.data_ptr(), wb, sp)
+    if rc != PIC_OK:
+        raise PicError(rc, "pic_huffman_decode")
+    if check:
+        rc = pic_huffman_status(ws.data_ptr(), sp)
+        if rc != PIC_OK:
+            raise PicError(rc, "pic_huffman_status")
     return out
 
 

@@ -344,6 +344,88 @@ def make_modulation(B: int, cf: int, seed: int) -> np.ndarray:
     return m.astype(np.float32)
 
 
+HUFF_WORDS_PER_SUBSEQ = 8   # streams of a batch start on multiples of this many words
+
+
+def huffman_code_lengths(counts: np.ndarray, p: int) -> np.ndarray:
+    """Code lengths <= p for symbols with the given counts, for generating
+    coded test inputs: Huffman's merge (heapq) for the depths, then lengths
+    clamped to p and, while Kraft's sum exceeds 1, the longest code below p
+    lengthened by one.  (A valid prefix code; the optimal one under the limit
+    is the encoder's business.)"""
+    import heapq
+    n = len(counts)
+    if n == 1:
+        return np.array([1], dtype=np.int64)
+    heap = [(int(c), i, [i]) for i, c in enumerate(counts)]
+    heapq.heapify(heap)
+    depth = np.zeros(n, dtype=np.int64)
+    tick = n
+    while len(heap) > 1:
+        a, _, la = heapq.heappop(heap)
+        b, _, lb = heapq.heappop(heap)
+        depth[la + lb] += 1
+        heapq.heappush(heap, (a + b, tick, la + lb))
+        tick += 1
+    ln = np.minimum(depth, p)
+    order = np.argsort(-ln, kind="stable")
+    while np.sum(2.0 ** -ln) > 1.0:
+        j = next(i for i in order if ln[i] < p)
+        ln[j] += 1
+        order = np.argsort(-ln, kind="stable")
+    return ln
+
+
+def huffman_pack(symbols: np.ndarray, p: int):
+    """One stream's image-specific canonical code and bits: returns
+    (tab_value, tab_len) in canonical order (length, then value), the words
+    (MSB first, padded to HUFF_WORDS_PER_SUBSEQ) and the number of bits."""
+    vals, inv, counts = np.unique(symbols, return_inverse=True, return_counts=True)
+    ln = huffman_code_lengths(counts, p)
+    order = np.lexsort((vals, ln))                 # canonical: by length, then value
+    code = np.zeros(len(vals), dtype=np.uint64)
+    c = 0
+    for k, i in enumerate(order):
+        if k > 0:
+            c = (c + 1) << int(ln[i] - ln[order[k - 1]])
+        code[i] = c
+    L = ln[inv].astype(np.uint64)
+    pos = np.cumsum(L) - L
+    n_bits = int(L.sum())
+    n_words = -(-max(n_bits, 1) // 32)
+    n_words = -(-n_words // HUFF_WORDS_PER_SUBSEQ) * HUFF_WORDS_PER_SUBSEQ
+    words = np.zeros(n_words + 1, dtype=np.uint64)
+    sh = np.uint64(64) - L - (pos & np.uint64(31))
+    v = code[inv] << sh
+    w = (pos >> np.uint64(5)).astype(np.int64)
+    np.bitwise_or.at(words, w, v >> np.uint64(32))
+    np.bitwise_or.at(words, w + 1, v & np.uint64(0xFFFFFFFF))
+    return (vals[order].astype(np.int32), ln[order].astype(np.int32),
+            words[:n_words].astype(np.uint32), n_bits)
+
+
+def huffman_streams(wl: Workload | str, batch: int | None = None, p: int = 12):
+    """The ZpR streams of zpr_streams, each Huffman-coded with its own
+    table (Sec. 3.3): returns a dict with the concatenated words, word_off
+    [B+1], n_bits [B], tab_value / tab_len [B][max_table] (zero-padded),
+    sym_off [B+1], the symbols themselves and eob."""
+    syms, counts, n_blk, eob = zpr_streams(wl, batch)
+    starts = np.r_[0, np.cumsum(counts)]
+    packs = [huffman_pack(syms[starts[b]:starts[b + 1]], p) for b in range(len(counts))]
+    max_table = max(len(t[0]) for t in packs)
+    B = len(packs)
+    tv = np.zeros((B, max_table), np.int32)
+    tl = np.zeros((B, max_table), np.int32)
+    for b, (v, ln, _, _) in enumerate(packs):
+        tv[b, :len(v)] = v
+        tl[b, :len(ln)] = ln
+    word_off = np.r_[0, np.cumsum([len(t[2]) for t in packs])].astype(np.int64)
+    return {"words": np.concatenate([t[2] for t in packs]), "word_off": word_off,
+            "n_bits": np.array([t[3] for t in packs], np.int64), "tab_value": tv,
+            "tab_len": tl, "sym_off": starts.astype(np.int64), "symbols": syms,
+            "n_blocks": n_blk, "eob": eob, "p": p}
+
+
 def sample_pixels(H: int, W: int, n: int, seed: int) -> np.ndarray:
     """Flat pixel indices (y * W + x) to check at full size: the four corners,
     the middle of every border, and n seeded random positions."""

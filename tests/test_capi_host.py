@@ -136,3 +136,13 @@ def test_output_format_is_validated(lib):
     a = pic.make_arch(2, 1, [2, 8, 3], max_H=8, max_W=8, output=3)
     h = pic._P()
     assert lib.pic_decode_create(pic.ctypes.byref(a), pic.ctypes.byref(h)) == pic.PIC_ERR_UNSUPPORTED
+
+
+def test_huffman_workspace_and_argument_checks(lib):
+    from paper_2609_09020_gb300 import pic
+    assert pic.pic_huffman_workspace_bytes(8, 1, 12) > 0
+    assert pic.pic_huffman_workspace_bytes(7, 1, 12) == -1   # not whole subsequences
+    assert pic.pic_huffman_workspace_bytes(8, 1, 13) == -1   # precision above 12
+    assert pic.pic_huffman_decode(None, 8, None, None, 1, None, None, 4, 12, None, None, None, 0,
+                                  None) == pic.PIC_ERR_INVALID_ARG
+    assert pic.pic_huffman_status(None, None) == pic.PIC_ERR_INVALID_ARG

@@ -78,3 +78,21 @@ def test_zpr_streams_are_the_oracle_encoding(orc):
 def test_zigzag_diagonals(orc):
     order = orc.zigzag()
     assert np.array_equal(wk.zigzag_diagonals(), order // 8 + order % 8)
+
+
+def test_huffman_pack_is_the_oracle_encoding(orc):
+    """The stream generator's table is a valid canonical code under the
+    precision (Kraft <= 1, canonical order) and its bits are exactly the
+    oracle's encoding with that table; the oracle decodes them back."""
+    rng = np.random.Generator(np.random.PCG64(89))
+    for p, syms in ((12, np.rint(rng.laplace(0, 4, 3000)).astype(np.int32)),
+                    (5, rng.integers(-3, 4, 500).astype(np.int32)),
+                    (4, np.full(37, 9, np.int32))):
+        tv, tl, words, nb = wk.huffman_pack(syms, p)
+        assert tl.max() <= p and np.sum(2.0 ** -tl.astype(float)) <= 1.0
+        ctv, ctl = orc.huffman_table(tv, tl)
+        assert np.array_equal(ctv, tv) and np.array_equal(ctl, tl)
+        w, nb2 = orc.huffman_encode(syms, tv, tl)
+        assert nb2 == nb and np.array_equal(words[:len(w)], w) and not words[len(w):].any()
+        assert len(words) % wk.HUFF_WORDS_PER_SUBSEQ == 0
+        assert np.array_equal(orc.huffman_decode(words, nb, tv, tl, syms.size), syms)
