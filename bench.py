@@ -228,7 +228,160 @@ STAGE_METRIC = {
     "pipeline": ("decoded megapixels/s from ZpR symbols (iZpR + iDCT + synthesis) at 1 GB300",
                  "MP/s"),
     "fuse": ("modulation fusion (App. A): per-image decoder weight blobs/s at 1 GB300", "images/s"),
+    "huffman": ("Huffman decoding (image-specific tables, self-synchronising): symbols/s at 1 GB300; "
+                "% of HBM roofline", "Msymbols/s"),
+    "bitstream": ("decoded megapixels/s from Huffman-coded bitstreams (Huffman + iZpR + iDCT + "
+                  "synthesis) at 1 GB300", "MP/s"),
 }
+
+
+def run_bitstream_stages(args):
+    """Huffman decoding of the 64-image batch's ZpR streams (one table per
+    image), alone ("huffman") or followed by iZpR, iDCT and the synthesis
+    ("bitstream": the whole decoder after the header)."""
+    import torch
+    from paper_2609_09020_gb300 import build, pic
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    build.build()
+    stage = args.stage
+    wl = wk.WORKLOADS["c5"]
+    B = wl.B
+    h = wk.huffman_streams(wl)
+    dx = wk.make_dct_inputs(wl)
+    n_blk, eob, p = h["n_blocks"], h["eob"], h["p"]
+    n_sym = int(h["sym_off"][-1])
+    stream = torch.cuda.current_stream(dev)
+    sp = stream.cuda_stream
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    words, word_off, n_bits = t(h["words"].view(np.int32)), t(h["word_off"]), t(h["n_bits"])
+    tv, tl, sym_off = t(h["tab_value"]), t(h["tab_len"]), t(h["sym_off"])
+    syms = torch.empty(n_sym, dtype=torch.int32, device=dev)
+    hwb = pic.pic_huffman_workspace_bytes(words.numel(), B, p)
+    hws = torch.empty(hwb, dtype=torch.uint8, device=dev)
+    full = stage == "bitstream"
+    if full:
+        coeffs = torch.empty((B * n_blk, 64), dtype=torch.int32, device=dev)
+        offsets = torch.empty(B * n_blk, dtype=torch.int64, device=dev)
+        zwb = pic.pic_izpr_workspace_bytes(n_sym)
+        zws = torch.empty(zwb, dtype=torch.uint8, device=dev)
+        steps_t = t(dx.steps)
+        lat = torch.empty((B, wl.n_latents), dtype=torch.float32, device=dev)
+        wts = t(dx.weights_for("fp16_tc"))
+        out = torch.empty((B, 3, wl.H, wl.W), dtype=torch.float32, device=dev)
+        dec = pic.Decoder.for_workload(wl, "fp16_tc", max_batch=B, latent="fp32")
+
+    def huff():
+        rc = pic.pic_huffman_decode(words.data_ptr(), words.numel(), word_off.data_ptr(),
+                                    n_bits.data_ptr(), B, tv.data_ptr(), tl.data_ptr(), tv.shape[1],
+                                    p, sym_off.data_ptr(), syms.data_ptr(), hws.data_ptr(), hwb, sp)
+        if rc != pic.PIC_OK:
+            raise pic.PicError(rc, "pic_huffman_decode")
+
+    def rest():
+        rc = pic.pic_izpr_decode(syms.data_ptr(), n_sym, eob, B * n_blk, coeffs.data_ptr(),
+                                 offsets.data_ptr(), zws.data_ptr(), zwb, sp)
+        if rc != pic.PIC_OK:
+            raise pic.PicError(rc, "pic_izpr_decode")
+        rc = pic.pic_idct_unpatchify(coeffs.data_ptr(), steps_t.data_ptr(), B, wl.H, wl.W, wl.L,
+                                     wl.C, lat.data_ptr(), sp)
+        if rc != pic.PIC_OK:
+            raise pic.PicError(rc, "pic_idct_unpatchify")
+        dec.decode_batch(lat, None, wts, wl.H, wl.W, out, stream=stream, B=B)
+
+    def one_step():
+        huff()
+        if full:
+            rest()
+
+    for _ in range(max(args.warmup, 3)):
+        one_step()
+    torch.cuda.synchronize()
+    if pic.pic_huffman_status(hws.data_ptr(), sp) != pic.PIC_OK:
+        raise RuntimeError("Huffman streams reported malformed")
+    if not torch.equal(syms.cpu(), torch.from_numpy(h["symbols"])):
+        raise RuntimeError("Huffman decode differs from the generated symbols")
+    if full:
+        if pic.pic_izpr_status(zws.data_ptr(), sp) != pic.PIC_OK:
+            raise RuntimeError("ZpR streams reported malformed")
+        dec.check(stream)
+    with ClockSampler(0) as clk:
+        ms = _event_time(one_step, args.steps, stream, torch)
+    stage_ms = {"huffman": _event_time(huff, args.steps, stream, torch)}
+    if full:
+        dec.check(stream)
+        stage_ms["izpr+idct+synthesis"] = ms - stage_ms["huffman"]
+    peaks = load_peaks()
+    hbytes = 4 * words.numel() + 8 * tv.numel() + 4 * n_sym + 24 * B
+    t_h = stage_ms["huffman"] * 1e-3
+    roof = {"bound": "hbm", "achieved": hbytes / t_h / 1e9, "peak": peaks["hbm_gbs"],
+            "unit": "GB/s", "peak_source": f"copy bandwidth, {peaks['source']}",
+            "kernel": "huff_lut + huff_decode (one call)", "avg_launch_us": t_h * 1e6,
+            "traffic": None, "algorithmic_bytes_per_launch": hbytes}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    if full:
+        value, unit = B * wl.H * wl.W / (ms * 1e-3) / 1e6, "MP/s"
+        roof["note"] = "roofline of the Huffman stage; the synthesis dominates the step"
+    else:
+        value, unit = n_sym / (ms * 1e-3) / 1e6, "Msymbols/s"
+    e2e = None
+    if not args.no_e2e:
+        src_h = torch.from_numpy(h["words"].view(np.int32)).pin_memory()
+        res_d = out if full else syms
+        res_h = torch.empty(res_d.shape, dtype=res_d.dtype).pin_memory()
+
+        def e2e_step():
+            words.copy_(src_h, non_blocking=True)
+            one_step()
+            res_h.copy_(res_d, non_blocking=True)
+            torch.cuda.current_stream().synchronize()
+
+        e2e_step()
+        k = max(3, min(args.steps, 10))
+        t0 = time.perf_counter()
+        for _ in range(k):
+            e2e_step()
+        el = (time.perf_counter() - t0) / k
+        units = B * wl.H * wl.W / 1e6 if full else n_sym / 1e6
+        e2e = {"value": units / el, "unit": unit,
+               "h2d_bytes_per_step": int(src_h.numel() * 4),
+               "d2h_bytes_per_step": int(res_h.numel() * res_h.element_size()),
+               "ms_per_step": 1e3 * el}
+    cpu = None
+    if not args.no_cpu_baseline:
+        import oracle
+        orc = oracle.load()
+        n, t0 = 0, time.perf_counter()
+        while time.perf_counter() - t0 < min(args.cpu_budget_s, 10.0):
+            b = n % B
+            m = int(np.count_nonzero(h["tab_len"][b]))
+            orc.huffman_decode(h["words"][h["word_off"][b]:h["word_off"][b + 1]], h["n_bits"][b],
+                               h["tab_value"][b, :m], h["tab_len"][b, :m],
+                               int(h["sym_off"][b + 1] - h["sym_off"][b]))
+            n += 1
+        el = time.perf_counter() - t0
+        per_img = n_sym / B
+        cpu = {"value": n * per_img / el / 1e6, "unit": "Msymbols/s", "cores": 1, "kind": "oracle",
+               "sample": f"{n} image stream(s) Huffman-decoded in {el:.1f} s (fp64-free C oracle, "
+                         "bit by bit, one thread)"}
+    line = {"metric": STAGE_METRIC[stage][0], "value": value, "unit": unit, "n_gpus": 1,
+            "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "int32 symbols" if not full else
+            "int32 symbols; f32 iDCT; f16 operands (hi+lo), f32 accumulate",
+            "data": "synthetic (seeded ZpR streams Huffman-coded with per-image tables)",
+            "config": {"workload": f"{stage}: {B} x {wl.W}x{wl.H}, {n_sym} symbols, "
+                                   f"{int(h['n_bits'].sum())} bits, p = {p}",
+                       "images": B, "symbols": n_sym, "bits": int(h["n_bits"].sum()),
+                       "bits_per_symbol": float(h["n_bits"].sum()) / n_sym,
+                       "max_table": int(h["tab_value"].shape[1]),
+                       "l2": "outputs larger than L2", "parallelism": "dp1"},
+            "roofline": roof, "clocks": clk.summary(), "e2e": e2e,
+            "gpu_launches": args.steps * (2 + (5 if full else 0)), "cpu_baseline": cpu,
+            "stage": stage, "stage_ms": stage_ms}
+    if full:
+        line["images_per_s"] = B / (ms * 1e-3)
+    print(json.dumps(line), flush=True)
 
 
 def run_fuse_stage(args):
@@ -455,7 +608,7 @@ def run_stage(args):
     if stage == "izpr":
         nbytes = 4 * n_sym + (256 + 8) * blocks
         value = blocks / (ms * 1e-3) / 1e6
-        launches = 4
+        launches = 3
     elif stage == "idct":
         nbytes = 256 * blocks + 4 * B * n_lat + 4 * B * wl.L
         value = blocks / (ms * 1e-3) / 1e6
@@ -463,7 +616,7 @@ def run_stage(args):
     else:
         nbytes = (4 * n_sym + 2 * B * wl.n_params + 4 * B * wl.L + 12 * B * wl.H * wl.W)
         value = B * wl.H * wl.W / (ms * 1e-3) / 1e6
-        launches = n_chunks * 6
+        launches = n_chunks * 5
     metric, unit = STAGE_METRIC[stage]
     if stage == "pipeline":
         flops = 2.0 * wl.macs_per_pixel * B * wl.H * wl.W
@@ -477,7 +630,7 @@ def run_stage(args):
     else:
         roof = {"bound": "hbm", "achieved": nbytes / (ms * 1e-3) / 1e9, "peak": peaks["hbm_gbs"],
                 "unit": "GB/s", "peak_source": f"copy bandwidth, {peaks['source']}",
-                "kernel": "izpr_count+izpr_scan+izpr_compact+izpr_expand (one call)"
+                "kernel": "izpr_count+izpr_scan+izpr_expand (one call)"
                 if stage == "izpr" else "idct_unpatchify_kernel",
                 "avg_launch_us": ms * 1e3}
     roof["frac"] = roof["achieved"] / roof["peak"]
@@ -559,7 +712,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--stage", default="decode",
-                    choices=["decode", "izpr", "idct", "pipeline", "fuse"],
+                    choices=["decode", "izpr", "idct", "pipeline", "fuse", "huffman",
+                             "bitstream"],
                     help="decode (default): the synthesis; the others time the stages before "
                          "it, alone or chained, on one GPU")
     ap.add_argument("--chunk", type=int, default=16,
@@ -570,7 +724,12 @@ def main():
             print(json.dumps({"stage": args.stage, "unavailable":
                               "stage benchmarks run our arm on one GPU only"}))
             return
-        run_fuse_stage(args) if args.stage == "fuse" else run_stage(args)
+        if args.stage == "fuse":
+            run_fuse_stage(args)
+        elif args.stage in ("huffman", "bitstream"):
+            run_bitstream_stages(args)
+        else:
+            run_stage(args)
         return
 
     wl = wk.WORKLOADS[args.workload]

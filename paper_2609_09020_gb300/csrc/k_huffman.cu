@@ -42,6 +42,10 @@ constexpr int kThreads = 256;
 constexpr int kMaxPasses = 64;
 constexpr int kMaxTable = 4096;
 constexpr int kMaxGrid = 8192;
+constexpr int kWbuf = kThreads * kQ + 2;  // stream words of one pass of 256 subsequences
+constexpr int kRound = 16;                // symbols a thread decodes between two warp stores
+constexpr int kRow = kRound + 1;          // staging row (padded against bank conflicts)
+constexpr int kStageInts = kThreads * kRow;
 enum : int { kBadCode = 1, kBadCount = 2, kNoSync = 4, kBadTable = 8 };
 
 struct Ws {
@@ -134,6 +138,7 @@ struct DecodeParams {
   int32_t* out;
   Ws ws;
   long long n_sub;
+  long long per_block;  // subsequences per CTA, a multiple of kThreads
 };
 
 __device__ __forceinline__ int image_of(const DecodeParams& P, long long word) {
@@ -150,37 +155,57 @@ __device__ __forceinline__ int32_t value_of(uint32_t e) {
   return static_cast<int32_t>(e << 8) >> 8;  // sign-extend the 24-bit value
 }
 
-// Decodes codewords of image b starting at bit `pos` while pos < ke; returns
-// the position after the last one.  With out != nullptr writes the values
-// (at most lim of them).  *bad is raised on a bit pattern that is no codeword.
-__device__ long long decode_span(const DecodeParams& P, const uint32_t* __restrict__ lut,
-                                 long long wbase, long long pos, long long ke, int* count,
-                                 int32_t* out, long long lim, bool* bad) {
+// Decodes codewords from bit `lpos` of the words staged in shared memory
+// (bit 0 = the top bit of sw[0]) while lpos < lke; returns the position
+// after the last codeword.  WRITE: stores the values into out (at most lim).
+// *bad is raised on a bit pattern that is no codeword.  The next p bits come
+// from one funnel shift of the two current words.
+template <bool WRITE>
+__device__ __forceinline__ int decode_span_s(const uint32_t* sw, int lpos, int lke, const uint32_t* lut,
+                                             int p, int* count, int32_t* out, long long lim, bool* bad) {
   int c = 0;
-  if (pos < ke) {
-    long long wp = wbase + (pos >> 5);
-    uint64_t cur = (static_cast<uint64_t>(__ldg(P.words + wp)) << 32) |
-                   (wp + 1 < P.n_words ? __ldg(P.words + wp + 1) : 0u);
-    const int shr = 64 - P.p;
-    while (pos < ke) {
-      const long long w = wbase + (pos >> 5);
-      if (w != wp) {  // crossed into the next word (codes are shorter than 32 bits)
-        wp = w;
-        cur = (cur << 32) | (wp + 1 < P.n_words ? __ldg(P.words + wp + 1) : 0u);
+  if (lpos < lke) {
+    int li = lpos >> 5;
+    uint32_t hi = sw[li], lo = sw[li + 1];
+    const int shr = 32 - p;
+    while (lpos < lke) {
+      const int wi = lpos >> 5;
+      if (wi != li) {  // crossed into the next word (codes are shorter than 32 bits)
+        li = wi;
+        hi = lo;
+        lo = sw[li + 1];
       }
-      const uint32_t e = __ldg(lut + static_cast<uint32_t>((cur << (pos & 31)) >> shr));
+      const uint32_t e = lut[__funnelshift_l(lo, hi, lpos & 31) >> shr];
       int len = static_cast<int>(e >> 24);
       if (len == 0) {
         *bad = true;
         len = 1;
       }
-      if (out != nullptr && c < lim) out[c] = value_of(e);
+      if constexpr (WRITE) {
+        if (c < lim) out[c] = value_of(e);
+      }
       ++c;
-      pos += len;
+      lpos += len;
     }
   }
   *count = c;
-  return pos;
+  return lpos;
+}
+
+// decode_span_s for subsequence positions of image b: pos (bits from the
+// image's first word wbase) <-> staged position (bits from word w0).
+template <bool WRITE>
+__device__ __forceinline__ long long decode_at(const uint32_t* sw, long long w0, long long wbase, long long pos,
+                                               long long ke, const uint32_t* lut, int p, int* count,
+                                               int32_t* out, long long lim, bool* bad) {
+  if (pos >= ke) {
+    *count = 0;
+    return pos;
+  }
+  const long long shift = (wbase - w0) * 32;  // staged bit = image bit + shift (>= 0 here)
+  const int lp = decode_span_s<WRITE>(sw, static_cast<int>(pos + shift), static_cast<int>(ke + shift), lut,
+                                      p, count, out, lim, bad);
+  return lp - shift;
 }
 
 __device__ long long block_sum_ll(long long v, long long* red) {
@@ -199,21 +224,50 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
   cg::grid_group grid = cg::this_grid();
   __shared__ long long red[kThreads / 32];
   __shared__ long long scan[kThreads];
+  extern __shared__ uint32_t s_lut[];  // the lookup tables of the first and last image of the range
   const Ws& ws = P.ws;
-  const long long per_block = (P.n_sub + gridDim.x - 1) / gridDim.x;
+  const long long per_block = P.per_block;
   const long long k_begin = static_cast<long long>(blockIdx.x) * per_block;
   const long long k_end = min(k_begin + per_block, P.n_sub);
   bool bad = false;
+  // every lookup is a dependent load in a decode chain: the CTA's images'
+  // tables go to shared memory (images between the first and the last of
+  // the range, which only tiny streams produce, read theirs from global)
+  const int tsize = 1 << P.p;
+  const int b_first = k_begin < k_end ? image_of(P, k_begin * kQ) : 0;
+  const int b_last = k_begin < k_end ? image_of(P, (k_end - 1) * kQ) : 0;
+  for (int i = threadIdx.x; i < tsize; i += blockDim.x) {
+    s_lut[i] = ws.lut[(static_cast<long long>(b_first) << P.p) + i];
+    s_lut[tsize + i] = ws.lut[(static_cast<long long>(b_last) << P.p) + i];
+  }
+  __syncthreads();
+  auto lut_of = [&](int b) -> const uint32_t* {
+    return b == b_first ? s_lut : (b == b_last ? s_lut + tsize : ws.lut + (static_cast<long long>(b) << P.p));
+  };
+  // each pass of 256 subsequences first stages its stream words (coalesced),
+  // so that no global load sits inside a decode chain
+  uint32_t* s_words = s_lut + 2 * tsize;
+  int* s_stage = reinterpret_cast<int*>(s_words + kWbuf);
+  auto stage_words = [&](long long k0) {
+    const long long w0 = k0 * kQ;
+    __syncthreads();
+    for (int i = threadIdx.x; i < kWbuf; i += blockDim.x)
+      s_words[i] = w0 + i < P.n_words ? __ldg(P.words + w0 + i) : 0u;
+    __syncthreads();
+  };
 
   // a. speculative decode of every subsequence from its first bit
-  for (long long k = k_begin + threadIdx.x; k < k_end; k += blockDim.x) {
+  for (long long k0 = k_begin; k0 < k_end; k0 += kThreads) {
+    stage_words(k0);
+    const long long k = k0 + threadIdx.x;
+    if (k >= k_end) continue;
     const int b = image_of(P, k * kQ);
     const long long wbase = __ldg(P.word_off + b), nb = __ldg(P.n_bits + b);
     const long long ks = (k * kQ - wbase) * 32, ke = min(ks + kS, nb);
     int c = 0;
     bool junk = false;
-    const long long ex = decode_span(P, ws.lut + (static_cast<long long>(b) << P.p), wbase, ks, ke, &c,
-                                     nullptr, 0, &junk);
+    const long long ex = decode_at<false>(s_words, k0 * kQ, wbase, ks, ke, lut_of(b), P.p, &c, nullptr, 0,
+                                          &junk);
     ws.exit0[k] = ex;
     ws.start[k] = ks;
     ws.cnt[k] = c;
@@ -227,18 +281,27 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
     const long long* ex_in = (pass & 1) ? ws.exit1 : ws.exit0;
     long long* ex_out = (pass & 1) ? ws.exit0 : ws.exit1;
     long long ch = 0;
-    for (long long k = k_begin + threadIdx.x; k < k_end; k += blockDim.x) {
-      const int b = image_of(P, k * kQ);
-      const long long wbase = __ldg(P.word_off + b), nb = __ldg(P.n_bits + b);
-      const long long ks = (k * kQ - wbase) * 32;
-      const long long st = ks == 0 || ks >= nb ? ws.start[k] : ex_in[k - 1];
-      if (st == ws.start[k]) {
-        ex_out[k] = ex_in[k];
-      } else {
+    for (long long k0 = k_begin; k0 < k_end; k0 += kThreads) {
+      const long long k = k0 + threadIdx.x;
+      int b = 0;
+      long long wbase = 0, nb = 0, ks = 0, st = 0;
+      bool redo = false;
+      if (k < k_end) {
+        b = image_of(P, k * kQ);
+        wbase = __ldg(P.word_off + b);
+        nb = __ldg(P.n_bits + b);
+        ks = (k * kQ - wbase) * 32;
+        st = ks == 0 || ks >= nb ? ws.start[k] : ex_in[k - 1];
+        redo = st != ws.start[k];
+        if (!redo) ex_out[k] = ex_in[k];
+      }
+      if (!__syncthreads_or(redo)) continue;  // nothing to redo in this pass of the CTA
+      stage_words(k0);
+      if (redo) {
         int c = 0;
         bool junk = false;
-        ex_out[k] = decode_span(P, ws.lut + (static_cast<long long>(b) << P.p), wbase, st,
-                                min(ks + kS, nb), &c, nullptr, 0, &junk);
+        ex_out[k] = decode_at<false>(s_words, k0 * kQ, wbase, st, min(ks + kS, nb), lut_of(b), P.p, &c,
+                                     nullptr, 0, &junk);
         ws.start[k] = st;
         ws.cnt[k] = c;
         ++ch;
@@ -283,48 +346,112 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
     atomicOr(ws.status, kBadCount);
   __syncthreads();
 
-  // d. final decode from the synchronised starts
-  for (long long k = k_begin + threadIdx.x; k < k_end; k += blockDim.x) {
-    const int b = image_of(P, k * kQ);
-    const long long wbase = __ldg(P.word_off + b), nb = __ldg(P.n_bits + b);
-    const long long ks = (k * kQ - wbase) * 32;
-    const long long o = ws.off[k];
-    const long long img_end = __ldg(P.sym_off + b + 1);
-    if (ks == 0 && o != __ldg(P.sym_off + b)) atomicOr(ws.status, kBadCount);
-    if (ks >= nb) continue;
-    int c = 0;
-    const long long room = o < img_end ? img_end - o : 0;
-    const long long ex = decode_span(P, ws.lut + (static_cast<long long>(b) << P.p), wbase, ws.start[k],
-                                     min(ks + kS, nb), &c, P.out + o, room, &bad);
-    if (c > room) atomicOr(ws.status, kBadCount);
-    if (ks + kS >= nb && ex != nb) atomicOr(ws.status, kBadCode);  // the last codeword overruns
+  // d. final decode from the synchronised starts.  Each thread decodes its
+  // subsequence in rounds of up to kRound symbols into its row of a per-warp
+  // shared buffer; the warp then stores two threads' rows per instruction
+  // (lanes 0-15 and 16-31: two 64-byte runs) instead of 32 scattered words.
+  int* wbuf = s_stage + (threadIdx.x >> 5) * 32 * kRow;
+  const int lane = threadIdx.x & 31;
+  for (long long k0 = k_begin; k0 < k_end; k0 += kThreads) {
+    stage_words(k0);
+    const long long k = k0 + threadIdx.x;
+    int lpos = 0, lke = 0, li = 0;
+    uint32_t hi = 0, lo = 0;
+    long long o = 0, room = 0, shift = 0, nb = 0, ks = 0;
+    const uint32_t* lut = s_lut;
+    bool more = false;
+    if (k < k_end) {
+      const int b = image_of(P, k * kQ);
+      const long long wbase = __ldg(P.word_off + b);
+      nb = __ldg(P.n_bits + b);
+      ks = (k * kQ - wbase) * 32;
+      o = ws.off[k];
+      const long long img_end = __ldg(P.sym_off + b + 1);
+      if (ks == 0 && o != __ldg(P.sym_off + b)) atomicOr(ws.status, kBadCount);
+      room = o < img_end ? img_end - o : 0;
+      shift = (wbase - k0 * kQ) * 32;
+      const long long st = ws.start[k], ke = min(ks + kS, nb);
+      lpos = static_cast<int>(st + shift);
+      lke = static_cast<int>(ke + shift);
+      lut = lut_of(b);
+      more = ks < nb && st < ke;
+      if (more) {
+        li = lpos >> 5;
+        hi = s_words[li];
+        lo = s_words[li + 1];
+      }
+    }
+    const int shr = 32 - P.p;
+    long long done = 0;
+    while (__any_sync(0xffffffffu, more)) {
+      int n = 0;
+      while (more && n < kRound) {
+        const int wi = lpos >> 5;
+        if (wi != li) {
+          li = wi;
+          hi = lo;
+          lo = s_words[li + 1];
+        }
+        const uint32_t e = lut[__funnelshift_l(lo, hi, lpos & 31) >> shr];
+        int len = static_cast<int>(e >> 24);
+        if (len == 0) {
+          bad = true;
+          len = 1;
+        }
+        wbuf[lane * kRow + n] = value_of(e);
+        ++n;
+        lpos += len;
+        more = lpos < lke;
+      }
+      __syncwarp();
+      const long long left = room - done;  // symbols this thread may still write
+#pragma unroll 4
+      for (int j = 0; j < 16; ++j) {
+        const int src = 2 * j + (lane >> 4), i = lane & 15;
+        const int ns = __shfl_sync(0xffffffffu, n, src);
+        const long long at = __shfl_sync(0xffffffffu, o + done, src);
+        const long long lim = __shfl_sync(0xffffffffu, left, src);
+        if (i < ns && i < lim) P.out[at + i] = wbuf[src * kRow + i];
+      }
+      done += n;
+      __syncwarp();
+    }
+    if (k < k_end && ks < nb) {
+      if (done > room) atomicOr(ws.status, kBadCount);
+      if (ks + kS >= nb && lpos - shift != nb) atomicOr(ws.status, kBadCode);  // the last codeword overruns
+    }
   }
   if (bad) atomicOr(ws.status, kBadCode);
 }
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Resident CTAs of huff_decode on the current device (the cooperative grid).
-int decode_grid(int* grid) {
+// Resident CTAs of huff_decode on the current device with `smem` bytes of
+// lookup tables each (the cooperative grid), per device and precision.
+int decode_grid(int p, size_t smem, int* grid) {
   constexpr int kMaxDev = 64;
-  static int cached[kMaxDev];
+  static int cached[kMaxDev][PIC_HUFF_MAX_PRECISION + 1];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) {
     cudaGetLastError();
     return PIC_ERR_CUDA;
   }
-  if (cached[dev] == 0) {
+  if (cached[dev][p] == 0) {
     int coop = 0, sms = 0, per_sm = 0;
-    if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess ||
+    // the attribute is the function's, for every precision: set it to the largest
+    constexpr int kMaxSmem = (4 * 2 << PIC_HUFF_MAX_PRECISION) + (kWbuf + kStageInts) * 4;
+    if (cudaFuncSetAttribute(huff_decode, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) !=
+            cudaSuccess ||
+        cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, huff_decode, kThreads, 0) != cudaSuccess) {
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, huff_decode, kThreads, smem) != cudaSuccess) {
       cudaGetLastError();
       return PIC_ERR_CUDA;
     }
     if (!coop || per_sm < 1) return PIC_ERR_UNSUPPORTED;
-    cached[dev] = sms * per_sm < kMaxGrid ? sms * per_sm : kMaxGrid;
+    cached[dev][p] = sms * per_sm < kMaxGrid ? sms * per_sm : kMaxGrid;
   }
-  *grid = cached[dev];
+  *grid = cached[dev][p];
   return PIC_OK;
 }
 
@@ -350,8 +477,10 @@ int pic_huffman_decode(const uint32_t* words, int64_t n_words, const int64_t* wo
     return PIC_ERR_INVALID_ARG;
   const long long n_sub = n_words / kQ;
   if (static_cast<long long>(workspace_bytes) < ws_size(n_sub, B, p)) return PIC_ERR_INVALID_ARG;
+  // 2 tables + the pass's words + the output staging rows
+  const size_t lut_smem = (sizeof(uint32_t) * 2 << p) + (kWbuf + kStageInts) * sizeof(uint32_t);
   int grid = 0;
-  int rc = decode_grid(&grid);
+  int rc = decode_grid(p, lut_smem, &grid);
   if (rc != PIC_OK) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   DecodeParams P{};
@@ -365,15 +494,19 @@ int pic_huffman_decode(const uint32_t* words, int64_t n_words, const int64_t* wo
   P.out = out;
   P.ws = ws_view(workspace, n_sub, B, p);
   P.n_sub = n_sub;
+  // whole passes of kThreads subsequences per CTA (no thread idles in a pass)
+  const long long passes = (n_sub + static_cast<long long>(grid) * kThreads - 1) /
+                           (static_cast<long long>(grid) * kThreads);
+  P.per_block = passes * kThreads;
   if (cudaMemsetAsync(workspace, 0, 16 + kMaxPasses * 4, s) != cudaSuccess) {  // status, pass counters
     cudaGetLastError();
     return PIC_ERR_CUDA;
   }
   huff_lut<<<B, kThreads, 0, s>>>(tab_value, tab_len, max_table, p, P.ws.lut, P.ws.status);
-  const long long g = n_sub < grid ? n_sub : grid;
+  const long long g = (n_sub + P.per_block - 1) / P.per_block;
   void* args[] = {&P};
   if (cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(huff_decode), dim3(static_cast<unsigned>(g)),
-                                  dim3(kThreads), args, 0, s) != cudaSuccess) {
+                                  dim3(kThreads), args, lut_smem, s) != cudaSuccess) {
     cudaGetLastError();
     return PIC_ERR_CUDA;
   }
