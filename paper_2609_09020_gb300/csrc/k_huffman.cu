@@ -119,11 +119,20 @@ __global__ void __launch_bounds__(kThreads)
   }
   __syncthreads();
   const int m = s_m;
-  for (int k = threadIdx.x; k < m; k += blockDim.x) {
-    const uint32_t e = (static_cast<uint32_t>(tl[k]) << 24) | (static_cast<uint32_t>(tv[k]) & 0xFFFFFFu);
-    for (int i = s_start[k]; i < s_start[k + 1]; ++i) out[i] = e;
+  // every entry finds its run by binary search over the run starts
+  for (int i = threadIdx.x; i < (1 << p); i += blockDim.x) {
+    uint32_t e = 0;  // no codeword
+    if (i < s_fill) {
+      int lo = 0, hi = m - 1;  // last k with s_start[k] <= i
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (s_start[mid] <= i) lo = mid;
+        else hi = mid - 1;
+      }
+      e = (static_cast<uint32_t>(tl[lo]) << 24) | (static_cast<uint32_t>(tv[lo]) & 0xFFFFFFu);
+    }
+    out[i] = e;
   }
-  for (int i = s_fill + threadIdx.x; i < (1 << p); i += blockDim.x) out[i] = 0;  // no codeword
 }
 
 // --------------------------------------------------------------- 2. decode
