@@ -179,6 +179,30 @@ def cpu_baseline(wl: wk.Workload, x: wk.Inputs, precision: str, budget_s: float)
             "images_per_s": n / el}
 
 
+# ---- the multi-process (weak-scaling) bookkeeping: each rank decodes its
+# own batch, nothing is exchanged on the data path, the timing is the max
+# over ranks and the rate counts every rank's pixels.
+def shard_workload(wl: wk.Workload, rank: int) -> wk.Workload:
+    """Rank r decodes its own batch: the workload's image seeds + 1000 r."""
+    return wl.replace(seeds=tuple(s + 1000 * rank for s in wl.seeds)) if rank else wl
+
+
+def max_over_ranks(v: float, world: int, device=None) -> float:
+    """The largest of the ranks' values (a MAX all-reduce; v itself at N = 1)."""
+    if world <= 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(px_per_rank: int, world: int, ms: float) -> float:
+    """Decoded megapixels/s over all ranks for a step that took ms (the max)."""
+    return world * px_per_rank / (ms * 1e-3) / 1e6
+
+
 def workload_desc(wl: wk.Workload, precision: str):
     mlp = "-".join(str(d) for d in wl.dims) + " " + wl.act
     return {"workload": f"{wl.name}: {wl.B} x {wl.W}x{wl.H}, {wl.L} levels x {wl.C} ch, MLP {mlp}, "
@@ -766,7 +790,7 @@ def main():
     build.build()  # no-op once built
 
     # Each rank decodes its own batch: image seeds offset by rank (weak scaling).
-    wl_r = wl.replace(seeds=tuple(s + 1000 * rank for s in wl.seeds)) if rank else wl
+    wl_r = shard_workload(wl, rank)
     x = wk.make_inputs(wl_r)
     B = x.latents.shape[0]
     dec = pic.Decoder.for_workload(wl, precision, max_batch=B)
@@ -793,13 +817,9 @@ def main():
         torch.cuda.synchronize(dev)
         barrier()
     dec.check(stream)
-    ms = ev0.elapsed_time(ev1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ev0.elapsed_time(ev1) / args.steps, world, dev)
     px_total = world * B * wl.H * wl.W
-    value = px_total / (ms * 1e-3) / 1e6
+    value = whole_job_rate(B * wl.H * wl.W, world, ms)
     images_per_s = world * B / (ms * 1e-3)
 
     # End to end through the C ABI with host buffers (pinned): H2D of the
@@ -825,11 +845,7 @@ def main():
         t0 = time.perf_counter()
         for _ in range(e_steps):
             host_call()
-        el = time.perf_counter() - t0
-        if world > 1:
-            t = torch.tensor([el], device=dev)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            el = float(t.item())
+        el = max_over_ranks(time.perf_counter() - t0, world, dev)
         h2d = lat_h.numel() * 4 + st_h.numel() * 4 + w_h.numel() * w_h.element_size()
         e2e = {"value": px_total * e_steps / el / 1e6, "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(out_h.numel() * 4),
