@@ -70,7 +70,7 @@ KERNEL_SOURCES = {
     "idct": ["k_idct.cu"],
     "izpr": ["k_izpr.cu"],
     "tc": ["k_tc.cuh", "tc_ptx.cuh", "pic_common.cuh", "pic_gelu.cuh", "pic_kernels.h"],
-    "fp32": ["k_fp32.cu", "pic_common.cuh", "pic_gelu.cuh", "pic_kernels.h"],
+    "fp32": ["k_fp32.cuh", "pic_common.cuh", "pic_gelu.cuh", "pic_kernels.h"],
 }
 
 

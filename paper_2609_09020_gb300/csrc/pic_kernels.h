@@ -20,7 +20,8 @@ struct KernelInfo {
   const void* fn;  // __global__ function taking (DecodeParams)
 };
 
-int fp32_kernels(KernelInfo* out, int cap);
+int fp32_kernels(KernelInfo* out, int cap);        // all of them
+int fp32_kernels_sweep(KernelInfo* out, int cap);  // the width ablation's (own translation unit)
 KernelInfo fp32_generic_kernel_info(int latent_format);
 int tc_kernels(KernelInfo* out, int cap);     // both latent formats
 int tc_kernels_fp32lat(KernelInfo* out, int cap);  // the fp32-latent ones (own translation unit)
