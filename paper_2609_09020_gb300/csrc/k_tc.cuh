@@ -265,6 +265,45 @@ __device__ __forceinline__ void output_layer_cc(const uint8_t* smem, uint32_t t_
   rgb[2] = r2.x + r2.y + wo[4 * N + 2];
 }
 
+// Hidden epilogue of one pixel (TMEM lane): accumulator -> activation ->
+// hi/lo split -> the next layer's A operand in TMEM (hi pairs at t_a, lo
+// pairs at t_a + N/2), 16 columns at a time (fewer live registers).
+template <class Net>
+__device__ __forceinline__ void hidden_epilogue(uint32_t t_acc, uint32_t t_a) {
+  constexpr int N = Net::N;
+#pragma unroll
+  for (int h0 = 0; h0 < N; h0 += 16) {
+    uint32_t acc[16];
+    tmem_ld16(t_acc + h0, acc);
+    tmem_ld_wait();
+    uint32_t hl[16];  // [0, 8): hi pairs, [8, 16): lo pairs
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      float a = __uint_as_float(acc[2 * q]);
+      float bb = __uint_as_float(acc[2 * q + 1]);
+      if constexpr (Net::ACT == ACT_GELU) {
+        a = gelu_poly(a);
+        bb = gelu_poly(bb);
+      }
+      // hi = fp16 truncation (ReLU folded in), lo = v - hi (packed subtraction)
+      split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[8 + q]);
+    }
+    tmem_st8(t_a + h0 / 2, hl);
+    tmem_st8(t_a + N / 2 + h0 / 2, hl + 8);
+  }
+  tmem_st_wait();
+}
+
+// The tile cursor (row yy, tile column xx) advanced by NWG tiles.
+template <int NWG>
+__device__ __forceinline__ void advance_tile(int& yy, int& xx, int tpr) {
+  xx += NWG;
+  while (xx >= tpr) {
+    xx -= tpr;
+    ++yy;
+  }
+}
+
 template <class Net, bool FL>
 __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
     tc_decode_kernel(const DecodeParams p) {
@@ -488,46 +527,12 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         return true;
       };
 
-      // Hidden epilogue: accumulator -> activation -> hi/lo -> TMEM operand.
-      auto hidden_epilogue = [&]() {
-#pragma unroll
-        for (int h0 = 0; h0 < N; h0 += 16) {  // 16 columns at a time (fewer live registers)
-          constexpr int HW = 16;
-          uint32_t acc[HW];
-#pragma unroll
-          for (int c0 = 0; c0 < HW; c0 += 16) tmem_ld16(t_acc + h0 + c0, acc + c0);
-          tmem_ld_wait();
-          uint32_t hl[HW];  // [0, HW/2): hi pairs, [HW/2, HW): lo pairs
-#pragma unroll
-          for (int q = 0; q < HW / 2; ++q) {
-            float a = __uint_as_float(acc[2 * q]);
-            float bb = __uint_as_float(acc[2 * q + 1]);
-            if constexpr (Net::ACT == ACT_GELU) {
-              a = gelu_poly(a);
-              bb = gelu_poly(bb);
-            }
-            // hi = fp16 truncation (ReLU folded in), lo = v - hi (packed subtraction)
-            split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[HW / 2 + q]);
-          }
-          // hi pair (h0/2 + q) -> column t_a + h0/2 + q; lo pair -> t_a + N/2 + h0/2 + q
-          tmem_st8(t_a + h0 / 2, hl);
-          tmem_st8(t_a + N / 2 + h0 / 2, hl + 8);
-        }
-        tmem_st_wait();
-      };
 
       // Tile cursor (row y, tile column tx) of this group's current tile and
       // of the one after it, advanced by NWG tiles without divisions.
       const int tpr = p.tiles_per_row;
       int cy = static_cast<int>((tile0 + w) / tpr);
       int ctx = static_cast<int>((tile0 + w) - static_cast<long long>(cy) * tpr);
-      auto advance = [&](int& yy, int& xx) {
-        xx += NWG;
-        while (xx >= tpr) {
-          xx -= tpr;
-          ++yy;
-        }
-      };
 
       bool ok = true;
       if (w < n_tiles) {
@@ -540,7 +545,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         const int y = cy;
         const int x0 = ctx * kTile;
         int ny = cy, ntx = ctx;
-        advance(ny, ntx);
+        advance_tile<NWG>(ny, ntx, tpr);
         const bool has_next = i + NWG < n_tiles;
         if (has_next) prefetch(ny, ntx * kTile);  // in flight during the first epilogue
 
@@ -553,7 +558,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             }
             acc_phase ^= 1u;
             tc_fence_after();
-            hidden_epilogue();
+            hidden_epilogue<Net>(t_acc, t_a);
             tc_fence_before();
             mbar_arrive(my_a);
             if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
@@ -581,7 +586,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           }
           acc_phase ^= 1u;
           tc_fence_after();
-          hidden_epilogue();
+          hidden_epilogue<Net>(t_acc, t_a);
           tc_fence_before();
           mbar_arrive(my_a);
           if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
