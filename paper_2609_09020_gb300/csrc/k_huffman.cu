@@ -90,46 +90,67 @@ __global__ void __launch_bounds__(kThreads)
     huff_lut(const int32_t* __restrict__ tab_value, const int32_t* __restrict__ tab_len,
              int max_table, int p, uint32_t* lut, int* status) {
   __shared__ int s_start[kMaxTable + 1];
-  __shared__ int s_m, s_fill;
-  const int b = blockIdx.x;
+  __shared__ uint32_t s_entry[kMaxTable];
+  __shared__ int s_warp[kThreads / 32];
+  __shared__ int s_m;
+  const int b = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int32_t* tv = tab_value + static_cast<long long>(b) * max_table;
   const int32_t* tl = tab_len + static_cast<long long>(b) * max_table;
-  uint32_t* out = lut + (static_cast<long long>(b) << p);
-  if (threadIdx.x == 0) {  // run starts: prefix sums of 2^(p - len)
-    int m = 0, bad = 0;
-    long long pos = 0;
-    for (; m < max_table; ++m) {
-      const int l = tl[m];
-      if (l == 0) break;
-      if (l < 1 || l > p) {
-        bad = 1;
-        break;
-      }
-      s_start[m] = static_cast<int>(pos);
-      pos += 1LL << (p - l);
-      if (pos > (1LL << p)) {  // Kraft's inequality violated
-        bad = 1;
-        break;
-      }
+  // the table ends at its first zero length
+  if (t == 0) s_m = max_table;
+  __syncthreads();
+  for (int k = t; k < max_table; k += blockDim.x)
+    if (tl[k] == 0) atomicMin(&s_m, k);
+  __syncthreads();
+  const int m = s_m;
+  // run sizes 2^(p - len) scanned into run starts, 256 entries at a time
+  bool bad = false;
+  int carry = 0;
+  for (int k0 = 0; k0 < m; k0 += kThreads) {
+    const int k = k0 + t;
+    int run = 0;
+    if (k < m) {
+      const int l = tl[k];
+      if (l < 1 || l > p) bad = true;
+      else run = 1 << (p - l);
+      s_entry[k] = (static_cast<uint32_t>(l) << 24) | (static_cast<uint32_t>(tv[k]) & 0xFFFFFFu);
     }
-    s_start[m] = static_cast<int>(pos > (1LL << p) ? (1LL << p) : pos);
-    s_m = bad ? 0 : m;
-    s_fill = bad ? 0 : s_start[m];  // a bad table decodes nothing: every entry "no codeword"
+    int x = run;  // inclusive warp scan, then across the warps
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) s_warp[warp] = x;
+    __syncthreads();
+    int before = 0, total = 0;
+    for (int i = 0; i < kThreads / 32; ++i) {
+      before += i < warp ? s_warp[i] : 0;
+      total += s_warp[i];
+    }
+    if (k < m) s_start[k] = min(carry + before + x - run, 1 << p);
+    carry = min(carry + total, (1 << p) + 1);  // capped: runs may sum past 2^p only in bad tables
+    __syncthreads();
+  }
+  bad = __syncthreads_or(bad) || carry > (1 << p);  // a bad length, or Kraft's inequality violated
+  if (t == 0) {
+    s_start[m] = bad ? 0 : carry;
     if (bad) atomicOr(status, kBadTable);
   }
   __syncthreads();
-  const int m = s_m;
+  const int fill = s_start[m];  // a bad table decodes nothing: every entry "no codeword"
+  uint32_t* out = lut + (static_cast<long long>(b) << p);
   // every entry finds its run by binary search over the run starts
-  for (int i = threadIdx.x; i < (1 << p); i += blockDim.x) {
+  for (int i = t; i < (1 << p); i += blockDim.x) {
     uint32_t e = 0;  // no codeword
-    if (i < s_fill) {
+    if (i < fill) {
       int lo = 0, hi = m - 1;  // last k with s_start[k] <= i
       while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
         if (s_start[mid] <= i) lo = mid;
         else hi = mid - 1;
       }
-      e = (static_cast<uint32_t>(tl[lo]) << 24) | (static_cast<uint32_t>(tv[lo]) & 0xFFFFFFu);
+      e = s_entry[lo];
     }
     out[i] = e;
   }
