@@ -735,6 +735,8 @@ def main():
     ap.add_argument("--ref-step-s", type=float, default=5.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-protocols", action="store_true",
+                    help="skip the per-call, CUDA-graph and serial-per-image rows")
     ap.add_argument("--stage", default="decode",
                     choices=["decode", "izpr", "idct", "pipeline", "fuse", "huffman",
                              "bitstream"],
@@ -818,6 +820,62 @@ def main():
         barrier()
     dec.check(stream)
     ms = max_over_ranks(ev0.elapsed_time(ev1) / args.steps, world, dev)
+
+    # Extra rows (rank 0, outside the timed region above): per-call
+    # percentiles, a CUDA-graph replay of the same calls, and the paper's
+    # serial protocol (synchronise, decode one image, synchronise; App. C).
+    protocols = None
+    if rank == 0 and not args.no_protocols:
+        call_ms = []
+        for _ in range(max(args.steps, 10)):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B)
+            e1.record(stream)
+            e1.synchronize()
+            call_ms.append(e0.elapsed_time(e1))
+        q = np.percentile(call_ms, [10, 50, 90])
+        graph = None
+        try:
+            g = torch.cuda.CUDAGraph()
+            side = torch.cuda.Stream(dev)
+            side.wait_stream(stream)
+            with torch.cuda.stream(side):
+                with torch.cuda.graph(g):
+                    for _ in range(4):
+                        dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, B=B)
+            stream.wait_stream(side)
+            g.replay()
+            torch.cuda.synchronize(dev)
+            reps = max(3, args.steps // 4)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            graph = {"ms_per_call": e0.elapsed_time(e1) / (4 * reps), "calls_per_graph": 4}
+        except Exception as exc:  # graph capture unsupported here: report, don't fail the bench
+            graph = {"unavailable": str(exc)[:200]}
+        dec.check(stream)
+        t_img = []
+        n_ser = min(B, 16)
+        w_img = [wts[b].clone() for b in range(n_ser)]  # each image's weights on its own (aligned)
+        for b in range(n_ser):
+            torch.cuda.synchronize(dev)
+            t0 = time.perf_counter()
+            dec.decode_batch(lat[b:b + 1], steps_t[b:b + 1], w_img[b], wl.H, wl.W, out[b:b + 1],
+                             stream=stream, B=1)
+            torch.cuda.synchronize(dev)
+            t_img.append(time.perf_counter() - t0)
+        protocols = {
+            "per_call_ms": {"p10": float(q[0]), "median": float(q[1]), "p90": float(q[2]),
+                            "calls": len(call_ms)},
+            "cuda_graph": graph,
+            "serial_per_image": {"ms_per_image": 1e3 * float(np.mean(t_img)),
+                                 "images_per_s": 1.0 / float(np.mean(t_img)), "images": len(t_img),
+                                 "note": "synchronise, decode one image, synchronise (the paper's "
+                                         "timing protocol; host clock)"}}
     px_total = world * B * wl.H * wl.W
     value = whole_job_rate(B * wl.H * wl.W, world, ms)
     images_per_s = world * B / (ms * 1e-3)
@@ -911,6 +969,8 @@ def main():
                 "images_per_s": images_per_s,
                 "roofline": roof, "clocks": clk.summary(), "e2e": e2e,
                 "gpu_launches": args.steps, "cpu_baseline": cpu}
+        if protocols is not None:
+            line["protocols"] = protocols
         print(json.dumps(line), flush=True)
     dec.close()
     if world > 1:
