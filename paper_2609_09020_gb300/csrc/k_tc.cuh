@@ -113,6 +113,14 @@ struct TcNet {
   static constexpr int WARPS_PER_SMSP = (THREADS / 32 + 3) / 4;
   static constexpr int MAXREG_RAW = 16384 / (32 * WARPS_PER_SMSP) / 8 * 8;
   static constexpr int MAXREG = MAXREG_RAW > 255 ? 255 : MAXREG_RAW;
+  // Registers moved at run time (setmaxnreg) from the issuing warpgroup,
+  // which needs few, to the decoding warpgroups.  The two budgets together
+  // must not exceed what the CTA was launched with (MAXREG per thread; the
+  // host refuses a build whose kernel does not use exactly MAXREG), or the
+  // increase would wait forever.
+  static constexpr int REG_ISSUE = 64;
+  static constexpr int REG_DECODE_RAW = (MAXREG * THREADS - REG_ISSUE * 32 * NISSUE) / (NWG * 128) / 8 * 8;
+  static constexpr int REG_DECODE = REG_DECODE_RAW > 248 ? 248 : REG_DECODE_RAW;
   static constexpr int CTRL = 256;
   static constexpr int B1_BYTES = N * K1 * 2;
   static constexpr int KB = N + 16;                      // [W | b 0..0]
@@ -138,6 +146,9 @@ struct TcNet {
   static_assert(N % 16 == 0 && N >= 16 && N <= 128, "hidden width must be 16..128, multiple of 16");
   static_assert(NL >= 2, "the tensor-core path needs at least one hidden layer");
   static_assert(TMEM_COLS <= 512, "tensor memory holds 512 columns");
+  static_assert(NISSUE == 4 && MMA_WARP % 4 == 0, "the issuing warps form one warpgroup");
+  static_assert(REG_DECODE >= MAXREG && REG_DECODE * NWG * 128 + REG_ISSUE * 32 * NISSUE <= MAXREG * THREADS,
+                "register split within the launch budget");
   static_assert(8 * (4 * NWG + NISSUE) <= 224, "control block holds the barriers");
 };
 
@@ -162,10 +173,11 @@ __device__ __forceinline__ __half ldh(const __half* p) {
   return __ushort_as_half(__ldg(reinterpret_cast<const unsigned short*>(p)));
 }
 
-// Fills the weight operands and biases of one image into shared memory (all threads).
+// Fills the weight operands and biases of one image into shared memory
+// (threads tid = 0 .. nthr-1 of the decoding warpgroups).
 template <class Net>
 __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
-                                                const int (&dims)[Net::NL + 1]) {
+                                                const int (&dims)[Net::NL + 1], int tid, int nthr) {
   constexpr int N = Net::N, D0 = Net::D0, K1 = Net::K1, NL = Net::NL, KB = Net::KB;
   const __half zero = __float2half_rn(0.0f);
   // layer 0: [W | W | b | 0]
@@ -173,7 +185,7 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
     const int d1 = dims[1];
     const __half* W0 = w;
     const __half* b0 = w + d1 * D0;
-    for (int e = threadIdx.x; e < N * K1; e += blockDim.x) {
+    for (int e = tid; e < N * K1; e += nthr) {
       const int n = e / K1, j = e - n * K1;
       __half v = zero;
       if (n < d1) {
@@ -193,12 +205,11 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
     if constexpr (Net::OUTCC) {
       if (out_layer) {  // 3 x din, fp16 -> fp32 (exact), in the pair layout of BO_BYTES
         float* wo = reinterpret_cast<float*>(smem + Net::OFF_BO);
-        for (int e = threadIdx.x; e < (N / 2) * 8; e += blockDim.x) {
+        for (int e = tid; e < (N / 2) * 8; e += nthr) {
           const int q = e >> 3, o = (e >> 1) & 3, j = 2 * q + (e & 1);
           wo[e] = (o < 3 && j < din) ? __half2float(ldh(p + o * din + j)) : 0.0f;
         }
-        if (threadIdx.x < 4)
-          wo[4 * N + threadIdx.x] = threadIdx.x < 3 ? __half2float(ldh(p + 3 * din + threadIdx.x)) : 0.0f;
+        if (tid < 4) wo[4 * N + tid] = tid < 3 ? __half2float(ldh(p + 3 * din + tid)) : 0.0f;
         break;
       }
     }
@@ -206,7 +217,7 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
     uint8_t* base = smem + (out_layer ? Net::OFF_BO : Net::OFF_BH + (k - 1) * Net::BH_BYTES);
     const __half* Wk = p;
     const __half* bk = p + dout * din;
-    for (int e = threadIdx.x; e < rows * KB; e += blockDim.x) {
+    for (int e = tid; e < rows * KB; e += nthr) {
       const int n = e / KB, j = e - n * KB;
       __half v = zero;
       if (n < dout) {
@@ -367,191 +378,223 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
   uint32_t a1_phase = 0;   // MMA warp: bit w = parity of a1_full[w]
   uint32_t a_phase = 0;    // MMA warp: bit w = parity of a_full[w]
 
-  for (long long seg = t_begin; seg < t_end;) {
-    const int b = static_cast<int>(seg / p.tiles_per_image);
-    const long long seg_end = min(t_end, static_cast<long long>(b + 1) * p.tiles_per_image);
-    __syncthreads();  // all MMAs and reads of the previous image's weights are done
-    {
-      int dims[NL + 1];
-#pragma unroll
-      for (int k = 0; k <= NL; ++k) dims[k] = p.dims[k];
-      load_weights_tc<Net>(smem, wts + b * p.params_per_image, dims);
-    }
-    fence_async_smem();
-    __syncthreads();
-    const int n_tiles = static_cast<int>(seg_end - seg);
-    const long long tile0 = seg - static_cast<long long>(b) * p.tiles_per_image;  // in-image index
-
-    if (warp < 4 * NWG) {
-      // ------------------------------------------------------------ warpgroup
-      const int w = warp >> 2;
-      const int r = ((warp & 3) << 5) | lane;  // tile row = TMEM lane = pixel
-      uint8_t* a1 = smem + Net::OFF_WG + w * Net::WG_BYTES;
-      const uint32_t a1_s = smem_addr(a1);
-      float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES);
-      const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
-      const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(w * 2 * N);
-      const uint32_t t_a = t_acc + N;  // hi in [0, N/2), lo in [N/2, N)
-      const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w,
-                     my_col = bar_col + 8 * w;
-      const int32_t* lat = p.latents + b * p.lat_per_image;
-      float step[L];
-#pragma unroll
-      for (int l = 0; l < L; ++l) step[l] = FL ? 1.0f : __ldg(p.steps + b * L + l);
-
-      // This thread's column items: level, column, and the level's geometry.
-      int it_l[JJ], it_i[JJ], it_W[JJ], it_H[JJ];
-      long long it_off[JJ];
-      float it_sy[JJ], it_sx[JJ];
-#pragma unroll
-      for (int j = 0; j < J; ++j) {
-        int e = r + kTile * j, l = 0, c = 0, i = 0;
-        if (e < NITEM) {
-#pragma unroll
-          for (int lv = 1; lv < L; ++lv)
-#pragma unroll
-            for (int cc = 0; cc < C; ++cc)
-              if (e >= CL::off(lv, cc) && e < CL::off(lv, cc) + ncol(lv)) {
-                l = lv;
-                c = cc;
-                i = e - CL::off(lv, cc);
-              }
-        }
-        it_l[j] = l;  // l == 0 marks an idle slot
-        it_i[j] = i;
-        const LevelGeom lg = p.lv[l];
-        it_W[j] = lg.W;
-        it_H[j] = lg.H;
-        it_off[j] = lg.off + static_cast<long long>(c) * lg.H * lg.W;
-        it_sy[j] = lg.sy;
-        it_sx[j] = lg.sx;
+  // Each role runs its own loop over the images of its tile range, so that
+  // it can hold its own register budget: the issuing warpgroup gives
+  // registers back, the decoding warpgroups take them (setmaxnreg).
+  if (warp < 4 * NWG) {
+    setmaxnreg_inc<Net::REG_DECODE>();
+    for (long long seg = t_begin; seg < t_end;) {
+      const int b = static_cast<int>(seg / p.tiles_per_image);
+      const long long seg_end = min(t_end, static_cast<long long>(b + 1) * p.tiles_per_image);
+      __syncthreads();  // all MMAs and reads of the previous image's weights are done
+      {
+        int dims[NL + 1];
+  #pragma unroll
+        for (int k = 0; k <= NL; ++k) dims[k] = p.dims[k];
+        load_weights_tc<Net>(smem, wts + b * p.params_per_image, dims, threadIdx.x, 4 * NWG * 32);
       }
-      // Relative x-taps of pixel r for each level (used when fast_x): the
-      // source coordinate (r + 1/2) / 2^l - 1/2 relative to column x0/2^l - 1.
-      int rel[L];
-      float fx[L];
-#pragma unroll
-      for (int l = 1; l < L; ++l) {
-        const float sx = (static_cast<float>(r) + 0.5f) * (1.0f / static_cast<float>(1 << l)) - 0.5f;
-        const float fl = floorf(sx);
-        rel[l] = static_cast<int>(fl) + 1;
-        fx[l] = sx - fl;
-      }
+      fence_async_smem();
+      __syncthreads();
+      const int n_tiles = static_cast<int>(seg_end - seg);
+      const long long tile0 = seg - static_cast<long long>(b) * p.tiles_per_image;  // in-image index
+      {
+        // ------------------------------------------------------------ warpgroup
+        const int w = warp >> 2;
+        const int r = ((warp & 3) << 5) | lane;  // tile row = TMEM lane = pixel
+        uint8_t* a1 = smem + Net::OFF_WG + w * Net::WG_BYTES;
+        const uint32_t a1_s = smem_addr(a1);
+        float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES);
+        const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
+        const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(w * 2 * N);
+        const uint32_t t_a = t_acc + N;  // hi in [0, N/2), lo in [N/2, N)
+        const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w,
+                       my_col = bar_col + 8 * w;
+        const int32_t* lat = p.latents + b * p.lat_per_image;
+        float step[L];
+  #pragma unroll
+        for (int l = 0; l < L; ++l) step[l] = FL ? 1.0f : __ldg(p.steps + b * L + l);
 
-      // Global loads tile (y, x0) needs -- the level-0 values of pixel r and
-      // the raw texel pairs of this thread's column items -- issued as
-      // asynchronous copies into this thread's column of the staging buffer
-      // (slot s of thread r at stage[s * 128 + r]); nothing waits on them
-      // until the features are computed.
-      const uint32_t stage_s = a1_s + Net::A1_BYTES + Net::COL_BYTES;
-      const int* stage = reinterpret_cast<const int*>(a1 + Net::A1_BYTES + Net::COL_BYTES);
-      auto prefetch = [&](int y, int x0) {
-        const int xc = min(x0 + r, p.W - 1);
-#pragma unroll
-        for (int c = 0; c < C; ++c)
-          cp_async4(stage_s + (c * kTile + r) * 4, lat + c * plane + static_cast<long long>(y) * p.W + xc);
-#pragma unroll
+        // This thread's column items: level, column, and the level's geometry.
+        int it_l[JJ], it_i[JJ], it_W[JJ], it_H[JJ];
+        long long it_off[JJ];
+        float it_sy[JJ], it_sx[JJ];
+  #pragma unroll
         for (int j = 0; j < J; ++j) {
-          const int l = it_l[j];
-          if (l > 0) {
-            const Tap ty = bilinear_tap(y, it_sy[j], it_H[j]);
-            const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, it_sx[j], it_W[j]).i0;
-            const int u = min(max(u_start + it_i[j], 0), it_W[j] - 1);
-            const int32_t* pl = lat + it_off[j] + u;
-            cp_async4(stage_s + ((C + 2 * j) * kTile + r) * 4, pl + ty.i0 * it_W[j]);
-            cp_async4(stage_s + ((C + 2 * j + 1) * kTile + r) * 4, pl + ty.i1 * it_W[j]);
+          int e = r + kTile * j, l = 0, c = 0, i = 0;
+          if (e < NITEM) {
+  #pragma unroll
+            for (int lv = 1; lv < L; ++lv)
+  #pragma unroll
+              for (int cc = 0; cc < C; ++cc)
+                if (e >= CL::off(lv, cc) && e < CL::off(lv, cc) + ncol(lv)) {
+                  l = lv;
+                  c = cc;
+                  i = e - CL::off(lv, cc);
+                }
           }
+          it_l[j] = l;  // l == 0 marks an idle slot
+          it_i[j] = i;
+          const LevelGeom lg = p.lv[l];
+          it_W[j] = lg.W;
+          it_H[j] = lg.H;
+          it_off[j] = lg.off + static_cast<long long>(c) * lg.H * lg.W;
+          it_sy[j] = lg.sy;
+          it_sx[j] = lg.sx;
         }
-        cp_async_commit();
-      };
-
-      // Features of tile (y, x0) from its prefetched loads -> A1 (shared).
-      // Returns false if a wait gave up.
-      auto features = [&](int y, int x0) -> bool {
-        cp_async_wait_all();  // this thread's staged loads have landed
-        // vertical pass into the column buffer
-#pragma unroll
-        for (int j = 0; j < J; ++j) {
-          const int l = it_l[j];
-          if (l > 0) {
-            const float beta = bilinear_tap(y, it_sy[j], it_H[j]).frac;
-            const int t0 = stage[(C + 2 * j) * kTile + r], t1 = stage[(C + 2 * j + 1) * kTile + r];
-            colbuf[r + kTile * j] = step[l] * lat_lerp<FL>(t0, t1, beta);
-          }
-        }
-        mbar_arrive(my_col);  // the group's column buffer is complete once all 128 arrived
-        if (!__all_sync(0xffffffffu, wait_bounded(my_col, col_phase, abort_flag, p.status)))
-          return false;
-        col_phase ^= 1u;
-        // horizontal pass + level 0
-        const int xc = min(x0 + r, p.W - 1);
-        float f[D0];
-#pragma unroll
-        for (int c = 0; c < C; ++c) f[c] = step[0] * lat_value<FL>(stage[c * kTile + r]);
-#pragma unroll
+        // Relative x-taps of pixel r for each level (used when fast_x): the
+        // source coordinate (r + 1/2) / 2^l - 1/2 relative to column x0/2^l - 1.
+        int rel[L];
+        float fx[L];
+  #pragma unroll
         for (int l = 1; l < L; ++l) {
-          int i0, i1;
-          float a;
-          if (fast_x) {
-            i0 = rel[l];
-            i1 = rel[l] + 1;
-            a = fx[l];
-          } else {
-            const LevelGeom lg = p.lv[l];
-            const int u_start = bilinear_tap(x0, lg.sx, lg.W).i0;
-            const Tap tx = bilinear_tap(xc, lg.sx, lg.W);
-            i0 = min(max(tx.i0 - u_start, 0), ncol(l) - 1);
-            i1 = min(max(tx.i1 - u_start, 0), ncol(l) - 1);
-            a = tx.frac;
-          }
-#pragma unroll
-          for (int c = 0; c < C; ++c) {
-            const float* cb = colbuf + CL::off(l, c);
-            const float v0 = cb[i0], v1 = cb[i1];
-            f[l * C + c] = fmaf(a, v1 - v0, v0);
-          }
+          const float sx = (static_cast<float>(r) + 0.5f) * (1.0f / static_cast<float>(1 << l)) - 0.5f;
+          const float fl = floorf(sx);
+          rel[l] = static_cast<int>(fl) + 1;
+          fx[l] = sx - fl;
         }
-        // hi/lo split, the constant-1 bias column, padding -> A1
-        float v[K1];
-#pragma unroll
-        for (int j = 0; j < K1; ++j) v[j] = 0.0f;
-#pragma unroll
-        for (int j = 0; j < D0; ++j) split_hi_lo(f[j], v[j], v[D0 + j]);
-        v[2 * D0] = 1.0f;
-#pragma unroll
-        for (int kc = 0; kc < K1 / 8; ++kc)
-          sts128(a1_s + kmaj(r, kc * 8, K1), pack_f16x2(v[kc * 8 + 0], v[kc * 8 + 1]),
-                 pack_f16x2(v[kc * 8 + 2], v[kc * 8 + 3]), pack_f16x2(v[kc * 8 + 4], v[kc * 8 + 5]),
-                 pack_f16x2(v[kc * 8 + 6], v[kc * 8 + 7]));
-        fence_async_smem();
-        return true;
-      };
+
+        // Global loads tile (y, x0) needs -- the level-0 values of pixel r and
+        // the raw texel pairs of this thread's column items -- issued as
+        // asynchronous copies into this thread's column of the staging buffer
+        // (slot s of thread r at stage[s * 128 + r]); nothing waits on them
+        // until the features are computed.
+        const uint32_t stage_s = a1_s + Net::A1_BYTES + Net::COL_BYTES;
+        const int* stage = reinterpret_cast<const int*>(a1 + Net::A1_BYTES + Net::COL_BYTES);
+        auto prefetch = [&](int y, int x0) {
+          const int xc = min(x0 + r, p.W - 1);
+  #pragma unroll
+          for (int c = 0; c < C; ++c)
+            cp_async4(stage_s + (c * kTile + r) * 4, lat + c * plane + static_cast<long long>(y) * p.W + xc);
+  #pragma unroll
+          for (int j = 0; j < J; ++j) {
+            const int l = it_l[j];
+            if (l > 0) {
+              const Tap ty = bilinear_tap(y, it_sy[j], it_H[j]);
+              const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, it_sx[j], it_W[j]).i0;
+              const int u = min(max(u_start + it_i[j], 0), it_W[j] - 1);
+              const int32_t* pl = lat + it_off[j] + u;
+              cp_async4(stage_s + ((C + 2 * j) * kTile + r) * 4, pl + ty.i0 * it_W[j]);
+              cp_async4(stage_s + ((C + 2 * j + 1) * kTile + r) * 4, pl + ty.i1 * it_W[j]);
+            }
+          }
+          cp_async_commit();
+        };
+
+        // Features of tile (y, x0) from its prefetched loads -> A1 (shared).
+        // Returns false if a wait gave up.
+        auto features = [&](int y, int x0) -> bool {
+          cp_async_wait_all();  // this thread's staged loads have landed
+          // vertical pass into the column buffer
+  #pragma unroll
+          for (int j = 0; j < J; ++j) {
+            const int l = it_l[j];
+            if (l > 0) {
+              const float beta = bilinear_tap(y, it_sy[j], it_H[j]).frac;
+              const int t0 = stage[(C + 2 * j) * kTile + r], t1 = stage[(C + 2 * j + 1) * kTile + r];
+              colbuf[r + kTile * j] = step[l] * lat_lerp<FL>(t0, t1, beta);
+            }
+          }
+          mbar_arrive(my_col);  // the group's column buffer is complete once all 128 arrived
+          if (!__all_sync(0xffffffffu, wait_bounded(my_col, col_phase, abort_flag, p.status)))
+            return false;
+          col_phase ^= 1u;
+          // horizontal pass + level 0
+          const int xc = min(x0 + r, p.W - 1);
+          float f[D0];
+  #pragma unroll
+          for (int c = 0; c < C; ++c) f[c] = step[0] * lat_value<FL>(stage[c * kTile + r]);
+  #pragma unroll
+          for (int l = 1; l < L; ++l) {
+            int i0, i1;
+            float a;
+            if (fast_x) {
+              i0 = rel[l];
+              i1 = rel[l] + 1;
+              a = fx[l];
+            } else {
+              const LevelGeom lg = p.lv[l];
+              const int u_start = bilinear_tap(x0, lg.sx, lg.W).i0;
+              const Tap tx = bilinear_tap(xc, lg.sx, lg.W);
+              i0 = min(max(tx.i0 - u_start, 0), ncol(l) - 1);
+              i1 = min(max(tx.i1 - u_start, 0), ncol(l) - 1);
+              a = tx.frac;
+            }
+  #pragma unroll
+            for (int c = 0; c < C; ++c) {
+              const float* cb = colbuf + CL::off(l, c);
+              const float v0 = cb[i0], v1 = cb[i1];
+              f[l * C + c] = fmaf(a, v1 - v0, v0);
+            }
+          }
+          // hi/lo split, the constant-1 bias column, padding -> A1
+          float v[K1];
+  #pragma unroll
+          for (int j = 0; j < K1; ++j) v[j] = 0.0f;
+  #pragma unroll
+          for (int j = 0; j < D0; ++j) split_hi_lo(f[j], v[j], v[D0 + j]);
+          v[2 * D0] = 1.0f;
+  #pragma unroll
+          for (int kc = 0; kc < K1 / 8; ++kc)
+            sts128(a1_s + kmaj(r, kc * 8, K1), pack_f16x2(v[kc * 8 + 0], v[kc * 8 + 1]),
+                   pack_f16x2(v[kc * 8 + 2], v[kc * 8 + 3]), pack_f16x2(v[kc * 8 + 4], v[kc * 8 + 5]),
+                   pack_f16x2(v[kc * 8 + 6], v[kc * 8 + 7]));
+          fence_async_smem();
+          return true;
+        };
 
 
-      // Tile cursor (row y, tile column tx) of this group's current tile and
-      // of the one after it, advanced by NWG tiles without divisions.
-      const int tpr = p.tiles_per_row;
-      int cy = static_cast<int>((tile0 + w) / tpr);
-      int ctx = static_cast<int>((tile0 + w) - static_cast<long long>(cy) * tpr);
+        // Tile cursor (row y, tile column tx) of this group's current tile and
+        // of the one after it, advanced by NWG tiles without divisions.
+        const int tpr = p.tiles_per_row;
+        int cy = static_cast<int>((tile0 + w) / tpr);
+        int ctx = static_cast<int>((tile0 + w) - static_cast<long long>(cy) * tpr);
 
-      bool ok = true;
-      if (w < n_tiles) {
-        prefetch(cy, ctx * kTile);
-        ok = features(cy, ctx * kTile);
-        if (ok) mbar_arrive(my_a1);
-      }
-      for (int i = w; i < n_tiles && ok; i += NWG) {
-        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
-        const int y = cy;
-        const int x0 = ctx * kTile;
-        int ny = cy, ntx = ctx;
-        advance_tile<NWG>(ny, ntx, tpr);
-        const bool has_next = i + NWG < n_tiles;
-        if (has_next) prefetch(ny, ntx * kTile);  // in flight during the first epilogue
+        bool ok = true;
+        if (w < n_tiles) {
+          prefetch(cy, ctx * kTile);
+          ok = features(cy, ctx * kTile);
+          if (ok) mbar_arrive(my_a1);
+        }
+        for (int i = w; i < n_tiles && ok; i += NWG) {
+          if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+          const int y = cy;
+          const int x0 = ctx * kTile;
+          int ny = cy, ntx = ctx;
+          advance_tile<NWG>(ny, ntx, tpr);
+          const bool has_next = i + NWG < n_tiles;
+          if (has_next) prefetch(ny, ntx * kTile);  // in flight during the first epilogue
 
-        if constexpr (Net::OUTCC) {
-          // hidden epilogues up to the last one, which runs the output layer
-          for (int k = 0; k < NL - 2 && ok; ++k) {
+          if constexpr (Net::OUTCC) {
+            // hidden epilogues up to the last one, which runs the output layer
+            for (int k = 0; k < NL - 2 && ok; ++k) {
+              if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
+                ok = false;
+                break;
+              }
+              acc_phase ^= 1u;
+              tc_fence_after();
+              hidden_epilogue<Net>(t_acc, t_a);
+              tc_fence_before();
+              mbar_arrive(my_a);
+              if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
+            }
+            if (!ok) break;
+            if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
+            acc_phase ^= 1u;
+            tc_fence_after();
+            float rgb[3];
+            output_layer_cc<Net>(smem, t_acc, rgb);
+            tc_fence_before();
+            if (NL == 2 && has_next) ok = features(ny, ntx * kTile);  // no hidden layer to overlap
+            if (has_next && ok) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
+            const int x = x0 + r;
+            if (x < p.W) store_rgb(p, b, y, x, rgb[0], rgb[1], rgb[2]);
+            cy = ny;
+            ctx = ntx;
+            if (!ok) break;
+            continue;
+          }
+          for (int k = 0; k < NL - 1 && ok; ++k) {
             if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
               ok = false;
               break;
@@ -564,114 +607,97 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
           }
           if (!ok) break;
+
+          // ---- output layer: bias, clamp, store ----
           if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
           acc_phase ^= 1u;
           tc_fence_after();
-          float rgb[3];
-          output_layer_cc<Net>(smem, t_acc, rgb);
+          uint32_t o[4];
+          tmem_ld4(t_acc, o);
+          tmem_ld_wait();
           tc_fence_before();
-          if (NL == 2 && has_next) ok = features(ny, ntx * kTile);  // no hidden layer to overlap
-          if (has_next && ok) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
+          if (has_next) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
           const int x = x0 + r;
-          if (x < p.W) store_rgb(p, b, y, x, rgb[0], rgb[1], rgb[2]);
+          if (x < p.W)
+            store_rgb(p, b, y, x, __uint_as_float(o[0]), __uint_as_float(o[1]), __uint_as_float(o[2]));
           cy = ny;
           ctx = ntx;
-          if (!ok) break;
-          continue;
-        }
-        for (int k = 0; k < NL - 1 && ok; ++k) {
-          if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
-            ok = false;
-            break;
-          }
-          acc_phase ^= 1u;
-          tc_fence_after();
-          hidden_epilogue<Net>(t_acc, t_a);
-          tc_fence_before();
-          mbar_arrive(my_a);
-          if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
-        }
-        if (!ok) break;
-
-        // ---- output layer: bias, clamp, store ----
-        if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
-        acc_phase ^= 1u;
-        tc_fence_after();
-        uint32_t o[4];
-        tmem_ld4(t_acc, o);
-        tmem_ld_wait();
-        tc_fence_before();
-        if (has_next) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
-        const int x = x0 + r;
-        if (x < p.W)
-          store_rgb(p, b, y, x, __uint_as_float(o[0]), __uint_as_float(o[1]), __uint_as_float(o[2]));
-        cy = ny;
-        ctx = ntx;
-      }
-    } else if (warp >= Net::MMA_WARP && warp < Net::MMA_WARP + Net::NISSUE) {
-      // --------------------------------------------------------------- MMA issuer
-      // Warp MMA_WARP + w issues every MMA of group w, in the group's order
-      // (its tiles in turn, layers in turn), sleeping in the mbarrier wait
-      // in between.  The whole warp runs the control flow (descriptors stay
-      // warp-uniform); one elected lane issues the MMAs and the commit.
-      // Descriptors depend on the start address only through their low
-      // field: base + (offset >> 4).
-      const int w = warp - Net::MMA_WARP;
-      constexpr uint32_t id_hidden = idesc_f16(128, N);
-      constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
-      const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG + w * Net::WG_BYTES, 128, 16 * K1);
-      const uint64_t dB1 = smem_desc(sbase + Net::OFF_B1, 128, 16 * K1);
-      const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * Net::KB);
-      const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * Net::KB);
-      const uint64_t dONES = smem_desc(sbase + Net::OFF_ONES, 128, 16 * 16);
-      constexpr uint64_t kStep = 256 >> 4;              // one K-step (16 fp16) = 256 B
-      constexpr uint64_t kLayer = Net::BH_BYTES >> 4;   // next hidden layer's weights
-      static_assert(Net::WG_BYTES % 16 == 0 && Net::BH_BYTES % 16 == 0, "16-byte aligned operands");
-      const uint32_t d = tmem + static_cast<uint32_t>(w * 2 * N);
-      const uint32_t ta = d + N;
-      const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w;
-      bool ok = true;
-      for (int i = w; i < n_tiles && ok; i += NWG) {
-        for (int k = 0; k < (Net::OUTCC ? NL - 1 : NL); ++k) {  // OUTCC: no output-layer MMA
-          const uint32_t bar = k == 0 ? my_a1 : my_a;
-          const uint32_t par = k == 0 ? (a1_phase & 1u) : (a_phase & 1u);
-          if (!__all_sync(0xffffffffu, wait_bounded(bar, par, abort_flag, p.status))) {
-            ok = false;
-            break;
-          }
-          if (k == 0) a1_phase ^= 1u;
-          else a_phase ^= 1u;
-          if (elect_one()) {
-            tc_fence_after();
-            if (k == 0) {
-#pragma unroll
-              for (int s = 0; s < K1 / 16; ++s) mma_f16(d, dA1 + s * kStep, dB1 + s * kStep, id_hidden, s > 0);
-            } else {
-              const bool out_layer = (k == NL - 1);
-              const uint64_t db = out_layer ? dBO : dBH + (k - 1) * kLayer;
-              const uint32_t id = out_layer ? id_out : id_hidden;
-#pragma unroll
-              for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + 8 * s, db + s * kStep, id, s > 0);  // hi
-#pragma unroll
-              for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
-              mma_f16(d, dONES, db + (N / 16) * kStep, id, 1);  // bias: [1 0..0] x [b 0..0]
-            }
-            mma_commit(my_c);
-          }
-          __syncwarp();
         }
       }
+      seg = seg_end;
     }
-    __syncwarp();
-    seg = seg_end;
-  }
-
-  if (warp >= Net::MMA_WARP && warp < Net::MMA_WARP + Net::NISSUE && elect_one()) {
-    // Every MMA this thread issued must be complete before the memory goes.
-    const uint32_t drain = bar_drain + 8 * (warp - Net::MMA_WARP);
-    mma_commit(drain);
-    int dummy = 0;
-    wait_bounded(drain, 0, reinterpret_cast<volatile int*>(&dummy), p.status);
+  } else {
+    setmaxnreg_dec<Net::REG_ISSUE>();
+    for (long long seg = t_begin; seg < t_end;) {
+      const int b = static_cast<int>(seg / p.tiles_per_image);
+      const long long seg_end = min(t_end, static_cast<long long>(b + 1) * p.tiles_per_image);
+      __syncthreads();  // all MMAs of the previous image are complete
+      __syncthreads();  // the decoding warps have loaded this image's weights
+      const int n_tiles = static_cast<int>(seg_end - seg);
+      {
+        // --------------------------------------------------------------- MMA issuer
+        // Warp MMA_WARP + w issues every MMA of group w, in the group's order
+        // (its tiles in turn, layers in turn), sleeping in the mbarrier wait
+        // in between.  The whole warp runs the control flow (descriptors stay
+        // warp-uniform); one elected lane issues the MMAs and the commit.
+        // Descriptors depend on the start address only through their low
+        // field: base + (offset >> 4).
+        const int w = warp - Net::MMA_WARP;
+        constexpr uint32_t id_hidden = idesc_f16(128, N);
+        constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
+        const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG + w * Net::WG_BYTES, 128, 16 * K1);
+        const uint64_t dB1 = smem_desc(sbase + Net::OFF_B1, 128, 16 * K1);
+        const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * Net::KB);
+        const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * Net::KB);
+        const uint64_t dONES = smem_desc(sbase + Net::OFF_ONES, 128, 16 * 16);
+        constexpr uint64_t kStep = 256 >> 4;              // one K-step (16 fp16) = 256 B
+        constexpr uint64_t kLayer = Net::BH_BYTES >> 4;   // next hidden layer's weights
+        static_assert(Net::WG_BYTES % 16 == 0 && Net::BH_BYTES % 16 == 0, "16-byte aligned operands");
+        const uint32_t d = tmem + static_cast<uint32_t>(w * 2 * N);
+        const uint32_t ta = d + N;
+        const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w;
+        bool ok = true;
+        for (int i = w; i < n_tiles && ok; i += NWG) {
+          for (int k = 0; k < (Net::OUTCC ? NL - 1 : NL); ++k) {  // OUTCC: no output-layer MMA
+            const uint32_t bar = k == 0 ? my_a1 : my_a;
+            const uint32_t par = k == 0 ? (a1_phase & 1u) : (a_phase & 1u);
+            if (!__all_sync(0xffffffffu, wait_bounded(bar, par, abort_flag, p.status))) {
+              ok = false;
+              break;
+            }
+            if (k == 0) a1_phase ^= 1u;
+            else a_phase ^= 1u;
+            if (elect_one()) {
+              tc_fence_after();
+              if (k == 0) {
+  #pragma unroll
+                for (int s = 0; s < K1 / 16; ++s) mma_f16(d, dA1 + s * kStep, dB1 + s * kStep, id_hidden, s > 0);
+              } else {
+                const bool out_layer = (k == NL - 1);
+                const uint64_t db = out_layer ? dBO : dBH + (k - 1) * kLayer;
+                const uint32_t id = out_layer ? id_out : id_hidden;
+  #pragma unroll
+                for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + 8 * s, db + s * kStep, id, s > 0);  // hi
+  #pragma unroll
+                for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
+                mma_f16(d, dONES, db + (N / 16) * kStep, id, 1);  // bias: [1 0..0] x [b 0..0]
+              }
+              mma_commit(my_c);
+            }
+            __syncwarp();
+          }
+        }
+      }
+      __syncwarp();
+      seg = seg_end;
+    }
+    if (elect_one()) {
+      // Every MMA this thread issued must be complete before the memory goes.
+      const uint32_t drain = bar_drain + 8 * (warp - Net::MMA_WARP);
+      mma_commit(drain);
+      int dummy = 0;
+      wait_bounded(drain, 0, reinterpret_cast<volatile int*>(&dummy), p.status);
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -693,6 +719,7 @@ KernelInfo make_tc(const char* name, const int* dims) {
   for (int i = 0; i <= NL; ++i) k.dims[i] = dims[i];
   k.act = ACT;
   k.threads = Net::THREADS;
+  k.regs_at_launch = Net::MAXREG;
   k.tile_px = kTile;
   k.smem_bytes = Net::SMEM;
   k.fn = reinterpret_cast<const void*>(&tc_decode_kernel<Net, FL>);

@@ -132,6 +132,19 @@ int launch(pic_decoder* h, const DecodeParams& p, cudaStream_t stream) {
 
 size_t weight_elem_bytes(const pic_arch& a) { return a.precision == PIC_PREC_FP16_TC ? 2 : 4; }
 
+// A kernel that moves registers between its warpgroups at run time assumes
+// the register count it was launched with; any other build is refused
+// (its register increase could otherwise never be granted).
+bool regs_match(const pic::KernelInfo& k) {
+  if (k.regs_at_launch == 0) return true;
+  cudaFuncAttributes a{};
+  if (cudaFuncGetAttributes(&a, k.fn) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.numRegs == k.regs_at_launch;
+}
+
 }  // namespace
 
 extern "C" {
@@ -207,6 +220,7 @@ int pic_decode_create(const pic_arch* arch, pic_decoder** out) {
     return PIC_ERR_UNSUPPORTED;
   }
   if (k.smem_bytes > static_cast<int>(prop.sharedMemPerBlockOptin)) return PIC_ERR_UNSUPPORTED;
+  if (!regs_match(k)) return PIC_ERR_UNSUPPORTED;
   if (cudaFuncSetAttribute(k.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, k.smem_bytes) !=
       cudaSuccess) {
     cudaGetLastError();
@@ -523,6 +537,7 @@ extern "C" int pic_decode_batch_noalloc(const pic_arch* arch, int B, const int32
     return PIC_ERR_UNSUPPORTED;
   }
   if (h.kern.smem_bytes > smem_optin) return PIC_ERR_UNSUPPORTED;
+  if (!regs_match(h.kern)) return PIC_ERR_UNSUPPORTED;
   if (cudaFuncSetAttribute(h.kern.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            h.kern.smem_bytes) != cudaSuccess) {
     cudaGetLastError();

@@ -15,6 +15,7 @@ struct KernelInfo {
   int dims[7];
   int act;
   int threads;     // threads per CTA
+  int regs_at_launch;  // registers per thread the kernel must be built with (0: any)
   int smem_bytes;  // dynamic shared memory per CTA
   int tile_px;     // pixels per tile (one tile = a run of one image row)
   const void* fn;  // __global__ function taking (DecodeParams)

@@ -90,6 +90,16 @@ __device__ __forceinline__ bool elect_one() {
   return pred != 0;
 }
 
+// Per-warpgroup register budget (all warps of the warpgroup execute it).
+template <int R>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R));
+}
+template <int R>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R));
+}
+
 // ---- tcgen05 ----------------------------------------------------------------
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
@@ -227,33 +237,30 @@ __device__ __forceinline__ float2 unpack_f16x2(uint32_t v) {
 // hi/lo split of a pair (a, b) of fp32 values for the split-operand MMA:
 // hi = RZ_fp16(x) (ReLU applied when RELU), lo = RN_fp16(x - hi) (ReLU too:
 // x - hi has x's sign).  Returns both as f16x2 with a in the low half.
+// x - hi comes from one mixed-precision FMA per element, hi * (-1) + x with
+// the fp16 hi widened exactly; the result is exact (x - hi is representable
+// in fp32), so no separate widening of hi is needed.
 template <bool RELU>
 __device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi2, uint32_t& lo2) {
   if constexpr (RELU) {
     asm("{\n\t"
-        ".reg .b16 h0, h1;\n\t.reg .f32 ha, hb, la, lb;\n\t.reg .b64 v, hh, l;\n\t"
+        ".reg .b16 h0, h1, m1;\n\t.reg .f32 la, lb;\n\t"
+        "mov.b16 m1, 0xBC00;\n\t"
         "cvt.rz.relu.f16x2.f32 %0, %3, %2;\n\t"
         "mov.b32 {h0, h1}, %0;\n\t"
-        "cvt.f32.f16 ha, h0;\n\t"
-        "cvt.f32.f16 hb, h1;\n\t"
-        "mov.b64 v, {%2, %3};\n\t"
-        "mov.b64 hh, {ha, hb};\n\t"
-        "sub.rn.f32x2 l, v, hh;\n\t"
-        "mov.b64 {la, lb}, l;\n\t"
+        "fma.rn.f32.f16 la, h0, m1, %2;\n\t"
+        "fma.rn.f32.f16 lb, h1, m1, %3;\n\t"
         "cvt.rn.relu.f16x2.f32 %1, lb, la;\n\t}\n"
         : "=r"(hi2), "=r"(lo2)
         : "f"(a), "f"(b));
   } else {
     asm("{\n\t"
-        ".reg .b16 h0, h1;\n\t.reg .f32 ha, hb, la, lb;\n\t.reg .b64 v, hh, l;\n\t"
+        ".reg .b16 h0, h1, m1;\n\t.reg .f32 la, lb;\n\t"
+        "mov.b16 m1, 0xBC00;\n\t"
         "cvt.rz.f16x2.f32 %0, %3, %2;\n\t"
         "mov.b32 {h0, h1}, %0;\n\t"
-        "cvt.f32.f16 ha, h0;\n\t"
-        "cvt.f32.f16 hb, h1;\n\t"
-        "mov.b64 v, {%2, %3};\n\t"
-        "mov.b64 hh, {ha, hb};\n\t"
-        "sub.rn.f32x2 l, v, hh;\n\t"
-        "mov.b64 {la, lb}, l;\n\t"
+        "fma.rn.f32.f16 la, h0, m1, %2;\n\t"
+        "fma.rn.f32.f16 lb, h1, m1, %3;\n\t"
         "cvt.rn.f16x2.f32 %1, lb, la;\n\t}\n"
         : "=r"(hi2), "=r"(lo2)
         : "f"(a), "f"(b));
