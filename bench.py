@@ -7,7 +7,7 @@ throughput workload (64 independent 768x512 images, 7 levels x 1 channel,
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c5]
                     [--precision fp16_tc|fp32] [--impl ours|reference]
-                    [--stage decode|izpr|idct|pipeline] [--chunk 16]
+                    [--stage decode|izpr|idct|pipeline] [--chunk 64]
 
 Prints one JSON line (rank 0).  ``value`` is decoded megapixels/s over all
 ranks (weak scaling: each rank decodes its own batch; no collective on the
@@ -787,7 +787,7 @@ def main():
                              "bitstream"],
                     help="decode (default): the synthesis; the others time the stages before "
                          "it, alone or chained, on one GPU")
-    ap.add_argument("--chunk", type=int, default=16,
+    ap.add_argument("--chunk", type=int, default=64,
                     help="pipeline stage: images per iZpR/iDCT/decode round")
     args = ap.parse_args()
     if args.stage != "decode":

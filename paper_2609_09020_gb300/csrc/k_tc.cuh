@@ -389,7 +389,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       __syncthreads();  // all MMAs and reads of the previous image's weights are done
       {
         int dims[NL + 1];
-  #pragma unroll
+#pragma unroll
         for (int k = 0; k <= NL; ++k) dims[k] = p.dims[k];
         load_weights_tc<Net>(smem, wts + b * p.params_per_image, dims, threadIdx.x, 4 * NWG * 32);
       }
@@ -411,20 +411,20 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
                        my_col = bar_col + 8 * w;
         const int32_t* lat = p.latents + b * p.lat_per_image;
         float step[L];
-  #pragma unroll
+#pragma unroll
         for (int l = 0; l < L; ++l) step[l] = FL ? 1.0f : __ldg(p.steps + b * L + l);
 
         // This thread's column items: level, column, and the level's geometry.
         int it_l[JJ], it_i[JJ], it_W[JJ], it_H[JJ];
         long long it_off[JJ];
         float it_sy[JJ], it_sx[JJ];
-  #pragma unroll
+#pragma unroll
         for (int j = 0; j < J; ++j) {
           int e = r + kTile * j, l = 0, c = 0, i = 0;
           if (e < NITEM) {
-  #pragma unroll
+#pragma unroll
             for (int lv = 1; lv < L; ++lv)
-  #pragma unroll
+#pragma unroll
               for (int cc = 0; cc < C; ++cc)
                 if (e >= CL::off(lv, cc) && e < CL::off(lv, cc) + ncol(lv)) {
                   l = lv;
@@ -445,7 +445,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         // source coordinate (r + 1/2) / 2^l - 1/2 relative to column x0/2^l - 1.
         int rel[L];
         float fx[L];
-  #pragma unroll
+#pragma unroll
         for (int l = 1; l < L; ++l) {
           const float sx = (static_cast<float>(r) + 0.5f) * (1.0f / static_cast<float>(1 << l)) - 0.5f;
           const float fl = floorf(sx);
@@ -462,10 +462,10 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         const int* stage = reinterpret_cast<const int*>(a1 + Net::A1_BYTES + Net::COL_BYTES);
         auto prefetch = [&](int y, int x0) {
           const int xc = min(x0 + r, p.W - 1);
-  #pragma unroll
+#pragma unroll
           for (int c = 0; c < C; ++c)
             cp_async4(stage_s + (c * kTile + r) * 4, lat + c * plane + static_cast<long long>(y) * p.W + xc);
-  #pragma unroll
+#pragma unroll
           for (int j = 0; j < J; ++j) {
             const int l = it_l[j];
             if (l > 0) {
@@ -485,7 +485,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         auto features = [&](int y, int x0) -> bool {
           cp_async_wait_all();  // this thread's staged loads have landed
           // vertical pass into the column buffer
-  #pragma unroll
+#pragma unroll
           for (int j = 0; j < J; ++j) {
             const int l = it_l[j];
             if (l > 0) {
@@ -501,9 +501,9 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           // horizontal pass + level 0
           const int xc = min(x0 + r, p.W - 1);
           float f[D0];
-  #pragma unroll
+#pragma unroll
           for (int c = 0; c < C; ++c) f[c] = step[0] * lat_value<FL>(stage[c * kTile + r]);
-  #pragma unroll
+#pragma unroll
           for (int l = 1; l < L; ++l) {
             int i0, i1;
             float a;
@@ -519,7 +519,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
               i1 = min(max(tx.i1 - u_start, 0), ncol(l) - 1);
               a = tx.frac;
             }
-  #pragma unroll
+#pragma unroll
             for (int c = 0; c < C; ++c) {
               const float* cb = colbuf + CL::off(l, c);
               const float v0 = cb[i0], v1 = cb[i1];
@@ -528,12 +528,12 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           }
           // hi/lo split, the constant-1 bias column, padding -> A1
           float v[K1];
-  #pragma unroll
+#pragma unroll
           for (int j = 0; j < K1; ++j) v[j] = 0.0f;
-  #pragma unroll
+#pragma unroll
           for (int j = 0; j < D0; ++j) split_hi_lo(f[j], v[j], v[D0 + j]);
           v[2 * D0] = 1.0f;
-  #pragma unroll
+#pragma unroll
           for (int kc = 0; kc < K1 / 8; ++kc)
             sts128(a1_s + kmaj(r, kc * 8, K1), pack_f16x2(v[kc * 8 + 0], v[kc * 8 + 1]),
                    pack_f16x2(v[kc * 8 + 2], v[kc * 8 + 3]), pack_f16x2(v[kc * 8 + 4], v[kc * 8 + 5]),
@@ -670,15 +670,15 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             if (elect_one()) {
               tc_fence_after();
               if (k == 0) {
-  #pragma unroll
+#pragma unroll
                 for (int s = 0; s < K1 / 16; ++s) mma_f16(d, dA1 + s * kStep, dB1 + s * kStep, id_hidden, s > 0);
               } else {
                 const bool out_layer = (k == NL - 1);
                 const uint64_t db = out_layer ? dBO : dBH + (k - 1) * kLayer;
                 const uint32_t id = out_layer ? id_out : id_hidden;
-  #pragma unroll
+#pragma unroll
                 for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + 8 * s, db + s * kStep, id, s > 0);  // hi
-  #pragma unroll
+#pragma unroll
                 for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
                 mma_f16(d, dONES, db + (N / 16) * kStep, id, 1);  // bias: [1 0..0] x [b 0..0]
               }
