@@ -3,21 +3,19 @@
 //
 // Algorithm 1 expands each block from its end-of-block marker offsets, which
 // the paper finds beforehand by a stream compaction.  Here:
-// 1. izpr_count: eob markers per 4096-symbol chunk (coalesced reads).
+// 1. izpr_count: eob markers per 2048-symbol chunk (coalesced reads).
 // 2. izpr_scan: one CTA, exclusive scan of the chunk counts = index of each
 //    chunk's first block; the marker total.
 // 3. izpr_expand: persistent CTAs do the compaction and the expansion
-//    together, chunk by chunk.  A CTA stages a chunk and the 96 symbols
-//    before it in shared memory by cp.async while it works on its previous
+//    together, chunk by chunk.  Each thread holds 16 consecutive symbols of
+//    the chunk in registers (loaded while the CTA expanded its previous
+//    chunk), stores them to shared memory with the 96 symbols before the
 //    chunk (a block has at most 64 symbols before its marker, so the marker
-//    ending the previous block is in that halo), ranks the chunk's markers
-//    with warp ballots (their stream indices are Algorithm 1's offsets), and
-//    expands the blocks 8 lanes per block: lane k owns symbols 8k..8k+7 of
-//    the block and counts the zigzag positions they cover (1 for a literal,
-//    n for the run code of n zeros), a scan over the 8 lanes turns the
-//    counts into positions, literals are scattered into a zeroed 64-entry
-//    block in shared memory through the zigzag table, and the block leaves
-//    as 256 contiguous bytes (two 16-byte stores per lane).
+//    ending the previous block is in that halo) and counts its markers; a
+//    CTA scan ranks them (their stream indices are Algorithm 1's offsets),
+//    and, as in Algorithm 1, one thread expands one block: literals go to
+//    the next zigzag position, a run code of n zeros skips n positions.  The
+//    blocks of a warp leave as whole 256-byte blocks in raster order.
 // The stream is read twice (steps 1 and 3); nothing else touches HBM but
 // the coefficients and offsets written.
 #include <cstdint>
@@ -30,7 +28,7 @@
 namespace pic {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 128;
 constexpr int kPerThread = 16;
 constexpr int kChunk = kThreads * kPerThread;  // symbols per compaction chunk
 
@@ -77,7 +75,6 @@ constexpr ZigzagTable make_zigzag() {
   }
   return t;
 }
-__constant__ ZigzagTable kZigzag = make_zigzag();
 
 // Exclusive scan of one int per thread over a 256-thread CTA; returns the
 // thread's prefix and writes the CTA total to *total.
@@ -107,232 +104,319 @@ __device__ int cta_exclusive_scan(int v, int* smem, int* total) {
   return before + x - v;
 }
 
+// 16 consecutive symbols from stream index i0 into r; positions past the
+// end read as `fill`.  16-byte loads when the stream is 16-byte aligned.
+__device__ __forceinline__ void load16(const int32_t* __restrict__ sym, long long n, long long i0,
+                                       bool vec, int fill, int (&r)[16]) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const long long i = i0 + 4 * q;
+    if (vec && i + 3 < n) {
+      const int4 v = __ldg(reinterpret_cast<const int4*>(sym + i));
+      r[4 * q] = v.x;
+      r[4 * q + 1] = v.y;
+      r[4 * q + 2] = v.z;
+      r[4 * q + 3] = v.w;
+    } else {
+#pragma unroll
+      for (int u = 0; u < 4; ++u) r[4 * q + u] = i + u < n ? __ldg(sym + i + u) : fill;
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kThreads) izpr_count(const int32_t* __restrict__ sym,
                                                        long long n, int32_t eob, int* counts) {
   __shared__ int smem[64];
-  const long long base = static_cast<long long>(blockIdx.x) * kChunk;
+  const long long i0 = static_cast<long long>(blockIdx.x) * kChunk + 16 * threadIdx.x;
+  int r[16];
+  load16(sym, n, i0, (reinterpret_cast<uintptr_t>(sym) & 15u) == 0, eob, r);
   int c = 0;
 #pragma unroll
-  for (int k = 0; k < kPerThread; ++k) {  // coalesced: thread t reads base + t + 256 k
-    const long long i = base + threadIdx.x + static_cast<long long>(kThreads) * k;
-    if (i < n && __ldg(sym + i) == eob) ++c;
-  }
+  for (int k = 0; k < 16; ++k) c += (r[k] == eob && i0 + k < n) ? 1 : 0;
   int total;
   cta_exclusive_scan(c, smem, &total);
   if (threadIdx.x == 0) counts[blockIdx.x] = total;
 }
 
 // One CTA: exclusive scan of the chunk counts into chunk bases; the total.
-__global__ void __launch_bounds__(1024) izpr_scan(const int* counts, long long n_chunks,
+// Tiles of 8192 counts are staged in shared memory by coalesced loads
+// (padded: entry j at j + j / 32); thread t scans entries 8t .. 8t+7.
+__global__ void __launch_bounds__(1024) izpr_scan(const int* __restrict__ counts, long long n_chunks,
                                                   long long* base, long long* total) {
-  __shared__ long long part[1024];
-  const long long per = (n_chunks + 1023) / 1024;
-  const long long lo = threadIdx.x * per, hi = lo + per < n_chunks ? lo + per : n_chunks;
-  long long s = 0;
-  for (long long j = lo; j < hi; ++j) s += counts[j];
-  part[threadIdx.x] = s;
-  __syncthreads();
-  for (int o = 1; o < 1024; o <<= 1) {  // Hillis-Steele inclusive scan of the parts
-    const long long y = threadIdx.x >= o ? part[threadIdx.x - o] : 0;
+  constexpr int kPer = 8, kTileN = 1024 * kPer;
+  __shared__ int s_c[kTileN + kTileN / 32];
+  __shared__ long long s_w[32];
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  long long carry = 0;
+  for (long long t0 = 0; t0 < n_chunks; t0 += kTileN) {
+    const long long m = min(static_cast<long long>(kTileN), n_chunks - t0);
+    int v[kPer];  // all loads in flight together, then the shared stores
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int j = t + 1024 * k;
+      v[k] = j < m ? __ldg(counts + t0 + j) : 0;
+    }
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int j = t + 1024 * k;
+      s_c[j + (j >> 5)] = v[k];
+    }
     __syncthreads();
-    part[threadIdx.x] += y;
+    long long s = 0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int j = kPer * t + k;
+      s += s_c[j + (j >> 5)];
+    }
+    long long x = s;  // inclusive scan: warp, then warp totals
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) s_w[warp] = x;
     __syncthreads();
+    if (warp == 0) {
+      long long w = s_w[lane];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const long long y = __shfl_up_sync(0xffffffffu, w, o);
+        if (lane >= o) w += y;
+      }
+      s_w[lane] = w;
+    }
+    __syncthreads();
+    long long run = carry + (warp > 0 ? s_w[warp - 1] : 0) + x - s;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int j = kPer * t + k;
+      if (j < m) base[t0 + j] = run;
+      run += s_c[j + (j >> 5)];
+    }
+    carry += s_w[31];
+    __syncthreads();  // s_c and s_w are free again
   }
-  long long run = part[threadIdx.x] - s;
-  for (long long j = lo; j < hi; ++j) {
-    base[j] = run;
-    run += counts[j];
-  }
-  if (threadIdx.x == 1023) *total = part[1023];
+  if (t == 0) *total = carry;
 }
 
-// Compaction and expansion in one pass over the stream.  A block holds at
-// most 64 symbols before its marker, so the marker that precedes a chunk's
-// first block lies within the kHalo symbols before the chunk (or the block
-// is malformed).  Persistent CTAs take chunks c, c + grid, ...; each stages
-// the halo and the chunk in shared memory by cp.async one chunk ahead
-// (double buffer), finds the chunk's markers in stream order (block
-// q = base[chunk] + rank), writes their offsets, and expands the chunk's
-// blocks straight from shared memory.
-constexpr int kHalo = 96;
-constexpr int kStageInts = kHalo + kChunk;
-// Staged symbol j sits at word j + j / 32: the lanes of a block, which read
-// symbols 8 apart, then fall in distinct banks.
-constexpr int kStagePadded = kStageInts + kStageInts / 32 + 1;
-__device__ __forceinline__ int pad(int j) { return j + (j >> 5); }
-constexpr int kExpandSmem = 2 * kStagePadded * 4          // symbols, double buffer
-                            + kChunk * 2                  // marker positions (u16)
-                            + 4 * (kThreads / 32) * 64 * 4  // one 64-entry block per octet
-                            + 64 * 4 + 64 + 16;           // scan scratch, zigzag table, halo marker
+// Compaction and expansion in one pass over the stream, as a segmented scan.
+// A block holds at most 64 symbols before its marker, so the marker that
+// precedes a chunk's first block lies within the kHalo symbols before the
+// chunk (or the block is malformed).  Persistent CTAs take chunks c,
+// c + grid, ...; for each:
+//  - every thread holds 16 consecutive symbols of the chunk in registers
+//    (loaded while the CTA worked on its previous chunk) and reduces them to
+//    (markers, positions covered since its last marker);
+//  - warp 0 finds the halo's last marker and the positions of the part of
+//    the chunk's first block that lies in the halo (they carry in);
+//  - a CTA-wide segmented scan of the (markers, positions) pairs gives each
+//    thread the block of its first symbol (block q of the chunk = block
+//    base[chunk] + q of the stream) and the zigzag position reached in it;
+//  - each thread walks its symbols: a literal goes to the block's next
+//    zigzag position, a run code of n zeros skips n positions, a marker
+//    closes the block (its stream index is Algorithm 1's offset);
+//  - the blocks, assembled in shared memory, leave as whole 256-byte blocks
+//    in raster order.
+// Symbols after the chunk's last marker belong to the next chunk's first
+// block; here they land in a spare block slot that is cleared, not written
+// out.  A chunk with more than kMaxBlk blocks (only possible with very short
+// blocks) is expanded in several passes over its block range.
+constexpr int kHalo = 96;                   // 3 symbols per lane of warp 0
+constexpr int kMaxBlk = 96;                 // blocks assembled per pass
+constexpr int kBlkStride = 68;              // words per block slot: equal raster
+                                            // entries of neighbouring blocks
+                                            // fall 4 banks apart
+constexpr int kExpandSmem = (kMaxBlk + 1) * kBlkStride * 4  // block slots + spare
+                            + 64 * 4                        // scan scratch
+                            + 64 + 16;                      // zigzag table, halo carry
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src) {
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_prev() {  // all but the newest group have landed
-  asm volatile("cp.async.wait_group 1;" ::: "memory");
-}
+// Segmented-scan combine: (m1, s1) then (m2, s2) -> markers m1 + m2, and
+// the positions covered since the last marker.
+struct Seg {
+  int m, s;
+};
+__device__ __forceinline__ Seg seg_cat(Seg a, Seg b) { return Seg{a.m + b.m, b.m > 0 ? b.s : a.s + b.s}; }
 
-__global__ void __launch_bounds__(kThreads, 4) izpr_expand(const int32_t* __restrict__ sym,
+__global__ void __launch_bounds__(kThreads, 6) izpr_expand(const int32_t* __restrict__ sym,
                                                         long long n, int32_t eob,
                                                         const long long* __restrict__ base,
                                                         const long long* total, long long n_blocks,
                                                         int32_t* __restrict__ coeffs,
                                                         int64_t* __restrict__ offsets, int* status) {
   extern __shared__ __align__(16) unsigned char smem[];
-  int* s_sym0 = reinterpret_cast<int*>(smem);
-  unsigned short* s_mk = reinterpret_cast<unsigned short*>(smem + 2 * kStagePadded * 4);
-  int(*s_blk)[64] = reinterpret_cast<int(*)[64]>(smem + 2 * kStagePadded * 4 + kChunk * 2);
-  int* s_scan = reinterpret_cast<int*>(smem + 2 * kStagePadded * 4 + kChunk * 2 +
-                                       4 * (kThreads / 32) * 64 * 4);
-  unsigned char* s_zz = reinterpret_cast<unsigned char*>(s_scan + 64);  // zigzag table
-  int* s_prev = reinterpret_cast<int*>(s_zz + 64);
+  int* s_buf = reinterpret_cast<int*>(smem);
+  int* s_scan = s_buf + (kMaxBlk + 1) * kBlkStride;
+  unsigned char* s_zz = reinterpret_cast<unsigned char*>(s_scan + 64);
+  int* s_carry = reinterpret_cast<int*>(s_zz + 64);
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  constexpr int kWarps = kThreads / 32;
   const long long n_chunks = (n + kChunk - 1) / kChunk;
-  if (t < 64) s_zz[t] = static_cast<unsigned char>(kZigzag.v[t]);
+  if (t < 64) s_zz[t] = static_cast<unsigned char>(make_zigzag().v[t]);
   if (blockIdx.x == 0 && t == 0) {
     if (*total != n_blocks) atomicOr(status, kBadCount);
     if (__ldg(sym + n - 1) != eob) atomicOr(status, kBadCount);  // symbols after the last marker
   }
+  for (int j = t; j < (kMaxBlk + 1) * kBlkStride / 4; j += kThreads)
+    reinterpret_cast<int4*>(s_buf)[j] = make_int4(0, 0, 0, 0);
+  const bool vec = (reinterpret_cast<uintptr_t>(sym) & 15u) == 0;
+  const uint32_t ueob16 = static_cast<uint32_t>(eob) - 16u;  // first run code
+  // Past the end of the stream the symbols read as a literal (eob - 17):
+  // never a marker, and only ever in the spare slot.
+  const int fill = static_cast<int>(static_cast<uint32_t>(eob) - 17u);
 
-  // stage chunk c into buffer dst: positions before the stream act as
-  // markers (the first block starts at 0); positions past its end hold 0
-  // and are never counted
-  auto stage = [&](long long c, int* dst) {
-    const long long c0 = c * kChunk;
-    const uint32_t d = smem_u32(dst);
-    for (int j = t; j < kStageInts; j += kThreads) {
-      const long long i = c0 - kHalo + j;
-      if (i >= 0 && i < n) cp_async4(d + 4 * pad(j), sym + i);
-      else dst[pad(j)] = i < 0 ? eob : 0;
-    }
+  // The halo of chunk c for warp 0 (lane l: symbols c0 - kHalo + 3 l .. + 2);
+  // before the stream they act as markers.
+  auto load_halo = [&](long long c, int (&h)[3]) {
+    const long long hi = c * kChunk - kHalo + 3 * lane;
+#pragma unroll
+    for (int u = 0; u < 3; ++u) h[u] = (warp != 0 || hi + u < 0) ? eob : __ldg(sym + hi + u);
   };
 
-  int buf = 0;
-  if (blockIdx.x < n_chunks) stage(blockIdx.x, s_sym0);
-  cp_async_commit();
-  for (long long c = blockIdx.x; c < n_chunks; c += gridDim.x, buf ^= 1) {
-    int* s_sym = s_sym0 + buf * kStagePadded;
-    if (c + gridDim.x < n_chunks) stage(c + gridDim.x, s_sym0 + (buf ^ 1) * kStagePadded);
-    cp_async_commit();
-    cp_async_wait_prev();
-    __syncthreads();  // chunk c is in s_sym
-    const long long c0 = c * kChunk;  // stream index of s_sym[kHalo]
+  // the next chunk's symbols, halo and first block index, loaded one chunk ahead
+  int cur[16], hcur[3];
+  long long bcur = 0;
+  if (blockIdx.x < n_chunks) {
+    load16(sym, n, static_cast<long long>(blockIdx.x) * kChunk + 16 * t, vec, fill, cur);
+    load_halo(blockIdx.x, hcur);
+    bcur = base[blockIdx.x];
+  }
+  for (long long c = blockIdx.x; c < n_chunks; c += gridDim.x) {
+    const long long c0 = c * kChunk;
+    const long long gb0 = bcur;
+    int x16[16], h[3];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) x16[i] = cur[i];
+#pragma unroll
+    for (int u = 0; u < 3; ++u) h[u] = hcur[u];
+    if (c + gridDim.x < n_chunks) {  // next chunk, in flight meanwhile
+      load16(sym, n, (c + gridDim.x) * kChunk + 16 * t, vec, fill, cur);
+      load_halo(c + gridDim.x, hcur);
+      bcur = base[c + gridDim.x];
+    }
 
-    // markers of the chunk in stream order: warp w scans symbols
-    // kHalo + 512 w .. + 511 in 16 steps of 32 (one per lane, conflict-free),
-    // ballots give each marker its rank
-    constexpr int kSpan = kChunk / (kThreads / 32);
-    unsigned mk_mask[kSpan / 32];
-    int wcount = 0;
+    // this thread's markers (bit i: symbol i) and positions since its last one
+    unsigned mk = 0;
+    int s = 0, vmax = x16[0];
 #pragma unroll
-    for (int st = 0; st < kSpan / 32; ++st) {
-      const int j = kHalo + kSpan * warp + 32 * st + lane;
-      mk_mask[st] = __ballot_sync(0xffffffffu, c0 + (j - kHalo) < n && s_sym[pad(j)] == eob);
-      wcount += __popc(mk_mask[st]);
+    for (int i = 0; i < 16; ++i) {
+      const int x = x16[i];
+      const uint32_t d = static_cast<uint32_t>(x) - ueob16;
+      const bool m = x == eob;
+      mk |= m ? 1u << i : 0u;
+      s = m ? 0 : s + (d < 16u ? static_cast<int>(d) + 1 : 1);
+      vmax = max(vmax, x);
     }
-    if (lane == 0) s_scan[warp] = wcount;
-    __syncthreads();
-    int run = 0, tot = 0;
+    bool bad = vmax > eob;
+    // warp-inclusive segmented scan
+    Seg inc{__popc(mk), s};
 #pragma unroll
-    for (int w2 = 0; w2 < kThreads / 32; ++w2) {
-      const int v = s_scan[w2];
-      run += w2 < warp ? v : 0;
-      tot += v;
+    for (int o = 1; o < 32; o <<= 1) {
+      const Seg y{__shfl_up_sync(0xffffffffu, inc.m, o), __shfl_up_sync(0xffffffffu, inc.s, o)};
+      if (lane >= o) inc = seg_cat(y, inc);
     }
-    const unsigned lt = (1u << lane) - 1u;
-#pragma unroll
-    for (int st = 0; st < kSpan / 32; ++st) {
-      const unsigned m = mk_mask[st];
-      if ((m >> lane) & 1u)
-        s_mk[run + __popc(m & lt)] = static_cast<unsigned short>(kHalo + kSpan * warp + 32 * st + lane);
-      run += __popc(m);
+    if (lane == 31) {
+      s_scan[2 * warp] = inc.m;
+      s_scan[2 * warp + 1] = inc.s;
     }
-    if (warp == 0) {  // the last marker of the halo, if any
+    // the halo (warp 0): its last marker, and the positions of the part of
+    // the chunk's first block that lies in it
+    int halo_pos = 0;
+    if (warp == 0) {
       int last = -1;
 #pragma unroll
-      for (int h = 0; h < kHalo / 32; ++h) {
-        const unsigned m = __ballot_sync(0xffffffffu, s_sym[pad(32 * h + lane)] == eob);
-        if (m) last = 32 * h + 31 - __clz(static_cast<int>(m));
+      for (int u = 0; u < 3; ++u)
+        if (h[u] == eob) last = 3 * lane + u;
+      last = __reduce_max_sync(0xffffffffu, last);
+      int sum = 0;
+#pragma unroll
+      for (int u = 0; u < 3; ++u) {
+        if (3 * lane + u <= last || last < 0) h[u] = eob;  // not part of the first block
+        const uint32_t d = static_cast<uint32_t>(h[u]) - ueob16;
+        sum += h[u] == eob ? 0 : (d < 16u ? static_cast<int>(d) + 1 : 1);
       }
-      if (lane == 0) *s_prev = last;
+      int x = sum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+      }
+      halo_pos = x - sum;  // zigzag position of this lane's first halo symbol
+      // a block with no marker in the halo has more than 64 symbols
+      if (lane == 31) *s_carry = last < 0 ? 65 : x;
     }
-    __syncthreads();
+    __syncthreads();  // warp totals and the halo carry
 
-    // expansion: 8 lanes per block (an "octet", 4 blocks per warp at a time);
-    // lane k of an octet owns symbols 8k .. 8k+7 of its block (a block has at
-    // most 64), counts the zigzag positions they cover, and after an
-    // exclusive scan over the octet scatters its literals.
-    const long long gb0 = base[c];
-    const int oct = lane >> 3, k = lane & 7;
-    const unsigned omask = 0xffu << (8 * oct);
-    int* blk = s_blk[4 * warp + oct];
-    for (int q0 = 4 * warp; q0 < tot; q0 += 4 * (kThreads / 32)) {  // warp-uniform trip count
-      const int q = q0 + oct;
-      const bool has = q < tot;
-      int start = 0, end = 0, len = 0;
-      bool bad = false;
-      if (has) {
-        end = s_mk[q];
-        const int prev = q == 0 ? *s_prev : s_mk[q - 1];
-        start = prev + 1;
-        len = end - start;
-        bad = prev < 0 || len > 64;
-      }
-      reinterpret_cast<int4*>(blk)[2 * k] = make_int4(0, 0, 0, 0);
-      reinterpret_cast<int4*>(blk)[2 * k + 1] = make_int4(0, 0, 0, 0);
-      int sv[8], cnt[8], sum = 0;
-      unsigned lit = 0;
+    // exclusive prefix of this thread: (block of its first symbol, position)
+    Seg pre{0, *s_carry};
+    int tot = 0;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int e = 8 * k + i;
-        sv[i] = 0;
-        cnt[i] = 0;
-        if (has && !bad && e < len) {
-          sv[i] = s_sym[pad(start + e)];
-          const bool run = sv[i] >= eob - 16 && sv[i] < eob;
-          cnt[i] = run ? sv[i] - (eob - 17) : 1;  // run of n zeros, or a literal
-          if (!run) lit |= 1u << i;
-          if (sv[i] > eob) bad = true;
-        }
-        sum += cnt[i];
-      }
-      int x = sum;  // inclusive scan over the octet
-#pragma unroll
-      for (int o = 1; o < 8; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, x, o, 8);
-        if (k >= o) x += y;
-      }
-      const int covered = __shfl_sync(0xffffffffu, x, 7, 8);
-      bad = (__ballot_sync(0xffffffffu, bad || covered > 64) & omask) != 0;
-      __syncwarp();  // the zeroed buffer is complete
-      if (!bad) {
-        int pos = x - sum;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          if (lit & (1u << i)) blk[s_zz[pos]] = sv[i];
-          pos += cnt[i];
-        }
-      }
-      __syncwarp();
-      if (has) {
-        if (bad && k == 0) atomicOr(status, kBadBlock);
-        const long long gb = gb0 + q;
-        if (gb < n_blocks) {
-          int4* dst = reinterpret_cast<int4*>(coeffs + gb * 64);
-          dst[2 * k] = reinterpret_cast<const int4*>(blk)[2 * k];
-          dst[2 * k + 1] = reinterpret_cast<const int4*>(blk)[2 * k + 1];
-          if (k == 0) offsets[gb] = c0 - kHalo + end;
-        } else if (k == 0) {
-          atomicOr(status, kBadCount);
-        }
-      }
-      __syncwarp();
+    for (int w2 = 0; w2 < kWarps; ++w2) {
+      const Seg v{s_scan[2 * w2], s_scan[2 * w2 + 1]};
+      if (w2 < warp) pre = seg_cat(pre, v);
+      tot += v.m;  // blocks of this chunk
     }
-    __syncthreads();  // s_mk, the octet buffers and this symbol buffer are free again
+    {
+      const Seg y{__shfl_up_sync(0xffffffffu, inc.m, 1), __shfl_up_sync(0xffffffffu, inc.s, 1)};
+      if (lane > 0) pre = seg_cat(pre, y);
+    }
+    // offsets (Algorithm 1): the stream index of each marker
+    {
+      int q = pre.m;
+      for (unsigned b = mk; b; b &= b - 1u, ++q) {
+        const long long gb = gb0 + q;
+        if (gb < n_blocks) offsets[gb] = c0 + 16 * t + (__ffs(b) - 1);
+        else atomicOr(status, kBadCount);
+      }
+    }
+
+    // expansion, kMaxBlk blocks of the chunk per pass; in a pass the blocks
+    // outside it (and the next chunk's first block) go to the spare slot
+    for (int p0 = 0; p0 < tot; p0 += kMaxBlk) {
+      const int p1 = min(tot, p0 + kMaxBlk);
+      const bool one_pass = tot <= kMaxBlk;  // then q - p0 never leaves [0, kMaxBlk]
+      if (p0 == 0 && warp == 0) {  // the first block's literals from the halo
+#pragma unroll
+        for (int u = 0; u < 3; ++u) {
+          const uint32_t d = static_cast<uint32_t>(h[u]) - ueob16;
+          if (h[u] != eob && d > 16u && halo_pos < 64) s_buf[s_zz[halo_pos]] = h[u];
+          halo_pos += h[u] == eob ? 0 : (d < 16u ? static_cast<int>(d) + 1 : 1);
+        }
+      }
+      int q = pre.m, pos = pre.s;
+      auto slot = [&](int qq) {
+        return one_pass ? qq * kBlkStride : ((qq >= p0 && qq < p1) ? qq - p0 : kMaxBlk) * kBlkStride;
+      };
+      int qb = slot(q);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int x = x16[i];
+        const uint32_t d = static_cast<uint32_t>(x) - ueob16;  // < 16: run code, 16: marker
+        const int zz = s_zz[pos & 63];
+        if (d > 16u) s_buf[qb + zz] = x;  // a literal (or a malformed value)
+        if (d == 16u) {
+          if (pos > 64) bad = true;
+          ++q;
+          pos = 0;
+          qb = slot(q);
+        } else {
+          pos += d < 16u ? static_cast<int>(d) + 1 : 1;
+        }
+      }
+      __syncthreads();  // the pass's blocks are assembled
+      // copy-out: two blocks per warp instruction, 16 bytes per lane; every
+      // slot used (the spare one too) is cleared for the next pass
+      const int last_slot = one_pass ? p1 - p0 : kMaxBlk;
+      for (int b = 2 * warp + (lane >> 4); b <= last_slot; b += 2 * kWarps) {
+        int4* src = reinterpret_cast<int4*>(s_buf + b * kBlkStride) + (lane & 15);
+        const int4 v = *src;
+        *src = make_int4(0, 0, 0, 0);
+        const long long gb = gb0 + p0 + b;
+        if (b < p1 - p0 && gb < n_blocks) reinterpret_cast<int4*>(coeffs + gb * 64)[lane & 15] = v;
+      }
+      __syncthreads();  // the slots are clear again
+    }
+    if (bad) atomicOr(status, kBadBlock);
+    __syncthreads();  // the scan scratch and the halo carry are free again
   }
 }
 

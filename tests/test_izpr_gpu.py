@@ -63,6 +63,33 @@ def test_edge_blocks(orc):
     _roundtrip(orc, b, eob=1000)             # any eob above the literals + 16
 
 
+def test_unaligned_stream(orc):
+    """Symbols starting 4 bytes past a 16-byte boundary (the scalar load path)."""
+    import torch
+    from paper_2609_09020_gb300 import pic
+    blocks = wk.dct_blocks(3000, 21)
+    eob = int(np.abs(blocks).max()) + 17
+    s = orc.zpr_encode(blocks, eob)
+    padded = torch.from_numpy(np.r_[np.int32(0), s].astype(np.int32)).to("cuda:0")
+    c, o = pic.izpr_decode(padded[1:], eob, blocks.shape[0])
+    assert padded[1:].data_ptr() % 16 != 0
+    assert np.array_equal(c.cpu().numpy(), blocks)
+    assert np.array_equal(o.cpu().numpy(), np.nonzero(s == eob)[0])
+
+
+def test_all_zero_blocks(orc):
+    """Every block empty: one marker per symbol, so every chunk holds as many
+    blocks as symbols (many expansion passes per chunk)."""
+    _roundtrip(orc, np.zeros((10000, 64), np.int32))
+
+
+def test_eob_zero(orc):
+    """eob = 0: the zeros past the end of the stream must not count as markers."""
+    rng = np.random.Generator(np.random.PCG64(9))
+    b = np.where(rng.random((777, 64)) < 0.3, rng.integers(-300, -17, (777, 64)), 0).astype(np.int32)
+    _roundtrip(orc, b, eob=0)
+
+
 def test_empty_stream():
     c, o = _gpu(np.zeros(0, np.int32), 40, 0)
     assert c.shape == (0, 64) and o.shape == (0,)
