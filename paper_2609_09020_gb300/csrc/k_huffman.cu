@@ -23,7 +23,10 @@
 //    d. every subsequence is decoded from its final start, writing values.
 // Each thread keeps a 64-bit window of the stream in registers and reloads
 // one word when its position crosses a word boundary (codes are at most 12
-// bits, so at most one word per codeword).
+// bits, so at most one word per codeword).  The counting decodes of a and b
+// use a pair table per image (the lengths of the first two codewords of
+// every p-bit window, when both lie inside it), so one lookup advances over
+// up to two codewords.
 #include <cstdint>
 
 #include <cooperative_groups.h>
@@ -185,34 +188,38 @@ __device__ __forceinline__ int32_t value_of(uint32_t e) {
   return static_cast<int32_t>(e << 8) >> 8;  // sign-extend the 24-bit value
 }
 
-// Decodes codewords from bit `lpos` of the words staged in shared memory
-// (bit 0 = the top bit of sw[0]) while lpos < lke; returns the position
-// after the last codeword.  WRITE: stores the values into out (at most lim).
-// *bad is raised on a bit pattern that is no codeword.  The next p bits come
-// from one funnel shift of the two current words.
-template <bool WRITE>
-__device__ __forceinline__ int decode_span_s(const uint32_t* sw, int lpos, int lke, const uint32_t* lut,
-                                             int p, int* count, int32_t* out, long long lim, bool* bad) {
+// The counting loop of decode_span_s, with (PAIR) or without the pair table.
+template <bool PAIR>
+__device__ __forceinline__ int decode_span_loop(const uint32_t* sw, int lpos, int lke, const uint32_t* lut,
+                                                const uint8_t* lut2, int p, int* count, bool* bad) {
   int c = 0;
-  if (lpos < lke) {
-    int li = lpos >> 5;
-    uint32_t hi = sw[li], lo = sw[li + 1];
-    const int shr = 32 - p;
-    while (lpos < lke) {
-      const int wi = lpos >> 5;
-      if (wi != li) {  // crossed into the next word (codes are shorter than 32 bits)
-        li = wi;
-        hi = lo;
-        lo = sw[li + 1];
+  int li = lpos >> 5;
+  uint32_t hi = sw[li], lo = sw[li + 1];
+  const int shr = 32 - p;
+  while (lpos < lke) {
+    const int wi = lpos >> 5;
+    if (wi != li) {  // crossed into the next word (a step covers at most p <= 12 bits)
+      li = wi;
+      hi = lo;
+      lo = sw[li + 1];
+    }
+    const uint32_t w = __funnelshift_l(lo, hi, lpos & 31) >> shr;
+    if constexpr (PAIR) {
+      const uint32_t e2 = lut2[w];
+      int l1 = static_cast<int>(e2 & 15u);
+      const int l2 = static_cast<int>(e2 >> 4);
+      if (l1 == 0) {
+        *bad = true;
+        l1 = 1;
       }
-      const uint32_t e = lut[__funnelshift_l(lo, hi, lpos & 31) >> shr];
-      int len = static_cast<int>(e >> 24);
+      const bool two = l2 != 0 && lpos + l1 < lke;
+      c += two ? 2 : 1;
+      lpos += two ? l1 + l2 : l1;
+    } else {
+      int len = static_cast<int>(lut[w] >> 24);
       if (len == 0) {
         *bad = true;
         len = 1;
-      }
-      if constexpr (WRITE) {
-        if (c < lim) out[c] = value_of(e);
       }
       ++c;
       lpos += len;
@@ -222,19 +229,35 @@ __device__ __forceinline__ int decode_span_s(const uint32_t* sw, int lpos, int l
   return lpos;
 }
 
+// Counts the codewords from bit `lpos` of the words staged in shared memory
+// (bit 0 = the top bit of sw[0]) while lpos < lke; returns the position
+// after the last codeword.  *bad is raised on a bit pattern that is no
+// codeword.  The next p bits come from one funnel shift of the two current
+// words.  With a pair table (lut2: the lengths of the first codeword of each
+// p-bit window and of the second one when it lies inside the same window),
+// one lookup advances over up to two codewords.
+__device__ __forceinline__ int decode_span_s(const uint32_t* sw, int lpos, int lke, const uint32_t* lut,
+                                             const uint8_t* lut2, int p, int* count, bool* bad) {
+  if (lpos >= lke) {
+    *count = 0;
+    return lpos;
+  }
+  return lut2 ? decode_span_loop<true>(sw, lpos, lke, lut, lut2, p, count, bad)
+              : decode_span_loop<false>(sw, lpos, lke, lut, lut2, p, count, bad);
+}
+
 // decode_span_s for subsequence positions of image b: pos (bits from the
 // image's first word wbase) <-> staged position (bits from word w0).
-template <bool WRITE>
 __device__ __forceinline__ long long decode_at(const uint32_t* sw, long long w0, long long wbase, long long pos,
-                                               long long ke, const uint32_t* lut, int p, int* count,
-                                               int32_t* out, long long lim, bool* bad) {
+                                               long long ke, const uint32_t* lut, const uint8_t* lut2, int p,
+                                               int* count, bool* bad) {
   if (pos >= ke) {
     *count = 0;
     return pos;
   }
   const long long shift = (wbase - w0) * 32;  // staged bit = image bit + shift (>= 0 here)
-  const int lp = decode_span_s<WRITE>(sw, static_cast<int>(pos + shift), static_cast<int>(ke + shift), lut,
-                                      p, count, out, lim, bad);
+  const int lp = decode_span_s(sw, static_cast<int>(pos + shift), static_cast<int>(ke + shift), lut, lut2, p,
+                               count, bad);
   return lp - shift;
 }
 
@@ -278,6 +301,24 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
   // so that no global load sits inside a decode chain
   uint32_t* s_words = s_lut + 2 * tsize;
   int* s_stage = reinterpret_cast<int*>(s_words + kWbuf);
+  // the pair tables of the two images: first codeword's length | the
+  // second's << 4 (0 when it does not lie inside the same p-bit window)
+  uint8_t* s_lut2 = reinterpret_cast<uint8_t*>(s_stage + kStageInts);
+  for (int i = threadIdx.x; i < 2 * tsize; i += blockDim.x) {
+    const uint32_t* L = s_lut + (i >= tsize ? tsize : 0);
+    const int w = i & (tsize - 1);
+    const int l1 = static_cast<int>(L[w] >> 24);
+    int l2 = 0;
+    if (l1 > 0 && l1 < P.p) {
+      const int l = static_cast<int>(L[(w << l1) & (tsize - 1)] >> 24);
+      if (l > 0 && l <= P.p - l1) l2 = l;
+    }
+    s_lut2[i] = static_cast<uint8_t>(l1 | (l2 << 4));
+  }
+  __syncthreads();
+  auto lut2_of = [&](int b) -> const uint8_t* {
+    return b == b_first ? s_lut2 : (b == b_last ? s_lut2 + tsize : nullptr);
+  };
   auto stage_words = [&](long long k0) {
     const long long w0 = k0 * kQ;
     __syncthreads();
@@ -296,8 +337,7 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
     const long long ks = (k * kQ - wbase) * 32, ke = min(ks + kS, nb);
     int c = 0;
     bool junk = false;
-    const long long ex = decode_at<false>(s_words, k0 * kQ, wbase, ks, ke, lut_of(b), P.p, &c, nullptr, 0,
-                                          &junk);
+    const long long ex = decode_at(s_words, k0 * kQ, wbase, ks, ke, lut_of(b), lut2_of(b), P.p, &c, &junk);
     ws.exit0[k] = ex;
     ws.start[k] = ks;
     ws.cnt[k] = c;
@@ -330,8 +370,8 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
       if (redo) {
         int c = 0;
         bool junk = false;
-        ex_out[k] = decode_at<false>(s_words, k0 * kQ, wbase, st, min(ks + kS, nb), lut_of(b), P.p, &c,
-                                     nullptr, 0, &junk);
+        ex_out[k] = decode_at(s_words, k0 * kQ, wbase, st, min(ks + kS, nb), lut_of(b), lut2_of(b), P.p, &c,
+                              &junk);
         ws.start[k] = st;
         ws.cnt[k] = c;
         ++ch;
@@ -469,7 +509,7 @@ int decode_grid(int p, size_t smem, int* grid) {
   if (cached[dev][p] == 0) {
     int coop = 0, sms = 0, per_sm = 0;
     // the attribute is the function's, for every precision: set it to the largest
-    constexpr int kMaxSmem = (4 * 2 << PIC_HUFF_MAX_PRECISION) + (kWbuf + kStageInts) * 4;
+    constexpr int kMaxSmem = (5 * 2 << PIC_HUFF_MAX_PRECISION) + (kWbuf + kStageInts) * 4;
     if (cudaFuncSetAttribute(huff_decode, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) !=
             cudaSuccess ||
         cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess ||
@@ -507,8 +547,8 @@ int pic_huffman_decode(const uint32_t* words, int64_t n_words, const int64_t* wo
     return PIC_ERR_INVALID_ARG;
   const long long n_sub = n_words / kQ;
   if (static_cast<long long>(workspace_bytes) < ws_size(n_sub, B, p)) return PIC_ERR_INVALID_ARG;
-  // 2 tables + the pass's words + the output staging rows
-  const size_t lut_smem = (sizeof(uint32_t) * 2 << p) + (kWbuf + kStageInts) * sizeof(uint32_t);
+  // 2 tables + the pass's words + the output staging rows + 2 pair tables
+  const size_t lut_smem = (sizeof(uint32_t) * 2 << p) + (kWbuf + kStageInts) * sizeof(uint32_t) + (2 << p);
   int grid = 0;
   int rc = decode_grid(p, lut_smem, &grid);
   if (rc != PIC_OK) return rc;
