@@ -400,17 +400,24 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
   for (long long k0 = k_begin; k0 < k_end; k0 += blockDim.x) {
     const long long k = k0 + threadIdx.x;
     const long long v = k < k_end ? ws.cnt[k] : 0;
-    __syncthreads();
-    scan[threadIdx.x] = v;
-    __syncthreads();
-    for (int o = 1; o < kThreads; o <<= 1) {  // inclusive scan (Hillis-Steele)
-      const long long y = threadIdx.x >= o ? scan[threadIdx.x - o] : 0;
-      __syncthreads();
-      scan[threadIdx.x] += y;
-      __syncthreads();
+    const int ln = threadIdx.x & 31, wp = threadIdx.x >> 5;
+    long long x = v;  // inclusive scan: warp shuffles, then the warp totals
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long y = __shfl_up_sync(0xffffffffu, x, o);
+      if (ln >= o) x += y;
     }
-    if (k < k_end) ws.off[k] = carry + scan[threadIdx.x] - v;
-    carry += scan[kThreads - 1];
+    __syncthreads();  // scan[] of the previous pass has been read
+    if (ln == 31) scan[wp] = x;
+    __syncthreads();
+    long long before = 0, all = 0;
+#pragma unroll
+    for (int i = 0; i < kThreads / 32; ++i) {
+      before += i < wp ? scan[i] : 0;
+      all += scan[i];
+    }
+    if (k < k_end) ws.off[k] = carry + before + x - v;
+    carry += all;
   }
   if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0 && carry != __ldg(P.sym_off + P.B))
     atomicOr(ws.status, kBadCount);
@@ -474,14 +481,19 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
         more = lpos < lke;
       }
       __syncwarp();
+      // this thread's output run: cap values at o + done.  Lanes hold
+      // consecutive subsequences, so o + done never falls below lane 0's and
+      // exceeds it by less than 2^13 (32 subsequences of at most 256
+      // codewords): one shuffle per row carries (offset from lane 0, cap).
       const long long left = room - done;  // symbols this thread may still write
+      const int cap = static_cast<int>(min(static_cast<long long>(n), max(left, 0LL)));
+      const long long at0 = __shfl_sync(0xffffffffu, o + done, 0);
+      const unsigned packed = (static_cast<unsigned>(o + done - at0) << 5) | static_cast<unsigned>(cap);
 #pragma unroll 4
       for (int j = 0; j < 16; ++j) {
         const int src = 2 * j + (lane >> 4), i = lane & 15;
-        const int ns = __shfl_sync(0xffffffffu, n, src);
-        const long long at = __shfl_sync(0xffffffffu, o + done, src);
-        const long long lim = __shfl_sync(0xffffffffu, left, src);
-        if (i < ns && i < lim) P.out[at + i] = wbuf[src * kRow + i];
+        const unsigned pk = __shfl_sync(0xffffffffu, packed, src);
+        if (i < static_cast<int>(pk & 31u)) P.out[at0 + (pk >> 5) + i] = wbuf[src * kRow + i];
       }
       done += n;
       __syncwarp();
