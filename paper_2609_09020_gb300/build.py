@@ -2,8 +2,8 @@
 
 Each translation unit is compiled by its own nvcc process, in parallel, then
 linked into one shared library with the C ABI of include/pic_decode.h,
-include/pic_izpr.h, include/pic_idct.h, include/pic_fuse.h and
-include/pic_huffman.h.
+include/pic_izpr.h, include/pic_idct.h, include/pic_fuse.h,
+include/pic_huffman.h and include/pic_measure.h.
 """
 from __future__ import annotations
 
@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libpic_gb300.so")
 SOURCES = ["pic_decode.cu", "k_fp32.cu", "k_fp32_sweep.cu", "k_tc.cu", "k_tc_f32lat.cu", "k_tc_sweep.cu", "k_izpr.cu",
-           "k_idct.cu", "k_fuse.cu", "k_huffman.cu"]
+           "k_idct.cu", "k_fuse.cu", "k_huffman.cu", "k_peak.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

@@ -115,6 +115,10 @@ def load_library():
     lib.pic_huffman_decode.restype = i
     lib.pic_huffman_status.argtypes = [_P, _P]
     lib.pic_huffman_status.restype = i
+    lib.pic_fma_peak_flops.argtypes = [i, i]
+    lib.pic_fma_peak_flops.restype = i64
+    lib.pic_fma_peak_launch.argtypes = [_P, i, i, _P]
+    lib.pic_fma_peak_launch.restype = i
     lib.pic_status_string.argtypes = [i]
     lib.pic_status_string.restype = ctypes.c_char_p
     _lib = lib
@@ -294,6 +298,30 @@ def pic_huffman_decode(words, n_words, word_off, n_bits, B, tab_value, tab_len, 
 
 def pic_huffman_status(workspace, stream=None) -> int:
     return load_library().pic_huffman_status(workspace, stream)
+
+
+def fma_peak_tflops(device=None, iters: int = 8192, reps: int = 5) -> float:
+    """Measured FP32 FMA throughput of the device (include/pic_measure.h):
+    8 CTAs of 256 threads per SM, 3 warm-up launches, then reps launches
+    timed with CUDA events on the current stream."""
+    import torch
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    blocks = 8 * torch.cuda.get_device_properties(dev).multi_processor_count
+    out = torch.empty(blocks, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    sp = ctypes.c_void_p(stream.cuda_stream)
+    lib = load_library()
+    for _ in range(3):
+        rc = lib.pic_fma_peak_launch(out.data_ptr(), blocks, iters, sp)
+        if rc != PIC_OK:
+            raise PicError(rc, "pic_fma_peak_launch")
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        lib.pic_fma_peak_launch(out.data_ptr(), blocks, iters, sp)
+    e1.record(stream)
+    e1.synchronize()
+    return lib.pic_fma_peak_flops(blocks, iters) * reps / (e0.elapsed_time(e1) * 1e-3) / 1e12
 
 
 def huffman_decode(words, word_off, n_bits, tab_value, tab_len, p, sym_off, stream=None,

@@ -146,3 +146,12 @@ def test_huffman_workspace_and_argument_checks(lib):
     assert pic.pic_huffman_decode(None, 8, None, None, 1, None, None, 4, 12, None, None, None, 0,
                                   None) == pic.PIC_ERR_INVALID_ARG
     assert pic.pic_huffman_status(None, None) == pic.PIC_ERR_INVALID_ARG
+
+
+def test_fma_peak_helper_without_gpu(lib):
+    """The FMA microbenchmark's flop count and argument checks (include/pic_measure.h)."""
+    from paper_2609_09020_gb300 import pic
+    assert pic.load_library().pic_fma_peak_flops(0, 1) == -1
+    assert pic.load_library().pic_fma_peak_flops(1, 0) == -1
+    assert pic.load_library().pic_fma_peak_flops(2, 3) == 2 * 256 * 3 * 16 * 8 * 2
+    assert pic.load_library().pic_fma_peak_launch(None, 1, 1, None) == pic.PIC_ERR_INVALID_ARG
