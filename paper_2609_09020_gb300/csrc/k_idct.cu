@@ -5,7 +5,8 @@
 //
 // The stage is bound by HBM: per patch it reads 256 B of int32 coefficients
 // and writes up to 256 B of fp32 latents, against 2 x 512 FMAs of the
-// separable transform.  One CTA pass takes 32 consecutive patches, 8 threads
+// separable transform (done as butterflies, below).  One CTA pass takes 32
+// consecutive patches, 8 threads
 // per patch (the 8 threads of a patch sit in one warp, so the exchanges
 // between the two 1-D passes need only __syncwarp):
 //   load    thread j reads 16 B at coefficient 4j and 32 + 4j of its patch
@@ -17,11 +18,13 @@
 //   store   lanes 2i and 2i+1 trade row halves so that each store
 //           instruction writes whole 32-byte rows: row 2i in the first,
 //           row 2i+1 in the second.
-// c[k][n] = a(k) cos((2n + 1) k pi / 16) lives in constant memory; every
-// index into it is warp-uniform, so each FMA reads its coefficient straight
-// from the constant bank.  The patch slot is padded to 72 floats so the
-// column accesses of pass 1 hit 32 distinct banks.
-#include <cmath>
+// Each 1-D transform x[n] = sum_k a(k) X[k] cos((2n + 1) k pi / 16) is the
+// even/odd split of the basis (cos((2(7-n) + 1) k pi / 16) = (-1)^k times
+// that of n): x[n] = E[n] + O[n], x[7-n] = E[n] - O[n] with E the 4-point
+// transform of X[0, 2, 4, 6] (split once more) and O a 4x4 product of
+// X[1, 3, 5, 7] -- 36 operations instead of 64 multiply-adds.  The patch
+// slot is padded to 72 floats so the column accesses of pass 1 hit 32
+// distinct banks.
 #include <cstdint>
 
 #include <cuda_runtime.h>
@@ -59,7 +62,29 @@ struct IdctParams {
   Plane pl[kPlanesMax];
 };
 
-__constant__ float kBasis[64];  // c[k][n] at k * 8 + n
+// 0.5 cos(k pi / 16), k = 1 .. 7 (k = 4 is also a(0) = 1 / sqrt(8))
+constexpr float kC1 = 4.903926402e-01f, kC2 = 4.619397663e-01f, kC3 = 4.157348062e-01f,
+                kC4 = 3.535533906e-01f, kC5 = 2.777851165e-01f, kC6 = 1.913417162e-01f,
+                kC7 = 9.754516101e-02f;
+
+// 8-point inverse DCT of X (frequencies) into x (samples), by the split above.
+__device__ __forceinline__ void idct8(const float (&X)[8], float (&x)[8]) {
+  const float ee0 = kC4 * (X[0] + X[4]), ee1 = kC4 * (X[0] - X[4]);
+  const float eo0 = fmaf(kC2, X[2], kC6 * X[6]), eo1 = fmaf(kC6, X[2], -kC2 * X[6]);
+  const float e0 = ee0 + eo0, e3 = ee0 - eo0, e1 = ee1 + eo1, e2 = ee1 - eo1;
+  const float o0 = fmaf(kC1, X[1], fmaf(kC3, X[3], fmaf(kC5, X[5], kC7 * X[7])));
+  const float o1 = fmaf(kC3, X[1], fmaf(-kC7, X[3], fmaf(-kC1, X[5], -kC5 * X[7])));
+  const float o2 = fmaf(kC5, X[1], fmaf(-kC1, X[3], fmaf(kC7, X[5], kC3 * X[7])));
+  const float o3 = fmaf(kC7, X[1], fmaf(-kC5, X[3], fmaf(kC3, X[5], -kC1 * X[7])));
+  x[0] = e0 + o0;
+  x[7] = e0 - o0;
+  x[1] = e1 + o1;
+  x[6] = e1 - o1;
+  x[2] = e2 + o2;
+  x[5] = e2 - o2;
+  x[3] = e3 + o3;
+  x[4] = e3 - o3;
+}
 
 // floor(n / d) for 32-bit n and d by one multiply-high with inv = ceil(2^64 / d)
 // (division by invariant integers, Granlund & Montgomery 1994: the error term
@@ -103,8 +128,12 @@ __global__ void __launch_bounds__(kThreads, 6)
     if (live) {
       b = static_cast<int>(udiv(g, p.blocks_per_image, p.bpi_inv));
       k = g - b * p.blocks_per_image;
-      for (int q = 1; q < p.n_planes; ++q)
-        if (k >= p.pl[q].blk0) pi = q;
+      int hi = p.n_planes - 1;  // last plane whose first patch is <= k
+      while (pi < hi) {
+        const int mid = (pi + hi + 1) >> 1;
+        if (k >= p.pl[mid].blk0) pi = mid;
+        else hi = mid - 1;
+      }
       step = __ldg(p.steps + b * p.L + p.pl[pi].level);
     }
     reinterpret_cast<float4*>(my)[j] =
@@ -119,13 +148,7 @@ __global__ void __launch_bounds__(kThreads, 6)
     float col[8], tr[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) col[u] = my[u * 8 + j];
-#pragma unroll
-    for (int m = 0; m < 8; ++m) {
-      float acc = 0.0f;
-#pragma unroll
-      for (int u = 0; u < 8; ++u) acc = fmaf(kBasis[u * 8 + m], col[u], acc);
-      tr[m] = acc;
-    }
+    idct8(col, tr);
     __syncwarp();
 #pragma unroll
     for (int m = 0; m < 8; ++m) my[m * 8 + j] = tr[m];
@@ -136,13 +159,7 @@ __global__ void __launch_bounds__(kThreads, 6)
     const float4 r1 = reinterpret_cast<const float4*>(my)[2 * j + 1];
     const float row[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
     float x[8];
-#pragma unroll
-    for (int n = 0; n < 8; ++n) {
-      float acc = 0.0f;
-#pragma unroll
-      for (int v = 0; v < 8; ++v) acc = fmaf(kBasis[v * 8 + n], row[v], acc);
-      x[n] = acc;
-    }
+    idct8(row, x);
     __syncwarp();  // the slot is refilled by the next pass
 
     // lanes 2i, 2i+1: the even lane sends its right half, the odd lane its left
@@ -181,31 +198,6 @@ __global__ void __launch_bounds__(kThreads, 6)
       }
     }
   }
-}
-
-// The basis table of the current device, written once per device.
-int ensure_basis() {
-  constexpr int kMaxDev = 64;
-  static bool done[kMaxDev];
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) {
-    cudaGetLastError();
-    return PIC_ERR_CUDA;
-  }
-  if (!done[dev]) {
-    float h[64];
-    const double pi = 3.14159265358979323846;
-    for (int k = 0; k < 8; ++k)
-      for (int n = 0; n < 8; ++n)
-        h[k * 8 + n] = static_cast<float>((k == 0 ? std::sqrt(0.125) : 0.5) *
-                                          std::cos((2 * n + 1) * k * pi / 16.0));
-    if (cudaMemcpyToSymbol(kBasis, h, sizeof(h)) != cudaSuccess) {
-      cudaGetLastError();
-      return PIC_ERR_CUDA;
-    }
-    done[dev] = true;
-  }
-  return PIC_OK;
 }
 
 bool sizes_ok(int H, int W, int L, int C) {
@@ -259,7 +251,6 @@ extern "C" int pic_idct_unpatchify(const int32_t* coeffs, const float* steps, in
   p.bpi_inv = udiv_inv(static_cast<unsigned>(blk));
   p.lat_per_image = off;
   p.total_blocks = static_cast<int>(blk * B);
-  if (ensure_basis() != PIC_OK) return PIC_ERR_CUDA;
 
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
