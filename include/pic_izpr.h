@@ -24,8 +24,9 @@
 extern "C" {
 #endif
 
-/* Bytes of device workspace pic_izpr_decode needs for n_symbols symbols
- * (the per-chunk marker counts of the compaction and a status word), or -1
+/* Bytes of device workspace pic_izpr_decode needs for n_symbols symbols (a
+ * status word and the compaction's marker counts: per 2048-symbol chunk its
+ * offset within its group of 8 chunks, per group its count and base), or -1
  * for n_symbols < 0. */
 int64_t pic_izpr_workspace_bytes(int64_t n_symbols);
 

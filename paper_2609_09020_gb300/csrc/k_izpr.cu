@@ -3,9 +3,10 @@
 //
 // Algorithm 1 expands each block from its end-of-block marker offsets, which
 // the paper finds beforehand by a stream compaction.  Here:
-// 1. izpr_count: eob markers per 2048-symbol chunk (coalesced reads).
-// 2. izpr_scan: one CTA, exclusive scan of the chunk counts = index of each
-//    chunk's first block; the marker total.
+// 1. izpr_count: eob markers per 2048-symbol chunk (16-byte loads), summed
+//    over groups of 8 chunks, with each chunk's offset within its group.
+// 2. izpr_scan: one CTA, exclusive scan of the group counts; a chunk's
+//    first block = its group's base + its offset in the group.
 // 3. izpr_expand: persistent CTAs do the compaction and the expansion
 //    together, chunk by chunk.  Each thread holds 16 consecutive symbols of
 //    the chunk in registers (loaded while the CTA expanded its previous
@@ -34,26 +35,33 @@ constexpr int kChunk = kThreads * kPerThread;  // symbols per compaction chunk
 
 enum : int { kBadBlock = 1, kBadCount = 2 };
 
-// Workspace: status word, marker total, chunk counts, chunk bases.
+// Chunks are counted in groups of kGroup (one CTA of kGroup x kThreads
+// threads per group), so the scan runs over the groups.
+constexpr int kGroup = 8;
+// Workspace: status word, marker total, group counts, each chunk's first
+// block within its group, group bases.
 struct Workspace {
   int* status;
   long long* total;
-  int* counts;
-  long long* base;
+  int* gcount;
+  int* local;
+  long long* gbase;
 };
 __host__ __device__ inline long long n_chunks_of(long long n) { return (n + kChunk - 1) / kChunk; }
+__host__ __device__ inline long long n_groups_of(long long n) { return (n_chunks_of(n) + kGroup - 1) / kGroup; }
+__host__ __device__ inline long long align16(long long b) { return (b + 15) / 16 * 16; }
 __host__ __device__ inline long long ws_bytes(long long n) {
-  const long long c = n_chunks_of(n);
-  return 32 + ((c * 4 + 15) / 16) * 16 + c * 8;
+  return 32 + align16(4 * n_groups_of(n)) + align16(4 * n_chunks_of(n)) + 8 * n_groups_of(n);
 }
 __host__ __device__ inline Workspace ws_view(void* w, long long n) {
   char* p = static_cast<char*>(w);
-  const long long c = n_chunks_of(n);
+  const long long g = n_groups_of(n), c = n_chunks_of(n);
   Workspace v;
   v.status = reinterpret_cast<int*>(p);
   v.total = reinterpret_cast<long long*>(p + 16);
-  v.counts = reinterpret_cast<int*>(p + 32);
-  v.base = reinterpret_cast<long long*>(p + 32 + ((c * 4 + 15) / 16) * 16);
+  v.gcount = reinterpret_cast<int*>(p + 32);
+  v.local = reinterpret_cast<int*>(p + 32 + align16(4 * g));
+  v.gbase = reinterpret_cast<long long*>(p + 32 + align16(4 * g) + align16(4 * c));
   return v;
 }
 
@@ -76,34 +84,6 @@ constexpr ZigzagTable make_zigzag() {
   return t;
 }
 
-// Exclusive scan of one int per thread over a 256-thread CTA; returns the
-// thread's prefix and writes the CTA total to *total.
-__device__ int cta_exclusive_scan(int v, int* smem, int* total) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int x = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, x, o);
-    if (lane >= o) x += y;
-  }
-  if (lane == 31) smem[warp] = x;
-  __syncthreads();
-  if (warp == 0) {
-    int w = lane < kThreads / 32 ? smem[lane] : 0;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, w, o);
-      if (lane >= o) w += y;
-    }
-    if (lane < kThreads / 32) smem[32 + lane] = w;  // inclusive warp totals
-  }
-  __syncthreads();
-  const int before = warp > 0 ? smem[32 + warp - 1] : 0;
-  *total = smem[32 + kThreads / 32 - 1];
-  __syncthreads();
-  return before + x - v;
-}
-
 // 16 consecutive symbols from stream index i0 into r; positions past the
 // end read as `fill`.  16-byte loads when the stream is 16-byte aligned.
 __device__ __forceinline__ void load16(const int32_t* __restrict__ sym, long long n, long long i0,
@@ -124,18 +104,37 @@ __device__ __forceinline__ void load16(const int32_t* __restrict__ sym, long lon
   }
 }
 
-__global__ void __launch_bounds__(kThreads) izpr_count(const int32_t* __restrict__ sym,
-                                                       long long n, int32_t eob, int* counts) {
-  __shared__ int smem[64];
-  const long long i0 = static_cast<long long>(blockIdx.x) * kChunk + 16 * threadIdx.x;
-  int r[16];
-  load16(sym, n, i0, (reinterpret_cast<uintptr_t>(sym) & 15u) == 0, eob, r);
-  int c = 0;
+// Markers of the kGroup chunks of group blockIdx.x: thread t counts 16
+// symbols of chunk kGroup g + t / kThreads; the group's total, and each
+// chunk's count of markers before it within the group.
+__global__ void __launch_bounds__(kGroup * kThreads, 2) izpr_count(const int32_t* __restrict__ sym, long long n,
+                                                                int32_t eob, long long n_chunks, int* gcount,
+                                                                int* local) {
+  __shared__ int s_warp[kGroup * kThreads / 32];
+  const int t = threadIdx.x, sub = t / kThreads, lane = t & 31;
+  const long long c = static_cast<long long>(blockIdx.x) * kGroup + sub;
+  const long long i0 = c * kChunk + 16 * (t % kThreads);
+  int cnt = 0;
+  if (c < n_chunks) {
+    int r[16];
+    load16(sym, n, i0, (reinterpret_cast<uintptr_t>(sym) & 15u) == 0, eob, r);
 #pragma unroll
-  for (int k = 0; k < 16; ++k) c += (r[k] == eob && i0 + k < n) ? 1 : 0;
-  int total;
-  cta_exclusive_scan(c, smem, &total);
-  if (threadIdx.x == 0) counts[blockIdx.x] = total;
+    for (int k = 0; k < 16; ++k) cnt += (r[k] == eob && i0 + k < n) ? 1 : 0;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+  if (lane == 0) s_warp[t >> 5] = cnt;
+  __syncthreads();
+  if (t == 0) {
+    constexpr int kWarpsPerChunk = kThreads / 32;
+    int run = 0;
+    for (int q = 0; q < kGroup; ++q) {
+      const long long cq = static_cast<long long>(blockIdx.x) * kGroup + q;
+      if (cq < n_chunks) local[cq] = run;
+      for (int w = 0; w < kWarpsPerChunk; ++w) run += s_warp[q * kWarpsPerChunk + w];
+    }
+    gcount[blockIdx.x] = run;
+  }
 }
 
 // One CTA: exclusive scan of the chunk counts into chunk bases; the total.
@@ -237,9 +236,10 @@ struct Seg {
 };
 __device__ __forceinline__ Seg seg_cat(Seg a, Seg b) { return Seg{a.m + b.m, b.m > 0 ? b.s : a.s + b.s}; }
 
-__global__ void __launch_bounds__(kThreads, 6) izpr_expand(const int32_t* __restrict__ sym,
+__global__ void __launch_bounds__(kThreads, 8) izpr_expand(const int32_t* __restrict__ sym,
                                                         long long n, int32_t eob,
-                                                        const long long* __restrict__ base,
+                                                        const long long* __restrict__ gbase,
+                                                        const int* __restrict__ local,
                                                         const long long* total, long long n_blocks,
                                                         int32_t* __restrict__ coeffs,
                                                         int64_t* __restrict__ offsets, int* status) {
@@ -278,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, 6) izpr_expand(const int32_t* __rest
   if (blockIdx.x < n_chunks) {
     load16(sym, n, static_cast<long long>(blockIdx.x) * kChunk + 16 * t, vec, fill, cur);
     load_halo(blockIdx.x, hcur);
-    bcur = base[blockIdx.x];
+    bcur = gbase[blockIdx.x / kGroup] + local[blockIdx.x];
   }
   for (long long c = blockIdx.x; c < n_chunks; c += gridDim.x) {
     const long long c0 = c * kChunk;
@@ -291,7 +291,7 @@ __global__ void __launch_bounds__(kThreads, 6) izpr_expand(const int32_t* __rest
     if (c + gridDim.x < n_chunks) {  // next chunk, in flight meanwhile
       load16(sym, n, (c + gridDim.x) * kChunk + 16 * t, vec, fill, cur);
       load_halo(c + gridDim.x, hcur);
-      bcur = base[c + gridDim.x];
+      bcur = gbase[(c + gridDim.x) / kGroup] + local[c + gridDim.x];
     }
 
     // this thread's markers (bit i: symbol i) and positions since its last one
@@ -480,12 +480,14 @@ int pic_izpr_decode(const int32_t* symbols, int64_t n_symbols, int32_t eob, int6
     return PIC_ERR_CUDA;
   }
   if (chunks > 0) {
-    izpr_count<<<static_cast<unsigned>(chunks), kThreads, 0, s>>>(symbols, n_symbols, eob, ws.counts);
-    izpr_scan<<<1, 1024, 0, s>>>(ws.counts, chunks, ws.base, ws.total);
+    const long long groups = n_groups_of(n_symbols);
+    izpr_count<<<static_cast<unsigned>(groups), kGroup * kThreads, 0, s>>>(symbols, n_symbols, eob, chunks,
+                                                                           ws.gcount, ws.local);
+    izpr_scan<<<1, 1024, 0, s>>>(ws.gcount, groups, ws.gbase, ws.total);
     int grid = 0;
     if (expand_grid(&grid) != PIC_OK) return PIC_ERR_CUDA;
     izpr_expand<<<static_cast<unsigned>(chunks < grid ? chunks : grid), kThreads, kExpandSmem, s>>>(
-        symbols, n_symbols, eob, ws.base, ws.total, n_blocks, coeffs, offsets, ws.status);
+        symbols, n_symbols, eob, ws.gbase, ws.local, ws.total, n_blocks, coeffs, offsets, ws.status);
   } else if (n_blocks > 0) {
     izpr_flag<<<1, 1, 0, s>>>(ws.status, kBadCount);  // no symbols, hence no markers
   }

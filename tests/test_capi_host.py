@@ -89,7 +89,12 @@ def test_izpr_workspace_and_argument_checks(lib):
     assert pic.pic_izpr_workspace_bytes(-1) == -1
     assert pic.pic_izpr_workspace_bytes(0) == 32
     assert pic.pic_izpr_workspace_bytes(1) >= 32 + 4 + 8
-    assert pic.pic_izpr_workspace_bytes(10 ** 8) > 10 ** 8 // 4096 * 12
+    # a status word and total, then per 2048-symbol chunk its offset in its
+    # group (int32), per group of 8 chunks its count (int32) and base (int64)
+    n = 10 ** 8
+    chunks = -(-n // 2048)
+    groups = -(-chunks // 8)
+    assert pic.pic_izpr_workspace_bytes(n) >= 32 + 4 * chunks + 12 * groups
     # rejected before any CUDA call
     assert pic.pic_izpr_decode(None, 10, 30, 1, None, None, None, 0, None) == pic.PIC_ERR_INVALID_ARG
     assert pic.pic_izpr_decode(None, -1, 30, 1, None, None, None, 0, None) == pic.PIC_ERR_INVALID_ARG
