@@ -47,7 +47,7 @@ int64_t pic_huffman_workspace_bytes(int64_t n_words, int B, int p);
  *   n_bits      : int64, device, [B]: coded bits of stream b
  *                 (<= 32 (word_off[b + 1] - word_off[b]))
  *   tab_value   : int32, device, [B][max_table]: the stored tables' symbol
- *                 values (|value| < 2^23), canonical order
+ *                 values (any int32), canonical order
  *   tab_len     : int32, device, [B][max_table]: code lengths, 1..p; the
  *                 first 0 (or max_table) ends an image's table
  *   p           : the precision, 1..12: every length <= p

@@ -5,8 +5,10 @@
 // 1. huff_lut (one CTA per image): the stored table -- values and lengths in
 //    canonical order -- is the run-length code of the 2^p-entry lookup table:
 //    symbol k covers 2^(p - len_k) consecutive entries.  Expanding the runs
-//    gives the table (entry = length << 24 | value), so one lookup of the
-//    next p bits decodes a symbol.  Kraft's inequality is checked here.
+//    gives the table (16-bit entry = length << 12 | k, the symbol's row in
+//    the stored table, whose value is read only when it is written out), so
+//    one lookup of the next p bits decodes a symbol.  Kraft's inequality is
+//    checked here.
 // 2. huff_decode (one cooperative launch; every CTA resident, grid-wide
 //    barriers between the phases):
 //    a. each thread decodes its 256-bit subsequences speculatively from their
@@ -55,7 +57,7 @@ struct Ws {
   int* status;           // [4]
   int* changed;          // [kMaxPasses]
   long long* block_sum;  // [kMaxGrid]
-  uint32_t* lut;         // [B][2^p]
+  uint16_t* lut;         // [B][2^p]
   long long* exit0;      // [n_sub]
   long long* exit1;      // [n_sub]
   long long* start;      // [n_sub]
@@ -65,7 +67,7 @@ struct Ws {
 
 long long ws_size(long long n_sub, int B, int p) {
   long long b = 16 + kMaxPasses * 4 + kMaxGrid * 8;
-  b += (static_cast<long long>(B) << p) * 4;
+  b += (static_cast<long long>(B) << p) * 2;
   b = (b + 15) / 16 * 16;
   b += n_sub * (8 * 4 + 4);
   return (b + 15) / 16 * 16;
@@ -77,8 +79,8 @@ __host__ __device__ inline Ws ws_view(void* w, long long n_sub, int B, int p) {
   v.status = reinterpret_cast<int*>(c);
   v.changed = reinterpret_cast<int*>(c + 16);
   v.block_sum = reinterpret_cast<long long*>(c + 16 + kMaxPasses * 4);
-  v.lut = reinterpret_cast<uint32_t*>(c + 16 + kMaxPasses * 4 + kMaxGrid * 8);
-  long long o = 16 + kMaxPasses * 4 + kMaxGrid * 8 + (static_cast<long long>(B) << p) * 4;
+  v.lut = reinterpret_cast<uint16_t*>(c + 16 + kMaxPasses * 4 + kMaxGrid * 8);
+  long long o = 16 + kMaxPasses * 4 + kMaxGrid * 8 + (static_cast<long long>(B) << p) * 2;
   o = (o + 15) / 16 * 16;
   v.exit0 = reinterpret_cast<long long*>(c + o);
   v.exit1 = v.exit0 + n_sub;
@@ -90,14 +92,12 @@ __host__ __device__ inline Ws ws_view(void* w, long long n_sub, int B, int p) {
 
 // ---------------------------------------------------------------- 1. tables
 __global__ void __launch_bounds__(kThreads)
-    huff_lut(const int32_t* __restrict__ tab_value, const int32_t* __restrict__ tab_len,
-             int max_table, int p, uint32_t* lut, int* status) {
+    huff_lut(const int32_t* __restrict__ tab_len, int max_table, int p, uint16_t* lut, int* status) {
   __shared__ int s_start[kMaxTable + 1];
-  __shared__ uint32_t s_entry[kMaxTable];
+  __shared__ uint16_t s_entry[kMaxTable];
   __shared__ int s_warp[kThreads / 32];
   __shared__ int s_m;
   const int b = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5;
-  const int32_t* tv = tab_value + static_cast<long long>(b) * max_table;
   const int32_t* tl = tab_len + static_cast<long long>(b) * max_table;
   // the table ends at its first zero length
   if (t == 0) s_m = max_table;
@@ -116,7 +116,7 @@ __global__ void __launch_bounds__(kThreads)
       const int l = tl[k];
       if (l < 1 || l > p) bad = true;
       else run = 1 << (p - l);
-      s_entry[k] = (static_cast<uint32_t>(l) << 24) | (static_cast<uint32_t>(tv[k]) & 0xFFFFFFu);
+      s_entry[k] = static_cast<uint16_t>((l << 12) | k);  // the value is tab_value[k]
     }
     int x = run;  // inclusive warp scan, then across the warps
 #pragma unroll
@@ -142,10 +142,10 @@ __global__ void __launch_bounds__(kThreads)
   }
   __syncthreads();
   const int fill = s_start[m];  // a bad table decodes nothing: every entry "no codeword"
-  uint32_t* out = lut + (static_cast<long long>(b) << p);
+  uint16_t* out = lut + (static_cast<long long>(b) << p);
   // every entry finds its run by binary search over the run starts
   for (int i = t; i < (1 << p); i += blockDim.x) {
-    uint32_t e = 0;  // no codeword
+    uint16_t e = 0;  // no codeword
     if (i < fill) {
       int lo = 0, hi = m - 1;  // last k with s_start[k] <= i
       while (lo < hi) {
@@ -168,6 +168,8 @@ struct DecodeParams {
   int B;
   int p;
   const long long* sym_off;
+  const int32_t* tab_value;  // [B][max_table]: a table entry's low 12 bits index its row
+  int max_table;
   int32_t* out;
   Ws ws;
   long long n_sub;
@@ -184,13 +186,9 @@ __device__ __forceinline__ int image_of(const DecodeParams& P, long long word) {
   return lo;
 }
 
-__device__ __forceinline__ int32_t value_of(uint32_t e) {
-  return static_cast<int32_t>(e << 8) >> 8;  // sign-extend the 24-bit value
-}
-
 // The counting loop of decode_span_s, with (PAIR) or without the pair table.
 template <bool PAIR>
-__device__ __forceinline__ int decode_span_loop(const uint32_t* sw, int lpos, int lke, const uint32_t* lut,
+__device__ __forceinline__ int decode_span_loop(const uint32_t* sw, int lpos, int lke, const uint16_t* lut,
                                                 const uint8_t* lut2, int p, int* count, bool* bad) {
   int c = 0;
   int li = lpos >> 5;
@@ -216,7 +214,7 @@ __device__ __forceinline__ int decode_span_loop(const uint32_t* sw, int lpos, in
       c += two ? 2 : 1;
       lpos += two ? l1 + l2 : l1;
     } else {
-      int len = static_cast<int>(lut[w] >> 24);
+      int len = static_cast<int>(lut[w] >> 12);
       if (len == 0) {
         *bad = true;
         len = 1;
@@ -236,7 +234,7 @@ __device__ __forceinline__ int decode_span_loop(const uint32_t* sw, int lpos, in
 // words.  With a pair table (lut2: the lengths of the first codeword of each
 // p-bit window and of the second one when it lies inside the same window),
 // one lookup advances over up to two codewords.
-__device__ __forceinline__ int decode_span_s(const uint32_t* sw, int lpos, int lke, const uint32_t* lut,
+__device__ __forceinline__ int decode_span_s(const uint32_t* sw, int lpos, int lke, const uint16_t* lut,
                                              const uint8_t* lut2, int p, int* count, bool* bad) {
   if (lpos >= lke) {
     *count = 0;
@@ -249,7 +247,7 @@ __device__ __forceinline__ int decode_span_s(const uint32_t* sw, int lpos, int l
 // decode_span_s for subsequence positions of image b: pos (bits from the
 // image's first word wbase) <-> staged position (bits from word w0).
 __device__ __forceinline__ long long decode_at(const uint32_t* sw, long long w0, long long wbase, long long pos,
-                                               long long ke, const uint32_t* lut, const uint8_t* lut2, int p,
+                                               long long ke, const uint16_t* lut, const uint8_t* lut2, int p,
                                                int* count, bool* bad) {
   if (pos >= ke) {
     *count = 0;
@@ -277,7 +275,8 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
   cg::grid_group grid = cg::this_grid();
   __shared__ long long red[kThreads / 32];
   __shared__ long long scan[kThreads];
-  extern __shared__ uint32_t s_lut[];  // the lookup tables of the first and last image of the range
+  extern __shared__ __align__(16) uint32_t s_dyn[];
+  uint16_t* s_lut = reinterpret_cast<uint16_t*>(s_dyn);  // tables of the first and last image of the range
   const Ws& ws = P.ws;
   const long long per_block = P.per_block;
   const long long k_begin = static_cast<long long>(blockIdx.x) * per_block;
@@ -294,23 +293,23 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
     s_lut[tsize + i] = ws.lut[(static_cast<long long>(b_last) << P.p) + i];
   }
   __syncthreads();
-  auto lut_of = [&](int b) -> const uint32_t* {
+  auto lut_of = [&](int b) -> const uint16_t* {
     return b == b_first ? s_lut : (b == b_last ? s_lut + tsize : ws.lut + (static_cast<long long>(b) << P.p));
   };
   // each pass of 256 subsequences first stages its stream words (coalesced),
   // so that no global load sits inside a decode chain
-  uint32_t* s_words = s_lut + 2 * tsize;
+  uint32_t* s_words = reinterpret_cast<uint32_t*>(s_lut + 2 * tsize);
   int* s_stage = reinterpret_cast<int*>(s_words + kWbuf);
   // the pair tables of the two images: first codeword's length | the
   // second's << 4 (0 when it does not lie inside the same p-bit window)
   uint8_t* s_lut2 = reinterpret_cast<uint8_t*>(s_stage + kStageInts);
   for (int i = threadIdx.x; i < 2 * tsize; i += blockDim.x) {
-    const uint32_t* L = s_lut + (i >= tsize ? tsize : 0);
+    const uint16_t* L = s_lut + (i >= tsize ? tsize : 0);
     const int w = i & (tsize - 1);
-    const int l1 = static_cast<int>(L[w] >> 24);
+    const int l1 = static_cast<int>(L[w] >> 12);
     int l2 = 0;
     if (l1 > 0 && l1 < P.p) {
-      const int l = static_cast<int>(L[(w << l1) & (tsize - 1)] >> 24);
+      const int l = static_cast<int>(L[(w << l1) & (tsize - 1)] >> 12);
       if (l > 0 && l <= P.p - l1) l2 = l;
     }
     s_lut2[i] = static_cast<uint8_t>(l1 | (l2 << 4));
@@ -435,7 +434,8 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
     int lpos = 0, lke = 0, li = 0;
     uint32_t hi = 0, lo = 0;
     long long o = 0, room = 0, shift = 0, nb = 0, ks = 0;
-    const uint32_t* lut = s_lut;
+    const uint16_t* lut = s_lut;
+    const int32_t* vals = P.tab_value;
     bool more = false;
     if (k < k_end) {
       const int b = image_of(P, k * kQ);
@@ -451,6 +451,7 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
       lpos = static_cast<int>(st + shift);
       lke = static_cast<int>(ke + shift);
       lut = lut_of(b);
+      vals = P.tab_value + static_cast<long long>(b) * P.max_table;
       more = ks < nb && st < ke;
       if (more) {
         li = lpos >> 5;
@@ -470,12 +471,12 @@ __global__ void __launch_bounds__(kThreads) huff_decode(const DecodeParams P) {
           lo = s_words[li + 1];
         }
         const uint32_t e = lut[__funnelshift_l(lo, hi, lpos & 31) >> shr];
-        int len = static_cast<int>(e >> 24);
+        int len = static_cast<int>(e >> 12);
         if (len == 0) {
           bad = true;
           len = 1;
         }
-        wbuf[lane * kRow + n] = value_of(e);
+        wbuf[lane * kRow + n] = __ldg(vals + (e & 0xFFFu));  // off the decode chain
         ++n;
         lpos += len;
         more = lpos < lke;
@@ -521,7 +522,7 @@ int decode_grid(int p, size_t smem, int* grid) {
   if (cached[dev][p] == 0) {
     int coop = 0, sms = 0, per_sm = 0;
     // the attribute is the function's, for every precision: set it to the largest
-    constexpr int kMaxSmem = (5 * 2 << PIC_HUFF_MAX_PRECISION) + (kWbuf + kStageInts) * 4;
+    constexpr int kMaxSmem = (3 * 2 << PIC_HUFF_MAX_PRECISION) + (kWbuf + kStageInts) * 4;
     if (cudaFuncSetAttribute(huff_decode, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) !=
             cudaSuccess ||
         cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess ||
@@ -560,7 +561,7 @@ int pic_huffman_decode(const uint32_t* words, int64_t n_words, const int64_t* wo
   const long long n_sub = n_words / kQ;
   if (static_cast<long long>(workspace_bytes) < ws_size(n_sub, B, p)) return PIC_ERR_INVALID_ARG;
   // 2 tables + the pass's words + the output staging rows + 2 pair tables
-  const size_t lut_smem = (sizeof(uint32_t) * 2 << p) + (kWbuf + kStageInts) * sizeof(uint32_t) + (2 << p);
+  const size_t lut_smem = (sizeof(uint16_t) * 2 << p) + (kWbuf + kStageInts) * sizeof(uint32_t) + (2 << p);
   int grid = 0;
   int rc = decode_grid(p, lut_smem, &grid);
   if (rc != PIC_OK) return rc;
@@ -573,6 +574,8 @@ int pic_huffman_decode(const uint32_t* words, int64_t n_words, const int64_t* wo
   P.B = B;
   P.p = p;
   P.sym_off = reinterpret_cast<const long long*>(sym_off);
+  P.tab_value = tab_value;
+  P.max_table = max_table;
   P.out = out;
   P.ws = ws_view(workspace, n_sub, B, p);
   P.n_sub = n_sub;
@@ -584,7 +587,7 @@ int pic_huffman_decode(const uint32_t* words, int64_t n_words, const int64_t* wo
     cudaGetLastError();
     return PIC_ERR_CUDA;
   }
-  huff_lut<<<B, kThreads, 0, s>>>(tab_value, tab_len, max_table, p, P.ws.lut, P.ws.status);
+  huff_lut<<<B, kThreads, 0, s>>>(tab_len, max_table, p, P.ws.lut, P.ws.status);
   const long long g = (n_sub + P.per_block - 1) / P.per_block;
   void* args[] = {&P};
   if (cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(huff_decode), dim3(static_cast<unsigned>(g)),

@@ -79,6 +79,18 @@ def test_edge_streams(orc, p):
     assert np.array_equal(got, np.concatenate(syms))
 
 
+def test_full_range_values():
+    """Symbol values anywhere in int32 (the lookup tables hold a symbol's
+    row in the stored table, not its value)."""
+    rng = np.random.Generator(np.random.PCG64(31))
+    alphabet = np.array([-2 ** 31, 2 ** 31 - 1, 2 ** 30, -2 ** 29 + 7, 0, 5, -(2 ** 23), 2 ** 23],
+                        np.int64).astype(np.int32)
+    s = alphabet[rng.integers(0, alphabet.size, 5000)]
+    d = _pack_batch([wk.huffman_pack(s, 12)], 12)
+    got = _gpu(d, np.array([0, s.size], np.int64))
+    assert np.array_equal(got, s)
+
+
 def test_malformed_streams_are_flagged():
     from paper_2609_09020_gb300 import pic
     rng = np.random.Generator(np.random.PCG64(97))
