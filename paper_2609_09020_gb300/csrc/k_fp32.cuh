@@ -210,7 +210,6 @@ __global__ void __launch_bounds__(kThreads) fp32_generic_kernel(const DecodePara
   const long long t_begin = blockIdx.x * chunk;
   const long long t_end = min(t_begin + chunk, p.total_tiles);
   const float* wts = static_cast<const float*>(p.weights);
-  const long long plane = static_cast<long long>(p.H) * p.W;
   int cur_b = -1;
   for (long long t = t_begin; t < t_end; ++t) {
     const int b = static_cast<int>(t / p.tiles_per_image);

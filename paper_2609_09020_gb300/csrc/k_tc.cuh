@@ -592,36 +592,36 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             cy = ny;
             ctx = ntx;
             if (!ok) break;
-            continue;
-          }
-          for (int k = 0; k < NL - 1 && ok; ++k) {
-            if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
-              ok = false;
-              break;
+          } else {
+            for (int k = 0; k < NL - 1 && ok; ++k) {
+              if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
+                ok = false;
+                break;
+              }
+              acc_phase ^= 1u;
+              tc_fence_after();
+              hidden_epilogue<Net>(t_acc, t_a);
+              tc_fence_before();
+              mbar_arrive(my_a);
+              if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
             }
+            if (!ok) break;
+
+            // ---- output layer: bias, clamp, store ----
+            if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
             acc_phase ^= 1u;
             tc_fence_after();
-            hidden_epilogue<Net>(t_acc, t_a);
+            uint32_t o[4];
+            tmem_ld4(t_acc, o);
+            tmem_ld_wait();
             tc_fence_before();
-            mbar_arrive(my_a);
-            if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
+            if (has_next) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
+            const int x = x0 + r;
+            if (x < p.W)
+              store_rgb(p, b, y, x, __uint_as_float(o[0]), __uint_as_float(o[1]), __uint_as_float(o[2]));
+            cy = ny;
+            ctx = ntx;
           }
-          if (!ok) break;
-
-          // ---- output layer: bias, clamp, store ----
-          if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
-          acc_phase ^= 1u;
-          tc_fence_after();
-          uint32_t o[4];
-          tmem_ld4(t_acc, o);
-          tmem_ld_wait();
-          tc_fence_before();
-          if (has_next) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
-          const int x = x0 + r;
-          if (x < p.W)
-            store_rgb(p, b, y, x, __uint_as_float(o[0]), __uint_as_float(o[1]), __uint_as_float(o[2]));
-          cy = ny;
-          ctx = ntx;
         }
       }
       seg = seg_end;
