@@ -418,6 +418,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         int it_l[JJ], it_i[JJ], it_W[JJ], it_H[JJ];
         long long it_off[JJ];
         float it_sy[JJ], it_sx[JJ];
+        float it_beta[JJ];  // vertical weight of each item for the tile last prefetched
 #pragma unroll
         for (int j = 0; j < J; ++j) {
           int e = r + kTile * j, l = 0, c = 0, i = 0;
@@ -470,6 +471,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             const int l = it_l[j];
             if (l > 0) {
               const Tap ty = bilinear_tap(y, it_sy[j], it_H[j]);
+              it_beta[j] = ty.frac;
               const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, it_sx[j], it_W[j]).i0;
               const int u = min(max(u_start + it_i[j], 0), it_W[j] - 1);
               const int32_t* pl = lat + it_off[j] + u;
@@ -489,7 +491,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           for (int j = 0; j < J; ++j) {
             const int l = it_l[j];
             if (l > 0) {
-              const float beta = bilinear_tap(y, it_sy[j], it_H[j]).frac;
+              const float beta = it_beta[j];  // set by the prefetch of this tile
               const int t0 = stage[(C + 2 * j) * kTile + r], t1 = stage[(C + 2 * j + 1) * kTile + r];
               colbuf[r + kTile * j] = step[l] * lat_lerp<FL>(t0, t1, beta);
             }
