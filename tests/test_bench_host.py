@@ -1,6 +1,6 @@
 """The bench's roofline arithmetic on the host: algorithmic work per launch
 from first principles (unpadded MACs; int32 latents, weights, steps and fp32
-RGB bytes moved once), and the binding time of SURVEY's c5 row."""
+RGB bytes moved once), and the binding time of the 64-image workload."""
 import importlib.util
 import os
 
