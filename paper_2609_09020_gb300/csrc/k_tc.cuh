@@ -158,7 +158,7 @@ struct TcNet {
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                              int* status) {
   for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    if (mbar_try_wait_sleep(bar, parity)) return true;
+    if (mbar_try_wait(bar, parity)) return true;
     if ((i & 63u) == 63u) {
       if (*abort_flag) return false;
       if (i > 4096) __nanosleep(64);
