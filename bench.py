@@ -306,6 +306,7 @@ def run_bitstream_stages(args):
         wts = t(dx.weights_for("fp16_tc"))
         out = torch.empty((B, 3, wl.H, wl.W), dtype=torch.float32, device=dev)
         dec = pic.Decoder.for_workload(wl, "fp16_tc", max_batch=B, latent="fp32")
+        dec.check_buffers(B, wl.H, wl.W, latents=lat, steps=None, weights=wts, out=out)
 
     def huff():
         rc = pic.pic_huffman_decode(words.data_ptr(), words.numel(), word_off.data_ptr(),
@@ -323,7 +324,7 @@ def run_bitstream_stages(args):
                                      wl.C, lat.data_ptr(), sp)
         if rc != pic.PIC_OK:
             raise pic.PicError(rc, "pic_idct_unpatchify")
-        dec.decode_batch(lat, None, wts, wl.H, wl.W, out, stream=stream, B=B)
+        dec.decode_batch(lat, None, wts, wl.H, wl.W, out, stream=stream, B=B, check=False)
 
     def one_step():
         huff()
@@ -360,6 +361,8 @@ def run_bitstream_stages(args):
                    "tv": t(h["tab_value"][b:b + 1]), "tl": t(h["tab_len"][b:b + 1]),
                    "sym_off": t(np.array([0, s1 - s0], np.int64)), "steps": t(dx.steps[b:b + 1]),
                    "w": t(dx.weights_for("fp16_tc")[b:b + 1])}
+            dec.check_buffers(1, wl.H, wl.W, latents=lat[:1], steps=None, weights=one["w"],
+                              out=out[:1])
             hwb1 = pic.pic_huffman_workspace_bytes(one["words"].numel(), 1, p)
             hws1 = torch.empty(hwb1, dtype=torch.uint8, device=dev)
 
@@ -379,7 +382,8 @@ def run_bitstream_stages(args):
                                              wl.L, wl.C, lat.data_ptr(), sp)
                 if rc != pic.PIC_OK:
                     raise pic.PicError(rc, "pic_idct_unpatchify")
-                dec.decode_batch(lat[:1], None, one["w"], wl.H, wl.W, out[:1], stream=stream, B=1)
+                dec.decode_batch(lat[:1], None, one["w"], wl.H, wl.W, out[:1], stream=stream, B=1,
+                                 check=False)
 
             run_one()  # warm this image's buffers
             torch.cuda.synchronize(dev)
@@ -623,6 +627,9 @@ def run_stage(args):
     ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
     dec = pic.Decoder.for_workload(wl, "fp16_tc", max_batch=chunk, latent="fp32") \
         if stage == "pipeline" else None
+    if dec is not None:
+        dec.check_buffers(chunk, wl.H, wl.W, latents=lat, steps=None, weights=wts[:chunk],
+                          out=out[:chunk])
 
     def izpr(s_ptr, n_sym, nb):
         rc = pic.pic_izpr_decode(s_ptr, n_sym, eob, nb, coeffs.data_ptr(), offsets.data_ptr(),
@@ -648,7 +655,7 @@ def run_stage(args):
                      nb * n_blk)
                 idct(coeffs.data_ptr(), steps_t.data_ptr() + 4 * b0 * wl.L, nb)
                 dec.decode_batch(lat, None, wts[b0:b0 + nb], wl.H, wl.W, out[b0:b0 + nb],
-                                 stream=stream, B=nb)
+                                 stream=stream, B=nb, check=False)
 
     for _ in range(max(args.warmup, 3)):
         one_step()
@@ -679,7 +686,7 @@ def run_stage(args):
                         idct(coeffs.data_ptr(), steps_t.data_ptr() + 4 * b0 * wl.L, nb)
                     else:
                         dec.decode_batch(lat, None, wts[b0:b0 + nb], wl.H, wl.W,
-                                         out[b0:b0 + nb], stream=stream, B=nb)
+                                         out[b0:b0 + nb], stream=stream, B=nb, check=False)
             return f
         for which in ("izpr", "idct", "decode"):
             stage_ms[which] = _event_time(part(which), args.steps, stream, torch)
@@ -859,9 +866,10 @@ def main():
     wts = torch.from_numpy(w_host).to(dev)
     out = torch.empty((B, 3, wl.H, wl.W), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
+    dec.check_buffers(B, wl.H, wl.W, latents=lat, steps=steps_t, weights=wts, out=out)
 
     for _ in range(max(args.warmup, 3)):
-        dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B)
+        dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B, check=False)
     dec.check(stream)
     torch.cuda.synchronize(dev)
 
@@ -871,7 +879,7 @@ def main():
         torch.cuda.synchronize(dev)
         ev0.record(stream)
         for _ in range(args.steps):
-            dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B)
+            dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B, check=False)
         ev1.record(stream)
         torch.cuda.synchronize(dev)
         barrier()
@@ -884,12 +892,12 @@ def main():
     protocols = None
     if rank == 0 and not args.no_protocols:
         for _ in range(20):  # warm-up calls
-            dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B)
+            dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B, check=False)
         call_ms = []
         for _ in range(200):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B)
+            dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, stream=stream, B=B, check=False)
             e1.record(stream)
             e1.synchronize()
             call_ms.append(e0.elapsed_time(e1))
@@ -902,7 +910,7 @@ def main():
             with torch.cuda.stream(side):
                 with torch.cuda.graph(g):
                     for _ in range(4):
-                        dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, B=B)
+                        dec.decode_batch(lat, steps_t, wts, wl.H, wl.W, out, B=B, check=False)
             stream.wait_stream(side)
             g.replay()
             torch.cuda.synchronize(dev)
@@ -921,10 +929,12 @@ def main():
         n_ser = min(B, 16)
         w_img = [wts[b].clone() for b in range(n_ser)]  # each image's weights on its own (aligned)
         for b in range(n_ser):
+            dec.check_buffers(1, wl.H, wl.W, latents=lat[b:b + 1], steps=steps_t[b:b + 1],
+                              weights=w_img[b], out=out[b:b + 1])
             torch.cuda.synchronize(dev)
             t0 = time.perf_counter()
             dec.decode_batch(lat[b:b + 1], steps_t[b:b + 1], w_img[b], wl.H, wl.W, out[b:b + 1],
-                             stream=stream, B=1)
+                             stream=stream, B=1, check=False)
             torch.cuda.synchronize(dev)
             t_img.append(time.perf_counter() - t0)
         protocols = {

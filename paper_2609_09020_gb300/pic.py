@@ -354,6 +354,47 @@ def huffman_decode(words, word_off, n_bits, tab_value, tab_len, p, sym_off, stre
 
 
 # ---- convenience wrapper over torch tensors --------------------------------
+def decode_buffer_bytes(arch: pic_arch, B, H, W) -> dict:
+    """Bytes each buffer of a B-image H x W decode must hold at least:
+    latents B x pic_latent_count x 4, steps B x L x 4 (int32 latents only),
+    weights B x pic_param_count x (2 for the tensor-core arch, else 4), out
+    B x 3 x H x W x (1 for uint8 output, else 4).  Sizes the C ABI would
+    refuse count as 0 (the call itself then reports the error)."""
+    B_, H_, W_ = max(B, 0), max(H, 0), max(W, 0)
+    n_lat = max(pic_latent_count(H, W, arch.num_levels, arch.channels_per_level), 0)
+    n_par = max(pic_param_count(arch), 0)
+    return {
+        "latents": 4 * B_ * n_lat,
+        "steps": 4 * B_ * arch.num_levels if arch.latent_format == PIC_LATENT_INT32 else 0,
+        "weights": (2 if arch.precision == PIC_PREC_FP16_TC else 4) * B_ * n_par,
+        "out": (1 if arch.output_format == PIC_OUT_U8_HWC else 4) * 3 * B_ * H_ * W_,
+    }
+
+
+def check_decode_buffers(need: dict, B, H, W, host=False, **bufs):
+    """Raises ValueError unless every named buffer (latents, steps, weights,
+    out: torch tensors, or numpy arrays on the host path) is contiguous,
+    lives on the device (host=False) or the host (host=True), and holds at
+    least ``need[name]`` bytes.  A missing (None) buffer passes only where
+    the call does not read it."""
+    for name, a in bufs.items():
+        if a is None:
+            if name != "steps" or need[name] > 0:
+                raise ValueError(f"{name}: required by this decoder")
+            continue
+        if isinstance(a, np.ndarray):
+            nbytes, contig, on_gpu = a.nbytes, a.flags["C_CONTIGUOUS"], False
+        else:
+            nbytes, contig, on_gpu = a.numel() * a.element_size(), a.is_contiguous(), a.is_cuda
+        if not contig:
+            raise ValueError(f"{name}: must be contiguous")
+        if on_gpu == host:
+            raise ValueError(f"{name}: must be a {'host' if host else 'CUDA'} buffer")
+        if nbytes < need[name]:
+            raise ValueError(f"{name}: holds {nbytes} bytes; a {B}-image {H}x{W} call needs "
+                             f"{need[name]}")
+
+
 def _stream_ptr(stream):
     if stream is None:
         import torch
@@ -363,7 +404,10 @@ def _stream_ptr(stream):
 
 class Decoder:
     """One decoder handle.  Tensors passed to the decode methods must be
-    contiguous CUDA tensors of the documented dtypes."""
+    contiguous CUDA tensors of the documented dtypes.  The C ABI receives bare
+    pointers and cannot see a buffer's size, so these methods refuse, before
+    anything is launched, a buffer that is smaller than the call reads or
+    writes, not contiguous, or on the wrong side of the host/device split."""
 
     def __init__(self, L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1,
                  max_W=1, max_batch=1, latent="int32", output="f32_chw"):
@@ -371,6 +415,7 @@ class Decoder:
                               output)
         self.latent = latent
         self.L, self.C, self.dims, self.precision = L, C, tuple(dims), precision
+        self._need = {}
         self.handle = pic_decode_create(self.arch)
 
     @classmethod
@@ -399,10 +444,27 @@ class Decoder:
         if rc != PIC_OK:
             raise PicError(rc, where)
 
-    def decode_batch(self, latents, steps, weights, H, W, out, stream=None, B=None):
-        """Enqueues a batch decode; arguments are torch CUDA tensors."""
+    def buffer_bytes(self, B, H, W) -> dict:
+        """``decode_buffer_bytes`` for this handle's arch (cached per shape)."""
+        key = (B, H, W)
+        need = self._need.get(key)
+        if need is None:
+            if len(self._need) >= 64:
+                self._need.clear()
+            need = self._need[key] = decode_buffer_bytes(self.arch, B, H, W)
+        return need
+
+    def check_buffers(self, B, H, W, host=False, **bufs):
+        check_decode_buffers(self.buffer_bytes(B, H, W), B, H, W, host, **bufs)
+
+    def decode_batch(self, latents, steps, weights, H, W, out, stream=None, B=None, check=True):
+        """Enqueues a batch decode; arguments are torch CUDA tensors.  With
+        check=False the buffer checks are skipped (a few microseconds of
+        host time per call): for loops that reuse buffers already checked."""
         if B is None:
             B = out.shape[0] if out.dim() == 4 else 1
+        if check:
+            self.check_buffers(B, H, W, latents=latents, steps=steps, weights=weights, out=out)
         sp = steps.data_ptr() if steps is not None else None
         rc = pic_decode_batch(self.handle, B, latents.data_ptr(), sp,
                               weights.data_ptr(), H, W, out.data_ptr(), _stream_ptr(stream))
@@ -410,7 +472,10 @@ class Decoder:
         return out
 
     def decode(self, latents, steps, weights, H, W, out, stream=None):
-        rc = pic_decode(self.handle, latents.data_ptr(), steps.data_ptr(), weights.data_ptr(),
+        """Enqueues a one-image decode; arguments are torch CUDA tensors."""
+        self.check_buffers(1, H, W, latents=latents, steps=steps, weights=weights, out=out)
+        sp = steps.data_ptr() if steps is not None else None
+        rc = pic_decode(self.handle, latents.data_ptr(), sp, weights.data_ptr(),
                         H, W, out.data_ptr(), _stream_ptr(stream))
         self._check(rc, "pic_decode")
         return out
@@ -422,11 +487,14 @@ class Decoder:
         chunks of images."""
         if B is None:
             B = latents.shape[0] if latents.ndim == 2 else 1
-        for a in (latents, steps, weights, out):
-            ok = a.flags["C_CONTIGUOUS"] if isinstance(a, np.ndarray) else a.is_contiguous()
-            if not ok:
-                raise ValueError("host buffers must be C-contiguous")
-        ptr = lambda a: a.ctypes.data if isinstance(a, np.ndarray) else a.data_ptr()
+        self.check_buffers(B, H, W, host=True, latents=latents, steps=steps, weights=weights,
+                           out=out)
+
+        def ptr(a):
+            if a is None:
+                return None
+            return a.ctypes.data if isinstance(a, np.ndarray) else a.data_ptr()
+
         rc = pic_decode_batch_host(self.handle, B, ptr(latents), ptr(steps), ptr(weights), H, W,
                                    ptr(out), _stream_ptr(stream))
         self._check(rc, "pic_decode_batch_host")
