@@ -50,7 +50,7 @@ typedef enum {
     PIC_ERR_INVALID_ARG = -1, /* NULL pointer, bad size, misaligned pointer, arch mismatch */
     PIC_ERR_UNSUPPORTED = -2, /* arch outside the supported envelope, or no sm_103 device */
     PIC_ERR_CUDA = -3,        /* a CUDA runtime call or kernel launch failed */
-    PIC_ERR_ALLOC = -4,       /* device or host allocation failed (create only) */
+    PIC_ERR_ALLOC = -4,       /* device allocation failed (create; first host-buffer call) */
     PIC_ERR_TIMEOUT = -5      /* a bounded device-side wait gave up (reported by pic_decode_check) */
 } pic_status;
 
