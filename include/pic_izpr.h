@@ -43,7 +43,8 @@ int64_t pic_izpr_workspace_bytes(int64_t n_symbols);
  *               16-byte aligned, caller-owned; it must not be shared by
  *               decodes that overlap on the GPU
  * A malformed stream (a block covering more than 64 positions, a value above
- * eob, or a marker count different from n_blocks) is recorded in the
+ * eob, a marker count different from n_blocks, or symbols after the last
+ * marker) is recorded in the
  * workspace and reported by pic_izpr_status; the coefficients of the blocks
  * concerned are then unspecified, but nothing is written out of bounds.
  * Errors: PIC_ERR_INVALID_ARG (NULL or misaligned pointers, negative sizes,
