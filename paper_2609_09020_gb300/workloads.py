@@ -122,7 +122,7 @@ WORKLOADS = {
 }
 
 # The decoding-speed ablation over the synthesis network's width (Sec. 4.3,
-# "Decoding speed for different width"): the paper's own g_s -- L = 8
+# its decode-speed-versus-width experiment): the paper's own g_s -- L = 8
 # single-channel latents, a 4-layer MLP with ReLU -- at widths 8, 16 (the
 # paper's choice), 32 and 64, on batches of 64 Kodak-sized images.
 for _w in (8, 16, 32, 64):

@@ -21,6 +21,27 @@ def test_workload_sizes(name, lat, params):
     assert wl.n_params == params
 
 
+@pytest.mark.parametrize("name,recipe", [
+    # image, levels x channels, MLP, activation, weight dtype, Laplace scale, clip, seeds
+    ("c1", (256, 256, 4, 1, (4, 16, 16, 3), "relu", "fp32", 2.0, 15, (0,))),
+    ("c2", (512, 768, 7, 1, (7, 40, 40, 3), "gelu", "fp32", 3.0, 31, (1,))),
+    ("c3", (1080, 1920, 7, 2, (14, 64, 64, 3), "relu", "fp32", 3.0, 31, (2,))),
+    ("c4", (2160, 3840, 8, 2, (16, 64, 64, 64, 3), "gelu", "fp32", 4.0, 63, (3,))),
+    ("c5", (512, 768, 7, 1, (7, 64, 64, 3), "relu", "fp16", 3.0, 31, tuple(range(100, 164)))),
+])
+def test_workload_recipes(name, recipe):
+    wl = wk.WORKLOADS[name]
+    assert (wl.H, wl.W, wl.L, wl.C, wl.dims, wl.act, wl.weight_dtype, wl.lap_scale, wl.clip,
+            wl.seeds) == recipe
+
+
+def test_width_sweep_is_the_papers_net_at_four_widths():
+    for w in (8, 16, 32, 64):
+        wl = wk.WORKLOADS[f"w{w}"]
+        assert (wl.H, wl.W, wl.L, wl.C, wl.act, wl.B) == (512, 768, 8, 1, "relu", 64)
+        assert wl.dims == (8, w, w, w, 3)
+
+
 def test_generator_is_deterministic_and_bounded():
     a = wk.make_inputs("c1")
     b = wk.make_inputs("c1")
