@@ -36,8 +36,8 @@
 //                        while the tensor core runs the current tile's
 //                        second layer, and handed over once the current
 //                        accumulator has been read.
-//   warp 4*NWG         : issues every MMA (one elected lane) to whichever
-//                        group has its operand ready, then tcgen05.commit.
+//   warps 4*NWG + w    : group w's issuing warp (together one warpgroup, which
+//                        gives registers to the decoders): waits, issues, commits.
 // Handshakes are mbarriers; every wait is bounded (on timeout the kernel
 // raises the handle's status word, skips the rest and still frees TMEM).
 #pragma once
