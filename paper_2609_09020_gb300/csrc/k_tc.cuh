@@ -296,7 +296,7 @@ __device__ __forceinline__ void hidden_epilogue(uint32_t t_acc, uint32_t t_a) {
         a = gelu_poly(a);
         bb = gelu_poly(bb);
       }
-      // hi = fp16 truncation (ReLU folded in), lo = v - hi (packed subtraction)
+      // hi = fp16 truncation (ReLU folded in), lo = fp16 of v - hi (one mixed FMA)
       split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[8 + q]);
     }
     tmem_st8(t_a + h0 / 2, hl);
@@ -639,7 +639,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       {
         // --------------------------------------------------------------- MMA issuer
         // Warp MMA_WARP + w issues every MMA of group w, in the group's order
-        // (its tiles in turn, layers in turn), sleeping in the mbarrier wait
+        // (its tiles in turn, layers in turn), polling the group's mbarriers
         // in between.  The whole warp runs the control flow (descriptors stay
         // warp-uniform); one elected lane issues the MMAs and the commit.
         // Descriptors depend on the start address only through their low
