@@ -23,12 +23,15 @@
 //    c. an exclusive scan of the codeword counts gives every subsequence's
 //       output position (each image's must equal its symbol offset);
 //    d. every subsequence is decoded from its final start, writing values.
-// Each thread keeps a 64-bit window of the stream in registers and reloads
-// one word when its position crosses a word boundary (codes are at most 12
-// bits, so at most one word per codeword).  The counting decodes of a and b
-// use a pair table per image (the lengths of the first two codewords of
-// every p-bit window, when both lie inside it), so one lookup advances over
-// up to two codewords.
+// Each CTA stages its images' lookup tables and, per pass, the stream words
+// of its 256 subsequences in shared memory.  Each thread keeps a 64-bit
+// window of the stream in registers and reloads one word when its position
+// crosses a word boundary (codes are at most 12 bits, so at most one word per
+// codeword).  The counting decodes of a and b use a pair table per image (the
+// lengths of the first two codewords of every p-bit window, when both lie
+// inside it), so one lookup advances over up to two codewords.  The final
+// decode d writes through per-warp staging rows, 16 symbols per thread per
+// round, so that each warp store writes two whole 64-byte runs.
 #include <cstdint>
 
 #include <cooperative_groups.h>
