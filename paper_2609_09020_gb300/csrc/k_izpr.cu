@@ -8,15 +8,17 @@
 // 2. izpr_scan: one CTA, exclusive scan of the group counts; a chunk's
 //    first block = its group's base + its offset in the group.
 // 3. izpr_expand: persistent CTAs do the compaction and the expansion
-//    together, chunk by chunk.  Each thread holds 16 consecutive symbols of
-//    the chunk in registers (loaded while the CTA expanded its previous
-//    chunk), stores them to shared memory with the 96 symbols before the
+//    together, chunk by chunk, as a segmented scan.  Each thread holds 16
+//    consecutive symbols of the chunk in registers (loaded while the CTA
+//    expanded its previous chunk) and reduces them to (markers, positions
+//    covered since its last marker); warp 0 reads the 96 symbols before the
 //    chunk (a block has at most 64 symbols before its marker, so the marker
-//    ending the previous block is in that halo) and counts its markers; a
-//    CTA scan ranks them (their stream indices are Algorithm 1's offsets),
-//    and, as in Algorithm 1, one thread expands one block: literals go to
-//    the next zigzag position, a run code of n zeros skips n positions.  The
-//    blocks of a warp leave as whole 256-byte blocks in raster order.
+//    ending the previous block is in that halo); a CTA-wide scan gives each
+//    thread the block and zigzag position of its first symbol, and each
+//    thread walks its symbols as Algorithm 1 walks a block: a literal goes to
+//    the next zigzag position, a run code of n zeros skips n positions, a
+//    marker closes the block (its stream index is Algorithm 1's offset).  The
+//    blocks, assembled in shared memory, leave as whole 256-byte blocks.
 // The stream is read twice (steps 1 and 3); nothing else touches HBM but
 // the coefficients and offsets written.
 #include <cstdint>
