@@ -200,7 +200,7 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 // ---------------------------------------------------------------------------
-// Generic fallback: any dims up to kMaxDim, runtime loops, weights in shared
+// Generic kernel: any dims up to kMaxDim, runtime loops, weights in shared
 // memory in the nn.Linear layout.  Slower (hidden values in local memory) but
 // covers every arch the C ABI accepts.
 template <bool FL>
