@@ -170,3 +170,60 @@ def test_split_meets_the_bar_with_margin_on_a_full_image(orc):
     assert err_split < 2e-5                 # the bar is 4e-3
     assert err_plain > 1e-3                 # plain fp16: within 4x of the bar
     assert err_plain > 100 * err_split
+
+
+def e4m3(v):
+    """Round to nearest even onto the OCP fp8 e4m3 grid (3 mantissa bits,
+    normal exponents -6..8, subnormal spacing 2^-9), saturating at 448."""
+    v = np.asarray(v, dtype=np.float64)
+    a = np.abs(v)
+    e = np.clip(np.floor(np.log2(np.maximum(a, 2.0 ** -30))), -6, 8)
+    step = 2.0 ** (e - 3)
+    return np.sign(v) * np.minimum(np.round(a / step) * step, 448.0)
+
+
+def test_e4m3_grid():
+    got = e4m3(np.array([448.0, 500.0, 1.0625, 1.1875, 2.0 ** -9, 2.0 ** -10 * 1.01, 3.0 * 2.0 ** -9,
+                         -0.3]))
+    # 1.0625 is halfway between 1 and 1.125 (even: 1); 1.1875 between 1.125
+    # and 1.25 (even: 1.25); 0.3 lies between 0.28125 and 0.3125 (nearer 0.3125)
+    assert got.tolist() == [448.0, 448.0, 1.0, 1.25, 2.0 ** -9, 2.0 ** -9, 3.0 * 2.0 ** -9, -0.3125]
+
+
+def _fp8_lo_operand_layers(layers, sa=2.0 ** 10, sw=2.0 ** 4):
+    """The MLP with hidden-layer operands hi (fp16, RZ) + lo in e4m3 (scaled
+    by sa) against e4m3 weights (scaled by sw), the products unscaled by
+    1/(sa sw) -- what a block-scaled fp8 MMA for the lo term computes with
+    constant power-of-two scales; the first layer keeps the fp16 split."""
+    def run(F32):
+        h = F32
+        for k, (W, bias) in enumerate(layers):
+            if k == 0:
+                z = W @ _split_operand(h) + bias[:, None]
+            else:
+                hi = rz16(h.astype(np.float32))
+                lo = h.astype(np.float32) - hi.astype(np.float32)
+                z = (W @ hi.astype(np.float64)
+                     + (e4m3(W * sw) @ e4m3(lo.astype(np.float64) * sa)) / (sw * sa)
+                     + bias[:, None])
+            h = np.maximum(z, 0).astype(np.float32) if k < len(layers) - 1 else z
+        return np.clip(h, 0.0, 1.0)
+    return run
+
+
+def test_fp8_lo_term_stays_inside_the_bar(orc):
+    """The next step for the tensor path: the lo term in fp8 keeps the error
+    near 2e-4 on a full c5 image (2.1e-4), some 20x inside the 4e-3 bar and
+    13x below plain fp16."""
+    wl = wk.WORKLOADS["c5"]
+    x = wk.make_inputs(wl, batch=1)
+    ref = orc.decode(x.latents[0], x.steps[0], x.oracle_weights("fp16_tc")[0], wl.H, wl.W,
+                     wl.L, wl.C, wl.dims, wl.act, nthreads=4).reshape(3, -1)
+    F = _features(orc, x, 0)
+    layers = _layers(x.weights_for("fp16_tc")[0].astype(np.float64), wl.dims)
+    run = _fp8_lo_operand_layers(layers)
+    err = max(float(np.abs(run(F[:, p:p + 32768]) - ref[:, p:p + 32768]).max())
+              for p in range(0, F.shape[1], 32768))
+    err_split = _max_error(F, layers, _split_operand, ref)
+    err_plain = _max_error(F, layers, _plain_operand, ref)
+    assert err_split < err < 4e-4 and 10 * err < err_plain
