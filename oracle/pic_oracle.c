@@ -11,8 +11,8 @@
  *   1. dequantisation of the integer latent symbols of every pyramid level
  *      (Fig. 1: the decoder reconstructs real latents from quantised symbols):
  *          y_l[c][v][u] = q_l[c][v][u] * step_l
- *   2. upsampling of every level to H x W (Sec. 3.1, after Eq. 1: "y_hat is
- *      upsampled to y_u in R^{C x H x W}").  The paper does not name the
+ *   2. upsampling of every level to H x W (Sec. 3.1, after Eq. 1: the levels
+ *      of y_hat are brought to one grid, y_u in R^{C x H x W}).  The paper does not name the
  *      kernel; this oracle uses bilinear interpolation with half-pixel
  *      centres and edge clamping, the size-based scale W_l / W and H_l / H.
  *   3. per-pixel concatenation of all levels into the feature vector that
@@ -309,9 +309,10 @@ int pic_oracle_decode_pixels(const int32_t *latents, const double *steps, const 
 /* ------------------------------------------------------------------------
  * ZpR and its inverse (Sec. 3.3, Fig. 2; App. B, Algorithm 1).
  *
- * A block is 8 x 8 quantised DCT coefficients, row-major ("raster").  ZpR
- * reorders a block in zigzag order, trims its trailing zeros and codes every
- * run of zeros by run length ("partial RLE": only zeros are run-coded).
+ * A block is 8 x 8 quantised DCT coefficients, row-major (raster order).
+ * ZpR reorders a block in zigzag order, trims its trailing zeros and codes
+ * every run of zeros by its length (a partial run-length code: only zeros
+ * are run-coded).
  * The stream uses one end-of-block marker value eob, larger than every
  * literal by at least 17: the 16 values eob-16 .. eob-1 code runs of 1..16
  * zeros (code eob - 17 + n for a run of n), any smaller value is a literal
