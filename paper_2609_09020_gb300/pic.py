@@ -3,7 +3,8 @@
 Argument marshalling only: every step of the decode runs in the library's CUDA
 kernels.  The functions keep the C names; ``Decoder`` wraps a handle and
 accepts torch CUDA tensors (PyTorch supplies device memory and streams) or,
-for ``decode_batch_host``, host numpy arrays.
+for ``decode_batch_host``, host numpy arrays, and checks each buffer's size,
+contiguity and device before the call (the C ABI sees bare pointers).
 
 Loading fails loudly (ImportError/OSError) when the library has not been
 built; there is no CPU fallback.
