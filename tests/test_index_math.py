@@ -1,5 +1,6 @@
-"""Integer index arithmetic of the inverse DCT kernel, restated and checked
-on the CPU (no GPU).
+"""Integer index arithmetic of the upstream kernels, restated and checked on
+the CPU (no GPU): the inverse DCT's division by invariant integers and the
+inverse ZpR's segmented-scan operator.
 
 Patch -> (image, plane row) uses division by invariant integers (Granlund &
 Montgomery 1994): for 32-bit n and d, floor(n / d) = the high 64 bits of
@@ -47,3 +48,54 @@ def test_edges_and_random_32_bit():
         for n in ns:
             if 0 <= n < (1 << 32):
                 assert udiv(n, inv) == n // d, (n, d)
+
+
+# ---- the inverse ZpR's segmented scan ---------------------------------------
+# Each thread of the expansion kernel reduces its 16 symbols to (m, s): the
+# number of end-of-block markers and the zigzag positions covered since its
+# last marker (a literal covers 1, the run code eob - 17 + n covers n).  The
+# pairs combine as (m1, s1) . (m2, s2) = (m1 + m2, s2 if m2 > 0 else s1 + s2);
+# a parallel (Hillis-Steele) scan with this operator is only valid if it is
+# associative.
+
+
+def seg_cat(a, b):
+    return (a[0] + b[0], b[1] if b[0] > 0 else a[1] + b[1])
+
+
+def summarise(symbols, eob):
+    m, s = 0, 0
+    for x in symbols:
+        if x == eob:
+            m, s = m + 1, 0
+        else:
+            d = x - (eob - 16)
+            s += d + 1 if 0 <= d < 16 else 1
+    return m, s
+
+
+def test_segment_combine_is_associative():
+    dom = [(m, s) for m in range(3) for s in range(5)]
+    for a in dom:
+        for b in dom:
+            for c in dom:
+                assert seg_cat(seg_cat(a, b), c) == seg_cat(a, seg_cat(b, c))
+
+
+def test_parallel_scan_equals_a_sequential_walk():
+    eob = 272
+    rng = np.random.default_rng(5)
+    for trial in range(40):
+        n_thr, per = 128, 16
+        kinds = rng.random(n_thr * per)
+        sym = np.where(kinds < 0.06, eob,
+                       np.where(kinds < 0.25, rng.integers(eob - 16, eob, kinds.size),
+                                rng.integers(-255, 256, kinds.size)))
+        parts = [summarise(sym[t * per:(t + 1) * per], eob) for t in range(n_thr)]
+        inc = list(parts)
+        o = 1
+        while o < n_thr:  # Hillis-Steele inclusive scan, as the warp shuffles do
+            inc = [seg_cat(inc[t - o], inc[t]) if t >= o else inc[t] for t in range(n_thr)]
+            o *= 2
+        for t in range(n_thr):
+            assert inc[t] == summarise(sym[:(t + 1) * per], eob)
