@@ -1,6 +1,7 @@
 """Integer index arithmetic of the upstream kernels, restated and checked on
-the CPU (no GPU): the inverse DCT's division by invariant integers and the
-inverse ZpR's segmented-scan operator.
+the CPU (no GPU): the inverse DCT's division by invariant integers, the
+inverse ZpR's segmented-scan operator and the bound on the Huffman final
+decode's packed row offsets.
 
 Patch -> (image, plane row) uses division by invariant integers (Granlund &
 Montgomery 1994): for 32-bit n and d, floor(n / d) = the high 64 bits of
@@ -99,3 +100,42 @@ def test_parallel_scan_equals_a_sequential_walk():
             o *= 2
         for t in range(n_thr):
             assert inc[t] == summarise(sym[:(t + 1) * per], eob)
+
+
+# ---- the Huffman final decode's packed row descriptor -----------------------
+# In the final decode each lane of a warp decodes one subsequence (consecutive
+# subsequences on consecutive lanes) in rounds of up to 16 symbols; per round
+# one shuffle carries ((o + done) - (o_0 + done_0)) << 5 | cap for the row a
+# lane stores, o being the subsequence's output offset (an exclusive scan of
+# the codeword counts, at most 256 per 256-bit subsequence) and done the
+# symbols it has stored.  The offset must be non-negative and below 2^13
+# (27 bits would still fit; 13 is the claim the kernel's comment makes).
+
+
+def _rounds(counts, base=0):
+    o = base + np.concatenate([[0], np.cumsum(counts)[:-1]])
+    done = np.zeros_like(counts)
+    worst, lo = 0, 0
+    while np.any(done < counts):
+        n = np.minimum(16, counts - done)
+        rel = (o + done) - (o[0] + done[0])
+        active = n > 0
+        worst = max(worst, int(rel[active].max()))
+        lo = min(lo, int(rel.min()))
+        assert np.all(n <= 16) and np.all(n >= 0)
+        done += n
+    return worst, lo
+
+
+def test_row_offsets_fit_the_packed_descriptor():
+    rng = np.random.default_rng(9)
+    cases = [np.full(32, 256), np.zeros(32, np.int64), np.r_[np.zeros(31, np.int64), 256],
+             np.r_[1, np.full(31, 256)], np.r_[np.full(31, 256), 1]]
+    cases += [rng.integers(0, 257, 32) for _ in range(2000)]
+    cases += [np.where(rng.random(32) < 0.5, 0, rng.integers(200, 257, 32)) for _ in range(500)]
+    worst = 0
+    for c in cases:
+        w, lo = _rounds(np.asarray(c, np.int64), base=int(rng.integers(0, 1 << 40)))
+        assert lo >= 0
+        worst = max(worst, w)
+    assert worst <= 31 * 256 < 1 << 13
