@@ -1,7 +1,7 @@
 """Integer index arithmetic of the upstream kernels, restated and checked on
-the CPU (no GPU): the inverse DCT's division by invariant integers, the
-inverse ZpR's segmented-scan operator and the bound on the Huffman final
-decode's packed row offsets.
+the CPU (no GPU): the inverse DCT's division by invariant integers and its
+8-point butterfly, the inverse ZpR's segmented-scan operator and the bound
+on the Huffman final decode's packed row offsets.
 
 Patch -> (image, plane row) uses division by invariant integers (Granlund &
 Montgomery 1994): for 32-bit n and d, floor(n / d) = the high 64 bits of
@@ -10,6 +10,9 @@ n * inv with inv = ceil(2^64 / d), computed on the host as (2^64 - 1) // d + 1
 0 <= e < d, the product over 2^64 is n / d + n e / (d 2^64), and the error
 term is below 2^-32 <= 1/d, so it never crosses the next integer.
 """
+import os
+import re
+
 import numpy as np
 
 M64 = (1 << 64) - 1
@@ -139,3 +142,45 @@ def test_row_offsets_fit_the_packed_descriptor():
         assert lo >= 0
         worst = max(worst, w)
     assert worst <= 31 * 256 < 1 << 13
+
+
+# ---- the inverse DCT's 8-point butterfly -------------------------------------
+# The kernel's idct8 splits the orthonormal 8-point DCT-III into an even part
+# E (frequencies 0, 2, 4, 6) and an odd part O (1, 3, 5, 7) with
+# x[n] = E[n] + O[n] and x[7 - n] = E[n] - O[n], using the constants
+# 0.5 cos(k pi / 16).  Restated here in fp64 and compared with scipy's
+# orthonormal inverse DCT; the fp32 constants in the source are checked
+# against the cosines.
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _idct8_butterfly(X, C):
+    ee0, ee1 = C[4] * (X[0] + X[4]), C[4] * (X[0] - X[4])
+    eo0, eo1 = C[2] * X[2] + C[6] * X[6], C[6] * X[2] - C[2] * X[6]
+    e = [ee0 + eo0, ee1 + eo1, ee1 - eo1, ee0 - eo0]
+    o = [C[1] * X[1] + C[3] * X[3] + C[5] * X[5] + C[7] * X[7],
+         C[3] * X[1] - C[7] * X[3] - C[1] * X[5] - C[5] * X[7],
+         C[5] * X[1] - C[1] * X[3] + C[7] * X[5] + C[3] * X[7],
+         C[7] * X[1] - C[5] * X[3] + C[3] * X[5] - C[1] * X[7]]
+    x = np.empty(8)
+    for n in range(4):
+        x[n], x[7 - n] = e[n] + o[n], e[n] - o[n]
+    return x
+
+
+def test_butterfly_is_the_orthonormal_inverse_dct():
+    from scipy.fft import idct
+    C = [0.5 * np.cos(k * np.pi / 16) for k in range(8)]
+    rng = np.random.default_rng(3)
+    for X in list(np.eye(8)) + [rng.standard_normal(8) for _ in range(200)]:
+        assert np.allclose(_idct8_butterfly(X, C), idct(X, norm="ortho"), rtol=0, atol=1e-12)
+
+
+def test_source_constants_are_the_cosines():
+    src = open(os.path.join(ROOT, "paper_2609_09020_gb300", "csrc", "k_idct.cu")).read()
+    got = dict((int(k), float(v)) for k, v in re.findall(r"kC(\d) = ([0-9.e+-]+)f", src))
+    assert sorted(got) == list(range(1, 8))
+    for k, v in got.items():
+        assert np.float32(v) == np.float32(0.5 * np.cos(k * np.pi / 16)), k
+    assert np.float32(got[4]) == np.float32(1 / np.sqrt(8))  # a(0), the DC scale
