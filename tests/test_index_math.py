@@ -1,4 +1,4 @@
-"""Integer index arithmetic of the upstream kernels, restated and checked on
+"""Index and transform arithmetic of the upstream kernels, restated and checked on
 the CPU (no GPU): the inverse DCT's division by invariant integers and its
 8-point butterfly, the inverse ZpR's segmented-scan operator and the bound
 on the Huffman final decode's packed row offsets.
