@@ -26,6 +26,7 @@ def gpu_decode(wl: wk.Workload, x: wk.Inputs, precision: str, clamp: bool = True
         out = np.empty((B, 3, wl.H, wl.W), dtype=np.float32)
         dec.decode_batch_host(np.ascontiguousarray(x.latents), np.ascontiguousarray(x.steps),
                               np.ascontiguousarray(w), wl.H, wl.W, out)
+        dec.check()
         dec.close()
         return out
     dev = torch.device("cuda:0")
