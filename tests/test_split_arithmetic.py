@@ -190,31 +190,36 @@ def test_e4m3_grid():
     assert got.tolist() == [448.0, 448.0, 1.0, 1.25, 2.0 ** -9, 2.0 ** -9, 3.0 * 2.0 ** -9, -0.3125]
 
 
-def _fp8_lo_operand_layers(layers, sa=2.0 ** 10, sw=2.0 ** 4):
-    """The MLP with hidden-layer operands hi (fp16, RZ) + lo in e4m3 (scaled
-    by sa) against e4m3 weights (scaled by sw), the products unscaled by
-    1/(sa sw) -- what a block-scaled fp8 MMA for the lo term computes with
-    constant power-of-two scales; the first layer keeps the fp16 split."""
+def _fp8_lo_operand_layers(layers, S=2.0 ** 8):
+    """The MLP as a tensor path with the lo term in fp8 would compute it.
+    Hidden activations stay scaled by S (ReLU commutes with a positive
+    scale): the hidden operand is hi = RZ16(S h) in fp16 against the fp16
+    weights W, plus lo = e4m3(S h - hi) against e4m3(W) (S h - hi is about
+    2^-11 S h, inside e4m3's normal range for S = 2^8, and exact in fp32);
+    the bias rows carry S b, the first layer's weights S W (exact: S is a
+    power of two), and only the 3 outputs are divided by S.  No rescaling
+    of the hidden values is needed, so the epilogue keeps its instruction
+    count; the lo MMAs take half the K-steps (32 e4m3 per step)."""
     def run(F32):
         h = F32
         for k, (W, bias) in enumerate(layers):
             if k == 0:
-                z = W @ _split_operand(h) + bias[:, None]
+                z = S * (W @ _split_operand(h)) + S * bias[:, None]
             else:
-                hi = rz16(h.astype(np.float32))
-                lo = h.astype(np.float32) - hi.astype(np.float32)
-                z = (W @ hi.astype(np.float64)
-                     + (e4m3(W * sw) @ e4m3(lo.astype(np.float64) * sa)) / (sw * sa)
-                     + bias[:, None])
-            h = np.maximum(z, 0).astype(np.float32) if k < len(layers) - 1 else z
+                hs = h.astype(np.float32)          # already scaled by S
+                assert np.abs(hs).max() < 65504
+                hi = rz16(hs)
+                lo = (hs - hi.astype(np.float32)).astype(np.float64)
+                z = W @ hi.astype(np.float64) + e4m3(W) @ e4m3(lo) + S * bias[:, None]
+            h = np.maximum(z, 0).astype(np.float32) if k < len(layers) - 1 else z / S
         return np.clip(h, 0.0, 1.0)
     return run
 
 
 def test_fp8_lo_term_stays_inside_the_bar(orc):
     """The next step for the tensor path: the lo term in fp8 keeps the error
-    near 2e-4 on a full c5 image (2.1e-4), some 20x inside the 4e-3 bar and
-    13x below plain fp16."""
+    near 2e-4 on a full c5 image (2.2e-4), some 20x inside the 4e-3 bar and
+    12x below plain fp16."""
     wl = wk.WORKLOADS["c5"]
     x = wk.make_inputs(wl, batch=1)
     ref = orc.decode(x.latents[0], x.steps[0], x.oracle_weights("fp16_tc")[0], wl.H, wl.W,
