@@ -160,3 +160,20 @@ def test_fma_peak_helper_without_gpu(lib):
     assert pic.load_library().pic_fma_peak_flops(1, 0) == -1
     assert pic.load_library().pic_fma_peak_flops(2, 3) == 2 * 256 * 3 * 16 * 8 * 2
     assert pic.load_library().pic_fma_peak_launch(None, 1, 1, None) == pic.PIC_ERR_INVALID_ARG
+
+
+def test_noalloc_entry_and_size_helpers_reject_bad_arguments(lib):
+    """pic_decode_batch_noalloc validates the arch before touching a device;
+    the size helpers answer -1 outside their domain."""
+    from paper_2609_09020_gb300 import pic
+    p = ctypes.c_void_p(256)
+    assert lib.pic_decode_batch_noalloc(None, 1, p, p, p, 8, 8, p, None) == pic.PIC_ERR_INVALID_ARG
+    bad = pic.make_arch(2, 1, (3, 8, 3), max_H=8, max_W=8)           # dims[0] != L*C
+    assert lib.pic_decode_batch_noalloc(ctypes.byref(bad), 1, p, p, p, 8, 8, p,
+                                        None) == pic.PIC_ERR_INVALID_ARG
+    wide = pic.make_arch(2, 1, (2, 256, 3), max_H=8, max_W=8)        # width above the envelope
+    assert lib.pic_decode_batch_noalloc(ctypes.byref(wide), 1, p, p, p, 8, 8, p,
+                                        None) == pic.PIC_ERR_UNSUPPORTED
+    assert lib.pic_param_count(None) == -1
+    assert pic.pic_latent_count(8, 8, 31, 1) == -1 and pic.pic_latent_count(8, 8, 1, 0) == -1
+    assert pic.pic_latent_count(1, 1, 30, 4) == 30 * 4   # every level of a 1x1 image is 1x1
