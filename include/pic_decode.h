@@ -127,7 +127,8 @@ int pic_decode_create(const pic_arch *arch, pic_decoder **out);
  *             planar [3][H][W] (R, G, B planes), fp32 [H][W][3], or uint8
  *             [H][W][3].
  * Errors: PIC_ERR_INVALID_ARG (NULL handle/pointer, misaligned pointer, H or W
- * out of range) with nothing launched; PIC_ERR_CUDA if the launch failed.
+ * out of range, or the current device is not the one the handle was created
+ * on) with nothing launched; PIC_ERR_CUDA if the launch failed.
  */
 int pic_decode(pic_decoder *h, const int32_t *latents, const float *steps, const void *weights,
                int H, int W, void *out_rgb, void *stream);
@@ -168,27 +169,46 @@ int pic_decode_batch_host(pic_decoder *h, int B, const int32_t *latents, const f
 int pic_decode_check(pic_decoder *h, void *stream);
 
 /*
- * Allocation-free decode (no counterpart in the paper; an interface for
- * callers that may not allocate device memory: code inside a CUDA-graph
- * stream capture, real-time or serving loops whose memory is fixed up front,
- * embedders that forbid the library from touching the allocator).
+ * Allocation-free decode (no counterpart in the paper).  For callers that
+ * cannot call cudaMalloc: a plug-in whose host application hands out all
+ * device memory from its own pool, a real-time loop that cannot accept
+ * cudaMalloc's implicit device synchronisation and unbounded latency, a
+ * service whose memory budget is fixed before it starts.
  * Same decode, layouts and argument rules as pic_decode_batch, with the
  * architecture passed directly instead of a handle (arch->max_H, max_W and
- * max_batch bound H, W and B as for a handle).  It allocates nothing: the
- * only global memory it uses besides the caller's buffers is a 256-byte
- * static device array built into the library (one status word of it per
- * call; calls needing more are refused), held by every GPU that loads the
- * library until the process exits.  The first call on a device looks up
- * that array's device address (make it before any stream capture); each
- * call clears the status word on `stream` first.  All calls share the
- * array, so calls that overlap on the GPU (different streams, no ordering)
- * race on it; a bounded wait that gives up in such a call is not reported.
+ * max_batch bound H, W and B as for a handle).  The caller passes inputs and
+ * outputs; the call allocates nothing (no cudaMalloc, no cudaFree, no
+ * allocating library routine).  The only global memory it uses besides the
+ * caller's buffers is a 256-byte static device array built into the library,
+ * which every GPU that loads the library holds until the process exits: one
+ * status word of it per device (a call that would need more is refused).
+ * The first call on a device, with that device current, looks up the
+ * array's device address, the device's capabilities and the kernel's launch
+ * attributes, and caches them; make that first call before any stream
+ * capture.
+ * The status word is zero when the library loads and is raised (never
+ * cleared) by a call in which a bounded device-side wait gives up; it stays
+ * raised until pic_decode_noalloc_check reads and clears it.  All calls on a
+ * device share the word, so a raised word says that some call since the
+ * last check gave up, not which one, and calls that overlap on the GPU
+ * (different streams, no ordering between them) race with a concurrent
+ * check's clear.
  * Errors: as pic_decode_batch (PIC_ERR_INVALID_ARG, PIC_ERR_UNSUPPORTED,
  * PIC_ERR_CUDA); nothing is launched on an argument error.
  */
 int pic_decode_batch_noalloc(const pic_arch *arch, int B, const int32_t *latents,
                              const float *steps, const void *weights, int H, int W,
                              void *out_rgb, void *stream);
+
+/*
+ * Status of the allocation-free calls on the current device (no counterpart
+ * in the paper): synchronises `stream`, then returns PIC_ERR_TIMEOUT if a
+ * bounded device-side wait gave up in any pic_decode_batch_noalloc call on
+ * this device since the last check (and clears the word, on `stream`), else
+ * PIC_OK.  Allocates nothing.
+ * Errors: PIC_ERR_CUDA.
+ */
+int pic_decode_noalloc_check(void *stream);
 
 /* Frees the handle and its device state.  NULL is a no-op.  Synchronises the
  * device first, so that no kernel of this handle is still running. */

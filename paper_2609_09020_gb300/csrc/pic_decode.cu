@@ -4,6 +4,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 #include <new>
 
 #include <cuda_runtime.h>
@@ -77,6 +78,14 @@ int check_decode_args(const pic_decoder* h, int B, const int32_t* latents, const
   if (H < 1 || W < 1 || H > h->arch.max_H || W > h->arch.max_W) return PIC_ERR_INVALID_ARG;
   if (!aligned(latents, 16) || !aligned(weights, 16) || !aligned(out, 16) || !aligned(steps, 4))
     return PIC_ERR_INVALID_ARG;
+  // The kernel would run on the current device with the handle's setup (and,
+  // for a handle, its status word) from another: refuse instead.
+  int cur = -1;
+  if (cudaGetDevice(&cur) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  if (cur != h->device) return PIC_ERR_INVALID_ARG;
   return PIC_OK;
 }
 
@@ -432,27 +441,46 @@ const char* pic_decode_kernel_name(const pic_decoder* h) { return h ? h->kern.na
 // ---------------------------------------------------------------------------
 // Allocation-free entry point.
 //
-// Some callers cannot allocate device memory at all: code running while a
-// stream is being captured into a CUDA graph (cudaMalloc is not capturable),
-// real-time or serving loops whose memory is fixed up front by a pool the
-// library must not bypass, and embedders that forbid the library from
-// touching the device allocator.  pic_decode_create() allocates (the
+// Some callers cannot call cudaMalloc: a plug-in inside a host application
+// that hands out all device memory from its own pool and forbids any other
+// allocation, a real-time loop that cannot accept cudaMalloc's implicit
+// device synchronisation and unbounded latency, or a service whose memory
+// budget is fixed before it starts.  pic_decode_create() allocates (the
 // handle's status word), so those callers use pic_decode_batch_noalloc()
 // instead.  It runs the same kernels; the only global memory it needs beyond
 // the caller's inputs and outputs -- the status word that a bounded wait in
 // the tensor-core kernel raises when it gives up -- lives in the static
 // device array below, which every GPU that loads this library holds until
-// the process exits.
+// the process exits.  A device global is zero when the module loads, so the
+// word starts at zero; pic_decode_noalloc_check() reads and clears it.
 namespace {
 
 constexpr int kStaticScratchInts = 64;  // 256 bytes; one call needs 1 word
 constexpr int kMaxStaticDevices = 64;
+constexpr int kNoallocKernelCache = 32;  // (device, kernel) pairs remembered
 
-struct StaticScratchSlot {
-  int ready;  // 0: not set up, 1: ok, -1: cudaGetSymbolAddress failed
-  int* ptr;   // device address of g_static_scratch on that device
+// What one device needs looked up once: its capabilities and the device
+// address of the static scratch (the array's name is only a host-side
+// stand-in).  Only successful look-ups are kept, so a failed first try
+// (no context yet, say) is retried by the next call.
+struct NoallocDevice {
+  bool ready;
+  int major, minor, sms, smem_optin;
+  int* scratch;
 };
-StaticScratchSlot g_static_slots[kMaxStaticDevices];
+// Per (device, kernel): the shared-memory attribute is set and the
+// occupancy and register count were read.
+struct NoallocKernel {
+  int dev;
+  const void* fn;
+  int per_sm;
+  bool regs_ok;
+};
+
+std::mutex g_noalloc_mutex;
+NoallocDevice g_noalloc_dev[kMaxStaticDevices];
+NoallocKernel g_noalloc_kern[kNoallocKernelCache];
+int g_noalloc_nkern = 0;
 
 }  // namespace
 
@@ -460,25 +488,58 @@ static __device__ __align__(256) int g_static_scratch[kStaticScratchInts];
 
 namespace {
 
-// Device address of the static scratch on `dev` (which is current).  The
-// array's name is only a host-side stand-in, so the address is looked up
-// once per device and cached.  Not thread-safe on the very first call per
-// device (two threads may both look it up; both get the same address).
-int static_scratch(int dev, int** out) {
+// Device facts and the static scratch address of `dev` (current), cached.
+int noalloc_device(int dev, NoallocDevice* out) {
   if (dev < 0 || dev >= kMaxStaticDevices) return PIC_ERR_UNSUPPORTED;
-  StaticScratchSlot& s = g_static_slots[dev];
-  if (s.ready == 0) {
+  std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+  NoallocDevice& d = g_noalloc_dev[dev];
+  if (!d.ready) {
+    NoallocDevice t{};
     void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr) {
+    if (cudaDeviceGetAttribute(&t.major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&t.minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&t.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&t.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+            cudaSuccess ||
+        cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr) {
       cudaGetLastError();
-      s.ready = -1;
-    } else {
-      s.ptr = static_cast<int*>(p);
-      s.ready = 1;
+      return PIC_ERR_CUDA;
+    }
+    t.scratch = static_cast<int*>(p);
+    t.ready = true;
+    d = t;
+  }
+  *out = d;
+  return PIC_OK;
+}
+
+// Occupancy of kernel `k` on `dev` (current), after setting its shared-memory
+// attribute; both done once per (device, kernel).
+int noalloc_kernel(int dev, const KernelInfo& k, int* per_sm) {
+  std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+  for (int i = 0; i < g_noalloc_nkern; ++i)
+    if (g_noalloc_kern[i].dev == dev && g_noalloc_kern[i].fn == k.fn) {
+      if (!g_noalloc_kern[i].regs_ok) return PIC_ERR_UNSUPPORTED;
+      *per_sm = g_noalloc_kern[i].per_sm;
+      return PIC_OK;
+    }
+  NoallocKernel e{dev, k.fn, 0, regs_match(k)};
+  if (e.regs_ok) {
+    if (cudaFuncSetAttribute(k.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, k.smem_bytes) !=
+        cudaSuccess) {
+      cudaGetLastError();
+      return PIC_ERR_CUDA;
+    }
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&e.per_sm, k.fn, k.threads, k.smem_bytes) !=
+            cudaSuccess ||
+        e.per_sm < 1) {
+      cudaGetLastError();
+      return PIC_ERR_UNSUPPORTED;
     }
   }
-  if (s.ready != 1) return PIC_ERR_CUDA;
-  *out = s.ptr;
+  if (g_noalloc_nkern < kNoallocKernelCache) g_noalloc_kern[g_noalloc_nkern++] = e;
+  if (!e.regs_ok) return PIC_ERR_UNSUPPORTED;
+  *per_sm = e.per_sm;
   return PIC_OK;
 }
 
@@ -503,16 +564,10 @@ extern "C" int pic_decode_batch_noalloc(const pic_arch* arch, int B, const int32
     cudaGetLastError();
     return PIC_ERR_UNSUPPORTED;
   }
-  int major = 0, minor = 0, sms = 0, smem_optin = 0;
-  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
-          cudaSuccess) {
-    cudaGetLastError();
-    return PIC_ERR_CUDA;
-  }
-  if (major != 10 || minor != 3) return PIC_ERR_UNSUPPORTED;
+  NoallocDevice d{};
+  int rc = noalloc_device(dev, &d);
+  if (rc != PIC_OK) return rc;
+  if (d.major != 10 || d.minor != 3) return PIC_ERR_UNSUPPORTED;
 
   // The same kernel selection as pic_decode_create, on a handle that lives
   // on this stack frame.
@@ -527,7 +582,7 @@ extern "C" int pic_decode_batch_noalloc(const pic_arch* arch, int B, const int32
   pic_decoder h{};
   h.arch = *arch;
   h.device = dev;
-  h.sm_count = sms;
+  h.sm_count = d.sms;
   if (chosen) {
     h.kern = *chosen;
   } else if (arch->precision == PIC_PREC_FP32) {
@@ -536,36 +591,42 @@ extern "C" int pic_decode_batch_noalloc(const pic_arch* arch, int B, const int32
   } else {
     return PIC_ERR_UNSUPPORTED;
   }
-  if (h.kern.smem_bytes > smem_optin) return PIC_ERR_UNSUPPORTED;
-  if (!regs_match(h.kern)) return PIC_ERR_UNSUPPORTED;
-  if (cudaFuncSetAttribute(h.kern.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           h.kern.smem_bytes) != cudaSuccess) {
-    cudaGetLastError();
-    return PIC_ERR_CUDA;
-  }
-  int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, h.kern.fn, h.kern.threads,
-                                                    h.kern.smem_bytes) != cudaSuccess ||
-      per_sm < 1) {
-    cudaGetLastError();
-    return PIC_ERR_UNSUPPORTED;
-  }
-  h.grid_cap = per_sm * sms;
-  h.n_params = pic_param_count(arch);
-
-  int* scratch = nullptr;
-  int rc = static_scratch(dev, &scratch);
-  if (rc != PIC_OK) return rc;
-  h.d_status = scratch;
-
+  if (h.kern.smem_bytes > d.smem_optin) return PIC_ERR_UNSUPPORTED;
   rc = check_decode_args(&h, B, latents, steps, weights, H, W, out_rgb);
   if (rc != PIC_OK) return rc;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(scratch, 0, kNeededInts * sizeof(int), s) != cudaSuccess) {  // starts at zero
+  int per_sm = 0;
+  rc = noalloc_kernel(dev, h.kern, &per_sm);
+  if (rc != PIC_OK) return rc;
+  h.grid_cap = per_sm * d.sms;
+  h.n_params = pic_param_count(arch);
+  h.d_status = d.scratch;
+
+  DecodeParams p;
+  fill_params(&h, p, B, latents, steps, weights, H, W, out_rgb);
+  return launch(&h, p, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" int pic_decode_noalloc_check(void* stream) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
     cudaGetLastError();
     return PIC_ERR_CUDA;
   }
-  DecodeParams p;
-  fill_params(&h, p, B, latents, steps, weights, H, W, out_rgb);
-  return launch(&h, p, s);
+  NoallocDevice d{};
+  int rc = noalloc_device(dev, &d);
+  if (rc != PIC_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int flag = 0;
+  if (cudaMemcpyAsync(&flag, d.scratch, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  if (flag == 0) return PIC_OK;
+  if (cudaMemsetAsync(d.scratch, 0, sizeof(int), s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return PIC_ERR_CUDA;
+  }
+  return PIC_ERR_TIMEOUT;
 }

@@ -87,6 +87,8 @@ def load_library():
     lib.pic_decode_batch_host.restype = i
     lib.pic_decode_batch_noalloc.argtypes = [ctypes.POINTER(pic_arch), i, _P, _P, _P, i, i, _P, _P]
     lib.pic_decode_batch_noalloc.restype = i
+    lib.pic_decode_noalloc_check.argtypes = [_P]
+    lib.pic_decode_noalloc_check.restype = i
     lib.pic_decode_check.argtypes = [_P, _P]
     lib.pic_decode_check.restype = i
     lib.pic_decode_destroy.argtypes = [_P]
@@ -174,6 +176,10 @@ def pic_decode_batch_noalloc(arch: pic_arch, B, latents, steps, weights, H, W, o
                              stream=None) -> int:
     return load_library().pic_decode_batch_noalloc(ctypes.byref(arch), B, latents, steps, weights,
                                                    H, W, out_rgb, stream)
+
+
+def pic_decode_noalloc_check(stream=None) -> int:
+    return load_library().pic_decode_noalloc_check(stream)
 
 
 def pic_decode_check(h, stream=None) -> int:
@@ -372,12 +378,13 @@ def decode_buffer_bytes(arch: pic_arch, B, H, W) -> dict:
     }
 
 
-def check_decode_buffers(need: dict, B, H, W, host=False, **bufs):
+def check_decode_buffers(need: dict, B, H, W, host=False, device=None, **bufs):
     """Raises ValueError unless every named buffer (latents, steps, weights,
     out: torch tensors, or numpy arrays on the host path) is contiguous,
-    lives on the device (host=False) or the host (host=True), and holds at
-    least ``need[name]`` bytes.  A missing (None) buffer passes only where
-    the call does not read it."""
+    lives on the device (host=False; on CUDA device index ``device`` when
+    that is given) or the host (host=True), and holds at least
+    ``need[name]`` bytes.  A missing (None) buffer passes only where the call
+    does not read it."""
     for name, a in bufs.items():
         if a is None:
             if name != "steps" or need[name] > 0:
@@ -391,6 +398,9 @@ def check_decode_buffers(need: dict, B, H, W, host=False, **bufs):
             raise ValueError(f"{name}: must be contiguous")
         if on_gpu == host:
             raise ValueError(f"{name}: must be a {'host' if host else 'CUDA'} buffer")
+        if on_gpu and device is not None and a.device.index != device:
+            raise ValueError(f"{name}: on cuda:{a.device.index}, but the decoder was created "
+                             f"on cuda:{device}")
         if nbytes < need[name]:
             raise ValueError(f"{name}: holds {nbytes} bytes; a {B}-image {H}x{W} call needs "
                              f"{need[name]}")
@@ -418,6 +428,8 @@ class Decoder:
         self.L, self.C, self.dims, self.precision = L, C, tuple(dims), precision
         self._need = {}
         self.handle = pic_decode_create(self.arch)
+        import torch
+        self.device = torch.cuda.current_device()  # the handle's device (current at create)
 
     @classmethod
     def for_workload(cls, wl, precision: str, clamp=True, max_batch=None, latent="int32",
@@ -456,7 +468,8 @@ class Decoder:
         return need
 
     def check_buffers(self, B, H, W, host=False, **bufs):
-        check_decode_buffers(self.buffer_bytes(B, H, W), B, H, W, host, **bufs)
+        check_decode_buffers(self.buffer_bytes(B, H, W), B, H, W, host,
+                             None if host else self.device, **bufs)
 
     def decode_batch(self, latents, steps, weights, H, W, out, stream=None, B=None, check=True):
         """Enqueues a batch decode; arguments are torch CUDA tensors.  With

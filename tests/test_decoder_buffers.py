@@ -17,8 +17,9 @@ def pic():
 class _FakeCuda:
     """Stands in for a CUDA tensor: only the metadata the checks read."""
 
-    def __init__(self, nbytes, contiguous=True):
+    def __init__(self, nbytes, contiguous=True, index=0):
         self._n, self._c, self.is_cuda = nbytes, contiguous, True
+        self.device = torch.device("cuda", index)
 
     def numel(self):
         return self._n
@@ -87,3 +88,17 @@ def test_host_path_takes_host_buffers(pic):
     with pytest.raises(ValueError, match="weights"):
         pic.check_decode_buffers(need, 1, 2, 2, host=True,
                                  **{**host, "weights": np.zeros(7, np.float32)})
+
+
+def test_device_buffers_must_be_on_the_decoders_gpu(pic):
+    """A tensor on another GPU than the handle's would be launched on with the
+    handle's setup: the wrapper refuses it (the C ABI refuses a call made
+    while another device is current)."""
+    need = {"latents": 64, "steps": 16, "weights": 32, "out": 48}
+    ok = {k: _FakeCuda(v, index=1) for k, v in need.items()}
+    pic.check_decode_buffers(need, 1, 2, 2, device=1, **ok)
+    pic.check_decode_buffers(need, 1, 2, 2, **ok)  # no device given: not checked
+    for name in need:
+        with pytest.raises(ValueError, match="cuda:0"):
+            pic.check_decode_buffers(need, 1, 2, 2, device=1,
+                                     **{**ok, name: _FakeCuda(need[name], index=0)})

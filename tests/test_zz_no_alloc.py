@@ -1,14 +1,16 @@
 """The allocation-free entry point, pic_decode_batch_noalloc.
 
-Callers that may not allocate device memory (inside a CUDA-graph stream
-capture, in serving loops whose memory is fixed up front, or in embedders
-that forbid the library from touching the allocator) decode through this
-entry point: it takes the architecture instead of a handle and keeps its
-only scratch -- the status word of the bounded waits -- in a static device
-array of the library.  Its output must match the handle-based
-pic_decode_batch within the tolerance of the other parity tests, on two
-calls in a row (the second call reuses the static array the first one left
-behind).
+Some callers cannot call cudaMalloc: a plug-in whose host application owns
+all device memory, a real-time loop that cannot take cudaMalloc's implicit
+device synchronisation, a service whose memory is fixed before it starts.
+They decode through this entry point: it takes the architecture instead of a
+handle and keeps its only scratch -- the status word of the bounded waits --
+in a static device array of the library, read and cleared by
+pic_decode_noalloc_check.  It launches the same kernel as the handle-based
+pic_decode_batch on the same inputs, so its output must equal that call's
+bit for bit, on two calls in a row (the second call reuses the static array
+the first one left behind), and the status read must report no wait that
+gave up.
 
 The file name makes pytest collect it last.
 """
@@ -17,7 +19,6 @@ import pytest
 
 from paper_2609_09020_gb300 import workloads as wk
 
-from decode_util import TOL, max_abs_diff
 
 pytestmark = pytest.mark.gpu
 
@@ -57,14 +58,16 @@ def test_noalloc_matches_handle_entry_point(wl, precision):
     dec.close()
 
     arch = pic.make_arch(wl.L, wl.C, wl.dims, wl.act, precision, True, wl.H, wl.W, B)
+    want = ref.cpu().numpy()
     for call in range(2):
         out = torch.full((B, 3, wl.H, wl.W), float("nan"), device=dev)
         rc = pic.pic_decode_batch_noalloc(arch, B, lat.data_ptr(), st.data_ptr(), w.data_ptr(),
                                           wl.H, wl.W, out.data_ptr(), stream)
         assert rc == pic.PIC_OK, (call, pic.pic_status_string(rc))
-        torch.cuda.synchronize()
-        d, where = max_abs_diff(out.cpu().numpy(), ref.cpu().numpy().astype(np.float64))
-        assert d <= TOL[precision], (call, d, where)
+        rc = pic.pic_decode_noalloc_check(stream)
+        assert rc == pic.PIC_OK, (call, pic.pic_status_string(rc))
+        got = out.cpu().numpy()
+        assert np.array_equal(got, want), (call, float(np.nanmax(np.abs(got - want))))
 
 
 def test_noalloc_rejects_bad_arguments():
