@@ -66,6 +66,92 @@ def algorithmic(wl: wk.Workload, batch: int):
     return flops, nbytes
 
 
+# FP32-pipe operations of one GELU evaluation in the kernels (pic_gelu.cuh):
+# z^2, the affine map, the Horner steps, the saturating fma and z * Phi.
+GELU_FP32_OPS = 4 + 12
+
+
+def executed_tensor_macs_per_px(wl: wk.Workload) -> int:
+    """MACs the tensor cores execute per pixel: layer 0 (K = round16(2 D0 + 1),
+    N = round16 of the width), hidden layers and (for wide, shallow nets) the
+    output layer (N = 16), with the hi and lo halves of K plus one K = 16 bias
+    step each."""
+    def r16(v):
+        return (v + 15) // 16 * 16
+    n_pad = r16(max(wl.dims[1:-1]))
+    mac = r16(2 * wl.dims[0] + 1) * n_pad
+    mac += (len(wl.dims) - 3) * (2 * n_pad + 16) * n_pad
+    if tc_output_on_tensor_cores(wl):
+        mac += (2 * n_pad + 16) * 16
+    return mac
+
+
+def tc_output_on_tensor_cores(wl: wk.Workload) -> bool:
+    """The tensor path runs the output layer as an MMA only for wide, shallow
+    nets (padded width > 32 and fewer than 4 layers); else on the CUDA cores."""
+    n_pad = (max(wl.dims[1:-1]) + 15) // 16 * 16
+    return n_pad > 32 and len(wl.dims) - 1 < 4
+
+
+def alu_ops_per_px(wl: wk.Workload, precision: str) -> int:
+    """Activation-inclusive CUDA-core work per pixel (FP32-pipe operations):
+    every hidden activation (GELU at GELU_FP32_OPS; ReLU is folded into a
+    conversion), plus on the tensor path the hi/lo split of every hidden value
+    that feeds an MMA (2 per value) and the output layer where it runs on the
+    CUDA cores (one FMA per weight), plus on the fp32 path every MLP MAC."""
+    hidden = list(wl.dims[1:-1])
+    act = GELU_FP32_OPS if wl.act == "gelu" else 0
+    ops = act * sum(hidden)
+    if precision == "fp16_tc":
+        if tc_output_on_tensor_cores(wl):
+            ops += 2 * sum(hidden)
+        else:
+            ops += 2 * sum(hidden[:-1]) + 3 * hidden[-1]
+    else:
+        ops += wl.macs_per_pixel
+    return ops
+
+
+def roofline_for(wl: wk.Workload, precision: str, B: int, ms: float, peaks: dict,
+                 fp32_tflops: float, fp32_src: str) -> dict:
+    """The roofline of one decode launch of B images that took ms: the binding
+    of (unpadded MLP FLOPs at the path's pipe peak, algorithmic bytes at the
+    HBM peak), and beside it the activation-inclusive ALU bound."""
+    flops, nbytes = algorithmic(wl, B)
+    t_s = ms * 1e-3
+    px = B * wl.H * wl.W
+    if precision == "fp16_tc":
+        peak_tf = peaks["bf16_tflops"]  # fp16 dense tensor rate = bf16 rate
+        roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": peak_tf,
+                "unit": "TFLOP/s", "peak_source": f"bf16 dense burst, {peaks['source']}"}
+    else:
+        peak_tf = fp32_tflops
+        roof = {"bound": "alu", "achieved": flops / t_s / 1e12, "peak": peak_tf,
+                "unit": "TFLOP/s", "peak_source": fp32_src}
+    t_pipe = flops / (peak_tf * 1e12)
+    t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
+    if t_hbm > t_pipe:
+        roof.update({"bound": "hbm", "achieved": nbytes / t_s / 1e9, "peak": peaks["hbm_gbs"],
+                     "unit": "GB/s", "peak_source": f"copy bandwidth, {peaks['source']}"})
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["algorithmic_flops_per_launch"] = flops
+    if precision == "fp16_tc":
+        roof["executed_tensor_flops_per_launch"] = 2.0 * executed_tensor_macs_per_px(wl) * px
+    roof["algorithmic_bytes_per_launch"] = nbytes
+    roof["binding_time_us"] = max(t_pipe, t_hbm) * 1e6
+    roof["avg_launch_us"] = ms * 1e3
+    # activation-inclusive ALU bound (FP32 pipe at the measured FMA rate;
+    # one operation = one lane-op, half an FMA's two FLOPs)
+    ops = alu_ops_per_px(wl, precision)
+    t_alu = ops * px / (fp32_tflops * 1e12 / 2)
+    t_bind = max(t_pipe, t_hbm, t_alu)
+    roof["alu_bound"] = {"ops_per_px": ops,
+                         "gelu_evals_per_launch": px * sum(wl.dims[1:-1]) if wl.act == "gelu" else 0,
+                         "t_alu_us": t_alu * 1e6, "binding_time_incl_alu_us": t_bind * 1e6,
+                         "frac_incl_alu": t_bind / t_s}
+    return roof
+
+
 KERNEL_SOURCES = {
     "idct": ["k_idct.cu"],
     "izpr": ["k_izpr.cu"],
@@ -794,6 +880,73 @@ def run_stage(args):
         dec.close()
 
 
+def fp32_peak(pic, dev):
+    """The FP32 FMA rate (TFLOP/s) of this GPU from the library's FMA
+    microbenchmark, else the formula; and a note saying which."""
+    try:
+        tf = pic.fma_peak_tflops(dev)
+        return tf, (f"FP32 FMA microbenchmark, measured (formula: {fp32_peak_tflops():.1f} "
+                    f"TFLOP/s = 152 SMs x 128 lanes x 2 FLOP x 2070 MHz)")
+    except Exception as exc:  # report the formula instead of failing the bench
+        return fp32_peak_tflops(), (f"FP32 FMA formula (152 SMs x 128 lanes x 2 FLOP x 2070 MHz; "
+                                    f"microbenchmark failed: {exc})")
+
+
+PER_CONFIG = ["c1", "c2", "c3", "c4", "c5"]
+
+
+def per_config_rows(pic, dev, stream, peaks, fp32_tf, fp32_src, reps=None):
+    """Every workload on both decoder paths, one row each: the median over
+    timed calls of one decode launch, each call preceded by a 256 MB write
+    that flushes L2 (the small workloads' inputs fit in L2), CUDA events on
+    the launching stream around the decode alone."""
+    import torch
+    flush = torch.empty(64 << 20, dtype=torch.float32, device=dev)  # 256 MB > L2
+    rows = []
+    for name in PER_CONFIG:
+        wl = wk.WORKLOADS[name]
+        x = wk.make_inputs(wl)
+        B = x.latents.shape[0]
+        lat = torch.from_numpy(x.latents).to(dev)
+        st = torch.from_numpy(x.steps).to(dev)
+        out = torch.empty((B, 3, wl.H, wl.W), dtype=torch.float32, device=dev)
+        for precision in ("fp16_tc", "fp32"):
+            w = torch.from_numpy(np.ascontiguousarray(x.weights_for(precision))).to(dev)
+            dec = pic.Decoder.for_workload(wl, precision, max_batch=B)
+            dec.check_buffers(B, wl.H, wl.W, latents=lat, steps=st, weights=w, out=out)
+            for _ in range(3):
+                dec.decode_batch(lat, st, w, wl.H, wl.W, out, stream=stream, B=B, check=False)
+            torch.cuda.synchronize(dev)
+            n = reps or (30 if wl.pixels > 5e6 else 60)
+            times = []
+            for _ in range(n):
+                flush.fill_(1.0)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                dec.decode_batch(lat, st, w, wl.H, wl.W, out, stream=stream, B=B, check=False)
+                e1.record(stream)
+                e1.synchronize()
+                times.append(e0.elapsed_time(e1))
+            dec.check(stream)
+            ms = float(np.median(times))
+            roof = roofline_for(wl, precision, B, ms, peaks, fp32_tf, fp32_src)
+            rows.append({"workload": name, "precision": precision, "kernel": dec.kernel_name,
+                         "images": B, "ms": ms, "ms_p10": float(np.percentile(times, 10)),
+                         "ms_p90": float(np.percentile(times, 90)), "calls": n,
+                         "mp_per_s": B * wl.H * wl.W / (ms * 1e-3) / 1e6,
+                         "images_per_s": B / (ms * 1e-3),
+                         "roofline": {k: roof[k] for k in ("bound", "achieved", "peak", "unit",
+                                                            "frac", "binding_time_us",
+                                                            "alu_bound")}})
+            dec.close()
+            del w
+        del lat, st, out
+    del flush
+    return {"rows": rows, "timing": "median of per-call CUDA events, L2 flushed (256 MB write) "
+                                    "before every call, 3 warm-up calls per row"}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -806,6 +959,8 @@ def main():
     ap.add_argument("--ref-step-s", type=float, default=5.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip the rows of every workload on both paths")
     ap.add_argument("--no-protocols", action="store_true",
                     help="skip the per-call, CUDA-graph and serial-per-image rows")
     ap.add_argument("--stage", default="decode",
@@ -985,52 +1140,43 @@ def main():
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(out_h.numel() * 4),
                "ms_per_step": 1e3 * el / e_steps}
 
+    # The same end to end with the uint8 HWC output (a quarter of the fp32
+    # RGB return over the host link), through its own handle.
+    e2e_u8 = None
+    if not args.no_e2e:
+        dec8 = pic.Decoder.for_workload(wl, precision, max_batch=B, output="u8_hwc")
+        out8_h = torch.empty((B, wl.H, wl.W, 3), dtype=torch.uint8).pin_memory()
+        p8 = out8_h.data_ptr()
+
+        def host_call_u8():
+            rc = pic.pic_decode_batch_host(dec8.handle, B, ptrs[0], ptrs[1], ptrs[2], wl.H, wl.W,
+                                           p8, sp)
+            if rc != pic.PIC_OK:
+                raise pic.PicError(rc, "pic_decode_batch_host")
+
+        host_call_u8()
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(e_steps):
+            host_call_u8()
+        el8 = max_over_ranks(time.perf_counter() - t0, world, dev)
+        dec8.check(stream)
+        e2e_u8 = {"value": px_total * e_steps / el8 / 1e6, "unit": UNIT,
+                  "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(out8_h.numel()),
+                  "ms_per_step": 1e3 * el8 / e_steps, "output": "uint8 [B][H][W][3]"}
+        dec8.close()
+
     peaks = load_peaks()
     flops, nbytes = algorithmic(wl, B)
-    t_s = ms * 1e-3
     kname = dec.kernel_name
-    if precision == "fp16_tc":
-        peak_tf = peaks["bf16_tflops"]  # fp16 dense tensor rate = bf16 rate
-        t_pipe = flops / (peak_tf * 1e12)
-        roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": peak_tf,
-                "unit": "TFLOP/s", "peak_source": f"bf16 dense burst, {peaks['source']}"}
-    else:
-        try:  # the FMA microbenchmark of include/pic_measure.h, on this GPU
-            peak_tf = pic.fma_peak_tflops(dev)
-            src = (f"FP32 FMA microbenchmark, measured (formula: {fp32_peak_tflops():.1f} "
-                   f"TFLOP/s = 152 SMs x 128 lanes x 2 FLOP x 2070 MHz)")
-        except Exception as exc:  # report the formula instead of failing the bench
-            peak_tf = fp32_peak_tflops()
-            src = f"FP32 FMA formula (152 SMs x 128 lanes x 2 FLOP x 2070 MHz; microbenchmark failed: {exc})"
-        t_pipe = flops / (peak_tf * 1e12)
-        roof = {"bound": "alu", "achieved": flops / t_s / 1e12, "peak": peak_tf,
-                "unit": "TFLOP/s", "peak_source": src}
-    t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
-    if t_hbm > t_pipe:
-        roof.update({"bound": "hbm", "achieved": nbytes / t_s / 1e9, "peak": peaks["hbm_gbs"],
-                     "unit": "GB/s", "peak_source": f"copy bandwidth, {peaks['source']}"})
-    roof["frac"] = roof["achieved"] / roof["peak"]
+    fp32_tf, fp32_src = fp32_peak(pic, dev)
+    roof = roofline_for(wl, precision, B, ms, peaks, fp32_tf, fp32_src)
     roof["traffic"] = recorded_traffic(kname, wl.name)
     roof["kernel"] = kname
-    roof["algorithmic_flops_per_launch"] = flops
-    if precision == "fp16_tc":
-        # MACs the tensor cores execute per pixel: layer 0 (K = round16(2 D0 + 1),
-        # N = round16 of the width), hidden layers and (for wide, shallow nets)
-        # the output layer (N = 16), with the hi and lo halves of K plus one
-        # K = 16 bias step each.
-        def r16(v):
-            return (v + 15) // 16 * 16
-        n_pad = r16(max(wl.dims[1:-1]))
-        mac = r16(2 * wl.dims[0] + 1) * n_pad
-        mac += (len(wl.dims) - 3) * (2 * n_pad + 16) * n_pad
-        # the output layer runs on the tensor cores only for wide, shallow
-        # nets (N > 32 and fewer than 4 layers); else on the CUDA cores
-        if n_pad > 32 and len(wl.dims) - 1 < 4:
-            mac += (2 * n_pad + 16) * 16
-        roof["executed_tensor_flops_per_launch"] = 2.0 * mac * B * wl.H * wl.W
-    roof["algorithmic_bytes_per_launch"] = nbytes
-    roof["binding_time_us"] = max(t_pipe, t_hbm) * 1e6
-    roof["avg_launch_us"] = ms * 1e3
+
+    per_config = None
+    if rank == 0 and not args.no_per_config:
+        per_config = per_config_rows(pic, dev, stream, peaks, fp32_tf, fp32_src)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -1050,6 +1196,10 @@ def main():
                 "images_per_s": images_per_s,
                 "roofline": roof, "clocks": clk.summary(), "e2e": e2e,
                 "gpu_launches": args.steps, "cpu_baseline": cpu}
+        if e2e_u8 is not None:
+            line["e2e_u8"] = e2e_u8
+        if per_config is not None:
+            line["per_config"] = per_config
         if protocols is not None:
             line["protocols"] = protocols
         print(json.dumps(line), flush=True)

@@ -93,9 +93,15 @@ __device__ __forceinline__ void dense_layer(const float* __restrict__ wt, const 
   }
 #pragma unroll
   for (int i = 0; i < D4 / 2; ++i) {
+    if constexpr (ACT == ACT_GELU && !LAST) acc[i] = gelu_poly2(acc[i]);
     const float2 v = unpack2(acc[i]);
-    if (2 * i < DOUT) out[2 * i] = LAST ? v.x : activate<ACT>(v.x);
-    if (2 * i + 1 < DOUT) out[2 * i + 1] = LAST ? v.y : activate<ACT>(v.y);
+    if constexpr (LAST || ACT == ACT_GELU) {
+      if (2 * i < DOUT) out[2 * i] = v.x;
+      if (2 * i + 1 < DOUT) out[2 * i + 1] = v.y;
+    } else {
+      if (2 * i < DOUT) out[2 * i] = activate<ACT>(v.x);
+      if (2 * i + 1 < DOUT) out[2 * i + 1] = activate<ACT>(v.y);
+    }
   }
 }
 

@@ -253,16 +253,13 @@ __device__ __forceinline__ void output_layer_cc(const uint8_t* smem, uint32_t t_
     tmem_ld_wait();
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
-      float a = __uint_as_float(acc[2 * q]);
-      float bb = __uint_as_float(acc[2 * q + 1]);
+      unsigned long long hv;
       if constexpr (Net::ACT == ACT_GELU) {
-        a = gelu_poly(a);
-        bb = gelu_poly(bb);
+        hv = gelu_poly2(pack2(__uint_as_float(acc[2 * q]), __uint_as_float(acc[2 * q + 1])));
       } else {
-        a = fmaxf(a, 0.0f);
-        bb = fmaxf(bb, 0.0f);
+        hv = pack2(fmaxf(__uint_as_float(acc[2 * q]), 0.0f),
+                   fmaxf(__uint_as_float(acc[2 * q + 1]), 0.0f));
       }
-      const unsigned long long hv = pack2(a, bb);
       const float4 wa = *reinterpret_cast<const float4*>(wo + 8 * (h0 / 2 + q));
       const float4 wb = *reinterpret_cast<const float4*>(wo + 8 * (h0 / 2 + q) + 4);
       s0 = fma2(pack2(wa.x, wa.y), hv, s0);
@@ -293,8 +290,9 @@ __device__ __forceinline__ void hidden_epilogue(uint32_t t_acc, uint32_t t_a) {
       float a = __uint_as_float(acc[2 * q]);
       float bb = __uint_as_float(acc[2 * q + 1]);
       if constexpr (Net::ACT == ACT_GELU) {
-        a = gelu_poly(a);
-        bb = gelu_poly(bb);
+        const float2 g = unpack2(gelu_poly2(pack2(a, bb)));
+        a = g.x;
+        bb = g.y;
       }
       // hi = fp16 truncation (ReLU folded in), lo = fp16 of v - hi (one mixed FMA)
       split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[8 + q]);

@@ -84,28 +84,6 @@ __device__ __forceinline__ float gelu_erf(float z) {
   return 0.5f * z * (1.0f + erff(z * 0.70710678118654752f));
 }
 
-// GELU z * Phi(z) without special-function units or branches:
-// erf(x) ~= x P(u) with u = 2 min(x^2, X^2) / X^2 - 1, x = z / sqrt 2, P the
-// degree-14 least-squares fit of gen_gelu_poly.py; Phi = saturate(1/2 + x P / 2)
-// (the saturation is the |erf| <= 1 clamp).  Max abs error ~1.1e-6.
-__device__ __forceinline__ float gelu_poly(float z) {
-  const float t = fminf(0.5f * z * z, kGeluX2);
-  const float u = fmaf(t, kGeluUScale, -1.0f);
-  const float p = gelu_poly_p(u);
-  const float phi = __saturatef(fmaf(z * 0.35355339059327376f, p, 0.5f));  // z / (2 sqrt 2)
-  return z * phi;
-}
-
-template <int ACT>
-__device__ __forceinline__ float activate(float z) {
-  if constexpr (ACT == ACT_GELU) return gelu_poly(z);
-  else return fmaxf(z, 0.0f);
-}
-
-__device__ __forceinline__ float activate_rt(float z, int act) {
-  return act == ACT_GELU ? gelu_poly(z) : fmaxf(z, 0.0f);
-}
-
 // ---- packed fp32 pairs (sm_100+ f32x2 instructions) ----------------------
 __device__ __forceinline__ unsigned long long pack2(float lo, float hi) {
   unsigned long long r;
@@ -130,6 +108,50 @@ __device__ __forceinline__ unsigned long long sub2(unsigned long long a, unsigne
   unsigned long long d;
   asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
+}
+
+// d = a * b on both halves.
+__device__ __forceinline__ unsigned long long mul2(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// GELU z * Phi(z) without special-function units or branches (the
+// polynomial P of gen_gelu_poly.py, max abs error ~1.1e-6 in fp32):
+//   t = min(z^2, Z^2), u = t * 2/Z^2 - 1, Phi = saturate(1/2 + z P(u)),
+// the saturation being both the clamp Phi in [0, 1] and the value beyond Z.
+__device__ __forceinline__ float gelu_poly(float z) {
+  const float t = fminf(z * z, kGeluZ2);
+  const float u = fmaf(t, kGeluUScale, -1.0f);
+  float p = gelu_coef(0);
+#pragma unroll
+  for (int i = 1; i <= kGeluDegree; ++i) p = fmaf(p, u, gelu_coef(i));
+  return z * __saturatef(fmaf(z, p, 0.5f));
+}
+
+// The same on a pair of values packed in 64 bits: the multiplies and the
+// Horner chain run as packed f32x2 instructions (one instruction, two
+// operations), with the same roundings as gelu_poly on each half.
+__device__ __forceinline__ unsigned long long gelu_poly2(unsigned long long v) {
+  const float2 zz = unpack2(mul2(v, v));
+  const unsigned long long t = pack2(fminf(zz.x, kGeluZ2), fminf(zz.y, kGeluZ2));
+  const unsigned long long u = fma2(t, pack2(kGeluUScale, kGeluUScale), pack2(-1.0f, -1.0f));
+  unsigned long long p = pack2(gelu_coef(0), gelu_coef(0));
+#pragma unroll
+  for (int i = 1; i <= kGeluDegree; ++i) p = fma2(p, u, pack2(gelu_coef(i), gelu_coef(i)));
+  const float2 z = unpack2(v), pp = unpack2(p);
+  return mul2(v, pack2(__saturatef(fmaf(z.x, pp.x, 0.5f)), __saturatef(fmaf(z.y, pp.y, 0.5f))));
+}
+
+template <int ACT>
+__device__ __forceinline__ float activate(float z) {
+  if constexpr (ACT == ACT_GELU) return gelu_poly(z);
+  else return fmaxf(z, 0.0f);
+}
+
+__device__ __forceinline__ float activate_rt(float z, int act) {
+  return act == ACT_GELU ? gelu_poly(z) : fmaxf(z, 0.0f);
 }
 
 // Bilinear source coordinate of output index x along one axis: the pixel

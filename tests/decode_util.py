@@ -43,9 +43,14 @@ def gpu_decode(wl: wk.Workload, x: wk.Inputs, precision: str, clamp: bool = True
 
 
 def oracle_full(orc, wl: wk.Workload, x: wk.Inputs, b: int, precision: str,
-                clamp: bool = True) -> np.ndarray:
+                clamp: bool = True, defined: bool = False) -> np.ndarray:
+    """The oracle's decode of image b with the weights the GPU path consumes
+    (``x.weights_for(precision)``), or, with defined=True, with the weights
+    the workload defines (its fp32 draw where the tensor path gets an fp16
+    copy of it)."""
+    w = x.oracle_weights(precision) if defined else x.weights_for(precision)
     return orc.decode(x.latents[b], x.steps[b].astype(np.float64),
-                      x.weights_for(precision)[b].astype(np.float64), wl.H, wl.W, wl.L, wl.C,
+                      w[b].astype(np.float64), wl.H, wl.W, wl.L, wl.C,
                       wl.dims, wl.act, clamp=clamp, nthreads=ORACLE_THREADS)
 
 

@@ -1,17 +1,16 @@
 """GPU parity of the fp32 CUDA-core decode (PIC_PREC_FP32) against the fp64
 oracle, element by element on the same seeded inputs, through the C ABI.
 
-Bar: max |GPU - oracle| <= 1e-4 on [0, 1] RGB.  Whole images where the
-oracle finishes in seconds; at the 2160p and 64-image sizes, in the launch
-configuration the benchmark times, sampled pixels the oracle decodes one by
-one.
+Bar: max |GPU - oracle| <= 1e-4 on [0, 1] RGB, on every pixel: whole images
+for c1-c3, the whole 3840x2160 image for c4, and all 64 images of the c5
+batch decoded in one launch (the launch configuration the benchmark times).
 """
 import numpy as np
 import pytest
 
 from paper_2609_09020_gb300 import workloads as wk
 
-from decode_util import TOL, gpu_decode, max_abs_diff, oracle_full, oracle_pixels
+from decode_util import TOL, gpu_decode, max_abs_diff, oracle_full
 
 pytestmark = pytest.mark.gpu
 P = "fp32"
@@ -51,19 +50,12 @@ def test_full_image_unclamped(orc, name):
     _check_full(orc, wk.WORKLOADS[name], clamp=False)
 
 
-@pytest.mark.parametrize("name,batch", [("c4", 1), ("c5", 64)])
-def test_full_size_sampled(orc, name, batch):
-    wl = wk.WORKLOADS[name]
-    x = wk.make_inputs(wl)
-    got = gpu_decode(wl, x, P)
-    assert not np.isnan(got).any()
+@pytest.mark.parametrize("name", ["c4", "c5"])
+def test_full_size_every_pixel(orc, name):
+    """c4 (3840x2160) and c5 (64 images in one launch): every pixel of every
+    image, including the 128-pixel tile seams of the 3840-wide rows."""
+    got = _check_full(orc, wk.WORKLOADS[name])
     assert got.min() >= 0.0 and got.max() <= 1.0
-    for b in range(0, batch, max(1, batch // 8)):
-        pix = wk.sample_pixels(wl.H, wl.W, 1500, seed=1000 + b)
-        want = oracle_pixels(orc, wl, x, b, P, pix)
-        g = got[b].reshape(3, -1)[:, pix].T
-        d, where = max_abs_diff(g, want)
-        assert d <= TOL[P], (name, b, d, where)
 
 
 # Edge and ragged shapes: 1-pixel images, sizes that are not multiples of the

@@ -1,13 +1,18 @@
 """GPU parity of the tensor-core decode (PIC_PREC_FP16_TC, tcgen05) against
-the fp64 oracle on the same seeded inputs (the fp16 weights the path
-consumes), through the C ABI.
+the fp64 oracle on the same seeded inputs, through the C ABI.
 
-Bars: max |GPU - oracle| <= 4e-3 on [0, 1] RGB and |PSNR(G, T) - PSNR(O, T)|
-<= 0.02 dB against a noisy target T = clamp(O + N(0, sigma^2)) at ~35 dB (the
-paper's operating range).  The split (hi + lo) fp16 operands carry ~22
-significant bits, so the error is also held to a much tighter design bound:
-plain fp16 operands would land near 4e-3 on these workloads, and a broken
-lo-term would show up here.
+Two references per image:
+- the decode as defined: the oracle on the weights the workload defines (its
+  fp32 draw for c1-c4, whose tensor path consumes an fp16 copy; the fp16
+  weights themselves for c5 and the fp16 edge cases).  Bars: max |GPU -
+  oracle| <= 4e-3 on [0, 1] RGB and |PSNR(G, T) - PSNR(O, T)| <= 0.02 dB
+  against a noisy target T = clamp(O + N(0, sigma^2)) at ~35 dB (the
+  paper's operating range).  The fp16 weight copy alone moves the c4 decode
+  by up to ~2.6e-3; this is the check of the decode the workload asks for.
+- the kernel's own arithmetic: the oracle on the fp16 weights the kernel
+  consumes.  The split (hi + lo) operands carry ~22 significant bits, so the
+  error is held to SPLIT_BOUND, far below the bar: plain fp16 operands would
+  land near 4e-3 on these workloads, and a broken lo-term would show up here.
 """
 import numpy as np
 import pytest
@@ -39,16 +44,20 @@ def _noisy_target(ref: np.ndarray, seed: int) -> np.ndarray:
 def _check(orc, wl, images=None, clamp=True):
     x = wk.make_inputs(wl)
     got = gpu_decode(wl, x, P, clamp=clamp)
+    # the kernel consumes a rounded copy of the defined weights (fp32 draws)
+    copy = not np.array_equal(x.weights_for(P).astype(np.float64), x.oracle_weights(P))
     worst = 0.0
     for b in (range(x.latents.shape[0]) if images is None else images):
-        want = oracle_full(orc, wl, x, b, P, clamp=clamp)
-        d, where = max_abs_diff(got[b], want)
+        want_in = oracle_full(orc, wl, x, b, P, clamp=clamp)  # the kernel's fp16 weights
+        want = oracle_full(orc, wl, x, b, P, clamp=clamp, defined=True) if copy else want_in
         scale = 1.0 if clamp else max(1.0, float(np.abs(want).max()))
-        assert d <= TOL[P] * scale, (wl.name, b, d, where)
-        assert d <= SPLIT_BOUND * scale, (wl.name, b, d, where, "split-precision bound")
+        d, where = max_abs_diff(got[b], want)
+        assert d <= TOL[P] * scale, (wl.name, b, d, where, "bar against the defined weights")
         if clamp:
             t = _noisy_target(want, 1000 + b)
-            assert abs(psnr(got[b], t) - psnr(want, t)) <= 0.02
+            assert abs(psnr(got[b], t) - psnr(want, t)) <= 0.02, (wl.name, b)
+        d_in, where = max_abs_diff(got[b], want_in)
+        assert d_in <= SPLIT_BOUND * scale, (wl.name, b, d_in, where, "split-precision bound")
         worst = max(worst, d)
     return worst
 
@@ -59,7 +68,10 @@ def test_c5_all_64_images(orc):
 
 
 def test_c4_full_image(orc):
-    """3840x2160, 8 levels x 2 channels, 16-64-64-64-3 GELU, fp16 weight copy."""
+    """3840x2160, 8 levels x 2 channels, 16-64-64-64-3 GELU: every pixel
+    against the oracle on the workload's fp32 weights (the 4e-3 / 0.02 dB
+    bars), and against the oracle on the fp16 copy the kernel consumes (the
+    split-precision bound)."""
     _check(orc, wk.WORKLOADS["c4"])
 
 
