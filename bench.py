@@ -893,6 +893,9 @@ def fp32_peak(pic, dev):
 
 
 PER_CONFIG = ["c1", "c2", "c3", "c4", "c5"]
+# extra tensor-path rows with the latent staging the library's default does
+# not pick for that architecture (TMA boxes vs per-thread copies)
+PER_CONFIG_STAGING = {"c5": "tma", "c3": "tma", "c4": "copies"}
 
 
 def per_config_rows(pic, dev, stream, peaks, fp32_tf, fp32_src, reps=None):
@@ -910,9 +913,12 @@ def per_config_rows(pic, dev, stream, peaks, fp32_tf, fp32_src, reps=None):
         lat = torch.from_numpy(x.latents).to(dev)
         st = torch.from_numpy(x.steps).to(dev)
         out = torch.empty((B, 3, wl.H, wl.W), dtype=torch.float32, device=dev)
-        for precision in ("fp16_tc", "fp32"):
+        runs = [("fp16_tc", "auto"), ("fp32", "auto")]
+        if name in PER_CONFIG_STAGING:
+            runs.insert(1, ("fp16_tc", PER_CONFIG_STAGING[name]))
+        for precision, staging in runs:
             w = torch.from_numpy(np.ascontiguousarray(x.weights_for(precision))).to(dev)
-            dec = pic.Decoder.for_workload(wl, precision, max_batch=B)
+            dec = pic.Decoder.for_workload(wl, precision, max_batch=B, staging=staging)
             dec.check_buffers(B, wl.H, wl.W, latents=lat, steps=st, weights=w, out=out)
             for _ in range(3):
                 dec.decode_batch(lat, st, w, wl.H, wl.W, out, stream=stream, B=B, check=False)
@@ -931,7 +937,8 @@ def per_config_rows(pic, dev, stream, peaks, fp32_tf, fp32_src, reps=None):
             dec.check(stream)
             ms = float(np.median(times))
             roof = roofline_for(wl, precision, B, ms, peaks, fp32_tf, fp32_src)
-            rows.append({"workload": name, "precision": precision, "kernel": dec.kernel_name,
+            rows.append({"workload": name, "precision": precision, "staging": staging,
+                         "kernel": dec.kernel_name,
                          "images": B, "ms": ms, "ms_p10": float(np.percentile(times, 10)),
                          "ms_p90": float(np.percentile(times, 90)), "calls": n,
                          "mp_per_s": B * wl.H * wl.W / (ms * 1e-3) / 1e6,

@@ -79,6 +79,21 @@ typedef enum {
 } pic_latent_format;
 
 typedef enum {
+    /* The library's choice per architecture (measured: TMA where it is as
+     * fast as per-thread copies, per-thread copies where TMA was slower). */
+    PIC_STAGING_AUTO = 0,
+    /* Every latent word a tile needs is loaded by the decoding threads'
+     * 4-byte asynchronous copies, one tile ahead. */
+    PIC_STAGING_COPIES = 1,
+    /* A tile's full-resolution row (every channel) arrives as TMA boxes
+     * issued two tiles ahead; the coarser levels' rows stay with per-thread
+     * copies.  Tensor-core path only, for the architectures that have a
+     * TMA-staged kernel (PIC_ERR_UNSUPPORTED at create otherwise); a call
+     * whose latent buffer holds 2^31 words or more falls back to copies. */
+    PIC_STAGING_TMA = 2
+} pic_staging;
+
+typedef enum {
     PIC_OUT_F32_CHW = 0, /* fp32 planar [3][H][W] (R, G, B planes) -- the default */
     PIC_OUT_F32_HWC = 1, /* fp32 interleaved [H][W][3] */
     PIC_OUT_U8_HWC = 2   /* uint8 interleaved [H][W][3]: round-half-even(255 clamp(v, 0, 1)) */
@@ -97,6 +112,7 @@ typedef struct {
     int max_batch;          /* largest B accepted by pic_decode_batch */
     int latent_format;      /* pic_latent_format; same layout and size (4 B) either way */
     int output_format;      /* pic_output_format (uint8 output always clamps) */
+    int staging;            /* pic_staging: how the tensor-core kernel stages latents */
 } pic_arch;
 
 /*
@@ -214,7 +230,9 @@ int pic_decode_noalloc_check(void *stream);
  * device first, so that no kernel of this handle is still running. */
 void pic_decode_destroy(pic_decoder *h);
 
-/* Name of the kernel selected at create (static string), or "" for NULL. */
+/* Name of the kernel the handle launches (static string), or "" for NULL:
+ * the TMA-staged kernel where the handle stages with TMA (a call whose
+ * latent buffer holds 2^31 words or more runs its per-thread-copy twin). */
 const char *pic_decode_kernel_name(const pic_decoder *h);
 
 /* sum_l C * ceil(H/2^l) * ceil(W/2^l), or -1 for invalid arguments. */

@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libpic_gb300.so")
-SOURCES = ["pic_decode.cu", "k_fp32.cu", "k_fp32_sweep.cu", "k_tc.cu", "k_tc_f32lat.cu", "k_tc_sweep.cu", "k_izpr.cu",
+SOURCES = ["pic_decode.cu", "k_fp32.cu", "k_fp32_sweep.cu", "k_tc.cu", "k_tc_f32lat.cu", "k_tc_sweep.cu", "k_tc_tma.cu", "k_izpr.cu",
            "k_idct.cu", "k_fuse.cu", "k_huffman.cu", "k_peak.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",

@@ -23,6 +23,7 @@ int tc_kernels(KernelInfo* out, int cap) {
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
   int k = 0;
   for (; k < n && k < cap; ++k) out[k] = list[k];
+  if (k < cap) k += tc_kernels_tma(out + k, cap - k);
   if (k < cap) k += tc_kernels_fp32lat(out + k, cap - k);
   if (k < cap) k += tc_kernels_sweep(out + k, cap - k);
   return k;

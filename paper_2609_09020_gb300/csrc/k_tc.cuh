@@ -40,6 +40,24 @@
 //                        gives registers to the decoders): waits, issues, commits.
 // Handshakes are mbarriers; every wait is bounded (on timeout the kernel
 // raises the handle's status word, skips the rest and still frees TMEM).
+//
+// Latent staging.  Each decoding thread loads its share of the next tile's
+// coarse-level source rows (levels l >= 1, read by many neighbouring tiles,
+// so mostly L1 hits) with 4-byte cp.async copies, one tile ahead.  The tile's
+// own full-resolution row (level 0, streamed from DRAM once) comes
+//   without TMA (TMA = false): the same way, one cp.async per thread;
+//   with TMA (TMA = true):     as one TMA box per channel (a 1-D tensor map
+//                              over the call's latents), which the group's
+//                              issuing warp loads into one of two buffers two
+//                              tiles ahead, right after the decoders have
+//                              handed over the tile that used that buffer.
+//                              The issuing warp also waits for the box of the
+//                              next tile and then arrives on the group's
+//                              col_ready barrier as its 129th participant, so
+//                              the decoders, which read level 0 after that
+//                              barrier, wait on nothing more than without TMA
+//                              (an extra wait per tile in the decoders cost
+//                              c5 9-14 %).
 #pragma once
 
 #include <cuda_fp16.h>
@@ -81,6 +99,20 @@ __host__ __device__ constexpr uint32_t kmaj(int row, int k, int K) {
 // [0, W_l - 1] when the buffer is filled, which reproduces the edge clamp of
 // the bilinear definition.
 __host__ __device__ constexpr int ncol(int l) { return (kTile >> l) + 4; }
+static_assert(kTile == kTcTile, "one tile size for the kernels and the host's TMA boxes");
+
+// One TMA buffer (TMA kernels): a slot per channel for the tile's level-0
+// row segment, each holding one box of kTmaRowBox 4-byte words and starting
+// on a 128-byte boundary (a tiled TMA copy's shared-memory destination must
+// be 128-byte aligned).
+template <int C>
+struct TmaSlots {
+  static constexpr int slot() { return (kTmaRowBox * 4 + 127) / 128 * 128; }
+  static constexpr int off(int c) { return c * slot(); }  // bytes
+  static constexpr int total() { return C * slot(); }
+  static constexpr int boxes() { return C; }
+  static constexpr int tx_bytes() { return C * kTmaRowBox * 4; }  // the stage mbarrier's count
+};
 
 template <int L, int C>
 struct ColLayout {
@@ -142,6 +174,10 @@ struct TcNet {
   static constexpr int STAGE_BYTES = STAGE_SLOTS * kTile * 4;
   static constexpr int WG_BYTES = A1_BYTES + COL_BYTES + STAGE_BYTES;
   static constexpr int SMEM = OFF_WG + NWG * WG_BYTES;
+  // TMA kernels: the per-thread staging slots give way to two TMA buffers
+  static constexpr int TBUF_BYTES = round_up(TmaSlots<C>::total(), 128);
+  static constexpr int WG_BYTES_TMA = WG_BYTES + 2 * TBUF_BYTES;
+  static constexpr int SMEM_TMA = OFF_WG + NWG * WG_BYTES_TMA;
   static constexpr int TMEM_COLS = pow2_at_least(NWG * 2 * N);
   static_assert(N % 16 == 0 && N >= 16 && N <= 128, "hidden width must be 16..128, multiple of 16");
   static_assert(NL >= 2, "the tensor-core path needs at least one hidden layer");
@@ -149,7 +185,10 @@ struct TcNet {
   static_assert(NISSUE == 4 && MMA_WARP % 4 == 0, "the issuing warps form one warpgroup");
   static_assert(REG_DECODE >= MAXREG && REG_DECODE * NWG * 128 + REG_ISSUE * 32 * NISSUE <= MAXREG * THREADS,
                 "register split within the launch budget");
-  static_assert(8 * (4 * NWG + NISSUE) <= 224, "control block holds the barriers");
+  static_assert(8 * (6 * NWG + NISSUE) <= 224, "control block holds the barriers");
+  static_assert(TmaSlots<C>::boxes() <= 32, "a tile's TMA boxes, one per lane of a warp");
+  static_assert(WG_BYTES % 128 == 0 && TBUF_BYTES % 128 == 0 && OFF_WG % 128 == 0,
+                "TMA buffers on 128-byte boundaries");
 };
 
 // Bounded mbarrier wait.  Returns false (and raises the abort flag and the
@@ -313,11 +352,13 @@ __device__ __forceinline__ void advance_tile(int& yy, int& xx, int tpr) {
   }
 }
 
-template <class Net, bool FL>
+template <class Net, bool FL, bool TMA>
 __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
-    tc_decode_kernel(const DecodeParams p) {
+    tc_decode_kernel(const DecodeParams p, const __grid_constant__ TmaParams tp) {
   constexpr int N = Net::N, NL = Net::NL, C = Net::C, L = Net::L, D0 = Net::D0, NWG = Net::NWG;
   constexpr int K1 = Net::K1;
+  constexpr int WGB = TMA ? Net::WG_BYTES_TMA : Net::WG_BYTES;
+  using TS = TmaSlots<C>;
   using CL = ColLayout<L, C>;
   constexpr int NITEM = CL::total();
   constexpr int J = (NITEM + kTile - 1) / kTile;  // column items per thread (0 if L == 1)
@@ -336,15 +377,20 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
   const uint32_t bar_c = sbase + 16 * NWG;
   const uint32_t bar_col = sbase + 24 * NWG;
   const uint32_t bar_drain = sbase + 32 * NWG;  // + 8 m for issuing warp m
+  // TMA kernels: per group two stage_full barriers (its boxes for the tile
+  // using buffer 0 / 1 have landed), at bar_stage + 16 w + 8 buffer
+  const uint32_t bar_stage = bar_drain + 8 * Net::NISSUE;
 
   if (threadIdx.x == 0) {
     for (int w = 0; w < NWG; ++w) {
       mbar_init(bar_a1 + 8 * w, 128);
       mbar_init(bar_a + 8 * w, 128);
       mbar_init(bar_c + 8 * w, 1);
-      mbar_init(bar_col + 8 * w, 128);
+      mbar_init(bar_col + 8 * w, TMA ? 129 : 128);  // TMA: + the issuing warp's arrival
     }
     for (int m = 0; m < Net::NISSUE; ++m) mbar_init(bar_drain + 8 * m, 1);
+    if constexpr (TMA)
+      for (int q = 0; q < 2 * NWG; ++q) mbar_init(bar_stage + 8 * q, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -375,6 +421,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
   uint32_t col_phase = 0;  // warpgroup threads: parity of their col_ready
   uint32_t a1_phase = 0;   // MMA warp: bit w = parity of a1_full[w]
   uint32_t a_phase = 0;    // MMA warp: bit w = parity of a_full[w]
+  uint32_t stage_phase = 0;  // TMA, issuing warps: bit q = parity of the next box set issued on q
+  uint32_t stage_wait = 0;   // TMA, issuing warps: bit q = parity of the next box set to wait for on q
 
   // Each role runs its own loop over the images of its tile range, so that
   // it can hold its own register budget: the issuing warpgroup gives
@@ -399,7 +447,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         // ------------------------------------------------------------ warpgroup
         const int w = warp >> 2;
         const int r = ((warp & 3) << 5) | lane;  // tile row = TMEM lane = pixel
-        uint8_t* a1 = smem + Net::OFF_WG + w * Net::WG_BYTES;
+        uint8_t* a1 = smem + Net::OFF_WG + w * WGB;
         const uint32_t a1_s = smem_addr(a1);
         float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES);
         const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
@@ -460,10 +508,12 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         const uint32_t stage_s = a1_s + Net::A1_BYTES + Net::COL_BYTES;
         const int* stage = reinterpret_cast<const int*>(a1 + Net::A1_BYTES + Net::COL_BYTES);
         auto prefetch = [&](int y, int x0) {
-          const int xc = min(x0 + r, p.W - 1);
+          if constexpr (!TMA) {  // else the level-0 row arrives as the issuing warp's TMA boxes
+            const int xc = min(x0 + r, p.W - 1);
 #pragma unroll
-          for (int c = 0; c < C; ++c)
-            cp_async4(stage_s + (c * kTile + r) * 4, lat + c * plane + static_cast<long long>(y) * p.W + xc);
+            for (int c = 0; c < C; ++c)
+              cp_async4(stage_s + (c * kTile + r) * 4, lat + c * plane + static_cast<long long>(y) * p.W + xc);
+          }
 #pragma unroll
           for (int j = 0; j < J; ++j) {
             const int l = it_l[j];
@@ -480,9 +530,20 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           cp_async_commit();
         };
 
-        // Features of tile (y, x0) from its prefetched loads -> A1 (shared).
-        // Returns false if a wait gave up.
-        auto features = [&](int y, int x0) -> bool {
+        // TMA kernels: the level-0 row of the group's k-th tile sits in TMA
+        // buffer k & 1 once the tile's col_ready phase has completed (the
+        // issuing warp arrives there only after the box has landed), channel
+        // c's box from latent word s_c & ~3 on, where
+        // s_c is the word of (c, y, x0) in the call's latent buffer; pixel r
+        // is box word (s_c & 3) + r.  Only the low two bits of the word index
+        // are used, so 32-bit wrap-around is harmless.
+        const uint8_t* tbuf = a1 + Net::A1_BYTES + Net::COL_BYTES + Net::STAGE_BYTES;
+        const unsigned img_word =
+            static_cast<unsigned>(b) * static_cast<unsigned>(p.lat_per_image);
+
+        // Features of the group's k-th tile (y, x0) from its staged loads ->
+        // A1 (shared).  Returns false if a wait gave up.
+        auto features = [&](int y, int x0, int k) -> bool {
           cp_async_wait_all();  // this thread's staged loads have landed
           // vertical pass into the column buffer
 #pragma unroll
@@ -502,7 +563,15 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           const int xc = min(x0 + r, p.W - 1);
           float f[D0];
 #pragma unroll
-          for (int c = 0; c < C; ++c) f[c] = step[0] * lat_value<FL>(stage[c * kTile + r]);
+          for (int c = 0; c < C; ++c) {
+            if constexpr (TMA) {
+              const unsigned sc = img_word + static_cast<unsigned>(c * plane + y * p.W + x0);
+              const int* slot = reinterpret_cast<const int*>(tbuf + (k & 1) * Net::TBUF_BYTES + TS::off(c));
+              f[c] = step[0] * lat_value<FL>(slot[(sc & 3u) + r]);
+            } else {
+              f[c] = step[0] * lat_value<FL>(stage[c * kTile + r]);
+            }
+          }
 #pragma unroll
           for (int l = 1; l < L; ++l) {
             int i0, i1;
@@ -542,7 +611,6 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           return true;
         };
 
-
         // Tile cursor (row y, tile column tx) of this group's current tile and
         // of the one after it, advanced by NWG tiles without divisions.
         const int tpr = p.tiles_per_row;
@@ -552,7 +620,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         bool ok = true;
         if (w < n_tiles) {
           prefetch(cy, ctx * kTile);
-          ok = features(cy, ctx * kTile);
+          ok = features(cy, ctx * kTile, 0);
           if (ok) mbar_arrive(my_a1);
         }
         for (int i = w; i < n_tiles && ok; i += NWG) {
@@ -562,6 +630,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           int ny = cy, ntx = ctx;
           advance_tile<NWG>(ny, ntx, tpr);
           const bool has_next = i + NWG < n_tiles;
+          const int knext = (i - w) / NWG + 1;  // the group's index of the next tile
           if (has_next) prefetch(ny, ntx * kTile);  // in flight during the first epilogue
 
           if constexpr (Net::OUTCC) {
@@ -576,7 +645,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
               hidden_epilogue<Net>(t_acc, t_a);
               tc_fence_before();
               mbar_arrive(my_a);
-              if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
+              if (k == 0 && has_next) ok = features(ny, ntx * kTile, knext);  // overlaps layer 1
             }
             if (!ok) break;
             if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
@@ -585,7 +654,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             float rgb[3];
             output_layer_cc<Net>(smem, t_acc, rgb);
             tc_fence_before();
-            if (NL == 2 && has_next) ok = features(ny, ntx * kTile);  // no hidden layer to overlap
+            if (NL == 2 && has_next) ok = features(ny, ntx * kTile, knext);  // no hidden layer to overlap
             if (has_next && ok) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
             const int x = x0 + r;
             if (x < p.W) store_rgb(p, b, y, x, rgb[0], rgb[1], rgb[2]);
@@ -603,7 +672,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
               hidden_epilogue<Net>(t_acc, t_a);
               tc_fence_before();
               mbar_arrive(my_a);
-              if (k == 0 && has_next) ok = features(ny, ntx * kTile);  // overlaps layer 1
+              if (k == 0 && has_next) ok = features(ny, ntx * kTile, knext);  // overlaps layer 1
             }
             if (!ok) break;
 
@@ -645,7 +714,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         const int w = warp - Net::MMA_WARP;
         constexpr uint32_t id_hidden = idesc_f16(128, N);
         constexpr uint32_t id_out = idesc_f16(128, Net::NOUT);
-        const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG + w * Net::WG_BYTES, 128, 16 * K1);
+        const uint64_t dA1 = smem_desc(sbase + Net::OFF_WG + w * WGB, 128, 16 * K1);
         const uint64_t dB1 = smem_desc(sbase + Net::OFF_B1, 128, 16 * K1);
         const uint64_t dBH = smem_desc(sbase + Net::OFF_BH, 128, 16 * Net::KB);
         const uint64_t dBO = smem_desc(sbase + Net::OFF_BO, 128, 16 * Net::KB);
@@ -656,7 +725,55 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         const uint32_t d = tmem + static_cast<uint32_t>(w * 2 * N);
         const uint32_t ta = d + N;
         const uint32_t my_a1 = bar_a1 + 8 * w, my_a = bar_a + 8 * w, my_c = bar_c + 8 * w;
+        // TMA kernels: the level-0 boxes of the group's tile i (of this
+        // segment) into buffer buf, one lane per channel; lane 0 first
+        // announces the buffer's byte count on its stage_full barrier.
+        auto issue_boxes = [&](int y, int x0, int buf) {
+          const uint32_t bar = bar_stage + 16 * w + 8 * buf;
+          const uint32_t dst = sbase + Net::OFF_WG + w * WGB + Net::WG_BYTES + buf * Net::TBUF_BYTES;
+          if (lane == 0) mbar_arrive_expect_tx(bar, TS::tx_bytes());
+          __syncwarp();
+          if (lane < C) {
+            // word indices fit in 32 bits: the host encodes the maps only for
+            // buffers of fewer than 2^31 words
+            const int start = b * static_cast<int>(p.lat_per_image) + lane * static_cast<int>(plane) +
+                              y * p.W + x0;
+            // Checked before the copy (never expected to fail: the slot
+            // layout and the host's 2^31-word limit rule it out): a
+            // misaligned destination or a negative start raises status bit 2
+            // and skips the copy, so the decoders' bounded wait reports it.
+            const uint32_t d_box = dst + TS::off(lane);
+            if ((d_box & 127u) == 0u && start >= 0) tma_load_1d(d_box, &tp.lat, start & ~3, bar);
+            else atomicOr(p.status, 2);
+          }
+          stage_phase ^= 1u << buf;  // parity of the next set on this buffer
+        };
+        // TMA kernels: waits (bounded) for the boxes of the group's tile in
+        // buffer buf, then arrives on the group's col_ready barrier for that
+        // tile.  Returns false if the wait gave up.
+        auto hand_over = [&](int buf) -> bool {
+          const uint32_t bar = bar_stage + 16 * w + 8 * buf;
+          const bool landed =
+              __all_sync(0xffffffffu, wait_bounded(bar, (stage_wait >> buf) & 1u, abort_flag, p.status));
+          if (!landed) return false;  // still in flight: the exit drain waits for it
+          stage_wait ^= 1u << buf;
+          if (lane == 0) mbar_arrive(bar_col + 8 * w);
+          return true;
+        };
+        // Cursor (row, tile column) of the next tile whose boxes this warp
+        // issues, advanced by NWG tiles without divisions (as the decoders').
+        int by = 0, btx = 0;
         bool ok = true;
+        if constexpr (TMA) {
+          const long long tile0 = seg - static_cast<long long>(b) * p.tiles_per_image;
+          by = static_cast<int>((tile0 + w) / p.tiles_per_row);
+          btx = static_cast<int>((tile0 + w) - static_cast<long long>(by) * p.tiles_per_row);
+          if (w < n_tiles) issue_boxes(by, btx * kTile, 0);
+          advance_tile<NWG>(by, btx, p.tiles_per_row);
+          if (w + NWG < n_tiles) issue_boxes(by, btx * kTile, 1);
+          advance_tile<NWG>(by, btx, p.tiles_per_row);
+          if (w < n_tiles) ok = hand_over(0);  // the first tile's features
+        }
         for (int i = w; i < n_tiles && ok; i += NWG) {
           for (int k = 0; k < (Net::OUTCC ? NL - 1 : NL); ++k) {  // OUTCC: no output-layer MMA
             const uint32_t bar = k == 0 ? my_a1 : my_a;
@@ -685,11 +802,40 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
               mma_commit(my_c);
             }
             __syncwarp();
+            if constexpr (TMA) {
+              if (k == 0) {
+                // The decoders have handed over this tile (its layer-0
+                // operand was written before a1_full), so the buffer it used
+                // takes the tile two ahead; and the next tile's boxes, issued
+                // a tile ago, are handed to the decoders' col_ready barrier.
+                const int kk = (i - w) / NWG;
+                if (i + 2 * NWG < n_tiles) {
+                  issue_boxes(by, btx * kTile, kk & 1);
+                  advance_tile<NWG>(by, btx, p.tiles_per_row);
+                }
+                if (i + NWG < n_tiles && !hand_over((kk + 1) & 1)) {
+                  ok = false;
+                  break;
+                }
+              }
+            }
           }
         }
       }
       __syncwarp();
       seg = seg_end;
+    }
+    if constexpr (TMA) {
+      // Box sets still in flight (issued, never waited for: a wait gave up
+      // first) land before the CTA's shared memory is released: wait for
+      // each, bounded.
+#pragma unroll
+      for (int q = 0; q < 2; ++q)
+        if (((stage_phase ^ stage_wait) >> q) & 1u) {
+          const uint32_t bar = bar_stage + 16 * (warp - Net::MMA_WARP) + 8 * q;
+          for (uint32_t it = 0; it < kSpinLimit; ++it)
+            if (mbar_try_wait(bar, (stage_wait >> q) & 1u)) break;
+        }
     }
     if (elect_one()) {
       // Every MMA this thread issued must be complete before the memory goes.
@@ -707,7 +853,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
   }
 }
 
-template <int C, int NL, int D0, int N, int ACT, int NWG, bool FL>
+template <int C, int NL, int D0, int N, int ACT, int NWG, bool FL, bool TMA = false>
 KernelInfo make_tc(const char* name, const int* dims) {
   using Net = TcNet<C, NL, D0, N, ACT, NWG>;
   KernelInfo k{};
@@ -721,8 +867,9 @@ KernelInfo make_tc(const char* name, const int* dims) {
   k.threads = Net::THREADS;
   k.regs_at_launch = Net::MAXREG;
   k.tile_px = kTile;
-  k.smem_bytes = Net::SMEM;
-  k.fn = reinterpret_cast<const void*>(&tc_decode_kernel<Net, FL>);
+  k.smem_bytes = TMA ? Net::SMEM_TMA : Net::SMEM;
+  k.tma = TMA ? 1 : 0;
+  k.fn = reinterpret_cast<const void*>(&tc_decode_kernel<Net, FL, TMA>);
   return k;
 }
 

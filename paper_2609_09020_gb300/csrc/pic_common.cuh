@@ -3,6 +3,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
 
@@ -13,6 +14,15 @@ namespace pic {
 constexpr int kMaxLevels = 12;
 constexpr int kMaxLayers = 6;
 constexpr int kMaxDim = 128;
+
+// Tensor-core tiles: 128 pixels of one image row (one tensor-memory lane
+// each).  The TMA-staged kernels load a tile's full-resolution row segment
+// (level 0) of each channel as one TMA box of kTmaRowBox 4-byte words: the
+// box starts at the segment's first word rounded down to a multiple of 4
+// (TMA's 16-byte rule), so 3 more words than the tile's 128 and a multiple
+// of 4 in all.
+constexpr int kTcTile = 128;
+constexpr int kTmaRowBox = kTcTile + 4;
 
 // Geometry of one pyramid level (Eq. 1 with the ceiling rule): size, offset
 // of the level inside one image's latent block, and the size ratios
@@ -42,6 +52,14 @@ struct DecodeParams {
   int dims[kMaxLayers + 1];
   int act;
   LevelGeom lv[kMaxLevels];
+};
+
+// Tensor map for the TMA staging of the tensor-core kernels: the whole
+// latent buffer of the call (every image's pyramid) as one 1-D tensor of
+// 4-byte words with boxes of kTmaRowBox words; a box reads zeros past the
+// buffer's end.
+struct TmaParams {
+  CUtensorMap lat;
 };
 
 enum { ACT_RELU = 0, ACT_GELU = 1 };

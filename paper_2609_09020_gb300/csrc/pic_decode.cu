@@ -7,6 +7,8 @@
 #include <mutex>
 #include <new>
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include "pic_common.cuh"
@@ -22,6 +24,15 @@ struct pic_decoder {
   int sm_count;
   KernelInfo kern;
   int grid_cap;          // resident CTAs over all SMs
+  // the TMA-staged twin of kern (tensor-core archs that have one), launched
+  // whenever the call's latent buffer can be described by tensor maps
+  bool has_tma;
+  KernelInfo kern_tma;
+  int grid_cap_tma;
+  // the last call's tensor map (it depends on the latent buffer and its size only)
+  const int32_t* tma_key_ptr;
+  long long tma_key_words;
+  pic::TmaParams tma_cache;
   int* d_status;         // bounded-wait failure flag (device word)
   long long n_params;    // per image
   // staging for pic_decode_batch_host (allocated on first use): one region
@@ -55,11 +66,13 @@ bool arch_valid(const pic_arch* a) {
   if (a->max_H > 65536 || a->max_W > 65536 || a->max_batch > 65536) return false;
   if (a->latent_format != PIC_LATENT_INT32 && a->latent_format != PIC_LATENT_FP32) return false;
   if (a->output_format < PIC_OUT_F32_CHW || a->output_format > PIC_OUT_U8_HWC) return false;
+  if (a->staging < PIC_STAGING_AUTO || a->staging > PIC_STAGING_TMA) return false;
   return true;
 }
 
-bool kernel_matches(const KernelInfo& k, const pic_arch* a) {
-  if (k.generic || k.precision != a->precision || k.latent_format != a->latent_format ||
+bool kernel_matches(const KernelInfo& k, const pic_arch* a, bool tma = false) {
+  if (k.generic || (k.tma != 0) != tma || k.precision != a->precision ||
+      k.latent_format != a->latent_format ||
       k.C != a->channels_per_level ||
       k.n_layers != a->num_layers || k.act != a->hidden_act)
     return false;
@@ -87,6 +100,43 @@ int check_decode_args(const pic_decoder* h, int B, const int32_t* latents, const
   }
   if (cur != h->device) return PIC_ERR_INVALID_ARG;
   return PIC_OK;
+}
+
+// cuTensorMapEncodeTiled from the driver, through the runtime (no link
+// against the driver library); null if the driver does not offer it.
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+      cudaGetLastError();
+      f = nullptr;
+    }
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }();
+  return fn;
+}
+
+// Tensor map for a TMA-staged tensor-core kernel (Sec. 3.1, Eq. 1: the
+// full-resolution level of image b is a C x H x W grid inside the call's
+// latent buffer): the whole buffer as one 1-D tensor of 4-byte words with
+// boxes of kTmaRowBox words, one box per tile row segment and channel.  Box
+// coordinates are 32-bit word indices, so the buffer must hold fewer than
+// 2^31 words; else (or if the driver offers no encoder, or the encode
+// fails) the caller launches the per-thread-copy kernel instead.
+bool encode_latent_map(pic::TmaParams& tp, const DecodeParams& p) {
+  const PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  const long long words = p.lat_per_image * p.B;
+  if (!enc || words < 1 || words >= (1LL << 31)) return false;
+  const cuuint64_t dim[1] = {static_cast<cuuint64_t>(words)};
+  const cuuint64_t stride[1] = {4};  // unused for a 1-D tensor
+  const cuuint32_t box[1] = {static_cast<cuuint32_t>(pic::kTmaRowBox)};
+  const cuuint32_t elem_stride[1] = {1u};
+  return enc(&tp.lat, CU_TENSOR_MAP_DATA_TYPE_INT32, 1, const_cast<int32_t*>(p.latents), dim, stride,
+             box, elem_stride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 void fill_params(const pic_decoder* h, DecodeParams& p, int B, const int32_t* latents,
@@ -127,11 +177,34 @@ void fill_params(const pic_decoder* h, DecodeParams& p, int B, const int32_t* la
 }
 
 int launch(pic_decoder* h, const DecodeParams& p, cudaStream_t stream) {
-  long long grid = p.total_tiles < h->grid_cap ? p.total_tiles : h->grid_cap;
+  const KernelInfo* k = &h->kern;
+  int cap = h->grid_cap;
+  // tensor-core kernels take the tensor maps as a second parameter (unused
+  // by the per-thread-copy kernels, but always passed, zeroed)
+  static const pic::TmaParams kNoMaps{};
+  const pic::TmaParams* tp = &kNoMaps;
+  if (h->has_tma) {
+    const long long words = p.lat_per_image * p.B;
+    bool ok = h->tma_key_ptr == p.latents && h->tma_key_words == words;
+    if (!ok) {
+      h->tma_key_ptr = nullptr;
+      ok = encode_latent_map(h->tma_cache, p);
+      if (ok) {
+        h->tma_key_ptr = p.latents;
+        h->tma_key_words = words;
+      }
+    }
+    if (ok) {
+      k = &h->kern_tma;
+      cap = h->grid_cap_tma;
+      tp = &h->tma_cache;
+    }
+  }
+  long long grid = p.total_tiles < cap ? p.total_tiles : cap;
   if (grid < 1) grid = 1;
-  void* args[] = {const_cast<DecodeParams*>(&p)};
-  cudaError_t e = cudaLaunchKernel(h->kern.fn, dim3(static_cast<unsigned>(grid)),
-                                   dim3(h->kern.threads), args, h->kern.smem_bytes, stream);
+  void* args[] = {const_cast<DecodeParams*>(&p), const_cast<pic::TmaParams*>(tp)};
+  cudaError_t e = cudaLaunchKernel(k->fn, dim3(static_cast<unsigned>(grid)), dim3(k->threads), args,
+                                   k->smem_bytes, stream);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return PIC_ERR_CUDA;
@@ -243,6 +316,28 @@ int pic_decode_create(const pic_arch* arch, pic_decoder** out) {
     return PIC_ERR_UNSUPPORTED;
   }
 
+  // the TMA-staged twin, where the arch has one
+  const KernelInfo* twin = nullptr;
+  int per_sm_tma = 0;
+  for (int i = 0; i < n && i < 32; ++i)
+    if (kernel_matches(table[i], arch, true)) {
+      twin = &table[i];
+      break;
+    }
+  if (arch->staging == PIC_STAGING_COPIES || (arch->staging == PIC_STAGING_AUTO && twin && !twin->tma_default))
+    twin = nullptr;
+  if (arch->staging == PIC_STAGING_TMA && !twin) return PIC_ERR_UNSUPPORTED;
+  if (twin && (twin->smem_bytes > static_cast<int>(prop.sharedMemPerBlockOptin) || !regs_match(*twin) ||
+               cudaFuncSetAttribute(twin->fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    twin->smem_bytes) != cudaSuccess ||
+               cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_tma, twin->fn, twin->threads,
+                                                             twin->smem_bytes) != cudaSuccess ||
+               per_sm_tma < 1)) {
+    cudaGetLastError();
+    if (arch->staging == PIC_STAGING_TMA) return PIC_ERR_UNSUPPORTED;
+    twin = nullptr;  // the per-thread-copy kernel serves every call
+  }
+
   pic_decoder* h = new (std::nothrow) pic_decoder();
   if (!h) return PIC_ERR_ALLOC;
   h->arch = *arch;
@@ -250,6 +345,11 @@ int pic_decode_create(const pic_arch* arch, pic_decoder** out) {
   h->sm_count = prop.multiProcessorCount;
   h->kern = k;
   h->grid_cap = per_sm * prop.multiProcessorCount;
+  if (twin) {
+    h->has_tma = true;
+    h->kern_tma = *twin;
+    h->grid_cap_tma = per_sm_tma * prop.multiProcessorCount;
+  }
   h->n_params = pic_param_count(arch);
   if (cudaMalloc(&h->d_status, sizeof(int)) != cudaSuccess) {
     cudaGetLastError();
@@ -434,7 +534,10 @@ void pic_decode_destroy(pic_decoder* h) {
   delete h;
 }
 
-const char* pic_decode_kernel_name(const pic_decoder* h) { return h ? h->kern.name : ""; }
+const char* pic_decode_kernel_name(const pic_decoder* h) {
+  if (!h) return "";
+  return h->has_tma ? h->kern_tma.name : h->kern.name;
+}
 
 }  // extern "C"
 
@@ -598,6 +701,22 @@ extern "C" int pic_decode_batch_noalloc(const pic_arch* arch, int B, const int32
   rc = noalloc_kernel(dev, h.kern, &per_sm);
   if (rc != PIC_OK) return rc;
   h.grid_cap = per_sm * d.sms;
+  // the TMA-staged twin, as pic_decode_create picks it (its tensor maps are
+  // encoded on the host for each call: no device memory)
+  for (int i = 0; i < n && i < 32; ++i)
+    if (kernel_matches(table[i], arch, true)) {
+      if (arch->staging == PIC_STAGING_COPIES ||
+          (arch->staging == PIC_STAGING_AUTO && !table[i].tma_default))
+        break;
+      int per_sm_tma = 0;
+      if (table[i].smem_bytes <= d.smem_optin && noalloc_kernel(dev, table[i], &per_sm_tma) == PIC_OK) {
+        h.has_tma = true;
+        h.kern_tma = table[i];
+        h.grid_cap_tma = per_sm_tma * d.sms;
+      }
+      break;
+    }
+  if (arch->staging == PIC_STAGING_TMA && !h.has_tma) return PIC_ERR_UNSUPPORTED;
   h.n_params = pic_param_count(arch);
   h.d_status = d.scratch;
 

@@ -18,7 +18,10 @@ struct KernelInfo {
   int regs_at_launch;  // registers per thread the kernel must be built with (0: any)
   int smem_bytes;  // dynamic shared memory per CTA
   int tile_px;     // pixels per tile (one tile = a run of one image row)
-  const void* fn;  // __global__ function taking (DecodeParams)
+  int tma;         // 1: stages the latents with TMA (needs valid TmaParams)
+  int tma_default; // (TMA kernels) 1: PIC_STAGING_AUTO picks it over its per-thread-copy twin
+  const void* fn;  // __global__ function taking (DecodeParams), or (DecodeParams,
+                   // TmaParams) for the tensor-core kernels (precision 1)
 };
 
 int fp32_kernels(KernelInfo* out, int cap);        // all of them
@@ -27,5 +30,6 @@ KernelInfo fp32_generic_kernel_info(int latent_format);
 int tc_kernels(KernelInfo* out, int cap);     // both latent formats
 int tc_kernels_fp32lat(KernelInfo* out, int cap);  // the fp32-latent ones (own translation unit)
 int tc_kernels_sweep(KernelInfo* out, int cap);    // the width ablation's (own translation unit)
+int tc_kernels_tma(KernelInfo* out, int cap);      // TMA-staged variants (own translation unit)
 
 }  // namespace pic

@@ -41,6 +41,12 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// Arrives on the mbarrier and adds `bytes` to the transaction count its
+// current phase waits for (the bytes an asynchronous copy will deliver).
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
 __device__ __forceinline__ void fence_mbar_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
@@ -59,6 +65,19 @@ __device__ __forceinline__ void cp_async_commit() {
 }
 __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
+// Tensor-map (TMA) load of the 1-D box of the map that starts at element x
+// into this CTA's shared memory at dst (16-byte aligned), completing the
+// box's bytes on the mbarrier bar.  The map lives in kernel parameter space
+// (__grid_constant__); x times the element size must be a multiple of 16
+// bytes.  Elements past the tensor's end read as zero.
+__device__ __forceinline__ void tma_load_1d(uint32_t dst, const void* tmap, int x, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.1d.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2}], [%3];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(bar)
+      : "memory");
 }
 
 // Named barrier over `count` threads (a warpgroup or the CTA).

@@ -39,6 +39,8 @@ PIC_OUT_F32_CHW = 0
 PIC_OUT_F32_HWC = 1
 PIC_OUT_U8_HWC = 2
 OUTPUTS = {"f32_chw": PIC_OUT_F32_CHW, "f32_hwc": PIC_OUT_F32_HWC, "u8_hwc": PIC_OUT_U8_HWC}
+PIC_STAGING_AUTO, PIC_STAGING_COPIES, PIC_STAGING_TMA = 0, 1, 2
+STAGINGS = {"auto": PIC_STAGING_AUTO, "copies": PIC_STAGING_COPIES, "tma": PIC_STAGING_TMA}
 
 
 class pic_arch(ctypes.Structure):
@@ -55,6 +57,7 @@ class pic_arch(ctypes.Structure):
         ("max_batch", ctypes.c_int),
         ("latent_format", ctypes.c_int),
         ("output_format", ctypes.c_int),
+        ("staging", ctypes.c_int),
     ]
 
 
@@ -136,7 +139,7 @@ class PicError(RuntimeError):
 
 
 def make_arch(L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1, max_W=1,
-              max_batch=1, latent="int32", output="f32_chw") -> pic_arch:
+              max_batch=1, latent="int32", output="f32_chw", staging="auto") -> pic_arch:
     a = pic_arch()
     a.num_levels, a.channels_per_level, a.num_layers = L, C, len(dims) - 1
     for k, d in enumerate(dims):
@@ -147,6 +150,7 @@ def make_arch(L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1, max
     a.max_H, a.max_W, a.max_batch = max_H, max_W, max_batch
     a.latent_format = LATENTS[latent] if isinstance(latent, str) else int(latent)
     a.output_format = OUTPUTS[output] if isinstance(output, str) else int(output)
+    a.staging = STAGINGS[staging] if isinstance(staging, str) else int(staging)
     return a
 
 
@@ -421,9 +425,9 @@ class Decoder:
     writes, not contiguous, or on the wrong side of the host/device split."""
 
     def __init__(self, L, C, dims, act="relu", precision="fp32", clamp=True, max_H=1,
-                 max_W=1, max_batch=1, latent="int32", output="f32_chw"):
+                 max_W=1, max_batch=1, latent="int32", output="f32_chw", staging="auto"):
         self.arch = make_arch(L, C, dims, act, precision, clamp, max_H, max_W, max_batch, latent,
-                              output)
+                              output, staging)
         self.latent = latent
         self.L, self.C, self.dims, self.precision = L, C, tuple(dims), precision
         self._need = {}
@@ -433,9 +437,9 @@ class Decoder:
 
     @classmethod
     def for_workload(cls, wl, precision: str, clamp=True, max_batch=None, latent="int32",
-                     output="f32_chw"):
+                     output="f32_chw", staging="auto"):
         return cls(wl.L, wl.C, wl.dims, wl.act, precision, clamp, wl.H, wl.W,
-                   max_batch or wl.B, latent, output)
+                   max_batch or wl.B, latent, output, staging)
 
     @property
     def kernel_name(self) -> str:

@@ -15,11 +15,12 @@ ORACLE_THREADS = max(1, min(16, os.cpu_count() or 1))
 
 
 def gpu_decode(wl: wk.Workload, x: wk.Inputs, precision: str, clamp: bool = True,
-               batch_host: bool = False) -> np.ndarray:
+               batch_host: bool = False, staging: str = "auto") -> np.ndarray:
     """Decodes every image of x on the GPU; returns fp32 [B][3][H][W] (host)."""
     import torch
     from paper_2609_09020_gb300.pic import Decoder
-    dec = Decoder.for_workload(wl, precision, clamp=clamp, max_batch=x.latents.shape[0])
+    dec = Decoder.for_workload(wl, precision, clamp=clamp, max_batch=x.latents.shape[0],
+                               staging=staging)
     B = x.latents.shape[0]
     w = x.weights_for(precision)
     if batch_host:

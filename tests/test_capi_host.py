@@ -174,6 +174,9 @@ def test_noalloc_entry_and_size_helpers_reject_bad_arguments(lib):
     wide = pic.make_arch(2, 1, (2, 256, 3), max_H=8, max_W=8)        # width above the envelope
     assert lib.pic_decode_batch_noalloc(ctypes.byref(wide), 1, p, p, p, 8, 8, p,
                                         None) == pic.PIC_ERR_UNSUPPORTED
+    staged = pic.make_arch(2, 1, (2, 16, 3), max_H=8, max_W=8, staging=3)  # no such staging
+    assert lib.pic_decode_batch_noalloc(ctypes.byref(staged), 1, p, p, p, 8, 8, p,
+                                        None) == pic.PIC_ERR_UNSUPPORTED
     assert lib.pic_param_count(None) == -1
     assert pic.pic_latent_count(8, 8, 31, 1) == -1 and pic.pic_latent_count(8, 8, 1, 0) == -1
     assert pic.pic_latent_count(1, 1, 30, 4) == 30 * 4   # every level of a 1x1 image is 1x1

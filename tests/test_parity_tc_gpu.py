@@ -117,3 +117,35 @@ def test_repeated_calls_are_deterministic():
     a = gpu_decode(wl, x, P)
     b = gpu_decode(wl, x, P)
     assert np.array_equal(a, b)
+
+
+# Latent staging: the TMA-staged kernels (the tile's full-resolution row as
+# TMA boxes) and the per-thread-copy kernels compute the same arithmetic on
+# the same words, so their outputs are equal bit for bit; every workload
+# architecture runs both, the one PIC_STAGING_AUTO does not pick on top of
+# the checks above.
+STAGING_CASES = [
+    wk.WORKLOADS["c5"].replace(seeds=(100, 101, 102), name="c5x3"),
+    wk.WORKLOADS["c4"],
+    wk.WORKLOADS["c3"],
+    wk.WORKLOADS["c2"],
+    wk.WORKLOADS["c1"],
+    EDGE[1],  # 3 x 200: one tile per row, ragged tail
+    EDGE[2],  # 129 x 131, batch of 3
+]
+
+
+@pytest.mark.parametrize("wl", STAGING_CASES, ids=lambda w: w.name)
+def test_tma_and_copy_staging_agree(orc, wl):
+    from paper_2609_09020_gb300.pic import Decoder
+    x = wk.make_inputs(wl)
+    tma = gpu_decode(wl, x, P, staging="tma")
+    cp = gpu_decode(wl, x, P, staging="copies")
+    assert np.array_equal(tma, cp), wl.name
+    want = oracle_full(orc, wl, x, 0, P)  # the kernels' own bound, image 0
+    d, where = max_abs_diff(tma[0], want)
+    assert d <= SPLIT_BOUND, (wl.name, d, where)
+    for staging, suffix in (("tma", "_tma"), ("copies", "")):
+        dec = Decoder.for_workload(wl, P, staging=staging)
+        assert dec.kernel_name.endswith(suffix) and ("_tma" in dec.kernel_name) == (staging == "tma")
+        dec.close()

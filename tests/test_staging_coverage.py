@@ -120,3 +120,88 @@ def test_workload_widths_take_the_expected_scheme():
     for W, L, fast in [(256, 4, True), (768, 7, True), (1920, 7, True), (3840, 8, True),
                        (131, 7, False), (383, 8, False), (200, 7, False), (1, 7, False)]:
         assert ((L - 1 <= 7) and W % (1 << (L - 1)) == 0) == fast
+
+
+# ---- TMA staging (the TMA-staged kernels).  Per tile, the group's issuing
+# warp loads every (level, channel, row) segment as one box of a 1-D tensor
+# map over the call's latent words: level 0 the tile's 128 words of row y,
+# level l >= 1 the words u_start .. u_start + NCOL(l) - 1 of rows i0 and i1 of
+# the tile row's vertical tap.  A box starts at the segment's first word s
+# rounded down to a multiple of 4 (TMA's 16-byte rule), so column k of the
+# segment is box word (s & 3) + k.
+
+def box_w(l):
+    """tma_box_w of the kernels: level 0 128 + 4 words; level l >= 1 NCOL(l)
+    + 3 rounded up to a multiple of 4."""
+    return TILE + 4 if l == 0 else -(-(ncol(l) + 3) // 4) * 4
+
+
+def test_box_widths():
+    assert [box_w(l) for l in range(10)] == [132, 72, 40, 24, 16, 12, 12, 8, 8, 8]
+    assert all(box_w(l) % 4 == 0 and box_w(l) <= 256 for l in range(13))
+    # the largest in-box index a read can take: 3 + (segment length - 1)
+    assert 3 + TILE - 1 < box_w(0)
+    assert all(3 + ncol(l) - 1 < box_w(l) for l in range(1, 13))
+
+
+@pytest.mark.parametrize("L", [2, 4, 7, 8, 12])
+def test_tma_segment_columns_stay_inside_the_box(L):
+    """The column the vertical pass reads, clamp(u_start + i, 0, W_l - 1) -
+    u_start, lies in [0, NCOL(l)) for every item i of every tile, both tap
+    schemes, so (s & 3) + column stays inside the box."""
+    for W in WIDTHS:
+        fast = (L - 1 <= 7) and W % (1 << (L - 1)) == 0
+        for l in range(1, L):
+            Wl = level_size(W, l)
+            ratio32 = np.float32(Wl / W)
+            for x0 in range(0, W, TILE):
+                u_start = (x0 >> l) - 1 if fast else int(tap32(x0, ratio32, Wl)[0])
+                assert u_start >= -1
+                col = np.clip(u_start + np.arange(ncol(l)), 0, Wl - 1) - u_start
+                assert col.min() >= 0 and col.max() < ncol(l), (W, L, l, x0)
+                for s in range(4):  # any alignment of the segment start
+                    assert (s & 3) + col.max() < box_w(l)
+
+
+def test_tma_box_reads_the_defined_words():
+    """Words s & ~3 .. of a buffer, read at (s & 3) + k, are words s + k: a
+    tile's segments come back whatever the alignment of their start,
+    including segments that begin one word before a row (u_start = -1,
+    never read: the clamp takes column 0) and segments at the buffer's end
+    (zero fill past it, never read either)."""
+    rng = np.random.default_rng(3)
+    buf = rng.integers(-63, 64, 1000)
+    for s in list(range(0, 40)) + [995, 996, 999]:
+        for bw in (8, 12, 72, 132):
+            x = s & ~3
+            box = np.array([buf[x + k] if x + k < buf.size else 0 for k in range(bw)])
+            n = min(bw - 3, buf.size - s)
+            assert np.array_equal(box[(s & 3) + np.arange(n)], buf[s:s + n])
+
+
+@pytest.mark.parametrize("L,C", [(4, 1), (7, 1), (8, 2), (12, 4)])
+def test_tma_boxes_and_slots(L, C):
+    """The issuing warp's lane q -> (level, channel, row) map hits every
+    segment of a tile exactly once, and the segments' slots in a buffer are
+    disjoint, start on 128 bytes (a tiled TMA copy's shared-memory
+    destination), hold their box and fill the buffer (TmaSlots)."""
+    rows = lambda l: 1 if l == 0 else 2
+    slot = lambda l: -(-box_w(l) * 4 // 128) * 128
+    def off(l, c, r):
+        o = sum(C * rows(k) * slot(k) for k in range(l))
+        return o + (c * rows(l) + r) * slot(l)
+    n = C * (2 * L - 1)
+    seen = []
+    for q in range(n):
+        if q < C:
+            l, c, r = 0, q, 0
+        else:
+            q2 = q - C
+            l, c, r = 1 + q2 // (2 * C), (q2 >> 1) % C, q2 & 1
+        assert 0 <= l < L and 0 <= c < C and r < rows(l)
+        seen.append((l, c, r))
+    assert len(set(seen)) == n == sum(C * rows(l) for l in range(L))
+    spans = sorted((off(l, c, r), off(l, c, r) + slot(l), box_w(l) * 4) for l, c, r in seen)
+    assert all(a % 128 == 0 and box <= e - a for a, e, box in spans)
+    assert all(spans[k][1] == spans[k + 1][0] for k in range(n - 1))
+    assert spans[0][0] == 0 and spans[-1][1] == off(L, 0, 0)
