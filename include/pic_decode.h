@@ -66,7 +66,15 @@ typedef enum {
      * fp32 accumulation.  Every activation operand (features and hidden
      * values) is split into two fp16 terms hi + lo, so the products carry
      * about 22 significant bits; the weights are used exactly as given. */
-    PIC_PREC_FP16_TC = 1
+    PIC_PREC_FP16_TC = 1,
+    /* fp16 weights; tensor cores as PIC_PREC_FP16_TC, with the lo term of
+     * every hidden operand in fp8 (e4m3) against an e4m3 copy of the
+     * weights, the hidden activations kept scaled by 2^6: about 15
+     * significant bits per product and half the lo MMAs.  For ReLU nets with
+     * a hidden width of 64 and the output layer on the tensor cores (the
+     * 7-64-64-3 architecture); hidden activations must stay below 1024 in
+     * magnitude. */
+    PIC_PREC_FP16_TC_LO8 = 2
 } pic_prec;
 
 typedef enum {
@@ -225,6 +233,22 @@ int pic_decode_batch_noalloc(const pic_arch *arch, int B, const int32_t *latents
  * Errors: PIC_ERR_CUDA.
  */
 int pic_decode_noalloc_check(void *stream);
+
+/*
+ * Test hook of the bounded device-side waits (no counterpart in the paper;
+ * production code never calls it).  Every tensor-core decode launched while
+ * withhold_arrival = 1 has one decoding thread of its first CTA skip one
+ * mbarrier arrival, so that a wait of that CTA runs out and the kernel takes
+ * its abort path (status word raised, remaining work skipped, outstanding
+ * MMAs and copies drained, tensor memory freed); spin_limit > 0 replaces the
+ * number of polls a wait makes before giving up (seconds' worth by default),
+ * so that the wait runs out in microseconds.  pic_decode_test_wait_fault(0,
+ * 0) restores production behaviour.  Process-wide, for all handles and the
+ * allocation-free entry point; not synchronised with decode calls in other
+ * host threads.
+ * Errors: PIC_ERR_INVALID_ARG (withhold_arrival not 0 or 1).
+ */
+int pic_decode_test_wait_fault(int withhold_arrival, unsigned spin_limit);
 
 /* Frees the handle and its device state.  NULL is a no-op.  Synchronises the
  * device first, so that no kernel of this handle is still running. */

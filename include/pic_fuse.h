@@ -26,7 +26,7 @@ extern "C" {
  * For B images:
  *   arch        : the decoder's architecture (num_layers >= 2); its precision
  *                 selects the output dtype (fp32, or IEEE half rounded to
- *                 nearest for PIC_PREC_FP16_TC)
+ *                 nearest for the tensor-core precisions)
  *   shared      : float, device, [pic_param_count(arch)] -- the g_s weights in
  *                 the layout of pic_decode.h
  *   mod         : float, device, [B][4][C'] with C' = dims[num_layers - 1]:

@@ -78,7 +78,7 @@ extern "C" int pic_fuse_modulation(const pic_arch* arch, int B, const float* sha
     if (k == n - 1) last = P;
     P += static_cast<long long>(arch->dims[k + 1]) * (arch->dims[k] + 1);
   }
-  const bool half = arch->precision == PIC_PREC_FP16_TC;
+  const bool half = arch->precision == PIC_PREC_FP16_TC || arch->precision == PIC_PREC_FP16_TC_LO8;
   if (!half && arch->precision != PIC_PREC_FP32) return PIC_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(weights_out) & 15u) != 0 ||
       (reinterpret_cast<uintptr_t>(shared) & 3u) != 0 || (reinterpret_cast<uintptr_t>(mod) & 3u) != 0)

@@ -17,7 +17,20 @@
 // and each layer computes W a_hi + W a_lo with fp32 accumulation, so the
 // products carry ~22 significant bits instead of fp16's 11.
 //
-// Operands of one 128-pixel tile (row r = pixel r = TMEM lane r):
+// Variant with the lo term in fp8 (LO8, PIC_PREC_FP16_TC_LO8; ReLU nets with
+// the output layer on the tensor cores): the hidden activations are kept
+// scaled by S = 2^6 -- the first layer's weights and every bias carry S
+// (exact, a power of two), ReLU commutes with it, and only the three outputs
+// are divided by S.  A hidden operand is a_hi = RZ_fp16(S h) against the
+// fp16 weights W plus a_lo = RN_e4m3(S h - a_hi) against an e4m3 copy of W
+// (kind::f8f6f4, K = 32 per instruction): half the lo MMAs and a quarter of
+// the lo operand's tensor memory, ~15 significant bits per product (S h -
+// a_hi is about 2^-11 S h, inside e4m3's range).  S |h| must stay below
+// fp16's 65504, i.e. |h| < 1024.
+//
+// Operands of one 128-pixel tile (row r = pixel r = TMEM lane r; LO8: hidden
+// A = [h_hi | h_lo] with h_lo in N/4 columns of four e4m3 each, and the lo
+// half of B the e4m3 copy of W_k, in its own shared tile):
 //   layer 0  A1 = [f_hi | f_lo | 1 | 0..]  smem, K1 = round16(2 D0 + 1); the bias
 //            B1 = [W_0  | W_0  | b_0 | 0..] b_0 rides along as the constant-1 column
 //   hidden   A  = [h_hi | h_lo]            TMEM, N/2 + N/2 columns (2 fp16 per column)
@@ -61,6 +74,7 @@
 #pragma once
 
 #include <cuda_fp16.h>
+#include <cuda_fp8.h>
 
 #include <type_traits>
 
@@ -74,7 +88,7 @@ namespace {
 using namespace tc;
 
 constexpr int kTile = 128;
-constexpr uint32_t kSpinLimit = 1u << 22;  // a few seconds of polling at most per wait
+constexpr uint32_t kSpinLimit = kWaitPolls;  // a few seconds of polling at most per wait
 
 __host__ __device__ constexpr int round_up(int v, int m) { return (v + m - 1) / m * m; }
 __host__ __device__ constexpr int pow2_at_least(int v) {
@@ -88,6 +102,11 @@ __host__ __device__ constexpr int pow2_at_least(int v) {
 // (row/8) * SBO + (k/8) * LBO with LBO = 128 B and SBO = 16 K bytes.
 __host__ __device__ constexpr uint32_t kmaj(int row, int k, int K) {
   return static_cast<uint32_t>((row >> 3) * (K * 16) + (k >> 3) * 128 + (row & 7) * 16 + (k & 7) * 2);
+}
+// The same for a [rows][K] tile of 8-bit elements: core matrix (row/8, k/16),
+// LBO = 128 B, SBO = 8 K bytes.
+__host__ __device__ constexpr uint32_t kmaj8(int row, int k, int K) {
+  return static_cast<uint32_t>((row >> 3) * (K * 8) + (k >> 4) * 128 + (row & 7) * 16 + (k & 15));
 }
 
 // Cooperative feature staging.  For level l >= 1 a 128-pixel row segment
@@ -125,9 +144,11 @@ struct ColLayout {
   static constexpr int total() { return off(L, 0); }
 };
 
-template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_>
+template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_, bool LO8_ = false>
 struct TcNet {
   static constexpr int C = C_, NL = NL_, D0 = D0_, N = N_, ACT = ACT_, NWG = NWG_;
+  static constexpr bool LO8 = LO8_;
+  static constexpr float kS = LO8 ? 64.0f : 1.0f;  // scale of the hidden activations (LO8)
   static constexpr int L = D0 / C;
   static constexpr int K1 = round_up(2 * D0 + 1, 16);
   // Output layer on the CUDA cores (fp32, one MMA round trip less per tile)
@@ -161,11 +182,17 @@ struct TcNet {
   // the CUDA cores fp32, per pair q of inputs 8 floats (w0 w0 | w1 w1 |
   // w2 w2 | 0 0 at inputs 2q, 2q+1), then the 3 biases
   static constexpr int BO_BYTES = OUTCC ? (N / 2) * 32 + 16 : NOUT * KB * 2;
+  // LO8: e4m3 copies of the hidden layers' and the output layer's W, K-major
+  // [rows][N] bytes (core matrices of 8 rows x 16 bytes)
+  static constexpr int BL_BYTES = LO8 ? N * N : 0;
+  static constexpr int BLO_BYTES = LO8 ? NOUT * N : 0;
   static constexpr int ONES_BYTES = kTile * 16 * 2;      // constant A tile [1 0..0] per row
   static constexpr int OFF_B1 = CTRL;
   static constexpr int OFF_BH = OFF_B1 + B1_BYTES;
   static constexpr int OFF_BO = OFF_BH + (NL - 2) * BH_BYTES;
-  static constexpr int OFF_ONES = round_up(OFF_BO + BO_BYTES, 128);
+  static constexpr int OFF_BL = round_up(OFF_BO + BO_BYTES, 128);
+  static constexpr int OFF_BLO = OFF_BL + (NL - 2) * BL_BYTES;
+  static constexpr int OFF_ONES = round_up(OFF_BLO + BLO_BYTES, 128);
   static constexpr int OFF_WG = round_up(OFF_ONES + ONES_BYTES, 128);
   static constexpr int A1_BYTES = kTile * K1 * 2;
   static constexpr int COL_BYTES = round_up(ColLayout<L, C>::total() * 4, 128);
@@ -181,6 +208,8 @@ struct TcNet {
   static constexpr int TMEM_COLS = pow2_at_least(NWG * 2 * N);
   static_assert(N % 16 == 0 && N >= 16 && N <= 128, "hidden width must be 16..128, multiple of 16");
   static_assert(NL >= 2, "the tensor-core path needs at least one hidden layer");
+  static_assert(!LO8 || (ACT == ACT_RELU && !OUTCC && N % 32 == 0),
+                "the fp8 lo term: ReLU nets, output layer on the tensor cores, K steps of 32");
   static_assert(TMEM_COLS <= 512, "tensor memory holds 512 columns");
   static_assert(NISSUE == 4 && MMA_WARP % 4 == 0, "the issuing warps form one warpgroup");
   static_assert(REG_DECODE >= MAXREG && REG_DECODE * NWG * 128 + REG_ISSUE * 32 * NISSUE <= MAXREG * THREADS,
@@ -191,12 +220,14 @@ struct TcNet {
                 "TMA buffers on 128-byte boundaries");
 };
 
-// Bounded mbarrier wait.  Returns false (and raises the abort flag and the
-// handle's status word) if the phase does not complete in time, or if
+// Bounded mbarrier wait: at most `limit` polls (the launch's spin_limit;
+// kWaitPolls in production).  Returns false (and raises the abort flag and
+// the handle's status word) if the phase does not complete in time, or if
 // another thread has already aborted.
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                             int* status) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+                                             int* status, uint32_t limit) {
+  if (mbar_test_wait(bar, parity)) return true;  // a completed phase: no blocking probe
+  for (uint32_t i = 0; i < limit; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((i & 63u) == 63u) {
       if (*abort_flag) return false;
@@ -219,7 +250,12 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
                                                 const int (&dims)[Net::NL + 1], int tid, int nthr) {
   constexpr int N = Net::N, D0 = Net::D0, K1 = Net::K1, NL = Net::NL, KB = Net::KB;
   const __half zero = __float2half_rn(0.0f);
-  // layer 0: [W | W | b | 0]
+  // LO8: S times an fp16 value (exact: S is a power of two and |v| < 1024)
+  auto scaled = [](__half v) {
+    if constexpr (Net::LO8) return __float2half_rn(__half2float(v) * Net::kS);
+    else return v;
+  };
+  // layer 0: [W | W | b | 0] (LO8: S W, S b)
   {
     const int d1 = dims[1];
     const __half* W0 = w;
@@ -228,14 +264,15 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
       const int n = e / K1, j = e - n * K1;
       __half v = zero;
       if (n < d1) {
-        if (j < D0) v = ldh(W0 + n * D0 + j);
-        else if (j < 2 * D0) v = ldh(W0 + n * D0 + (j - D0));
-        else if (j == 2 * D0) v = ldh(b0 + n);
+        if (j < D0) v = scaled(ldh(W0 + n * D0 + j));
+        else if (j < 2 * D0) v = scaled(ldh(W0 + n * D0 + (j - D0)));
+        else if (j == 2 * D0) v = scaled(ldh(b0 + n));
       }
       *reinterpret_cast<__half*>(smem + Net::OFF_B1 + kmaj(n, j, K1)) = v;
     }
   }
-  // hidden layers and output: [W | b 0..0], zero padded to N (or 16) rows
+  // hidden layers and output: [W | b 0..0] (LO8: S b), zero padded to N (or
+  // 16) rows; LO8 also the e4m3 copy of W, [rows][N] bytes
   const __half* p = w + dims[1] * D0 + dims[1];
 #pragma unroll
   for (int k = 1; k < NL; ++k) {
@@ -261,9 +298,19 @@ __device__ __forceinline__ void load_weights_tc(uint8_t* smem, const __half* w,
       __half v = zero;
       if (n < dout) {
         if (j < din) v = ldh(Wk + n * din + j);
-        else if (j == N) v = ldh(bk + n);
+        else if (j == N) v = scaled(ldh(bk + n));
       }
       *reinterpret_cast<__half*>(base + kmaj(n, j, KB)) = v;
+    }
+    if constexpr (Net::LO8) {
+      uint8_t* lo = smem + (out_layer ? Net::OFF_BLO : Net::OFF_BL + (k - 1) * Net::BL_BYTES);
+      for (int e = tid; e < rows * N; e += nthr) {
+        const int n = e / N, j = e - n * N;
+        uint8_t v = 0;
+        if (n < dout && j < din)
+          v = __nv_cvt_float_to_fp8(__half2float(ldh(Wk + n * din + j)), __NV_SATFINITE, __NV_E4M3);
+        lo[kmaj8(n, j, N)] = v;
+      }
     }
     p = bk + dout;
   }
@@ -338,6 +385,30 @@ __device__ __forceinline__ void hidden_epilogue(uint32_t t_acc, uint32_t t_a) {
     }
     tmem_st8(t_a + h0 / 2, hl);
     tmem_st8(t_a + N / 2 + h0 / 2, hl + 8);
+  }
+  tmem_st_wait();
+}
+
+// LO8: hidden epilogue with the lo terms in e4m3: hi pairs at t_a (N/2
+// columns), lo quads at t_a + N/2 (N/4 columns), 16 values at a time.
+template <class Net>
+__device__ __forceinline__ void hidden_epilogue_lo8(uint32_t t_acc, uint32_t t_a) {
+  constexpr int N = Net::N;
+#pragma unroll
+  for (int h0 = 0; h0 < N; h0 += 16) {
+    uint32_t acc[16];
+    tmem_ld16(t_acc + h0, acc);
+    tmem_ld_wait();
+    uint32_t hi[8], lo[4];
+#pragma unroll
+    for (int q = 0; q < 8; q += 2) {
+      uint16_t l0, l1;
+      split_pair_e4m3(__uint_as_float(acc[2 * q]), __uint_as_float(acc[2 * q + 1]), hi[q], l0);
+      split_pair_e4m3(__uint_as_float(acc[2 * q + 2]), __uint_as_float(acc[2 * q + 3]), hi[q + 1], l1);
+      lo[q / 2] = static_cast<uint32_t>(l0) | (static_cast<uint32_t>(l1) << 16);
+    }
+    tmem_st8(t_a + h0 / 2, hi);
+    tmem_st4(t_a + N / 2 + h0 / 4, lo);
   }
   tmem_st_wait();
 }
@@ -556,7 +627,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             }
           }
           mbar_arrive(my_col);  // the group's column buffer is complete once all 128 arrived
-          if (!__all_sync(0xffffffffu, wait_bounded(my_col, col_phase, abort_flag, p.status)))
+          if (!__all_sync(0xffffffffu, wait_bounded(my_col, col_phase, abort_flag, p.status, p.spin_limit)))
             return false;
           col_phase ^= 1u;
           // horizontal pass + level 0
@@ -621,7 +692,11 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         if (w < n_tiles) {
           prefetch(cy, ctx * kTile);
           ok = features(cy, ctx * kTile, 0);
-          if (ok) mbar_arrive(my_a1);
+          // p.test_fault (tests of the bounded waits only; 0 in every
+          // production launch): one thread of CTA 0's first group withholds
+          // its first a1_full arrival, so the issuing warp's wait runs out
+          const bool withhold = p.test_fault && blockIdx.x == 0 && w == 0 && r == 5 && seg == t_begin;
+          if (ok && !withhold) mbar_arrive(my_a1);
         }
         for (int i = w; i < n_tiles && ok; i += NWG) {
           if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
@@ -636,7 +711,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           if constexpr (Net::OUTCC) {
             // hidden epilogues up to the last one, which runs the output layer
             for (int k = 0; k < NL - 2 && ok; ++k) {
-              if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
+              if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status, p.spin_limit))) {
                 ok = false;
                 break;
               }
@@ -648,7 +723,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
               if (k == 0 && has_next) ok = features(ny, ntx * kTile, knext);  // overlaps layer 1
             }
             if (!ok) break;
-            if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
+            if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status, p.spin_limit))) break;
             acc_phase ^= 1u;
             tc_fence_after();
             float rgb[3];
@@ -663,21 +738,22 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             if (!ok) break;
           } else {
             for (int k = 0; k < NL - 1 && ok; ++k) {
-              if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) {
+              if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status, p.spin_limit))) {
                 ok = false;
                 break;
               }
               acc_phase ^= 1u;
               tc_fence_after();
-              hidden_epilogue<Net>(t_acc, t_a);
+              if constexpr (Net::LO8) hidden_epilogue_lo8<Net>(t_acc, t_a);
+              else hidden_epilogue<Net>(t_acc, t_a);
               tc_fence_before();
               mbar_arrive(my_a);
               if (k == 0 && has_next) ok = features(ny, ntx * kTile, knext);  // overlaps layer 1
             }
             if (!ok) break;
 
-            // ---- output layer: bias, clamp, store ----
-            if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status))) break;
+            // ---- output layer: bias, clamp, store (LO8: the accumulator holds S o) ----
+            if (!__all_sync(0xffffffffu, wait_bounded(my_c, acc_phase, abort_flag, p.status, p.spin_limit))) break;
             acc_phase ^= 1u;
             tc_fence_after();
             uint32_t o[4];
@@ -686,8 +762,10 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             tc_fence_before();
             if (has_next) mbar_arrive(my_a1);  // accumulator read: the next tile's layer 0 may start
             const int x = x0 + r;
+            constexpr float inv_s = 1.0f / Net::kS;  // exact: a power of two
             if (x < p.W)
-              store_rgb(p, b, y, x, __uint_as_float(o[0]), __uint_as_float(o[1]), __uint_as_float(o[2]));
+              store_rgb(p, b, y, x, __uint_as_float(o[0]) * inv_s, __uint_as_float(o[1]) * inv_s,
+                        __uint_as_float(o[2]) * inv_s);
             cy = ny;
             ctx = ntx;
           }
@@ -695,6 +773,9 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       }
       seg = seg_end;
     }
+    // A wait that gave up may leave this thread's next-tile copies in
+    // flight: they land before the CTA's shared memory is released.
+    cp_async_wait_all();
   } else {
     setmaxnreg_dec<Net::REG_ISSUE>();
     for (long long seg = t_begin; seg < t_end;) {
@@ -721,6 +802,11 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         const uint64_t dONES = smem_desc(sbase + Net::OFF_ONES, 128, 16 * 16);
         constexpr uint64_t kStep = 256 >> 4;              // one K-step (16 fp16) = 256 B
         constexpr uint64_t kLayer = Net::BH_BYTES >> 4;   // next hidden layer's weights
+        // LO8: the e4m3 copies, K-major with N bytes per row (one K step of
+        // 32 e4m3 = two core matrices = 256 B, as for fp16)
+        const uint64_t dBL = smem_desc(sbase + Net::OFF_BL, 128, 8 * N);
+        const uint64_t dBLO = smem_desc(sbase + Net::OFF_BLO, 128, 8 * N);
+        constexpr uint64_t kLayerL = (Net::BL_BYTES >> 4);
         static_assert(Net::WG_BYTES % 16 == 0 && Net::BH_BYTES % 16 == 0, "16-byte aligned operands");
         const uint32_t d = tmem + static_cast<uint32_t>(w * 2 * N);
         const uint32_t ta = d + N;
@@ -754,7 +840,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         auto hand_over = [&](int buf) -> bool {
           const uint32_t bar = bar_stage + 16 * w + 8 * buf;
           const bool landed =
-              __all_sync(0xffffffffu, wait_bounded(bar, (stage_wait >> buf) & 1u, abort_flag, p.status));
+              __all_sync(0xffffffffu, wait_bounded(bar, (stage_wait >> buf) & 1u, abort_flag, p.status, p.spin_limit));
           if (!landed) return false;  // still in flight: the exit drain waits for it
           stage_wait ^= 1u << buf;
           if (lane == 0) mbar_arrive(bar_col + 8 * w);
@@ -778,7 +864,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           for (int k = 0; k < (Net::OUTCC ? NL - 1 : NL); ++k) {  // OUTCC: no output-layer MMA
             const uint32_t bar = k == 0 ? my_a1 : my_a;
             const uint32_t par = k == 0 ? (a1_phase & 1u) : (a_phase & 1u);
-            if (!__all_sync(0xffffffffu, wait_bounded(bar, par, abort_flag, p.status))) {
+            if (!__all_sync(0xffffffffu, wait_bounded(bar, par, abort_flag, p.status, p.spin_limit))) {
               ok = false;
               break;
             }
@@ -795,8 +881,14 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
                 const uint32_t id = out_layer ? id_out : id_hidden;
 #pragma unroll
                 for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + 8 * s, db + s * kStep, id, s > 0);  // hi
+                if constexpr (Net::LO8) {  // lo in e4m3: K = 32 per MMA, 8 columns of A each
+                  const uint64_t dl = out_layer ? dBLO : dBL + (k - 1) * kLayerL;
 #pragma unroll
-                for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
+                  for (int s = 0; s < N / 32; ++s) mma_e4m3_ta(d, ta + N / 2 + 8 * s, dl + s * kStep, id, 1);
+                } else {
+#pragma unroll
+                  for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
+                }
                 mma_f16(d, dONES, db + (N / 16) * kStep, id, 1);  // bias: [1 0..0] x [b 0..0]
               }
               mma_commit(my_c);
@@ -842,7 +934,7 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
       const uint32_t drain = bar_drain + 8 * (warp - Net::MMA_WARP);
       mma_commit(drain);
       int dummy = 0;
-      wait_bounded(drain, 0, reinterpret_cast<volatile int*>(&dummy), p.status);
+      wait_bounded(drain, 0, reinterpret_cast<volatile int*>(&dummy), p.status, kSpinLimit);
     }
   }
   tc_fence_before();
@@ -853,12 +945,12 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
   }
 }
 
-template <int C, int NL, int D0, int N, int ACT, int NWG, bool FL, bool TMA = false>
+template <int C, int NL, int D0, int N, int ACT, int NWG, bool FL, bool TMA = false, bool LO8 = false>
 KernelInfo make_tc(const char* name, const int* dims) {
-  using Net = TcNet<C, NL, D0, N, ACT, NWG>;
+  using Net = TcNet<C, NL, D0, N, ACT, NWG, LO8>;
   KernelInfo k{};
   k.name = name;
-  k.precision = 1;
+  k.precision = LO8 ? 2 : 1;
   k.latent_format = FL ? 1 : 0;
   k.C = C;
   k.n_layers = NL;

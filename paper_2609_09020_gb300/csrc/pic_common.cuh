@@ -52,7 +52,13 @@ struct DecodeParams {
   int dims[kMaxLayers + 1];
   int act;
   LevelGeom lv[kMaxLevels];
+  unsigned spin_limit;         // polls a bounded device-side wait makes before giving up
+  int test_fault;              // tests of the bounded waits only (0 in production)
 };
+
+// Polls a bounded device-side wait makes before it gives up (with a short
+// sleep between polls after the first few thousand): seconds at most.
+constexpr unsigned kWaitPolls = 1u << 22;
 
 // Tensor map for the TMA staging of the tensor-core kernels: the whole
 // latent buffer of the call (every image's pyramid) as one 1-D tensor of

@@ -4,6 +4,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 #include <new>
 
@@ -49,6 +50,11 @@ struct pic_decoder {
 
 namespace {
 
+// Test hook of the bounded device-side waits (pic_decode_test_wait_fault):
+// nonzero only while a test makes a wait run out on purpose.
+std::atomic<int> g_test_fault{0};
+std::atomic<unsigned> g_test_spin_limit{0};
+
 int level_size(int n, int l) { return static_cast<int>((static_cast<long long>(n) + (1LL << l) - 1) >> l); }
 
 bool arch_valid(const pic_arch* a) {
@@ -60,7 +66,9 @@ bool arch_valid(const pic_arch* a) {
   for (int k = 0; k <= a->num_layers; ++k)
     if (a->dims[k] < 1 || a->dims[k] > pic::kMaxDim) return false;
   if (a->hidden_act != PIC_ACT_RELU && a->hidden_act != PIC_ACT_GELU) return false;
-  if (a->precision != PIC_PREC_FP32 && a->precision != PIC_PREC_FP16_TC) return false;
+  if (a->precision != PIC_PREC_FP32 && a->precision != PIC_PREC_FP16_TC &&
+      a->precision != PIC_PREC_FP16_TC_LO8)
+    return false;
   if (a->clamp_output != 0 && a->clamp_output != 1) return false;
   if (a->max_H < 1 || a->max_W < 1 || a->max_batch < 1) return false;
   if (a->max_H > 65536 || a->max_W > 65536 || a->max_batch > 65536) return false;
@@ -174,6 +182,9 @@ void fill_params(const pic_decoder* h, DecodeParams& p, int B, const int32_t* la
   p.tiles_per_row = (W + tp - 1) / tp;
   p.tiles_per_image = static_cast<long long>(p.tiles_per_row) * H;
   p.total_tiles = p.tiles_per_image * B;
+  const unsigned test_limit = g_test_spin_limit.load(std::memory_order_relaxed);
+  p.spin_limit = test_limit ? test_limit : pic::kWaitPolls;
+  p.test_fault = g_test_fault.load(std::memory_order_relaxed);
 }
 
 int launch(pic_decoder* h, const DecodeParams& p, cudaStream_t stream) {
@@ -212,7 +223,7 @@ int launch(pic_decoder* h, const DecodeParams& p, cudaStream_t stream) {
   return PIC_OK;
 }
 
-size_t weight_elem_bytes(const pic_arch& a) { return a.precision == PIC_PREC_FP16_TC ? 2 : 4; }
+size_t weight_elem_bytes(const pic_arch& a) { return a.precision == PIC_PREC_FP32 ? 4 : 2; }
 
 // A kernel that moves registers between its warpgroups at run time assumes
 // the register count it was launched with; any other build is refused
@@ -523,6 +534,13 @@ int pic_decode_check(pic_decoder* h, void* stream) {
     }
     return PIC_ERR_TIMEOUT;
   }
+  return PIC_OK;
+}
+
+int pic_decode_test_wait_fault(int withhold_arrival, unsigned spin_limit) {
+  if (withhold_arrival != 0 && withhold_arrival != 1) return PIC_ERR_INVALID_ARG;
+  g_test_spin_limit.store(spin_limit, std::memory_order_relaxed);
+  g_test_fault.store(withhold_arrival, std::memory_order_relaxed);
   return PIC_OK;
 }
 

@@ -147,6 +147,18 @@ __device__ __forceinline__ void mma_f16_ta(uint32_t d_tmem, uint32_t a_tmem, uin
       "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// D[tmem] (+)= A[tmem] * B[smem desc]^T with e4m3 A and B (kind::f8f6f4),
+// fp32 accumulate: K = 32 per instruction, four e4m3 of K per 32-bit column
+// of A (element 4c + j in byte j).
+__device__ __forceinline__ void mma_e4m3_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 // Arrives on the mbarrier once every MMA issued so far by this thread has completed.
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
@@ -181,6 +193,11 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
 __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* r) {
   asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
                "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+               : "memory");
+}
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint32_t* r) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr), "r"(r[0]),
+               "r"(r[1]), "r"(r[2]), "r"(r[3])
                : "memory");
 }
 __device__ __forceinline__ void tmem_st_wait() {
@@ -271,6 +288,24 @@ __device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi2, uint
         : "=r"(hi2), "=r"(lo2)
         : "f"(a), "f"(b));
   }
+}
+
+// hi/lo split of a pair (a, b) with the lo terms in e4m3 (ReLU applied):
+// hi = RZ_fp16(relu(x)) as f16x2, lo = RN_e4m3(relu(x - hi)) as two bytes
+// (a's in the low byte).  x - hi is exact in fp32 (one mixed-precision FMA
+// per element, as in split_pair); e4m3 keeps 4 significant bits of it, so
+// hi + lo carries about 15 of x.  Values must stay below fp16's range.
+__device__ __forceinline__ void split_pair_e4m3(float a, float b, uint32_t& hi2, uint16_t& lo2) {
+  asm("{\n\t"
+      ".reg .b16 h0, h1, m1;\n\t.reg .f32 la, lb;\n\t"
+      "mov.b16 m1, 0xBC00;\n\t"
+      "cvt.rz.relu.f16x2.f32 %0, %3, %2;\n\t"
+      "mov.b32 {h0, h1}, %0;\n\t"
+      "fma.rn.f32.f16 la, h0, m1, %2;\n\t"
+      "fma.rn.f32.f16 lb, h1, m1, %3;\n\t"
+      "cvt.rn.satfinite.relu.e4m3x2.f32 %1, lb, la;\n\t}\n"
+      : "=r"(hi2), "=h"(lo2)
+      : "f"(a), "f"(b));
 }
 
 __device__ __forceinline__ void sts128(uint32_t saddr, uint32_t a, uint32_t b, uint32_t c,

@@ -29,11 +29,12 @@ PIC_ACT_RELU = 0
 PIC_ACT_GELU = 1
 PIC_PREC_FP32 = 0
 PIC_PREC_FP16_TC = 1
+PIC_PREC_FP16_TC_LO8 = 2
 PIC_LATENT_INT32 = 0
 PIC_LATENT_FP32 = 1
 
 ACTS = {"relu": PIC_ACT_RELU, "gelu": PIC_ACT_GELU}
-PRECS = {"fp32": PIC_PREC_FP32, "fp16_tc": PIC_PREC_FP16_TC}
+PRECS = {"fp32": PIC_PREC_FP32, "fp16_tc": PIC_PREC_FP16_TC, "fp16_tc_lo8": PIC_PREC_FP16_TC_LO8}
 LATENTS = {"int32": PIC_LATENT_INT32, "fp32": PIC_LATENT_FP32}
 PIC_OUT_F32_CHW = 0
 PIC_OUT_F32_HWC = 1
@@ -92,6 +93,8 @@ def load_library():
     lib.pic_decode_batch_noalloc.restype = i
     lib.pic_decode_noalloc_check.argtypes = [_P]
     lib.pic_decode_noalloc_check.restype = i
+    lib.pic_decode_test_wait_fault.argtypes = [i, ctypes.c_uint]
+    lib.pic_decode_test_wait_fault.restype = i
     lib.pic_decode_check.argtypes = [_P, _P]
     lib.pic_decode_check.restype = i
     lib.pic_decode_destroy.argtypes = [_P]
@@ -184,6 +187,10 @@ def pic_decode_batch_noalloc(arch: pic_arch, B, latents, steps, weights, H, W, o
 
 def pic_decode_noalloc_check(stream=None) -> int:
     return load_library().pic_decode_noalloc_check(stream)
+
+
+def pic_decode_test_wait_fault(withhold_arrival: int, spin_limit: int) -> int:
+    return load_library().pic_decode_test_wait_fault(withhold_arrival, spin_limit)
 
 
 def pic_decode_check(h, stream=None) -> int:
@@ -286,7 +293,7 @@ def fuse_modulation(arch: pic_arch, shared, mod, out=None, stream=None):
     import torch
     B = mod.shape[0]
     P = pic_param_count(arch)
-    dt = torch.float16 if arch.precision == PIC_PREC_FP16_TC else torch.float32
+    dt = torch.float32 if arch.precision == PIC_PREC_FP32 else torch.float16
     if out is None:
         out = torch.empty((B, P), dtype=dt, device=mod.device)
     rc = pic_fuse_modulation(arch, B, shared.data_ptr(), mod.data_ptr(), out.data_ptr(),
@@ -377,7 +384,7 @@ def decode_buffer_bytes(arch: pic_arch, B, H, W) -> dict:
     return {
         "latents": 4 * B_ * n_lat,
         "steps": 4 * B_ * arch.num_levels if arch.latent_format == PIC_LATENT_INT32 else 0,
-        "weights": (2 if arch.precision == PIC_PREC_FP16_TC else 4) * B_ * n_par,
+        "weights": (4 if arch.precision == PIC_PREC_FP32 else 2) * B_ * n_par,
         "out": (1 if arch.output_format == PIC_OUT_U8_HWC else 4) * 3 * B_ * H_ * W_,
     }
 

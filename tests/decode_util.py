@@ -9,7 +9,7 @@ import numpy as np
 from paper_2609_09020_gb300 import workloads as wk
 
 # Tolerances on [0, 1] RGB, max |GPU - oracle| (the decode's stated bars).
-TOL = {"fp32": 1e-4, "fp16_tc": 4e-3}
+TOL = {"fp32": 1e-4, "fp16_tc": 4e-3, "fp16_tc_lo8": 4e-3}
 # Oracle threads: the host cores of whatever machine runs the tests.
 ORACLE_THREADS = max(1, min(16, os.cpu_count() or 1))
 

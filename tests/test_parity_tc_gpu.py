@@ -149,3 +149,54 @@ def test_tma_and_copy_staging_agree(orc, wl):
         dec = Decoder.for_workload(wl, P, staging=staging)
         assert dec.kernel_name.endswith(suffix) and ("_tma" in dec.kernel_name) == (staging == "tma")
         dec.close()
+
+
+# The fp8 lo term (PIC_PREC_FP16_TC_LO8, the 7-64-64-3 architecture): the
+# hidden operands carry about 15 significant bits (fp16 hi + e4m3 lo, the
+# activations scaled by 2^6), so its own bound is wider than the split's.
+# A CPU emulation of exactly this arithmetic on 8 of the 64 c5 images
+# (tests/test_split_arithmetic.py) reaches 3.4e-4 against the oracle; the
+# kernel is held to LO8_BOUND = 1e-3, a quarter of the 4e-3 bar, on top of
+# the bar and the PSNR check.
+LO8 = "fp16_tc_lo8"
+LO8_BOUND = 1e-3
+
+
+def _check_lo8(orc, wl, clamp=True):
+    from paper_2609_09020_gb300.pic import Decoder
+    x = wk.make_inputs(wl)
+    got = gpu_decode(wl, x, LO8, clamp=clamp)
+    dec = Decoder.for_workload(wl, LO8)
+    assert dec.kernel_name.endswith("_lo8")
+    dec.close()
+    worst = 0.0
+    for b in range(x.latents.shape[0]):
+        want = oracle_full(orc, wl, x, b, P, clamp=clamp)  # fp16 weights: the definition
+        scale = 1.0 if clamp else max(1.0, float(np.abs(want).max()))
+        d, where = max_abs_diff(got[b], want)
+        assert d <= LO8_BOUND * scale, (wl.name, b, d, where)
+        if clamp:
+            t = _noisy_target(want, 1000 + b)
+            assert abs(psnr(got[b], t) - psnr(want, t)) <= 0.02, (wl.name, b)
+        worst = max(worst, d)
+    return worst
+
+
+def test_lo8_c5_all_64_images(orc):
+    _check_lo8(orc, wk.WORKLOADS["c5"])
+
+
+def test_lo8_c5_unclamped(orc):
+    _check_lo8(orc, wk.WORKLOADS["c5"].replace(seeds=(100, 101), name="c5x2"), clamp=False)
+
+
+@pytest.mark.parametrize("wl", EDGE[:3], ids=lambda w: w.name)
+def test_lo8_edge_shapes(orc, wl):
+    _check_lo8(orc, wl)
+
+
+def test_lo8_needs_its_architecture():
+    """Only the 7-64-64-3 ReLU architecture has an fp8-lo kernel."""
+    from paper_2609_09020_gb300 import pic
+    with pytest.raises(pic.PicError):
+        pic.Decoder.for_workload(wk.WORKLOADS["c4"], LO8)

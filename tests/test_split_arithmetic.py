@@ -190,12 +190,12 @@ def test_e4m3_grid():
     assert got.tolist() == [448.0, 448.0, 1.0, 1.25, 2.0 ** -9, 2.0 ** -9, 3.0 * 2.0 ** -9, -0.3125]
 
 
-def _fp8_lo_operand_layers(layers, S=2.0 ** 8):
+def _fp8_lo_operand_layers(layers, S=2.0 ** 6):
     """The MLP as a tensor path with the lo term in fp8 would compute it.
     Hidden activations stay scaled by S (ReLU commutes with a positive
     scale): the hidden operand is hi = RZ16(S h) in fp16 against the fp16
     weights W, plus lo = e4m3(S h - hi) against e4m3(W) (S h - hi is about
-    2^-11 S h, inside e4m3's normal range for S = 2^8, and exact in fp32);
+    2^-11 S h, inside e4m3's range for S = 2^6 (the kernel's), exact in fp32);
     the bias rows carry S b, the first layer's weights S W (exact: S is a
     power of two), and only the 3 outputs are divided by S.  No rescaling
     of the hidden values is needed, so the epilogue keeps its instruction
@@ -217,9 +217,9 @@ def _fp8_lo_operand_layers(layers, S=2.0 ** 8):
 
 
 def test_fp8_lo_term_stays_inside_the_bar(orc):
-    """The next step for the tensor path: the lo term in fp8 keeps the error
-    near 2e-4 on a full c5 image (2.2e-4), some 20x inside the 4e-3 bar and
-    12x below plain fp16."""
+    """The arithmetic of the tensor path's fp8 lo term (PIC_PREC_FP16_TC_LO8)
+    keeps the error near 2e-4 on a full c5 image (2.2e-4), some 20x inside
+    the 4e-3 bar and 12x below plain fp16 (over 8 of the 64 images: 3.4e-4)."""
     wl = wk.WORKLOADS["c5"]
     x = wk.make_inputs(wl, batch=1)
     ref = orc.decode(x.latents[0], x.steps[0], x.oracle_weights("fp16_tc")[0], wl.H, wl.W,
