@@ -109,15 +109,20 @@ __host__ __device__ constexpr uint32_t kmaj8(int row, int k, int K) {
   return static_cast<uint32_t>((row >> 3) * (K * 8) + (k >> 4) * 128 + (row & 7) * 16 + (k & 15));
 }
 
-// Cooperative feature staging.  For level l >= 1 a 128-pixel row segment
-// needs at most NCOL(l) = 128/2^l + 4 source columns.  The warpgroup first
-// interpolates those columns vertically (rows v0, v1 of the level, weight
-// beta) into a small shared buffer -- one item per (level, channel, column),
-// spread over the 128 threads -- and every pixel then interpolates
-// horizontally between two buffer entries.  Column indices are clamped into
-// [0, W_l - 1] when the buffer is filled, which reproduces the edge clamp of
-// the bilinear definition.
-__host__ __device__ constexpr int ncol(int l) { return (kTile >> l) + 4; }
+// Feature staging per segment of the tile row: a warp's 32 pixels (offset
+// 32 (warp & 3) within the tile; single-channel nets) or the group's whole
+// 128 (nets with more channels, whose per-warp buffers would take more
+// staging registers).  A segment of SEG pixels needs at most NCOL(l) =
+// SEG/2^l + 4 source columns of level l >= 1.  Its threads first
+// interpolate those columns vertically (rows v0, v1 of the level, weight
+// beta) into the segment's small shared buffer -- one item per (level,
+// channel, column), spread over them -- and every pixel then interpolates
+// horizontally between two buffer entries.  A warp segment needs only a
+// __syncwarp between the two passes (the group barrier it replaces measured
+// 4-5 % of the c5 time); a group segment waits on the group's col_ready
+// mbarrier.  Column indices are clamped into [0, W_l - 1] when the buffer is
+// filled, which reproduces the edge clamp of the bilinear definition.
+__host__ __device__ constexpr int ncol(int l, int seg) { return (seg >> l) + 4; }
 static_assert(kTile == kTcTile, "one tile size for the kernels and the host's TMA boxes");
 
 // One TMA buffer (TMA kernels): a slot per channel for the tile's level-0
@@ -133,13 +138,13 @@ struct TmaSlots {
   static constexpr int tx_bytes() { return C * kTmaRowBox * 4; }  // the stage mbarrier's count
 };
 
-template <int L, int C>
+template <int L, int C, int SEG>
 struct ColLayout {
-  // float offset of (level l, channel c) inside the column buffer
+  // float offset of (level l, channel c) inside a segment's column buffer
   static constexpr int off(int l, int c) {
     int o = 0;
-    for (int k = 1; k < l; ++k) o += C * ncol(k);
-    return o + c * ncol(l);
+    for (int k = 1; k < l; ++k) o += C * ncol(k, SEG);
+    return o + c * ncol(l, SEG);
   }
   static constexpr int total() { return off(L, 0); }
 };
@@ -148,6 +153,8 @@ template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_, bool LO8_ = fals
 struct TcNet {
   static constexpr int C = C_, NL = NL_, D0 = D0_, N = N_, ACT = ACT_, NWG = NWG_;
   static constexpr bool LO8 = LO8_;
+  static constexpr int SEG = C == 1 ? 32 : kTile;  // staging segment: a warp's pixels or the group's
+  static constexpr int NSEG = kTile / SEG;         // segments (column buffers) per group
   static constexpr float kS = LO8 ? 64.0f : 1.0f;  // scale of the hidden activations (LO8)
   static constexpr int L = D0 / C;
   static constexpr int K1 = round_up(2 * D0 + 1, 16);
@@ -195,8 +202,8 @@ struct TcNet {
   static constexpr int OFF_ONES = round_up(OFF_BLO + BLO_BYTES, 128);
   static constexpr int OFF_WG = round_up(OFF_ONES + ONES_BYTES, 128);
   static constexpr int A1_BYTES = kTile * K1 * 2;
-  static constexpr int COL_BYTES = round_up(ColLayout<L, C>::total() * 4, 128);
-  static constexpr int NITEM_PER_THREAD = (ColLayout<L, C>::total() + kTile - 1) / kTile;
+  static constexpr int COL_BYTES = round_up(NSEG * ColLayout<L, C, SEG>::total() * 4, 128);
+  static constexpr int NITEM_PER_THREAD = (ColLayout<L, C, SEG>::total() + SEG - 1) / SEG;
   static constexpr int STAGE_SLOTS = C + 2 * NITEM_PER_THREAD;  // raw int32 loads per thread
   static constexpr int STAGE_BYTES = STAGE_SLOTS * kTile * 4;
   static constexpr int WG_BYTES = A1_BYTES + COL_BYTES + STAGE_BYTES;
@@ -430,9 +437,10 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
   constexpr int K1 = Net::K1;
   constexpr int WGB = TMA ? Net::WG_BYTES_TMA : Net::WG_BYTES;
   using TS = TmaSlots<C>;
-  using CL = ColLayout<L, C>;
-  constexpr int NITEM = CL::total();
-  constexpr int J = (NITEM + kTile - 1) / kTile;  // column items per thread (0 if L == 1)
+  constexpr int SEG = Net::SEG;
+  using CL = ColLayout<L, C, SEG>;
+  constexpr int NITEM = CL::total();  // column items of one segment
+  constexpr int J = (NITEM + SEG - 1) / SEG;  // column items per thread (0 if L == 1)
   constexpr int JJ = J > 0 ? J : 1;
   extern __shared__ __align__(1024) uint8_t smem[];
 
@@ -520,7 +528,12 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         const int r = ((warp & 3) << 5) | lane;  // tile row = TMEM lane = pixel
         uint8_t* a1 = smem + Net::OFF_WG + w * WGB;
         const uint32_t a1_s = smem_addr(a1);
-        float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES);
+        // this thread's segment: its column buffer, its offset xo in the tile
+        // row, and the thread's place sr in it
+        const int sid = SEG == kTile ? 0 : (warp & 3);
+        float* colbuf = reinterpret_cast<float*>(a1 + Net::A1_BYTES) + sid * NITEM;
+        const int xo = sid * SEG;
+        const int sr = r - xo;
         const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
         const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(w * 2 * N);
         const uint32_t t_a = t_acc + N;  // hi in [0, N/2), lo in [N/2, N)
@@ -538,13 +551,13 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
         float it_beta[JJ];  // vertical weight of each item for the tile last prefetched
 #pragma unroll
         for (int j = 0; j < J; ++j) {
-          int e = r + kTile * j, l = 0, c = 0, i = 0;
+          int e = sr + SEG * j, l = 0, c = 0, i = 0;
           if (e < NITEM) {
 #pragma unroll
             for (int lv = 1; lv < L; ++lv)
 #pragma unroll
               for (int cc = 0; cc < C; ++cc)
-                if (e >= CL::off(lv, cc) && e < CL::off(lv, cc) + ncol(lv)) {
+                if (e >= CL::off(lv, cc) && e < CL::off(lv, cc) + ncol(lv, SEG)) {
                   l = lv;
                   c = cc;
                   i = e - CL::off(lv, cc);
@@ -560,12 +573,15 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
           it_sx[j] = lg.sx;
         }
         // Relative x-taps of pixel r for each level (used when fast_x): the
-        // source coordinate (r + 1/2) / 2^l - 1/2 relative to column x0/2^l - 1.
+        // source coordinate of pixel x0 + r, relative to column (x0 + xo)/2^l
+        // - 1, is ((xo mod 2^l) + lane + 1/2) / 2^l - 1/2 + 1 (x0 is a
+        // multiple of 128 >= 2^l, so this does not depend on the tile).
         int rel[L];
         float fx[L];
 #pragma unroll
         for (int l = 1; l < L; ++l) {
-          const float sx = (static_cast<float>(r) + 0.5f) * (1.0f / static_cast<float>(1 << l)) - 0.5f;
+          const int off = (xo & ((1 << l) - 1)) + sr;
+          const float sx = (static_cast<float>(off) + 0.5f) * (1.0f / static_cast<float>(1 << l)) - 0.5f;
           const float fl = floorf(sx);
           rel[l] = static_cast<int>(fl) + 1;
           fx[l] = sx - fl;
@@ -591,7 +607,8 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             if (l > 0) {
               const Tap ty = bilinear_tap(y, it_sy[j], it_H[j]);
               it_beta[j] = ty.frac;
-              const int u_start = fast_x ? (x0 >> l) - 1 : bilinear_tap(x0, it_sx[j], it_W[j]).i0;
+              const int u_start =
+                  fast_x ? ((x0 + xo) >> l) - 1 : bilinear_tap(x0 + xo, it_sx[j], it_W[j]).i0;
               const int u = min(max(u_start + it_i[j], 0), it_W[j] - 1);
               const int32_t* pl = lat + it_off[j] + u;
               cp_async4(stage_s + ((C + 2 * j) * kTile + r) * 4, pl + ty.i0 * it_W[j]);
@@ -623,13 +640,20 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
             if (l > 0) {
               const float beta = it_beta[j];  // set by the prefetch of this tile
               const int t0 = stage[(C + 2 * j) * kTile + r], t1 = stage[(C + 2 * j + 1) * kTile + r];
-              colbuf[r + kTile * j] = step[l] * lat_lerp<FL>(t0, t1, beta);
+              colbuf[sr + SEG * j] = step[l] * lat_lerp<FL>(t0, t1, beta);
             }
           }
-          mbar_arrive(my_col);  // the group's column buffer is complete once all 128 arrived
-          if (!__all_sync(0xffffffffu, wait_bounded(my_col, col_phase, abort_flag, p.status, p.spin_limit)))
-            return false;
-          col_phase ^= 1u;
+          if constexpr (TMA || SEG == kTile) {
+            // the group's barrier: the group's column buffer is complete, and
+            // (TMA) the issuing warp hands over the tile's level-0 boxes there
+            // (its 129th arrival)
+            mbar_arrive(my_col);
+            if (!__all_sync(0xffffffffu, wait_bounded(my_col, col_phase, abort_flag, p.status, p.spin_limit)))
+              return false;
+            col_phase ^= 1u;
+          } else {
+            __syncwarp();  // this warp's column buffer is complete
+          }
           // horizontal pass + level 0
           const int xc = min(x0 + r, p.W - 1);
           float f[D0];
@@ -653,10 +677,10 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
               a = fx[l];
             } else {
               const LevelGeom lg = p.lv[l];
-              const int u_start = bilinear_tap(x0, lg.sx, lg.W).i0;
+              const int u_start = bilinear_tap(x0 + xo, lg.sx, lg.W).i0;
               const Tap tx = bilinear_tap(xc, lg.sx, lg.W);
-              i0 = min(max(tx.i0 - u_start, 0), ncol(l) - 1);
-              i1 = min(max(tx.i1 - u_start, 0), ncol(l) - 1);
+              i0 = min(max(tx.i0 - u_start, 0), ncol(l, SEG) - 1);
+              i1 = min(max(tx.i1 - u_start, 0), ncol(l, SEG) - 1);
               a = tx.frac;
             }
 #pragma unroll

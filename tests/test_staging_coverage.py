@@ -205,3 +205,70 @@ def test_tma_boxes_and_slots(L, C):
     assert all(a % 128 == 0 and box <= e - a for a, e, box in spans)
     assert all(spans[k][1] == spans[k + 1][0] for k in range(n - 1))
     assert spans[0][0] == 0 and spans[-1][1] == off(L, 0, 0)
+
+
+# ---- Per-warp column buffers.  Each warp of a group (its 32 consecutive
+# pixels, offset xo = 32 w within the 128-pixel tile) fills its own column
+# buffer of NCOLW(l) = 32/2^l + 4 entries from its own left tap, so no
+# barrier across the group's warps is needed: the fast scheme's relative taps
+# use the pixel's offset within a 2^l-aligned span, (xo mod 2^l) + lane,
+# which is tile-invariant because the tile origin is a multiple of 128.
+SEG = 32
+
+
+def ncolw(l):
+    return (SEG >> l) + 4
+
+
+def warp_row(row, W, l, fast, ratio32):
+    """The horizontal pass of every pixel of a W-wide row at level l, warp by
+    warp, as the kernel indexes each warp's column buffer; returns the values
+    and whether any buffer index had to be clamped."""
+    Wl = row.size
+    out = np.empty(W)
+    clamped = False
+    for x0 in range(0, W, TILE):
+        for xo in range(0, TILE, SEG):
+            X = x0 + xo
+            lane = np.arange(SEG)
+            if fast:
+                u_start = (X >> l) - 1
+                sx = (((xo % (1 << l)) + lane) + 0.5) / (1 << l) - 0.5  # exact (dyadic)
+                fl = np.floor(sx)
+                i0 = fl.astype(np.int64) + 1
+                i1 = i0 + 1
+                a = sx - fl
+            else:
+                u_start = int(tap32(X, ratio32, Wl)[0])
+                xc = np.minimum(X + lane, W - 1)
+                t0, t1, a = tap32(xc, ratio32, Wl)
+                i0, i1 = t0 - u_start, t1 - u_start
+            lim = ncolw(l) - 1
+            valid = X + lane < W  # pixels past the row's end are never stored
+            bad = (i0 < 0) | (i0 > lim) | (i1 < 0) | (i1 > lim)
+            clamped |= bool(np.any(bad & valid))
+            i0, i1 = np.clip(i0, 0, lim), np.clip(i1, 0, lim)
+            buf = row[np.clip(u_start + np.arange(ncolw(l)), 0, Wl - 1)]
+            vals = buf[i0] + a * (buf[i1] - buf[i0])
+            n = max(0, min(SEG, W - X))
+            out[X:X + n] = vals[:n]
+    return out, clamped
+
+
+@pytest.mark.parametrize("L", [2, 4, 7, 8, 12])
+def test_warp_buffers_cover_every_tap(L):
+    rng = np.random.default_rng(100 + L)
+    for W in WIDTHS:
+        fast = (L - 1 <= 7) and W % (1 << (L - 1)) == 0
+        for l in range(1, L):
+            Wl = level_size(W, l)
+            ratio32 = np.float32(Wl / W)
+            row = rng.standard_normal(Wl)
+            got, clamped = warp_row(row, W, l, fast, ratio32)
+            assert not clamped, (W, L, l, fast)
+            x = np.arange(W)
+            e0, e1, ea = exact_taps(x, W, Wl)
+            want = row[e0] + ea * (row[e1] - row[e0])
+            slope = np.max(np.abs(np.diff(row))) if Wl > 1 else 0.0
+            tol = 2.0 ** -22 * (Wl + 2) * slope + 1e-12
+            assert np.max(np.abs(got - want)) <= tol, (W, L, l, fast)
