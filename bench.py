@@ -895,7 +895,7 @@ def fp32_peak(pic, dev):
 PER_CONFIG = ["c1", "c2", "c3", "c4", "c5"]
 # extra tensor-path rows with the latent staging the library's default does
 # not pick for that architecture (TMA boxes vs per-thread copies)
-PER_CONFIG_STAGING = {"c5": "tma", "c3": "tma", "c4": "copies"}
+PER_CONFIG_STAGING = {"c5": "tma", "c3": "tma", "c4": "tma"}
 
 
 def per_config_rows(pic, dev, stream, peaks, fp32_tf, fp32_src, reps=None):
