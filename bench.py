@@ -949,9 +949,31 @@ def per_config_rows(pic, dev, stream, peaks, fp32_tf, fp32_src, reps=None):
             dec.close()
             del w
         del lat, st, out
+    # The floor of this timing method: a near-empty launch of the library's
+    # FMA microbenchmark kernel (152 CTAs x 256 threads, 128 FMAs a thread)
+    # timed the same way (L2 flushed, events around the launch alone).
+    out = torch.empty(152, dtype=torch.float32, device=dev)
+    lib = pic.load_library()
+    sp = stream.cuda_stream
+    for _ in range(3):
+        lib.pic_fma_peak_launch(out.data_ptr(), 152, 1, sp)
+    torch.cuda.synchronize(dev)
+    floor = []
+    for _ in range(60):
+        flush.fill_(1.0)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        lib.pic_fma_peak_launch(out.data_ptr(), 152, 1, sp)
+        e1.record(stream)
+        e1.synchronize()
+        floor.append(e0.elapsed_time(e1))
     del flush
     return {"rows": rows, "timing": "median of per-call CUDA events, L2 flushed (256 MB write) "
-                                    "before every call, 3 warm-up calls per row"}
+                                    "before every call, 3 warm-up calls per row",
+            "launch_floor": {"ms": float(np.median(floor)),
+                             "kernel": "FMA microbenchmark, 152 CTAs x 256 threads, 128 FMAs a "
+                                       "thread, timed the same way"}}
 
 
 def main():
