@@ -155,6 +155,10 @@ struct TcNet {
   static constexpr bool LO8 = LO8_;
   static constexpr int SEG = C == 1 ? 32 : kTile;  // staging segment: a warp's pixels or the group's
   static constexpr int NSEG = kTile / SEG;         // segments (column buffers) per group
+  // Hidden operand layout in tensor memory: per 16-value chunk the hi and the
+  // lo columns adjacent (one 16-column store; single-channel nets, measured
+  // 1 % faster on c5), else all hi columns, then all lo columns.
+  static constexpr bool ADJ = C == 1 && !LO8;
   static constexpr float kS = LO8 ? 64.0f : 1.0f;  // scale of the hidden activations (LO8)
   static constexpr int L = D0 / C;
   static constexpr int K1 = round_up(2 * D0 + 1, 16);
@@ -367,8 +371,9 @@ __device__ __forceinline__ void output_layer_cc(const uint8_t* smem, uint32_t t_
 }
 
 // Hidden epilogue of one pixel (TMEM lane): accumulator -> activation ->
-// hi/lo split -> the next layer's A operand in TMEM (hi pairs at t_a, lo
-// pairs at t_a + N/2), 16 columns at a time (fewer live registers).
+// hi/lo split -> the next layer's A operand in TMEM, 16 values at a time
+// (fewer live registers): chunk c's hi pairs at t_a + 16c and lo pairs at
+// t_a + 16c + 8 (Net::ADJ), else hi pairs at t_a + 8c, lo at t_a + N/2 + 8c.
 template <class Net>
 __device__ __forceinline__ void hidden_epilogue(uint32_t t_acc, uint32_t t_a) {
   constexpr int N = Net::N;
@@ -390,8 +395,12 @@ __device__ __forceinline__ void hidden_epilogue(uint32_t t_acc, uint32_t t_a) {
       // hi = fp16 truncation (ReLU folded in), lo = fp16 of v - hi (one mixed FMA)
       split_pair<Net::ACT != ACT_GELU>(a, bb, hl[q], hl[8 + q]);
     }
-    tmem_st8(t_a + h0 / 2, hl);
-    tmem_st8(t_a + N / 2 + h0 / 2, hl + 8);
+    if constexpr (Net::ADJ) {
+      tmem_st16(t_a + h0, hl);
+    } else {
+      tmem_st8(t_a + h0 / 2, hl);
+      tmem_st8(t_a + N / 2 + h0 / 2, hl + 8);
+    }
   }
   tmem_st_wait();
 }
@@ -904,14 +913,16 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
                 const uint64_t db = out_layer ? dBO : dBH + (k - 1) * kLayer;
                 const uint32_t id = out_layer ? id_out : id_hidden;
 #pragma unroll
-                for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + 8 * s, db + s * kStep, id, s > 0);  // hi
+                for (int s = 0; s < N / 16; ++s)  // hi
+                  mma_f16_ta(d, ta + (Net::ADJ ? 16 * s : 8 * s), db + s * kStep, id, s > 0);
                 if constexpr (Net::LO8) {  // lo in e4m3: K = 32 per MMA, 8 columns of A each
                   const uint64_t dl = out_layer ? dBLO : dBL + (k - 1) * kLayerL;
 #pragma unroll
                   for (int s = 0; s < N / 32; ++s) mma_e4m3_ta(d, ta + N / 2 + 8 * s, dl + s * kStep, id, 1);
                 } else {
 #pragma unroll
-                  for (int s = 0; s < N / 16; ++s) mma_f16_ta(d, ta + N / 2 + 8 * s, db + s * kStep, id, 1);  // lo
+                  for (int s = 0; s < N / 16; ++s)  // lo
+                    mma_f16_ta(d, ta + (Net::ADJ ? 16 * s + 8 : N / 2 + 8 * s), db + s * kStep, id, 1);
                 }
                 mma_f16(d, dONES, db + (N / 16) * kStep, id, 1);  // bias: [1 0..0] x [b 0..0]
               }
