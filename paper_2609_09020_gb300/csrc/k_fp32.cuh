@@ -142,7 +142,7 @@ __device__ __forceinline__ void dense_acc(const float* __restrict__ X, const flo
       }
     }
   }
-#pragma unroll 1
+#pragma unroll 2
   for (int kb = 0; kb < Ly::K / BLK; ++kb) {
     const int sw = SWZ ? (kb & 7) : 0;
     const float* xb = X + kb * BLK * kThreads;
