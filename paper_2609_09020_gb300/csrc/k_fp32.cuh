@@ -11,21 +11,23 @@
 //      shared-memory activation buffer X (one row of 128 floats per
 //      feature), so features never reach HBM;
 //   2. each hidden layer of g_s (Sec. 4.1) is a 128-pixel x N contraction
-//      on the CUDA cores, register-tiled: thread (pg, ng) accumulates TP
-//      pixels x TN neurons (TP = NG, NG x TN = N; 8 x 8 for N = 64) over the
-//      K inputs, reading TP activations and TN weights from shared memory
-//      per input, so one load feeds TN (resp. TP) FMAs instead of one;
-//      packed f32x2 FMAs do two neurons of one pixel per instruction.  The
-//      bias seeds the accumulators; the activation is applied in registers
-//      and the layer's output rows are written back over X;
+//      on the CUDA cores, register-tiled: warp ng owns the neurons
+//      ng*TN .. ng*TN + TN - 1 (TN = N / 4) and its lane pg the 4 pixels
+//      4pg .. 4pg + 3, and accumulates those 4 x TN outputs over the K
+//      inputs.  Per input a lane loads its 4 activations (one 16-byte load;
+//      a quarter-warp reads 128 consecutive bytes) and the warp's TN weights
+//      (16-byte loads at one address for the whole warp, a broadcast), so
+//      each load feeds TN (resp. 4) FMAs; packed f32x2 FMAs do two neurons of
+//      one pixel per instruction.  The bias seeds the accumulators; the
+//      activation is applied in registers and the layer's output rows are
+//      written back over X (again 128 consecutive bytes per quarter-warp);
 //   3. the output layer (3 neurons) is folded into the last hidden layer's
-//      epilogue: each thread forms the 3 partial sums over its TN neurons for
-//      its TP pixels, and thread p adds the NG partials of pixel p, the bias,
-//      clamps and stores the planar RGB row (coalesced).
+//      epilogue: each lane forms the 3 partial sums over its warp's TN
+//      neurons for its 4 pixels, and thread p adds the 4 warps' partials of
+//      pixel p and the bias, clamps and stores the planar RGB row
+//      (coalesced).
 // Weights live in shared memory for the whole tile range (reloaded when the
-// image changes).  Activation rows are 16-byte chunks XOR-swizzled by the
-// writing thread's neuron group, so the epilogue stores and the K-loop loads
-// both run without bank conflicts.
+// image changes).
 //
 // Work split: the tiles of all images are numbered image-major and each CTA
 // takes one contiguous range of them (a CTA sees at most a couple of images
@@ -40,23 +42,24 @@ namespace pic {
 namespace {
 
 constexpr int kThreads = 128;  // threads per CTA = pixels per tile = floats per activation row
+constexpr int kWarps = kThreads / 32;  // neuron groups of a layer
+constexpr int kTP = 4;                 // pixels per lane
 
-// Neuron groups of a hidden layer of width n: thread (pg, ng) owns TP = NG
-// pixels and TN = n / NG neurons (NG x TN = n, 128 / NG pixel groups).
-__host__ __device__ constexpr int ng_for(int n) { return n >= 64 ? 8 : (n >= 16 ? 4 : 2); }
-
-// One hidden layer: K inputs, N outputs.  Shared-memory image: K weight rows
-// then the bias row, each row holding, per 4-float chunk c and neuron group
-// ng, neurons ng*TN + 4c .. 4c+3 (zero past TN): [row][c][ng][4].  A warp's
-// load of chunk c is 32 (or fewer) consecutive words.
+// One hidden layer: K inputs, N outputs, warp ng computing neurons
+// ng*TN .. ng*TN + TN - 1.  Shared-memory image: K weight rows then the bias
+// row, each row holding per warp a segment of SEGF floats (its TN neurons,
+// zero padded to whole 16-byte chunks): [row][ng][SEGF].
 template <int K_, int N_>
 struct Dense {
   static constexpr int K = K_, N = N_;
-  static constexpr int NG = ng_for(N_), TN = N_ / NG, TP = NG, TN2 = TN / 2;
+  static constexpr int TN = N_ / kWarps, TN2 = TN / 2;
   static constexpr int NCH = (TN + 3) / 4;
-  static constexpr int ROWF = NCH * NG * 4;
+  static constexpr int SEGF = 4 * NCH;
+  static constexpr int ROWF = kWarps * SEGF;
   static constexpr int FLOATS = (K + 1) * ROWF;
-  static_assert(N_ % NG == 0 && TN % 2 == 0, "hidden width must split into even neuron groups");
+  // inputs per iteration of the K loop
+  static constexpr int UNR = K <= 16 ? K : (K % 16 == 0 ? 16 : (K % 8 == 0 ? 8 : 1));
+  static_assert(N_ % (2 * kWarps) == 0, "hidden width must be a multiple of 8");
 };
 
 // Copies one hidden layer from the nn.Linear layout (W [N][K] row-major,
@@ -65,8 +68,7 @@ template <class Ly>
 __device__ __forceinline__ void load_dense(float* __restrict__ sm, const float* __restrict__ w) {
   for (int e = threadIdx.x; e < Ly::FLOATS; e += kThreads) {
     const int k = e / Ly::ROWF, r = e - k * Ly::ROWF;
-    const int c = r / (4 * Ly::NG), r2 = r - c * 4 * Ly::NG;
-    const int ng = r2 >> 2, j = 4 * c + (r2 & 3);
+    const int ng = r / Ly::SEGF, j = r - ng * Ly::SEGF;
     const int n = ng * Ly::TN + j;
     float v = 0.0f;
     if (j < Ly::TN) v = k < Ly::K ? w[n * Ly::K + k] : w[Ly::N * Ly::K + n];
@@ -86,93 +88,54 @@ __device__ __forceinline__ void load_out(float* __restrict__ sm, const float* __
   }
 }
 
-// The TP activations of pixel group pg in a 128-float row whose 16-byte
-// chunks are XOR-swizzled by sw: TP = 8 -> chunks 2pg, 2pg+1; TP = 4 ->
-// chunk pg; TP = 2 -> half of chunk pg / 2.
-template <int TP>
-__device__ __forceinline__ void load_px(const float* __restrict__ row, int pg, int sw, float (&a)[TP]) {
-  if constexpr (TP == 8) {
-    const float4 u = *reinterpret_cast<const float4*>(row + (((2 * pg) ^ sw) << 2));
-    const float4 v = *reinterpret_cast<const float4*>(row + (((2 * pg + 1) ^ sw) << 2));
-    a[0] = u.x; a[1] = u.y; a[2] = u.z; a[3] = u.w;
-    a[4] = v.x; a[5] = v.y; a[6] = v.z; a[7] = v.w;
-  } else if constexpr (TP == 4) {
-    const float4 u = *reinterpret_cast<const float4*>(row + ((pg ^ sw) << 2));
-    a[0] = u.x; a[1] = u.y; a[2] = u.z; a[3] = u.w;
-  } else {
-    static_assert(TP == 2, "pixels per thread: 2, 4 or 8");
-    const float2 u = *reinterpret_cast<const float2*>(row + (((pg >> 1) ^ sw) << 2) + ((pg & 1) << 1));
-    a[0] = u.x; a[1] = u.y;
-  }
-}
-
-template <int TP>
-__device__ __forceinline__ void store_px(float* __restrict__ row, int pg, int sw, const float (&a)[TP]) {
-  if constexpr (TP == 8) {
-    *reinterpret_cast<float4*>(row + (((2 * pg) ^ sw) << 2)) = make_float4(a[0], a[1], a[2], a[3]);
-    *reinterpret_cast<float4*>(row + (((2 * pg + 1) ^ sw) << 2)) = make_float4(a[4], a[5], a[6], a[7]);
-  } else if constexpr (TP == 4) {
-    *reinterpret_cast<float4*>(row + ((pg ^ sw) << 2)) = make_float4(a[0], a[1], a[2], a[3]);
-  } else {
-    *reinterpret_cast<float2*>(row + (((pg >> 1) ^ sw) << 2) + ((pg & 1) << 1)) = make_float2(a[0], a[1]);
-  }
-}
-
-// Float offset of pixel p in a row swizzled by sw.
-__device__ __forceinline__ int px_off(int p, int sw) { return (((p >> 2) ^ sw) << 2) | (p & 3); }
-
-// acc = b + X^T W over the layer's K input rows X[0 .. K) (row k swizzled by
-// (k / BLK) & 7, or not at all when SWZ is false), for the thread's TP pixels
-// and TN neurons; acc[p][j] packs neurons 2j, 2j+1 of pixel p.
-template <class Ly, int BLK, bool SWZ>
+// acc = b + X^T W over the layer's K input rows X[0 .. K), for lane pg's 4
+// pixels and warp ng's TN neurons; acc[p][j] packs neurons 2j, 2j+1 of
+// pixel 4pg + p.
+template <class Ly>
 __device__ __forceinline__ void dense_acc(const float* __restrict__ X, const float* __restrict__ Wl,
-                                          int pg, int ng,
-                                          unsigned long long (&acc)[Ly::TP][Ly::TN2]) {
-  constexpr int TP = Ly::TP, TN2 = Ly::TN2, NCH = Ly::NCH, NG = Ly::NG, ROWF = Ly::ROWF;
-  static_assert(Ly::K % BLK == 0, "input blocks must tile K");
+                                          int pg, int ng, unsigned long long (&acc)[kTP][Ly::TN2]) {
+  constexpr int TN2 = Ly::TN2, NCH = Ly::NCH, ROWF = Ly::ROWF;
+  const float* wseg = Wl + ng * Ly::SEGF;  // warp-uniform
   {
-    const float* bias = Wl + Ly::K * ROWF + 4 * ng;
+    const float* bias = wseg + Ly::K * ROWF;
 #pragma unroll
     for (int c = 0; c < NCH; ++c) {
-      const ulonglong2 b = *reinterpret_cast<const ulonglong2*>(bias + c * 4 * NG);
+      const ulonglong2 b = *reinterpret_cast<const ulonglong2*>(bias + 4 * c);
 #pragma unroll
-      for (int p = 0; p < TP; ++p) {
+      for (int p = 0; p < kTP; ++p) {
         if (2 * c < TN2) acc[p][2 * c] = b.x;
         if (2 * c + 1 < TN2) acc[p][2 * c + 1] = b.y;
       }
     }
   }
-#pragma unroll 2
-  for (int kb = 0; kb < Ly::K / BLK; ++kb) {
-    const int sw = SWZ ? (kb & 7) : 0;
-    const float* xb = X + kb * BLK * kThreads;
-    const float* wb = Wl + kb * BLK * ROWF + 4 * ng;
+  const float* xa = X + 4 * pg;
+#pragma unroll 1
+  for (int k0 = 0; k0 < Ly::K; k0 += Ly::UNR) {
 #pragma unroll
-    for (int kk = 0; kk < BLK; ++kk) {
-      float a[TP];
-      load_px<TP>(xb + kk * kThreads, pg, sw, a);
+    for (int kk = 0; kk < Ly::UNR; ++kk) {
+      const float4 a = *reinterpret_cast<const float4*>(xa + (k0 + kk) * kThreads);
       unsigned long long w[2 * NCH];
 #pragma unroll
       for (int c = 0; c < NCH; ++c) {
-        const ulonglong2 v = *reinterpret_cast<const ulonglong2*>(wb + kk * ROWF + c * 4 * NG);
+        const ulonglong2 v = *reinterpret_cast<const ulonglong2*>(wseg + (k0 + kk) * ROWF + 4 * c);
         w[2 * c] = v.x;
         w[2 * c + 1] = v.y;
       }
+      const unsigned long long ad[kTP] = {pack2(a.x, a.x), pack2(a.y, a.y), pack2(a.z, a.z),
+                                          pack2(a.w, a.w)};
 #pragma unroll
-      for (int p = 0; p < TP; ++p) {
-        const unsigned long long ad = pack2(a[p], a[p]);
+      for (int p = 0; p < kTP; ++p)
 #pragma unroll
-        for (int j = 0; j < TN2; ++j) acc[p][j] = fma2(ad, w[j], acc[p][j]);
-      }
+        for (int j = 0; j < TN2; ++j) acc[p][j] = fma2(ad[p], w[j], acc[p][j]);
     }
   }
 }
 
 // The activation on every accumulator pair.
 template <class Ly, int ACT>
-__device__ __forceinline__ void activate_acc(unsigned long long (&acc)[Ly::TP][Ly::TN2]) {
+__device__ __forceinline__ void activate_acc(unsigned long long (&acc)[kTP][Ly::TN2]) {
 #pragma unroll
-  for (int p = 0; p < Ly::TP; ++p)
+  for (int p = 0; p < kTP; ++p)
 #pragma unroll
     for (int j = 0; j < Ly::TN2; ++j) {
       if constexpr (ACT == ACT_GELU) {
@@ -189,47 +152,46 @@ __device__ __forceinline__ float half_of(unsigned long long v, int hi) {
   return hi ? f.y : f.x;
 }
 
-// Hidden-layer output: neuron ng*TN + j of the thread's pixels goes to row
-// ng*TN + j of X, swizzled by ng & 7 (= (row / TN) & 7).
+// Hidden-layer output: neuron ng*TN + j of lane pg's pixels goes to row
+// ng*TN + j of X.
 template <class Ly>
 __device__ __forceinline__ void store_hidden(float* __restrict__ X, int pg, int ng,
-                                             const unsigned long long (&acc)[Ly::TP][Ly::TN2]) {
-  const int sw = ng & 7;
+                                             const unsigned long long (&acc)[kTP][Ly::TN2]) {
 #pragma unroll
   for (int j = 0; j < Ly::TN; ++j) {
-    float v[Ly::TP];
+    float v[kTP];
 #pragma unroll
-    for (int p = 0; p < Ly::TP; ++p) v[p] = half_of(acc[p][j >> 1], j & 1);
-    store_px<Ly::TP>(X + (ng * Ly::TN + j) * kThreads, pg, sw, v);
+    for (int p = 0; p < kTP; ++p) v[p] = half_of(acc[p][j >> 1], j & 1);
+    *reinterpret_cast<float4*>(X + (ng * Ly::TN + j) * kThreads + 4 * pg) = make_float4(v[0], v[1], v[2], v[3]);
   }
 }
 
-// Output-layer partial sums of the thread's TN neurons for its TP pixels:
-// row 3 ng + c of X holds output c's partial from group ng, swizzled by
-// ng & 7 (= (row / 3) & 7).
+// Output-layer partial sums of warp ng's TN neurons for lane pg's pixels:
+// row 3 ng + c of X holds output c's partial from warp ng.
 template <class Ly>
 __device__ __forceinline__ void store_out_partials(float* __restrict__ X, const float* __restrict__ Wout,
                                                    int pg, int ng,
-                                                   const unsigned long long (&acc)[Ly::TP][Ly::TN2]) {
-  float part[3][Ly::TP];
+                                                   const unsigned long long (&acc)[kTP][Ly::TN2]) {
+  float part[3][kTP];
 #pragma unroll
   for (int c = 0; c < 3; ++c)
 #pragma unroll
-    for (int p = 0; p < Ly::TP; ++p) part[c][p] = 0.0f;
+    for (int p = 0; p < kTP; ++p) part[c][p] = 0.0f;
 #pragma unroll
   for (int j = 0; j < Ly::TN; ++j) {
     const float4 w = *reinterpret_cast<const float4*>(Wout + 4 * (ng * Ly::TN + j));
 #pragma unroll
-    for (int p = 0; p < Ly::TP; ++p) {
+    for (int p = 0; p < kTP; ++p) {
       const float h = half_of(acc[p][j >> 1], j & 1);
       part[0][p] = fmaf(h, w.x, part[0][p]);
       part[1][p] = fmaf(h, w.y, part[1][p]);
       part[2][p] = fmaf(h, w.z, part[2][p]);
     }
   }
-  const int sw = ng & 7;
 #pragma unroll
-  for (int c = 0; c < 3; ++c) store_px<Ly::TP>(X + (3 * ng + c) * kThreads, pg, sw, part[c]);
+  for (int c = 0; c < 3; ++c)
+    *reinterpret_cast<float4*>(X + (3 * ng + c) * kThreads + 4 * pg) =
+        make_float4(part[c][0], part[c][1], part[c][2], part[c][3]);
 }
 
 template <int C, int NL, int D0, int D1, int D2, int D3, int D4, int ACT>
@@ -237,15 +199,14 @@ struct Fp32Net {
   static_assert(NL >= 2 && NL <= 4, "1 to 3 hidden layers");
   static constexpr int L = D0 / C;
   using H1 = Dense<D0, D1>;
-  using H2 = Dense<D1, (NL >= 3 ? D2 : 4)>;  // used only when NL >= 3
-  using H3 = Dense<D2, (NL >= 4 ? D3 : 4)>;  // used only when NL >= 4
+  using H2 = Dense<D1, (NL >= 3 ? D2 : 8)>;  // used only when NL >= 3
+  using H3 = Dense<D2, (NL >= 4 ? D3 : 8)>;  // used only when NL >= 4
   static constexpr int KOUT = NL == 2 ? D1 : (NL == 3 ? D2 : D3);  // width of the last hidden layer
-  static constexpr int NG_LAST = ng_for(KOUT);
   static constexpr int HMAX = (D1 > D2 ? D1 : D2) > D3 ? (D1 > D2 ? D1 : D2) : D3;
   // Rows of X: hidden outputs use [0, width); the output partials
-  // [0, 3 NG_LAST); the features [F0, F0 + D0), clear of the partials so
+  // [0, 3 kWarps); the features [F0, F0 + D0), clear of the partials so
   // that the next tile's features need no barrier after the RGB pass.
-  static constexpr int F0 = (3 * NG_LAST > HMAX - D0) ? 3 * NG_LAST : HMAX - D0;
+  static constexpr int F0 = (3 * kWarps > HMAX - D0) ? 3 * kWarps : HMAX - D0;
   static constexpr int XROWS = F0 + D0;
   static constexpr int OFF_H2 = H1::FLOATS;
   static constexpr int OFF_H3 = OFF_H2 + (NL >= 3 ? H2::FLOATS : 0);
@@ -272,6 +233,7 @@ __global__ void __launch_bounds__(kThreads, (Fp32Net<C, NL, D0, D1, D2, D3, D4, 
   const float* const Wout = sm_w + Net::OFF_OUT;
 
   const int tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
   const long long chunk = (p.total_tiles + gridDim.x - 1) / gridDim.x;
   const long long t_begin = blockIdx.x * chunk;
   const long long t_end = min(t_begin + chunk, p.total_tiles);
@@ -332,33 +294,33 @@ __global__ void __launch_bounds__(kThreads, (Fp32Net<C, NL, D0, D1, D2, D3, D4, 
 
     // ---- step 4: the synthesis MLP ----
     {
-      unsigned long long acc[H1::TP][H1::TN2];
-      dense_acc<H1, D0, false>(X + Net::F0 * kThreads, sm_w, tid / H1::NG, tid % H1::NG, acc);
+      unsigned long long acc[kTP][H1::TN2];
+      dense_acc<H1>(X + Net::F0 * kThreads, sm_w, lane, warp, acc);
       activate_acc<H1, ACT>(acc);
       __syncthreads();
       if constexpr (NL == 2)
-        store_out_partials<H1>(X, Wout, tid / H1::NG, tid % H1::NG, acc);
+        store_out_partials<H1>(X, Wout, lane, warp, acc);
       else
-        store_hidden<H1>(X, tid / H1::NG, tid % H1::NG, acc);
+        store_hidden<H1>(X, lane, warp, acc);
       __syncthreads();
     }
     if constexpr (NL >= 3) {
-      unsigned long long acc[H2::TP][H2::TN2];
-      dense_acc<H2, H1::TN, true>(X, sm_w + Net::OFF_H2, tid / H2::NG, tid % H2::NG, acc);
+      unsigned long long acc[kTP][H2::TN2];
+      dense_acc<H2>(X, sm_w + Net::OFF_H2, lane, warp, acc);
       activate_acc<H2, ACT>(acc);
       __syncthreads();
       if constexpr (NL == 3)
-        store_out_partials<H2>(X, Wout, tid / H2::NG, tid % H2::NG, acc);
+        store_out_partials<H2>(X, Wout, lane, warp, acc);
       else
-        store_hidden<H2>(X, tid / H2::NG, tid % H2::NG, acc);
+        store_hidden<H2>(X, lane, warp, acc);
       __syncthreads();
     }
     if constexpr (NL >= 4) {
-      unsigned long long acc[H3::TP][H3::TN2];
-      dense_acc<H3, H2::TN, true>(X, sm_w + Net::OFF_H3, tid / H3::NG, tid % H3::NG, acc);
+      unsigned long long acc[kTP][H3::TN2];
+      dense_acc<H3>(X, sm_w + Net::OFF_H3, lane, warp, acc);
       activate_acc<H3, ACT>(acc);
       __syncthreads();
-      store_out_partials<H3>(X, Wout, tid / H3::NG, tid % H3::NG, acc);
+      store_out_partials<H3>(X, Wout, lane, warp, acc);
       __syncthreads();
     }
 
@@ -367,11 +329,10 @@ __global__ void __launch_bounds__(kThreads, (Fp32Net<C, NL, D0, D1, D2, D3, D4, 
       const float* bo = Wout + Net::KOUT * 4;
       float o0 = bo[0], o1 = bo[1], o2 = bo[2];
 #pragma unroll
-      for (int g = 0; g < Net::NG_LAST; ++g) {
-        const int off = px_off(tid, g & 7);
-        o0 += X[(3 * g) * kThreads + off];
-        o1 += X[(3 * g + 1) * kThreads + off];
-        o2 += X[(3 * g + 2) * kThreads + off];
+      for (int g = 0; g < kWarps; ++g) {
+        o0 += X[(3 * g) * kThreads + tid];
+        o1 += X[(3 * g + 1) * kThreads + tid];
+        o2 += X[(3 * g + 2) * kThreads + tid];
       }
       store_rgb(p, b, y, x, o0, o1, o2);
     }
