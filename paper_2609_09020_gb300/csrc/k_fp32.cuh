@@ -30,8 +30,9 @@
 // image changes).
 //
 // Work split: the tiles of all images are numbered image-major and each CTA
-// takes one contiguous range of them (a CTA sees at most a couple of images
-// and loads each one's weights once).  Grid = resident CTAs over all SMs.
+// takes one contiguous range of them, all ranges within one tile of the same
+// length (a CTA sees at most a couple of images and loads each one's weights
+// once).  Grid = resident CTAs over all SMs.
 
 #pragma once
 
@@ -234,9 +235,9 @@ __global__ void __launch_bounds__(kThreads, (Fp32Net<C, NL, D0, D1, D2, D3, D4, 
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
-  const long long chunk = (p.total_tiles + gridDim.x - 1) / gridDim.x;
-  const long long t_begin = blockIdx.x * chunk;
-  const long long t_end = min(t_begin + chunk, p.total_tiles);
+  // balanced contiguous ranges: every CTA gets floor or ceil of tiles / CTAs
+  const long long t_begin = blockIdx.x * p.total_tiles / gridDim.x;
+  const long long t_end = (blockIdx.x + 1LL) * p.total_tiles / gridDim.x;
   const float* wts = static_cast<const float*>(p.weights);
   const long long plane = static_cast<long long>(p.H) * p.W;
   int cur_b = -1;
@@ -346,9 +347,9 @@ __global__ void __launch_bounds__(kThreads, (Fp32Net<C, NL, D0, D1, D2, D3, D4, 
 template <bool FL>
 __global__ void __launch_bounds__(kThreads) fp32_generic_kernel(const DecodeParams p) {
   extern __shared__ __align__(16) float sm_w[];
-  const long long chunk = (p.total_tiles + gridDim.x - 1) / gridDim.x;
-  const long long t_begin = blockIdx.x * chunk;
-  const long long t_end = min(t_begin + chunk, p.total_tiles);
+  // balanced contiguous ranges: every CTA gets floor or ceil of tiles / CTAs
+  const long long t_begin = blockIdx.x * p.total_tiles / gridDim.x;
+  const long long t_end = (blockIdx.x + 1LL) * p.total_tiles / gridDim.x;
   const float* wts = static_cast<const float*>(p.weights);
   int cur_b = -1;
   for (long long t = t_begin; t < t_end; ++t) {
