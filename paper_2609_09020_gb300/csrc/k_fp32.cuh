@@ -341,6 +341,151 @@ __global__ void __launch_bounds__(kThreads, (Fp32Net<C, NL, D0, D1, D2, D3, D4, 
 }
 
 // ---------------------------------------------------------------------------
+// Narrow nets (every hidden layer at most 16 wide): one thread per pixel with
+// the features and every activation in registers, no activation buffer and
+// no barrier per tile.  A 16-wide layer is only 16 FMAs per input, so the
+// tiled kernel's fixed per-tile work (staging, barriers, partial sums) would
+// outweigh the contraction.  Weights sit transposed in shared memory and are
+// read with broadcast 16-byte loads; packed f32x2 FMAs do two outputs per
+// instruction.
+
+__host__ __device__ constexpr int round4(int d) { return (d + 3) & ~3; }
+
+// Shared-memory image of one layer: W^T [din][round4(dout)] then the bias
+// [round4(dout)], zero padded.
+__host__ __device__ constexpr int px_layer_floats(int din, int dout) { return (din + 1) * round4(dout); }
+
+__device__ __forceinline__ void load_px_layer(float* __restrict__ sm, const float* __restrict__ w, int din,
+                                              int dout) {
+  const int d4 = round4(dout);
+  for (int e = threadIdx.x; e < (din + 1) * d4; e += kThreads) {
+    const int j = e / d4, i = e - j * d4;  // row j of W^T (j == din: the bias row), column i
+    float v = 0.0f;
+    if (i < dout) v = (j < din) ? w[i * din + j] : w[dout * din + i];
+    sm[e] = v;
+  }
+}
+
+// out = act(W in + b), or W in + b for the output layer.
+template <int DIN, int DOUT, int ACT, bool LAST, int MAXW>
+__device__ __forceinline__ void dense_px(const float* __restrict__ wt, const float (&in)[MAXW],
+                                         float (&out)[MAXW]) {
+  constexpr int D4 = round4(DOUT);
+  unsigned long long acc[D4 / 2];
+#pragma unroll
+  for (int i = 0; i < D4 / 4; ++i) {
+    const ulonglong2 b = *reinterpret_cast<const ulonglong2*>(wt + DIN * D4 + 4 * i);
+    acc[2 * i] = b.x;
+    acc[2 * i + 1] = b.y;
+  }
+#pragma unroll
+  for (int j = 0; j < DIN; ++j) {
+    const unsigned long long hh = pack2(in[j], in[j]);
+#pragma unroll
+    for (int i = 0; i < D4 / 4; ++i) {
+      const ulonglong2 w = *reinterpret_cast<const ulonglong2*>(wt + j * D4 + 4 * i);
+      acc[2 * i] = fma2(w.x, hh, acc[2 * i]);
+      acc[2 * i + 1] = fma2(w.y, hh, acc[2 * i + 1]);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < D4 / 2; ++i) {
+    if constexpr (ACT == ACT_GELU && !LAST) acc[i] = gelu_poly2(acc[i]);
+    const float2 v = unpack2(acc[i]);
+    const bool relu = !LAST && ACT == ACT_RELU;
+    if (2 * i < DOUT) out[2 * i] = relu ? fmaxf(v.x, 0.0f) : v.x;
+    if (2 * i + 1 < DOUT) out[2 * i + 1] = relu ? fmaxf(v.y, 0.0f) : v.y;
+  }
+}
+
+template <int C, int NL, int D0, int D1, int D2, int D3, int D4, int ACT>
+struct PxNet {
+  static constexpr int L = D0 / C;
+  static constexpr int MW = (D0 > 16 ? D0 : 16);  // widest vector a thread holds
+  static constexpr int OFF2 = px_layer_floats(D0, D1);
+  static constexpr int OFF3 = OFF2 + px_layer_floats(D1, D2);
+  static constexpr int OFF4 = OFF3 + (NL >= 3 ? px_layer_floats(D2, D3) : 0);
+  static constexpr int smem_floats() { return OFF4 + (NL >= 4 ? px_layer_floats(D3, D4) : 0); }
+};
+
+template <int C, int NL, int D0, int D1, int D2, int D3, int D4, int ACT, bool FL>
+__global__ void __launch_bounds__(kThreads) fp32_px_kernel(const DecodeParams p) {
+  using Net = PxNet<C, NL, D0, D1, D2, D3, D4, ACT>;
+  constexpr int L = Net::L;
+  constexpr int MW = Net::MW;
+  extern __shared__ __align__(16) float sm_w[];
+
+  const long long t_begin = blockIdx.x * p.total_tiles / gridDim.x;
+  const long long t_end = (blockIdx.x + 1LL) * p.total_tiles / gridDim.x;
+  const float* wts = static_cast<const float*>(p.weights);
+  const long long plane = static_cast<long long>(p.H) * p.W;
+  int cur_b = -1;
+
+  for (long long t = t_begin; t < t_end; ++t) {
+    const int b = static_cast<int>(t / p.tiles_per_image);
+    const long long r = t - static_cast<long long>(b) * p.tiles_per_image;
+    const int y = static_cast<int>(r / p.tiles_per_row);
+    const int x = static_cast<int>(r - static_cast<long long>(y) * p.tiles_per_row) * kThreads +
+                  threadIdx.x;
+    if (b != cur_b) {  // uniform across the CTA
+      __syncthreads();
+      const float* w = wts + b * p.params_per_image;
+      load_px_layer(sm_w, w, D0, D1);
+      w += D1 * D0 + D1;
+      load_px_layer(sm_w + Net::OFF2, w, D1, D2);
+      w += D2 * D1 + D2;
+      if constexpr (NL >= 3) {
+        load_px_layer(sm_w + Net::OFF3, w, D2, D3);
+        w += D3 * D2 + D3;
+      }
+      if constexpr (NL >= 4) load_px_layer(sm_w + Net::OFF4, w, D3, D4);
+      __syncthreads();
+      cur_b = b;
+    }
+    if (x >= p.W) continue;
+
+    // ---- steps 1-3: dequantise, upsample and concatenate every level ----
+    const int32_t* lat = p.latents + b * p.lat_per_image;
+    float h[MW], g[MW];
+#pragma unroll
+    for (int l = 0; l < L; ++l) {
+      const LevelGeom lg = p.lv[l];
+      const float step = FL ? 1.0f : __ldg(p.steps + b * L + l);
+      if (l == 0) {  // level 0 has the output size: the upsampling is the identity
+#pragma unroll
+        for (int c = 0; c < C; ++c)
+          h[c] = step * lat_value<FL>(__ldg(lat + c * plane + static_cast<long long>(y) * p.W + x));
+      } else {
+        const Tap tx = bilinear_tap(x, lg.sx, lg.W);
+        const Tap ty = bilinear_tap(y, lg.sy, lg.H);
+#pragma unroll
+        for (int c = 0; c < C; ++c)
+          h[l * C + c] = step * bilinear_sample<FL>(lat + lg.off + static_cast<long long>(c) * lg.H * lg.W,
+                                                    lg.W, tx, ty);
+      }
+    }
+
+    // ---- step 4: the synthesis MLP (ping-pong between h and g) ----
+    dense_px<D0, D1, ACT, false>(sm_w, h, g);
+    if constexpr (NL == 2) {
+      dense_px<D1, D2, ACT, true>(sm_w + Net::OFF2, g, h);
+    } else {
+      dense_px<D1, D2, ACT, false>(sm_w + Net::OFF2, g, h);
+      if constexpr (NL == 3) {
+        dense_px<D2, D3, ACT, true>(sm_w + Net::OFF3, h, g);
+        for (int c = 0; c < 3; ++c) h[c] = g[c];
+      } else {
+        dense_px<D2, D3, ACT, false>(sm_w + Net::OFF3, h, g);
+        dense_px<D3, D4, ACT, true>(sm_w + Net::OFF4, g, h);
+      }
+    }
+
+    // ---- step 5: clamp and store (planar rows are coalesced) ----
+    store_rgb(p, b, y, x, h[0], h[1], h[2]);
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Generic kernel: any dims up to kMaxDim, runtime loops, weights in shared
 // memory in the nn.Linear layout.  Slower (hidden values in local memory) but
 // covers every arch the C ABI accepts.
@@ -396,6 +541,7 @@ __global__ void __launch_bounds__(kThreads) fp32_generic_kernel(const DecodePara
 template <int C, int NL, int D0, int D1, int D2, int D3, int D4, int ACT, bool FL = false>
 KernelInfo make_fp32(const char* name) {
   using Net = Fp32Net<C, NL, D0, D1, D2, D3, D4, ACT>;
+  constexpr bool narrow = Net::HMAX <= 16;  // the one-thread-per-pixel kernel
   KernelInfo k{};
   k.name = name;
   k.precision = 0;
@@ -407,8 +553,13 @@ KernelInfo make_fp32(const char* name) {
   k.act = ACT;
   k.threads = kThreads;
   k.tile_px = kThreads;
-  k.smem_bytes = Net::smem_floats() * 4;
-  k.fn = reinterpret_cast<const void*>(&fp32_decode_kernel<C, NL, D0, D1, D2, D3, D4, ACT, FL>);
+  if constexpr (narrow) {
+    k.smem_bytes = PxNet<C, NL, D0, D1, D2, D3, D4, ACT>::smem_floats() * 4;
+    k.fn = reinterpret_cast<const void*>(&fp32_px_kernel<C, NL, D0, D1, D2, D3, D4, ACT, FL>);
+  } else {
+    k.smem_bytes = Net::smem_floats() * 4;
+    k.fn = reinterpret_cast<const void*>(&fp32_decode_kernel<C, NL, D0, D1, D2, D3, D4, ACT, FL>);
+  }
   return k;
 }
 
