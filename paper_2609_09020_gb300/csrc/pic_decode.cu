@@ -400,9 +400,33 @@ constexpr long long kChunkAlign = 256;
 
 long long align_up(long long v, long long a) { return (v + a - 1) / a * a; }
 
-// Per-chunk stride of a staging buffer holding `per_image` bytes per image
-// for up to `imgs` images of a chunk.
-long long chunk_stride(long long per_image, int imgs) { return align_up(per_image * imgs, kChunkAlign); }
+// Bytes of a staging buffer holding `per_image` bytes for each of `imgs`
+// images in up to kHostChunks chunks, each chunk starting on a
+// kChunkAlign-byte boundary.
+long long staging_bytes(long long per_image, int imgs) {
+  return align_up(per_image * imgs, kChunkAlign) + kHostChunks * kChunkAlign;
+}
+
+// Chunks of pic_decode_batch_host: image b0[c] .. b0[c+1] - 1 for chunk c.
+// The first chunks are one and two images, so that the copy-back (the
+// slowest stage: fp32 RGB is the largest buffer) starts after one image has
+// been copied in and decoded; the rest of the batch is split evenly over the
+// remaining chunks.  Returns the number of chunks.
+int host_chunks(int B, int (&b0)[kHostChunks + 1]) {
+  int n = 0, b = 0;
+  b0[0] = 0;
+  for (const int first : {1, 2}) {
+    if (b >= B) break;
+    b += first < B - b ? first : B - b;
+    b0[++n] = b;
+  }
+  const int left = B - b, rest = kHostChunks - n;
+  for (int i = 1; i <= rest && b < B; ++i) {
+    const int e = (B - left) + static_cast<int>(static_cast<long long>(left) * i / rest);
+    if (e > b) b0[++n] = b = e;
+  }
+  return n;
+}
 
 void free_host_pipeline(pic_decoder* h) {
   cudaFree(h->s_lat);
@@ -438,18 +462,15 @@ int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const f
   if (B < 1 || B > h->arch.max_batch || H < 1 || W < 1 || H > h->arch.max_H || W > h->arch.max_W)
     return PIC_ERR_INVALID_ARG;
   const pic_arch& a = h->arch;
-  const int per_chunk_max = (a.max_batch + kHostChunks - 1) / kHostChunks;
   const long long out_elem = a.output_format == PIC_OUT_U8_HWC ? 1 : 4;
   if (!h->s_lat) {
     const long long lat = pic_latent_count(a.max_H, a.max_W, a.num_levels, a.channels_per_level);
     bool ok =
-        cudaMalloc(&h->s_lat, kHostChunks * chunk_stride(lat * 4, per_chunk_max)) == cudaSuccess &&
-        cudaMalloc(&h->s_steps, kHostChunks * chunk_stride(a.num_levels * 4LL, per_chunk_max)) ==
-            cudaSuccess &&
-        cudaMalloc(&h->s_w, kHostChunks * chunk_stride(h->n_params * static_cast<long long>(weight_elem_bytes(a)),
-                                                       per_chunk_max)) == cudaSuccess &&
-        cudaMalloc(&h->s_out, kHostChunks * chunk_stride(3LL * a.max_H * a.max_W * 4, per_chunk_max)) ==
-            cudaSuccess;
+        cudaMalloc(&h->s_lat, staging_bytes(lat * 4, a.max_batch)) == cudaSuccess &&
+        cudaMalloc(&h->s_steps, staging_bytes(a.num_levels * 4LL, a.max_batch)) == cudaSuccess &&
+        cudaMalloc(&h->s_w, staging_bytes(h->n_params * static_cast<long long>(weight_elem_bytes(a)),
+                                          a.max_batch)) == cudaSuccess &&
+        cudaMalloc(&h->s_out, staging_bytes(3LL * a.max_H * a.max_W * 4, a.max_batch)) == cudaSuccess;
     if (ok && !h->p_ready) {
       ok = cudaStreamCreateWithFlags(&h->p_in, cudaStreamNonBlocking) == cudaSuccess &&
            cudaStreamCreateWithFlags(&h->p_run, cudaStreamNonBlocking) == cudaSuccess &&
@@ -468,12 +489,8 @@ int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const f
   const long long st_img = a.num_levels * 4LL;
   const long long w_img = h->n_params * static_cast<long long>(weight_elem_bytes(a));
   const long long out_img = 3LL * H * W * out_elem;
-  const long long lat_max = pic_latent_count(a.max_H, a.max_W, a.num_levels, a.channels_per_level) * 4;
-  const long long s_lat_stride = chunk_stride(lat_max, per_chunk_max);
-  const long long s_st_stride = chunk_stride(st_img, per_chunk_max);
-  const long long s_w_stride = chunk_stride(w_img, per_chunk_max);
-  const long long s_out_stride = chunk_stride(3LL * a.max_H * a.max_W * 4, per_chunk_max);
-  const int per_chunk = (B + kHostChunks - 1) / kHostChunks;
+  int b0s[kHostChunks + 1];
+  const int n_chunks = host_chunks(B, b0s);
   const bool have_steps = steps != nullptr;
   cudaEvent_t* ev = h->p_ev;  // [0]: start; then (in, run, out) per chunk
 
@@ -483,13 +500,19 @@ int pic_decode_batch_host(pic_decoder* h, int B, const int32_t* latents, const f
   };
   if (cudaEventRecord(ev[0], s) != cudaSuccess || cudaStreamWaitEvent(h->p_in, ev[0], 0) != cudaSuccess)
     return cuda_fail();
+  // chunk c's staging starts on a kChunkAlign boundary after chunk c - 1's
+  long long o_lat = 0, o_st = 0, o_w = 0, o_out = 0;
   int c = 0;
-  for (int b0 = 0; b0 < B; b0 += per_chunk, ++c) {
-    const int nb = B - b0 < per_chunk ? B - b0 : per_chunk;
-    unsigned char* d_lat = h->s_lat + c * s_lat_stride;
-    unsigned char* d_st = h->s_steps + c * s_st_stride;
-    unsigned char* d_w = h->s_w + c * s_w_stride;
-    unsigned char* d_out = h->s_out + c * s_out_stride;
+  for (; c < n_chunks; ++c) {
+    const int b0 = b0s[c], nb = b0s[c + 1] - b0s[c];
+    unsigned char* d_lat = h->s_lat + o_lat;
+    unsigned char* d_st = h->s_steps + o_st;
+    unsigned char* d_w = h->s_w + o_w;
+    unsigned char* d_out = h->s_out + o_out;
+    o_lat = align_up(o_lat + nb * lat_img, kChunkAlign);
+    o_st = align_up(o_st + nb * st_img, kChunkAlign);
+    o_w = align_up(o_w + nb * w_img, kChunkAlign);
+    o_out = align_up(o_out + nb * out_img, kChunkAlign);
     cudaEvent_t e_in = ev[1 + 3 * c], e_run = ev[2 + 3 * c], e_out = ev[3 + 3 * c];
     if (cudaMemcpyAsync(d_lat, reinterpret_cast<const unsigned char*>(latents) + b0 * lat_img, nb * lat_img,
                         cudaMemcpyHostToDevice, h->p_in) != cudaSuccess ||

@@ -75,6 +75,35 @@ def test_edge_shapes(orc, wl):
     _check_full(orc, wl)
 
 
+# Ragged shapes on every specialised architecture, with the kernel each one
+# must run on: the register-tiled contraction (a hidden layer wider than 16;
+# a row's last tile is partly past the image edge) and the one-thread-per-
+# pixel kernel (nets no wider than 16).  The batched cases put many images
+# into one CTA's tile range, so the weights are reloaded mid-range.
+EDGE_SPECIALISED = [
+    (wk.custom("c2arch_9x200", 9, 200, 7, 1, (7, 40, 40, 3), act="gelu"), "fp32_7x40x40x3_gelu"),
+    (wk.custom("c3arch_7x130", 7, 130, 7, 2, (14, 64, 64, 3)), "fp32_14x64x64x3_relu"),
+    (wk.custom("c4arch_5x383", 5, 383, 8, 2, (16, 64, 64, 64, 3), act="gelu", clip=63,
+               lap_scale=4.0), "fp32_16x64x64x64x3_gelu"),
+    (wk.custom("w32arch_6x250", 6, 250, 8, 1, (8, 32, 32, 32, 3)), "fp32_8x32x32x32x3_relu"),
+    (wk.custom("w64arch_3x131", 3, 131, 8, 1, (8, 64, 64, 64, 3)), "fp32_8x64x64x64x3_relu"),
+    (wk.custom("w8arch_4x140", 4, 140, 8, 1, (8, 8, 8, 8, 3)), "fp32_8x8x8x8x3_relu"),
+    (wk.custom("w16arch_2x77", 2, 77, 8, 1, (8, 16, 16, 16, 3)), "fp32_8x16x16x16x3_relu"),
+    (wk.custom("c5arch_x40_2x129", 2, 129, 7, 1, (7, 64, 64, 3), seed=30, batch=40),
+     "fp32_7x64x64x3_relu"),
+    (wk.custom("c1arch_x24_3x5", 3, 5, 4, 1, (4, 16, 16, 3), seed=70, batch=24), "fp32_4x16x16x3_relu"),
+]
+
+
+@pytest.mark.parametrize("wl,kernel", EDGE_SPECIALISED, ids=lambda c: getattr(c, "name", c))
+def test_edge_shapes_specialised(orc, wl, kernel):
+    from paper_2609_09020_gb300.pic import Decoder
+    dec = Decoder.for_workload(wl, P, max_batch=len(wl.seeds))
+    assert dec.kernel_name == kernel
+    dec.close()
+    _check_full(orc, wl)
+
+
 def test_generic_kernel_arch(orc):
     """An arch with no compile-time specialisation runs on the generic kernel."""
     from paper_2609_09020_gb300.pic import Decoder
