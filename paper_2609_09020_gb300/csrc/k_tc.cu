@@ -18,7 +18,7 @@ int tc_kernels(KernelInfo* out, int cap) {
       make_tc<1, 3, 7, 64, ACT_RELU, 4, false, false, true>("tc05_7x64x64x3_relu_lo8", d_c5),
       make_tc<2, 4, 16, 64, ACT_GELU, 4, false>("tc05_16x64x64x64x3_gelu", d_c4),
       make_tc<2, 3, 14, 64, ACT_RELU, 4, false>("tc05_14x64x64x3_relu", d_c3),
-      make_tc<1, 3, 7, 48, ACT_GELU, 4, false>("tc05_7x40x40x3_gelu", d_c2),
+      make_tc<1, 3, 7, 48, ACT_GELU, 4, false, false, false, 40>("tc05_7x40x40x3_gelu", d_c2),
       make_tc<1, 3, 4, 16, ACT_RELU, 4, false>("tc05_4x16x16x3_relu", d_c1),
   };
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));

@@ -149,10 +149,15 @@ struct ColLayout {
   static constexpr int total() { return off(L, 0); }
 };
 
-template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_, bool LO8_ = false>
+template <int C_, int NL_, int D0_, int N_, int ACT_, int NWG_, bool LO8_ = false, int NR_ = N_>
 struct TcNet {
   static constexpr int C = C_, NL = NL_, D0 = D0_, N = N_, ACT = ACT_, NWG = NWG_;
   static constexpr bool LO8 = LO8_;
+  // hidden neurons the net has (N is that rounded up to the MMA's N step):
+  // columns NR .. N - 1 hold zero weights and bias, so their accumulators are
+  // exactly +0 and the epilogues write +0 there without computing anything
+  static constexpr int NR = NR_;
+  static_assert(NR_ >= 1 && NR_ <= N_, "real hidden width within the tile");
   static constexpr int SEG = C == 1 ? 32 : kTile;  // staging segment: a warp's pixels or the group's
   static constexpr int NSEG = kTile / SEG;         // segments (column buffers) per group
   // Hidden operand layout in tensor memory: per 16-value chunk the hi and the
@@ -350,6 +355,7 @@ __device__ __forceinline__ void output_layer_cc(const uint8_t* smem, uint32_t t_
     tmem_ld_wait();
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
+      if (h0 + 2 * q >= Net::NR) continue;  // padding: act(+0) = +0 adds nothing
       unsigned long long hv;
       if constexpr (Net::ACT == ACT_GELU) {
         hv = gelu_poly2(pack2(__uint_as_float(acc[2 * q]), __uint_as_float(acc[2 * q + 1])));
@@ -385,6 +391,11 @@ __device__ __forceinline__ void hidden_epilogue(uint32_t t_acc, uint32_t t_a) {
     uint32_t hl[16];  // [0, 8): hi pairs, [8, 16): lo pairs
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
+      if (h0 + 2 * q >= Net::NR) {  // padding columns: act(+0) = +0, split into +0 and +0
+        hl[q] = 0u;
+        hl[8 + q] = 0u;
+        continue;
+      }
       float a = __uint_as_float(acc[2 * q]);
       float bb = __uint_as_float(acc[2 * q + 1]);
       if constexpr (Net::ACT == ACT_GELU) {
@@ -980,9 +991,10 @@ __global__ void __launch_bounds__(Net::THREADS) __maxnreg__(Net::MAXREG)
   }
 }
 
-template <int C, int NL, int D0, int N, int ACT, int NWG, bool FL, bool TMA = false, bool LO8 = false>
+template <int C, int NL, int D0, int N, int ACT, int NWG, bool FL, bool TMA = false, bool LO8 = false,
+          int NR = N>
 KernelInfo make_tc(const char* name, const int* dims) {
-  using Net = TcNet<C, NL, D0, N, ACT, NWG, LO8>;
+  using Net = TcNet<C, NL, D0, N, ACT, NWG, LO8, NR>;
   KernelInfo k{};
   k.name = name;
   k.precision = LO8 ? 2 : 1;

@@ -15,7 +15,7 @@ const int d_w64[] = {8, 64, 64, 64, 3};
 
 int tc_kernels_sweep(KernelInfo* out, int cap) {
   const KernelInfo list[] = {
-      make_tc<1, 4, 8, 16, ACT_RELU, 4, false>("tc05_8x8x8x8x3_relu", d_w8),
+      make_tc<1, 4, 8, 16, ACT_RELU, 4, false, false, false, 8>("tc05_8x8x8x8x3_relu", d_w8),
       make_tc<1, 4, 8, 16, ACT_RELU, 4, false>("tc05_8x16x16x16x3_relu", d_w16),
       make_tc<1, 4, 8, 32, ACT_RELU, 4, false>("tc05_8x32x32x32x3_relu", d_w32),
       make_tc<1, 4, 8, 64, ACT_RELU, 4, false>("tc05_8x64x64x64x3_relu", d_w64),

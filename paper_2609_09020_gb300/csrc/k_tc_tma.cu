@@ -26,7 +26,7 @@ int tc_kernels_tma(KernelInfo* out, int cap) {
       tma_auto(make_tc<1, 3, 7, 64, ACT_RELU, 4, false, true>("tc05_7x64x64x3_relu_tma", d_c5), false),
       tma_auto(make_tc<2, 4, 16, 64, ACT_GELU, 4, false, true>("tc05_16x64x64x64x3_gelu_tma", d_c4), false),
       tma_auto(make_tc<2, 3, 14, 64, ACT_RELU, 4, false, true>("tc05_14x64x64x3_relu_tma", d_c3), false),
-      tma_auto(make_tc<1, 3, 7, 48, ACT_GELU, 4, false, true>("tc05_7x40x40x3_gelu_tma", d_c2), false),
+      tma_auto(make_tc<1, 3, 7, 48, ACT_GELU, 4, false, true, false, 40>("tc05_7x40x40x3_gelu_tma", d_c2), false),
       tma_auto(make_tc<1, 3, 4, 16, ACT_RELU, 4, false, true>("tc05_4x16x16x3_relu_tma", d_c1), true),
   };
   const int n = static_cast<int>(sizeof(list) / sizeof(list[0]));
