@@ -1,8 +1,9 @@
 """pic_decode_batch_host runs copy-in, decode and copy-out of chunks of
 images on three streams; its output must be bit-identical to the device
-path (same kernels), for batch sizes that do not divide into the chunks,
-weight blobs whose size makes per-chunk offsets unaligned, and every output
-and latent format."""
+path (same kernels), for batch sizes that end inside the first chunks (one
+image, then two), that do not divide into the remaining chunks, weight blobs
+whose size makes per-chunk offsets unaligned, and every output and latent
+format."""
 import numpy as np
 import pytest
 
@@ -43,7 +44,7 @@ def _both(wl, precision, output="f32_chw", latent="int32", B=None, max_batch=Non
     return host.numpy(), dev.cpu().numpy()
 
 
-@pytest.mark.parametrize("B", [1, 5, 13, 64])
+@pytest.mark.parametrize("B", [1, 2, 3, 5, 13, 17, 64])
 def test_host_pipeline_equals_device_path_tc(B):
     got, ref = _both(wk.WORKLOADS["c5"], "fp16_tc", B=B, max_batch=64)
     assert np.array_equal(got, ref)
