@@ -67,8 +67,9 @@ def algorithmic(wl: wk.Workload, batch: int):
 
 
 # FP32-pipe operations of one GELU evaluation in the kernels (pic_gelu.cuh):
-# z^2, the affine map, the Horner steps, the saturating fma and z * Phi.
-GELU_FP32_OPS = 4 + 12
+# z^2, the Horner steps of P (5) and Q (4), P * (1 / Q), the saturating fma
+# and z * Phi; the reciprocal itself runs on the special-function unit.
+GELU_FP32_OPS = 4 + 5 + 4
 
 
 def executed_tensor_macs_per_px(wl: wk.Workload) -> int:

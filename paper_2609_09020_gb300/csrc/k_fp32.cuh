@@ -140,7 +140,7 @@ __device__ __forceinline__ void activate_acc(unsigned long long (&acc)[kTP][Ly::
 #pragma unroll
     for (int j = 0; j < Ly::TN2; ++j) {
       if constexpr (ACT == ACT_GELU) {
-        acc[p][j] = gelu_poly2(acc[p][j]);
+        acc[p][j] = gelu_approx2(acc[p][j]);
       } else {
         const float2 v = unpack2(acc[p][j]);
         acc[p][j] = pack2(fmaxf(v.x, 0.0f), fmaxf(v.y, 0.0f));
@@ -390,7 +390,7 @@ __device__ __forceinline__ void dense_px(const float* __restrict__ wt, const flo
   }
 #pragma unroll
   for (int i = 0; i < D4 / 2; ++i) {
-    if constexpr (ACT == ACT_GELU && !LAST) acc[i] = gelu_poly2(acc[i]);
+    if constexpr (ACT == ACT_GELU && !LAST) acc[i] = gelu_approx2(acc[i]);
     const float2 v = unpack2(acc[i]);
     const bool relu = !LAST && ACT == ACT_RELU;
     if (2 * i < DOUT) out[2 * i] = relu ? fmaxf(v.x, 0.0f) : v.x;

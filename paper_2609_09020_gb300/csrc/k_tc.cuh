@@ -358,7 +358,7 @@ __device__ __forceinline__ void output_layer_cc(const uint8_t* smem, uint32_t t_
       if (h0 + 2 * q >= Net::NR) continue;  // padding: act(+0) = +0 adds nothing
       unsigned long long hv;
       if constexpr (Net::ACT == ACT_GELU) {
-        hv = gelu_poly2(pack2(__uint_as_float(acc[2 * q]), __uint_as_float(acc[2 * q + 1])));
+        hv = gelu_approx2(pack2(__uint_as_float(acc[2 * q]), __uint_as_float(acc[2 * q + 1])));
       } else {
         hv = pack2(fmaxf(__uint_as_float(acc[2 * q]), 0.0f),
                    fmaxf(__uint_as_float(acc[2 * q + 1]), 0.0f));
@@ -399,7 +399,7 @@ __device__ __forceinline__ void hidden_epilogue(uint32_t t_acc, uint32_t t_a) {
       float a = __uint_as_float(acc[2 * q]);
       float bb = __uint_as_float(acc[2 * q + 1]);
       if constexpr (Net::ACT == ACT_GELU) {
-        const float2 g = unpack2(gelu_poly2(pack2(a, bb)));
+        const float2 g = unpack2(gelu_approx2(pack2(a, bb)));
         a = g.x;
         bb = g.y;
       }

@@ -141,41 +141,54 @@ __device__ __forceinline__ unsigned long long mul2(unsigned long long a, unsigne
   return d;
 }
 
-// GELU z * Phi(z) without special-function units or branches (the
-// polynomial P of gen_gelu_poly.py, max abs error ~1.1e-6 in fp32):
-//   t = min(z^2, Z^2), u = t * 2/Z^2 - 1, Phi = saturate(1/2 + z P(u)),
+// 1 / x on the special-function unit (rcp.approx: within an ulp; x >= 1
+// wherever the GELU uses it).
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+
+// GELU z * Phi(z) without branches (the rational function of gen_gelu.py,
+// max abs error ~1.2e-6 in fp32):
+//   s = min(z^2, Z^2), Phi = saturate(1/2 + z P(s) / Q(s)),
 // the saturation being both the clamp Phi in [0, 1] and the value beyond Z.
-__device__ __forceinline__ float gelu_poly(float z) {
-  const float t = fminf(z * z, kGeluZ2);
-  const float u = fmaf(t, kGeluUScale, -1.0f);
-  float p = gelu_coef(0);
+// 13 FP32-pipe operations and one reciprocal per value.
+__device__ __forceinline__ float gelu_approx(float z) {
+  const float s = fminf(z * z, kGeluZ2);
+  float pn = gelu_p(0), qd = gelu_q(0);
 #pragma unroll
-  for (int i = 1; i <= kGeluDegree; ++i) p = fmaf(p, u, gelu_coef(i));
-  return z * __saturatef(fmaf(z, p, 0.5f));
+  for (int i = 1; i <= kGeluDegP; ++i) pn = fmaf(pn, s, gelu_p(i));
+#pragma unroll
+  for (int i = 1; i <= kGeluDegQ; ++i) qd = fmaf(qd, s, gelu_q(i));
+  return z * __saturatef(fmaf(z, pn * rcp_approx(qd), 0.5f));
 }
 
 // The same on a pair of values packed in 64 bits: the multiplies and the
-// Horner chain run as packed f32x2 instructions (one instruction, two
-// operations), with the same roundings as gelu_poly on each half.
-__device__ __forceinline__ unsigned long long gelu_poly2(unsigned long long v) {
+// Horner chains run as packed f32x2 instructions (one instruction, two
+// operations), with the same roundings as gelu_approx on each half.
+__device__ __forceinline__ unsigned long long gelu_approx2(unsigned long long v) {
   const float2 zz = unpack2(mul2(v, v));
-  const unsigned long long t = pack2(fminf(zz.x, kGeluZ2), fminf(zz.y, kGeluZ2));
-  const unsigned long long u = fma2(t, pack2(kGeluUScale, kGeluUScale), pack2(-1.0f, -1.0f));
-  unsigned long long p = pack2(gelu_coef(0), gelu_coef(0));
+  const unsigned long long s = pack2(fminf(zz.x, kGeluZ2), fminf(zz.y, kGeluZ2));
+  unsigned long long pn = pack2(gelu_p(0), gelu_p(0)), qd = pack2(gelu_q(0), gelu_q(0));
 #pragma unroll
-  for (int i = 1; i <= kGeluDegree; ++i) p = fma2(p, u, pack2(gelu_coef(i), gelu_coef(i)));
-  const float2 z = unpack2(v), pp = unpack2(p);
-  return mul2(v, pack2(__saturatef(fmaf(z.x, pp.x, 0.5f)), __saturatef(fmaf(z.y, pp.y, 0.5f))));
+  for (int i = 1; i <= kGeluDegP; ++i) pn = fma2(pn, s, pack2(gelu_p(i), gelu_p(i)));
+#pragma unroll
+  for (int i = 1; i <= kGeluDegQ; ++i) qd = fma2(qd, s, pack2(gelu_q(i), gelu_q(i)));
+  const float2 q = unpack2(qd);
+  const float2 r = unpack2(mul2(pn, pack2(rcp_approx(q.x), rcp_approx(q.y))));
+  const float2 z = unpack2(v);
+  return mul2(v, pack2(__saturatef(fmaf(z.x, r.x, 0.5f)), __saturatef(fmaf(z.y, r.y, 0.5f))));
 }
 
 template <int ACT>
 __device__ __forceinline__ float activate(float z) {
-  if constexpr (ACT == ACT_GELU) return gelu_poly(z);
+  if constexpr (ACT == ACT_GELU) return gelu_approx(z);
   else return fmaxf(z, 0.0f);
 }
 
 __device__ __forceinline__ float activate_rt(float z, int act) {
-  return act == ACT_GELU ? gelu_poly(z) : fmaxf(z, 0.0f);
+  return act == ACT_GELU ? gelu_approx(z) : fmaxf(z, 0.0f);
 }
 
 // Bilinear source coordinate of output index x along one axis: the pixel
