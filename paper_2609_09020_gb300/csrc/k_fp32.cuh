@@ -2,10 +2,12 @@
 // instantiated in k_fp32.cu (the decode workloads' architectures, the
 // generic kernel, the registry) and k_fp32_sweep.cu (the width ablation).
 //
-// The decode fused on the fp32 CUDA cores.
+// The decode fused on the fp32 CUDA cores, in two kernels: the
+// register-tiled contraction below (nets with a hidden layer wider than 16)
+// and, further down, one thread per pixel for narrower nets.
 //
-// A CTA of 128 threads decodes tiles of 128 consecutive pixels of one image
-// row.  Per tile:
+// Register-tiled: a CTA of 128 threads decodes tiles of 128 consecutive
+// pixels of one image row.  Per tile:
 //   1. features: thread p dequantises and upsamples every pyramid level for
 //      pixel p (Sec. 3.1, Eq. 1) and writes the feature vector into a
 //      shared-memory activation buffer X (one row of 128 floats per
