@@ -170,13 +170,16 @@ int pic_decode_batch(pic_decoder *h, int B, const int32_t *latents, const float 
 
 /*
  * End-to-end convenience for callers holding HOST buffers (same layouts as
- * pic_decode_batch, host pointers, preferably pinned): copies the inputs to
- * device buffers owned by the handle, decodes, copies the RGB back, and
- * synchronises `stream` before returning.  The batch runs as a pipeline over
- * up to 16 chunks of images on three internal streams (copy-in, decode,
- * copy-out), ordered after the work already queued on `stream`, so that the
- * copies of one chunk overlap the decode of another; the output is identical
- * to pic_decode_batch's.  The staging buffers and streams are allocated on
+ * pic_decode_batch, host pointers): copies the inputs to device buffers owned
+ * by the handle, decodes, copies the RGB back, and synchronises `stream`
+ * before returning.  The batch runs as a pipeline over up to 16 chunks of
+ * images on three internal streams (copy-in, decode, copy-out), ordered after
+ * the work already queued on `stream`, so that the copies of one chunk
+ * overlap the decode of another; the first two chunks are one and two images,
+ * so that the copy-back starts early.  The output is identical to
+ * pic_decode_batch's.  The copies overlap only when the host buffers are
+ * page-locked (cudaHostAlloc / cudaHostRegister); with pageable memory the
+ * result is the same but the copies run one after another.  The staging buffers and streams are allocated on
  * first use (for max_batch images of max_H x max_W) and kept until destroy;
  * calls on one handle must not overlap.
  * Errors: as pic_decode_batch, plus PIC_ERR_ALLOC.
